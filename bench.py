@@ -1,0 +1,386 @@
+"""Throughput of the Gram-Space codebook hot path on GB300.
+
+Headline workload: large-batch fused project + similarity + argmax, bipolar
+codebook M = 256, D = 8192, 65,536 queries (codeword + N(0,1) noise), fp32
+queries resident in HBM (2 GiB, larger than the 129 MB L2, so no flush is
+needed between steps).  One step = one gs_project_similarity call over the
+whole batch (argmax + maxval written).  The basis build is initialisation
+(paper Sec. 3.3) and is timed separately.
+
+Prints ONE JSON line (rank 0).  `value` is queries/s over all ranks; `e2e`
+repeats the measurement through the same API with the queries in pinned host
+memory, copied in and the results copied out inside the timed region.
+`--impl reference` times the float64 CPU oracle instead (the reference arm).
+
+Multi-GPU: every rank runs its own copy of the workload (independent query
+batches, no collective on the data path): weak scaling.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "project+similarity queries/s"
+WORKLOAD = "large-batch fused project+similarity+argmax, bipolar M=256, D=8192, 65536 queries (sigma=1)"
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--path", default="auto", choices=["auto", "simt", "tensor"])
+    p.add_argument("--no-rows", action="store_true", help="skip the per-row side measurements")
+    p.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline leg")
+    return p.parse_args()
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return {"hbm_gbs": float(d["hbm_gbs"]), "bf16_tflops": float(d["bf16_tflops"]),
+                "bf16_tflops_sustained": float(d.get("bf16_tflops_sustained", d["bf16_tflops"])),
+                "src": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "src": "fallback"}
+
+
+def traffic_record(kernel_file, key):
+    """DRAM traffic per launch from a committed ncu summary, valid only while the
+    kernel source is unchanged (sha256 recorded next to the number)."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)[key]
+        src = os.path.join(ROOT, "paper_2608_01528_gb300", "csrc", kernel_file)
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        return rec["bytes_per_launch"] if rec.get("source_sha256") == h else None
+    except Exception:
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples while the timed region runs."""
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.file = None
+
+    def __enter__(self):
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.file, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if getattr(self, "_summary", None) is not None:
+            return self._summary
+        if self.proc is None or self.file is None:
+            return None
+        self.file.seek(0)
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.file.read().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        os.unlink(self.file.name)
+        self.file = None
+        if not sm:
+            return None
+        self._summary = {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                         "samples": len(sm)}
+        return self._summary
+
+
+def cpu_baseline(seconds=10.0):
+    """The float64 oracle on the host cores, on a bounded sample of the workload."""
+    import numpy as np
+    import synth
+    from oracle import oracle as O
+    C = synth.large_codebook()
+    Q, R, cn = O.build_basis(C)
+    w = synth.large(rows=(0, 256))
+    t0 = time.perf_counter()
+    O.project_similarity(w["X"], Q, R, cn)
+    t1 = time.perf_counter() - t0
+    n = int(max(256, min(65536, 256 * seconds / max(t1, 1e-3))) // 256 * 256)
+    w = synth.large(rows=(0, n))
+    t0 = time.perf_counter()
+    out = O.project_similarity(w["X"], Q, R, cn)
+    dt = time.perf_counter() - t0
+    assert np.array_equal(out["argmax"], w["labels"])
+    return {"value": n / dt, "unit": "queries/s", "cores": O.num_threads(), "kind": "oracle",
+            "sample": f"first {n} of 65536 queries (float64 oracle: project + similarity + argmax)",
+            "seconds": round(dt, 3)}
+
+
+def run_reference(args):
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return
+    import numpy as np
+    import synth
+    from oracle import oracle as O
+    C = synth.large_codebook()
+    Q, R, cn = O.build_basis(C)
+    n = 1024
+    w = synth.large(rows=(0, n))
+    for _ in range(args.warmup):
+        O.project_similarity(w["X"][:256], Q, R, cn)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        out = O.project_similarity(w["X"], Q, R, cn)
+        times.append(time.perf_counter() - t0)
+    assert np.array_equal(out["argmax"], w["labels"])
+    dt = sum(times)
+    v = n * args.steps / dt
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "queries/s", "n_gpus": 0,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD, "sample_rows_per_step": n},
+            "cpu_baseline": {"value": v, "unit": "queries/s", "cores": O.num_threads(), "kind": "oracle",
+                             "sample": f"first {n} of 65536 queries per step"},
+            "e2e": {"value": v, "unit": "queries/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+        return
+    ws, rank, local = dist_env()
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu:
+        # the oracle leg runs before CUDA is touched (no forked workers after GPU init)
+        cpu = cpu_baseline()
+
+    import numpy as np
+    import torch
+    import synth
+    from paper_2608_01528_gb300 import gramspace as gs
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+
+    w = synth.large()
+    N, D = w["X"].shape
+    M = w["C"].shape[0]
+    Xh = torch.from_numpy(w["X"]).pin_memory()
+    X = Xh.to(dev)
+    C = torch.from_numpy(w["C"]).to(dev)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    basis = gs.build_basis(C)
+    torch.cuda.synchronize()
+    build_ms = 1e3 * (time.perf_counter() - t0)
+    r = basis.r
+    am = torch.empty(N, dtype=torch.int32, device=dev)
+    mv = torch.empty(N, dtype=torch.float32, device=dev)
+    outs = {"argmax": am, "maxval": mv}
+    stream = torch.cuda.current_stream()
+
+    def step():
+        gs.project_similarity(basis, X, path=args.path, out=outs)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    gs.stream_status()
+    ok = bool(np.array_equal(am.cpu().numpy(), w["labels"]))
+
+    def barrier():
+        if pg is not None:
+            pg.barrier()
+        torch.cuda.synchronize()
+
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        barrier()
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+        e1.record(stream)
+        barrier()
+    ms = e0.elapsed_time(e1)
+    if pg is not None:
+        t = torch.tensor([ms], device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        ms = float(t.item())
+    gs.stream_status()
+    per_step_ms = ms / args.steps
+    value = N * ws * args.steps / (ms / 1e3)
+
+    # end to end through the same API: pinned host queries in, argmax/maxval out
+    amh = torch.empty(N, dtype=torch.int32).pin_memory()
+    mvh = torch.empty(N, dtype=torch.float32).pin_memory()
+
+    def step_e2e():
+        X.copy_(Xh, non_blocking=True)
+        gs.project_similarity(basis, X, path=args.path, out=outs)
+        amh.copy_(am, non_blocking=True)
+        mvh.copy_(mv, non_blocking=True)
+
+    for _ in range(2):
+        step_e2e()
+    barrier()
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ke = max(3, args.steps // 4)
+    f0.record(stream)
+    for _ in range(ke):
+        step_e2e()
+    f1.record(stream)
+    barrier()
+    ms_e2e = f0.elapsed_time(f1)
+    if pg is not None:
+        t = torch.tensor([ms_e2e], device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        ms_e2e = float(t.item())
+    e2e = {"value": N * ws * ke / (ms_e2e / 1e3), "unit": "queries/s",
+           "h2d_bytes_per_step": N * D * 4, "d2h_bytes_per_step": N * 8}
+    ok = ok and bool(np.array_equal(amh.numpy(), w["labels"]))
+
+    # roofline of the dominant (only, on the tensor-core path) kernel of the step
+    peaks = load_peaks()
+    alg_bytes = N * D * 4 + N * 8 + r * D * 2 + M * r * 4
+    achieved = alg_bytes / (per_step_ms / 1e3) / 1e9
+    tc = args.path == "tensor" or (args.path == "auto" and basis.r <= 256)
+    kernel = "k_ps_tc" if tc else "k_gemm (simt)"
+    roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": round(achieved / peaks["hbm_gbs"], 4), "peak_src": peaks["src"],
+            "traffic": traffic_record("gs_tc.cu", "k_ps_tc/large") if tc else None, "kernel": kernel,
+            "algorithmic_bytes_per_launch": alg_bytes}
+
+    rows = None
+    if not args.no_rows and rank == 0:
+        rows = side_rows(gs, dev)
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "queries/s", "n_gpus": ws, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": per_step_ms, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f16xf16->f32 (proj), f32 (scores)",
+                "data": "synthetic",
+                "config": {"workload": WORKLOAD, "N": N, "D": D, "M": M, "r": r, "path": args.path,
+                           "l2": "inputs (2 GiB) larger than L2; no flush", "parallelism": f"replicas x{ws}"},
+                "hbm_gbs": round(achieved, 1), "codebook_bytes_ratio": {
+                    "coefficient_D_over_r": D / r, "total_MD_over_rD_plus_Mr": (M * D) / (r * D + M * r)},
+                "roofline": roof, "e2e": e2e, "gpu_launches": args.steps * (1 if tc else 3),
+                "build_ms": round(build_ms, 2), "argmax_matches_labels": ok}
+        if cpu is not None:
+            line["cpu_baseline"] = cpu
+        clocks = clk.summary()
+        if clocks is not None:
+            line["clocks"] = clocks
+        if rows:
+            line["rows"] = rows
+        print(json.dumps(line), flush=True)
+    if pg is not None:
+        pg.destroy_process_group()
+
+
+def side_rows(gs, dev):
+    """One timed measurement per other hot-path row (small, HBM-resident inputs)."""
+    import torch
+    import synth
+    out = {}
+
+    def timeit(fn, reps=10):
+        for _ in range(3):
+            fn()
+        s = torch.cuda.current_stream()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(s)
+        for _ in range(reps):
+            fn()
+        b.record(s)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps
+
+    # build (init-time) on the rank-deficient binary codebook
+    C4, _ = synth.rankdef_codebook()
+    C4d = torch.from_numpy(C4).to(dev)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    b4 = gs.build_basis(C4d)
+    torch.cuda.synchronize()
+    out["build_rankdef_ms"] = round(1e3 * (time.perf_counter() - t0), 2)
+    out["build_rankdef_r"] = b4.r
+    # reconstruct 16,384 x 922 -> 16,384 x 10,000
+    T = torch.randn(16384, b4.r, device=dev)
+    Xh = torch.empty(16384, 10000, device=dev)
+    ms = timeit(lambda: gs.reconstruct(b4, T, out=Xh))
+    out["reconstruct_rankdef_ms"] = round(ms, 4)
+    out["reconstruct_rankdef_gflops"] = round(2 * 16384 * b4.r * 10000 / (ms / 1e3) / 1e9, 1)
+    # prob-vectorize + attention on the attention workload (64 x 1024, r = 512)
+    a = synth.attention()
+    b5 = gs.build_basis(torch.from_numpy(a["C"]).to(dev))
+    Pq = torch.from_numpy(a["Pq"]).to(dev)
+    Vq = torch.empty(Pq.shape[0], b5.r, dtype=torch.bfloat16, device=dev)
+    ms = timeit(lambda: gs.prob_vectorize(b5, Pq, out=Vq))
+    out["probvec_attention_ms"] = round(ms, 4)
+    out["probvec_attention_gbs"] = round((Pq.numel() * 4 + Vq.numel() * 2) / (ms / 1e3) / 1e9, 1)
+    V3 = Vq.reshape(64, 1024, -1)
+    A = torch.empty(64, 1024, 1024, device=dev)
+    ms = timeit(lambda: gs.attention_scores(V3, V3, 1 / 64.0, out=A))
+    out["attention_ms"] = round(ms, 4)
+    out["attention_gbs"] = round((2 * V3.numel() * 2 + A.numel() * 4) / (ms / 1e3) / 1e9, 1)
+    out["attention_tflops"] = round(2 * 64 * 1024 * 1024 * b5.r / (ms / 1e3) / 1e12, 1)
+    del b4, b5
+    return out
+
+
+if __name__ == "__main__":
+    main()

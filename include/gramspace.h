@@ -1,0 +1,190 @@
+/*
+ * gramspace.h -- C ABI of the GB300 (sm_103a) Gram-Space codebook library.
+ *
+ * Gram-Space (Wang & Li, "Gram-Space: Structure-Preserving Codebook
+ * Compression for Memory-Efficient Neuro-Symbolic AI") replaces a VSA codebook
+ * by an orthonormal basis of its span and the codewords' coordinates in that
+ * basis ("Gram-loc"), runs matrix-space operators (similarity, probability
+ * vectorization, attention scores) on the coordinates, and reconstructs
+ * full vectors only before component-wise operators.
+ *
+ * Notation.  The paper stores the codebook as W (D x M, one atom per column),
+ * the basis as U (D x k) and the Gram-loc codebook T = U^T W (k x M) (Sec. 3.1,
+ * Eq. 1).  This library stores every matrix row-major with one vector per
+ * row:  C = W^T (M x D),  Q = U^T (r x D, r = k),  R = T^T (M x r),  C = R Q.
+ * The Gram-loc of a query x (t = U^T x, Sec. 3.1) is the row y = x Q^T.
+ *
+ * Conventions shared by every entry point:
+ *  - Array arguments are DEVICE pointers owned by the caller unless a
+ *    function says otherwise.  The library owns only what a gs_basis holds.
+ *  - Matrices are row-major; ld* arguments are leading dimensions in
+ *    elements (ld >= number of columns).
+ *  - Work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *    stream) and returns before it finishes.  Argument errors are detected on
+ *    the host and returned immediately with nothing enqueued.
+ *  - Errors that only the device can see (a bounded wait that ran out, an
+ *    input outside a fast path's numeric range) set a per-device error word;
+ *    gs_stream_status() synchronises the stream and returns and clears it.
+ *  - Only gs_build_basis (and gs_basis_reserve_host_staging) allocate device
+ *    memory; the other calls allocate nothing.  N = 0 is a valid no-op.
+ *  - All functions are callable from any host thread; a gs_basis must not be
+ *    destroyed while work that uses it is in flight.
+ */
+#ifndef GRAMSPACE_H
+#define GRAMSPACE_H
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Every entry point is exported from the shared library; everything else in
+ * it has hidden visibility. */
+#if defined(__GNUC__)
+#define GS_API __attribute__((visibility("default")))
+#else
+#define GS_API
+#endif
+
+typedef enum gs_status {
+    GS_OK = 0,
+    GS_ERR_INVALID_ARG = 1,  /* null pointer, negative size or unknown enum/flag   */
+    GS_ERR_ALIGNMENT = 2,    /* pointer or leading dimension not aligned as stated */
+    GS_ERR_SHAPE = 3,        /* sizes inconsistent with the basis or beyond limits */
+    GS_ERR_NOMEM = 4,        /* a device allocation failed                          */
+    GS_ERR_CUDA = 5,         /* a CUDA runtime / driver call failed                 */
+    GS_ERR_TIMEOUT = 6,      /* a bounded device-side wait gave up (device word)    */
+    GS_ERR_RANGE = 7,        /* an input exceeded the fp16 range of the tensor-core
+                                path (|x| > 65504); results of that call are invalid,
+                                rerun it with GS_PATH_SIMT (device word)            */
+    GS_ERR_UNSUPPORTED = 8   /* no sm_103 device, or a forced path cannot run      */
+} gs_status;
+
+typedef enum gs_dtype { GS_F32 = 0, GS_BF16 = 1 } gs_dtype;
+
+typedef enum gs_score_mode {
+    GS_SCORE_RAW = 0,      /* S = scale * <y, R_i>                          */
+    GS_SCORE_COSINE = 1,   /* S = scale * <y, R_i> / (||x|| * ||c_i||)      */
+    GS_SCORE_SOFTMAX = 2   /* S = softmax_i(scale * <y, R_i>) over M atoms  */
+} gs_score_mode;
+
+/* gs_build_basis flags */
+#define GS_BUILD_NORMALIZE_ROWS 0x1u /* build on c_i / ||c_i|| ("each atomic vector
+                                        undergoes normalization", Sec. 3.1)       */
+
+/* path-selection flags of the apply calls (at most one) */
+#define GS_PATH_AUTO 0x0u   /* pick by problem size                                 */
+#define GS_PATH_SIMT 0x1u   /* fp32 CUDA-core kernels: fp32 accumulation, any range */
+#define GS_PATH_TENSOR 0x2u /* tcgen05 tensor-core kernels (GS_ERR_UNSUPPORTED when
+                               the shape has no tensor-core kernel)                 */
+
+typedef struct gs_basis gs_basis;
+
+/*
+ * Basis construction (Sec. 3.1, Eq. 1; built once "during initialization" by
+ * Gram-Schmidt, Sec. 3.3; rank k = algebraic rank, Sec. 3.2).
+ *
+ * Orthonormalises the rows of C (M x D, fp32, ld = ldc) in row order by
+ * Gram-Schmidt with two projection passes per row (reorthogonalisation),
+ * computed in fp64 on the device in panels of rows.  Row i is accepted as a
+ * new basis direction when the norm left after both passes exceeds
+ * rank_tol * ||c_i||; otherwise it is dependent and keeps only its
+ * coefficients.  Produces Q (r x D) with Q Q^T = I_r, R (M x r, lower echelon,
+ * positive pivots) with C = R Q, ||c_i|| per row, and r.
+ *
+ * rank_tol: relative tolerance (> 0; 1e-6 is the library's default reading).
+ * flags: 0 or GS_BUILD_NORMALIZE_ROWS.
+ * out: receives a new handle owning Q, R, the norms and the derived operand
+ *      copies of the tensor-core kernels.  Destroy with gs_basis_destroy.
+ * Synchronises `stream` once (to learn r).  Requires 1 <= M, 1 <= D, ldc >= D.
+ * Errors: GS_ERR_INVALID_ARG, GS_ERR_SHAPE, GS_ERR_NOMEM, GS_ERR_CUDA,
+ *         GS_ERR_UNSUPPORTED (no sm_103 device).
+ */
+GS_API gs_status gs_build_basis(const float* C, int M, int D, int ldc, float rank_tol,
+                         unsigned flags, void* stream, gs_basis** out);
+
+/*
+ * Read-only view of a basis: sizes and device pointers to Q (r x D, ld = D),
+ * R (M x r, ld = r) and cnorm (M, fp32 ||c_i||).  Any output pointer may be
+ * NULL.  The pointers stay valid until gs_basis_destroy.
+ */
+GS_API gs_status gs_basis_info(const gs_basis* h, int* M, int* D, int* r, const float** Q,
+                        const float** R, const float** cnorm);
+
+/* Releases a handle and its device memory (synchronises its device first). */
+GS_API gs_status gs_basis_destroy(gs_basis* h);
+
+/*
+ * Fused project + similarity (Sec. 3.1: t = U^T x; Sec. 2.2 scaled dot-product
+ * similarity; Sec. 3.2, Eq. 2-3: scores computed on Gram-loc equal the
+ * uncompressed ones).
+ *
+ * X: N x D queries (fp32, ld = ldx).  Computes Y = X Q^T (N x r) and scores
+ * against the M codewords in Gram-loc, S = Y R^T, then per `mode`
+ * (gs_score_mode) with `scale`; COSINE divides by the full D-dimensional
+ * ||x_n|| and by ||c_i||.  Optional outputs (NULL to skip):
+ *   Y      N x r fp32, ld = ldy          argmax  N int32 (lowest index on ties)
+ *   S      N x M fp32, ld = lds          maxval  N fp32 (S at argmax)
+ * At least one output must be non-NULL.  When r = 0 every score is 0 (softmax:
+ * 1/M) and argmax is 0.
+ * Tensor-core path (GS_PATH_AUTO picks it for large N with r <= 256): X is
+ * rounded to fp16 on the fly (|x| must stay below 65504, else GS_ERR_RANGE is
+ * raised on the device word), Q is a fixed fp16 copy with unbiased dithered
+ * rounding, fp32 accumulation; the scores S = Y R^T are taken in fp32.
+ * Requires X 16-byte aligned and ldx % 4 == 0 on the tensor-core path.
+ */
+GS_API gs_status gs_project_similarity(const gs_basis* h, const float* X, long long N, int ldx,
+                                int mode, float scale, unsigned flags, float* Y, int ldy,
+                                float* S, int lds, int* argmax, float* maxval, void* stream);
+
+/*
+ * Probability vectorization on Gram-loc (Sec. 2.2: weighted sum of codewords
+ * with attribute probabilities as weights; Sec. 3.1 / 3.3: run on Gram-loc).
+ * V = P R: P is N x M (fp32, ld = ldp), V is N x r of type v_dtype
+ * (GS_F32 or GS_BF16, ld = ldv).  V is the Gram-loc of P C.
+ * fp32 V: fp32 CUDA-core arithmetic.  bf16 V: bf16 tensor-core product with
+ * fp32 accumulation when GS_PATH_AUTO/TENSOR and the shape allows it.
+ */
+GS_API gs_status gs_prob_vectorize(const gs_basis* h, const float* P, long long N, int ldp, void* V,
+                            int v_dtype, int ldv, unsigned flags, void* stream);
+
+/*
+ * Reconstruction, the "decompose" step (Sec. 3.1 and Sec. 3.3: x = U t before
+ * component-wise operators).  Xhat = T Q: T is N x r coefficients of type
+ * t_dtype (GS_F32 or GS_BF16, ld = ldt), Xhat is N x D fp32 (ld = ldxh).
+ * Reconstructing R itself returns the codebook C (exact up to rounding).
+ */
+GS_API gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt,
+                         float* Xhat, int ldxh, unsigned flags, void* stream);
+
+/*
+ * Attention scores between compressed vectors (Sec. 2.2 attention score;
+ * Sec. 3.2: attention computed by matrix multiplication is preserved on
+ * Gram-loc).  For each of B sequences: A[b] = scale * Yq[b] Yk[b]^T
+ * (Lq x Lk, fp32), followed by a row softmax over the Lk keys when
+ * apply_softmax != 0.  Yq is B x Lq x r and Yk is B x Lk x r, both of type
+ * in_dtype (GS_F32 or GS_BF16) with row stride ldy elements; A is
+ * B x Lq x Lk fp32, dense.  scale = 1/sqrt(D) reproduces full-dimension
+ * attention.  Tensor-core path: bf16 inputs, fp32 accumulation.
+ */
+GS_API gs_status gs_attention_scores(const void* Yq, const void* Yk, int in_dtype, int B, int Lq,
+                              int Lk, int r, int ldy, float scale, int apply_softmax, float* A,
+                              unsigned flags, void* stream);
+
+/*
+ * Synchronises `stream` (NULL = the whole device) and returns the first error
+ * the device recorded since the last call (GS_ERR_TIMEOUT, GS_ERR_RANGE), or
+ * GS_ERR_CUDA if the stream itself failed; clears the recorded word.
+ */
+GS_API gs_status gs_stream_status(void* stream);
+
+/* Static, human-readable name of a status code. */
+GS_API const char* gs_status_string(gs_status s);
+
+/* Library version, major*10000 + minor*100 + patch. */
+GS_API int gs_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GRAMSPACE_H */

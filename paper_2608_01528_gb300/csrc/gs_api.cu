@@ -1,0 +1,283 @@
+// gs_api.cu -- the C ABI declared in include/gramspace.h: argument checks,
+// device selection, path dispatch and status handling.  No arithmetic of the
+// method lives here; every step runs in the kernels of gs_build.cu,
+// gs_simt.cu and gs_tc.cu.
+
+#include <math.h>
+#include <stdint.h>
+
+#include <algorithm>
+
+#include "gs_internal.h"
+
+namespace {
+
+// Makes h's device current for the duration of a call and restores the caller's.
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = true;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) { ok = false; return; }
+        if (prev != dev && cudaSetDevice(dev) != cudaSuccess) ok = false;
+    }
+    ~DeviceGuard() {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+gs_status from_cuda(cudaError_t e) {
+    if (e == cudaSuccess) return GS_OK;
+    if (e == cudaErrorMemoryAllocation) return GS_ERR_NOMEM;
+    return GS_ERR_CUDA;
+}
+
+bool device_supported(int dev) {
+    int major = 0, minor = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess) return false;
+    if (cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess) return false;
+    return major == 10 && minor == 3;
+}
+
+bool valid_path(unsigned flags) {
+    return flags == GS_PATH_AUTO || flags == GS_PATH_SIMT || flags == GS_PATH_TENSOR;
+}
+
+void free_basis(gs_basis* h) {
+    if (!h) return;
+    cudaFree(h->Q);
+    cudaFree(h->R);
+    cudaFree(h->cnorm);
+    cudaFree(h->rlen);
+    cudaFree(h->rlen_chunk);
+    cudaFree(h->Q16);
+    cudaFree(h->Q16t);
+    cudaFree(h->scratch);
+    cudaFree(h->tc_Rpad);
+    cudaFree(h->tc_jlen16);
+    delete h;
+}
+
+constexpr long long kMaxGemmRows = 65535LL * 64;  // grid.y limit of the SIMT GEMM
+
+}  // namespace
+
+extern "C" {
+
+int gs_version(void) { return 100; }
+
+const char* gs_status_string(gs_status s) {
+    switch (s) {
+        case GS_OK: return "GS_OK";
+        case GS_ERR_INVALID_ARG: return "GS_ERR_INVALID_ARG";
+        case GS_ERR_ALIGNMENT: return "GS_ERR_ALIGNMENT";
+        case GS_ERR_SHAPE: return "GS_ERR_SHAPE";
+        case GS_ERR_NOMEM: return "GS_ERR_NOMEM";
+        case GS_ERR_CUDA: return "GS_ERR_CUDA";
+        case GS_ERR_TIMEOUT: return "GS_ERR_TIMEOUT";
+        case GS_ERR_RANGE: return "GS_ERR_RANGE";
+        case GS_ERR_UNSUPPORTED: return "GS_ERR_UNSUPPORTED";
+    }
+    return "GS_ERR_UNKNOWN";
+}
+
+gs_status gs_build_basis(const float* C, int M, int D, int ldc, float rank_tol, unsigned flags,
+                         void* stream, gs_basis** out) {
+    if (!out) return GS_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (!C || M < 1 || D < 1 || ldc < D) return M < 1 || D < 1 || ldc < D ? GS_ERR_SHAPE : GS_ERR_INVALID_ARG;
+    if (!(rank_tol > 0.f) || !isfinite(rank_tol)) return GS_ERR_INVALID_ARG;
+    if (flags & ~GS_BUILD_NORMALIZE_ROWS) return GS_ERR_INVALID_ARG;
+    if ((uintptr_t)C % sizeof(float)) return GS_ERR_ALIGNMENT;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return GS_ERR_CUDA;
+    if (!device_supported(dev)) return GS_ERR_UNSUPPORTED;
+    gs_basis* h = new gs_basis();
+    h->device = dev;
+    gs_status st = gs::build_basis(C, M, D, ldc, (double)rank_tol, (flags & GS_BUILD_NORMALIZE_ROWS) != 0,
+                                   (cudaStream_t)stream, h);
+    if (st == GS_OK && gs::tc_available(dev)) st = gs::tc_prepare(h);
+    if (st != GS_OK) {
+        free_basis(h);
+        return st;
+    }
+    *out = h;
+    return GS_OK;
+}
+
+gs_status gs_basis_info(const gs_basis* h, int* M, int* D, int* r, const float** Q, const float** R,
+                        const float** cnorm) {
+    if (!h) return GS_ERR_INVALID_ARG;
+    if (M) *M = h->M;
+    if (D) *D = h->D;
+    if (r) *r = h->r;
+    if (Q) *Q = h->Q;
+    if (R) *R = h->R;
+    if (cnorm) *cnorm = h->cnorm;
+    return GS_OK;
+}
+
+gs_status gs_basis_destroy(gs_basis* h) {
+    if (!h) return GS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    cudaDeviceSynchronize();
+    free_basis(h);
+    return GS_OK;
+}
+
+gs_status gs_project_similarity(const gs_basis* h, const float* X, long long N, int ldx, int mode,
+                                float scale, unsigned flags, float* Y, int ldy, float* S, int lds,
+                                int* argmax, float* maxval, void* stream) {
+    if (!h || !valid_path(flags)) return GS_ERR_INVALID_ARG;
+    if (mode < GS_SCORE_RAW || mode > GS_SCORE_SOFTMAX || !isfinite(scale)) return GS_ERR_INVALID_ARG;
+    if (N < 0 || ldx < h->D) return GS_ERR_SHAPE;
+    if ((Y && ldy < h->r) || (S && lds < h->M)) return GS_ERR_SHAPE;
+    if (N == 0) return GS_OK;
+    if (!Y && !S && !argmax && !maxval) return GS_ERR_INVALID_ARG;
+    if (!X) return GS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    if (!g.ok) return GS_ERR_CUDA;
+    cudaStream_t s = (cudaStream_t)stream;
+    const int r = h->r, M = h->M, D = h->D;
+
+    const bool tc_shape = r >= 1 && r <= 256 && h->has_tmap_q16 && (uintptr_t)X % 16 == 0 && ldx % 4 == 0;
+    const bool big = (double)N * D >= (double)(1 << 24);
+    if (flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && big && tc_shape)) {
+        if (!tc_shape) return (uintptr_t)X % 16 || ldx % 4 ? GS_ERR_ALIGNMENT : GS_ERR_UNSUPPORTED;
+        return from_cuda(gs::launch_ps_tc(h, X, N, ldx, mode, scale, Y, ldy, S, lds, argmax, maxval, s));
+    }
+    if (r <= 32) {
+        return from_cuda(gs::launch_ps_warp(X, N, ldx, D, h->Q, r, h->R, h->ldr, M, h->cnorm, mode, scale,
+                                            Y, ldy, S, lds, argmax, maxval, s));
+    }
+    // generic chunked fp32 path: Y = X Q^T, S = Y R^T (+ cosine / scale), row finish
+    const long long chunk = std::min(h->chunk_rows, kMaxGemmRows);
+    for (long long c0 = 0; c0 < N; c0 += chunk) {
+        const long long nc = std::min(chunk, N - c0);
+        float* scr = h->scratch;
+        float* Ybuf = Y ? Y + c0 * ldy : scr;
+        const long long ldyb = Y ? ldy : r;
+        scr += Y ? 0 : nc * r;
+        float* xn = nullptr;
+        if (mode == GS_SCORE_COSINE) {
+            xn = scr;
+            scr += nc;
+            cudaError_t e = gs::launch_rownorm(X + c0 * ldx, nc, ldx, D, xn, s);
+            if (e != cudaSuccess) return from_cuda(e);
+        }
+        gs::GemmArgs a{};
+        a.A = X + c0 * ldx; a.a_type = gs::MAT_F32; a.lda = ldx;
+        a.B = h->Q; a.b_type = gs::MAT_F32; a.ldb = D; a.b_trans = true;
+        a.C = Ybuf; a.c_type = gs::MAT_F32; a.ldc = ldyb;
+        a.m = nc; a.n = r; a.k = D; a.batch = 1; a.alpha = 1.f;
+        cudaError_t e = gs::launch_gemm_simt(a, s);
+        if (e != cudaSuccess) return from_cuda(e);
+        if (!S && !argmax && !maxval) continue;
+        float* Sbuf = S ? S + c0 * lds : scr;
+        const long long ldsb = S ? lds : M;
+        gs::GemmArgs b{};
+        b.A = Ybuf; b.a_type = gs::MAT_F32; b.lda = ldyb;
+        b.B = h->R; b.b_type = gs::MAT_F32; b.ldb = h->ldr; b.b_trans = true; b.b_rowlen = h->rlen;
+        b.C = Sbuf; b.c_type = gs::MAT_F32; b.ldc = ldsb;
+        b.m = nc; b.n = M; b.k = r; b.batch = 1; b.alpha = scale;
+        if (mode == GS_SCORE_COSINE) { b.rownorm = xn; b.colnorm = h->cnorm; }
+        e = gs::launch_gemm_simt(b, s);
+        if (e != cudaSuccess) return from_cuda(e);
+        if (argmax || maxval || mode == GS_SCORE_SOFTMAX) {
+            e = gs::launch_row_finish(Sbuf, nc, M, (int)ldsb, mode == GS_SCORE_SOFTMAX,
+                                      argmax ? argmax + c0 : nullptr, maxval ? maxval + c0 : nullptr, s);
+            if (e != cudaSuccess) return from_cuda(e);
+        }
+    }
+    return GS_OK;
+}
+
+gs_status gs_prob_vectorize(const gs_basis* h, const float* P, long long N, int ldp, void* V, int v_dtype,
+                            int ldv, unsigned flags, void* stream) {
+    if (!h || !valid_path(flags)) return GS_ERR_INVALID_ARG;
+    if (v_dtype != GS_F32 && v_dtype != GS_BF16) return GS_ERR_INVALID_ARG;
+    if (N < 0 || ldp < h->M || ldv < h->r) return GS_ERR_SHAPE;
+    if (N == 0 || h->r == 0) return GS_OK;
+    if (!P || !V) return GS_ERR_INVALID_ARG;
+    if (flags == GS_PATH_TENSOR) return GS_ERR_UNSUPPORTED;
+    DeviceGuard g(h->device);
+    if (!g.ok) return GS_ERR_CUDA;
+    cudaStream_t s = (cudaStream_t)stream;
+    for (long long c0 = 0; c0 < N; c0 += kMaxGemmRows) {
+        const long long nc = std::min(kMaxGemmRows, N - c0);
+        gs::GemmArgs a{};
+        a.A = P + c0 * ldp; a.a_type = gs::MAT_F32; a.lda = ldp;
+        a.B = h->R; a.b_type = gs::MAT_F32; a.ldb = h->ldr; a.b_trans = false;
+        a.C = (char*)V + (size_t)c0 * ldv * (v_dtype == GS_F32 ? 4 : 2);
+        a.c_type = v_dtype == GS_F32 ? gs::MAT_F32 : gs::MAT_BF16; a.ldc = ldv;
+        a.m = nc; a.n = h->r; a.k = h->M; a.batch = 1; a.alpha = 1.f;
+        cudaError_t e = gs::launch_gemm_simt(a, s);
+        if (e != cudaSuccess) return from_cuda(e);
+    }
+    return GS_OK;
+}
+
+gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt, float* Xhat,
+                         int ldxh, unsigned flags, void* stream) {
+    if (!h || !valid_path(flags)) return GS_ERR_INVALID_ARG;
+    if (t_dtype != GS_F32 && t_dtype != GS_BF16) return GS_ERR_INVALID_ARG;
+    if (N < 0 || ldt < h->r || ldxh < h->D) return GS_ERR_SHAPE;
+    if (N == 0) return GS_OK;
+    if (!T || !Xhat) return GS_ERR_INVALID_ARG;
+    if (flags == GS_PATH_TENSOR) return GS_ERR_UNSUPPORTED;
+    DeviceGuard g(h->device);
+    if (!g.ok) return GS_ERR_CUDA;
+    cudaStream_t s = (cudaStream_t)stream;
+    for (long long c0 = 0; c0 < N; c0 += kMaxGemmRows) {
+        const long long nc = std::min(kMaxGemmRows, N - c0);
+        gs::GemmArgs a{};
+        a.A = (const char*)T + (size_t)c0 * ldt * (t_dtype == GS_F32 ? 4 : 2);
+        a.a_type = t_dtype == GS_F32 ? gs::MAT_F32 : gs::MAT_BF16; a.lda = ldt;
+        a.B = h->Q; a.b_type = gs::MAT_F32; a.ldb = h->D; a.b_trans = false;
+        a.C = Xhat + c0 * ldxh; a.c_type = gs::MAT_F32; a.ldc = ldxh;
+        a.m = nc; a.n = h->D; a.k = h->r; a.batch = 1; a.alpha = 1.f;
+        cudaError_t e = gs::launch_gemm_simt(a, s);
+        if (e != cudaSuccess) return from_cuda(e);
+    }
+    return GS_OK;
+}
+
+gs_status gs_attention_scores(const void* Yq, const void* Yk, int in_dtype, int B, int Lq, int Lk, int r,
+                              int ldy, float scale, int apply_softmax, float* A, unsigned flags,
+                              void* stream) {
+    if (!valid_path(flags)) return GS_ERR_INVALID_ARG;
+    if (in_dtype != GS_F32 && in_dtype != GS_BF16) return GS_ERR_INVALID_ARG;
+    if (B < 0 || Lq < 0 || Lk < 0 || r < 0 || ldy < r || !isfinite(scale)) return GS_ERR_SHAPE;
+    if ((long long)B * Lq * Lk == 0) return GS_OK;
+    if (!Yq || !Yk || !A) return GS_ERR_INVALID_ARG;
+    if (B > 65535 || Lq > kMaxGemmRows) return GS_ERR_SHAPE;
+    if (flags == GS_PATH_TENSOR) return GS_ERR_UNSUPPORTED;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return GS_ERR_CUDA;
+    if (!device_supported(dev)) return GS_ERR_UNSUPPORTED;
+    cudaStream_t s = (cudaStream_t)stream;
+    gs::GemmArgs a{};
+    const int t = in_dtype == GS_F32 ? gs::MAT_F32 : gs::MAT_BF16;
+    a.A = Yq; a.a_type = t; a.lda = ldy; a.a_bstride = (long long)Lq * ldy;
+    a.B = Yk; a.b_type = t; a.ldb = ldy; a.b_bstride = (long long)Lk * ldy; a.b_trans = true;
+    a.C = A; a.c_type = gs::MAT_F32; a.ldc = Lk; a.c_bstride = (long long)Lq * Lk;
+    a.m = Lq; a.n = Lk; a.k = r; a.batch = B; a.alpha = scale;
+    cudaError_t e = gs::launch_gemm_simt(a, s);
+    if (e != cudaSuccess) return from_cuda(e);
+    if (apply_softmax) {
+        e = gs::launch_row_softmax(A, (long long)B * Lq, Lk, Lk, s);
+        if (e != cudaSuccess) return from_cuda(e);
+    }
+    return GS_OK;
+}
+
+gs_status gs_stream_status(void* stream) {
+    cudaError_t e = stream ? cudaStreamSynchronize((cudaStream_t)stream) : cudaDeviceSynchronize();
+    if (e != cudaSuccess) return GS_ERR_CUDA;
+    const unsigned w = gs::take_device_error_build() | gs::take_device_error_tc();
+    if (w & GS_DEV_ERR_TIMEOUT) return GS_ERR_TIMEOUT;
+    if (w & GS_DEV_ERR_RANGE) return GS_ERR_RANGE;
+    return GS_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,389 @@
+// gs_build.cu -- basis construction (paper Sec. 3.1, Eq. 1; Sec. 3.3 "during
+// initialization ... Gram-Schmidt orthogonalization of the codebook").
+//
+// Row-order Gram-Schmidt with two projection passes per row and a relative
+// rank tolerance, in fp64 on the device.  Rows are taken in panels of
+// kPanel.  For each panel:
+//   1. load the panel rows V (fp64) and their norms ||c_i||;
+//   2. twice (reorthogonalisation): H = V Q_old^T (tiled fp64 dot products
+//      over D-slices, then a slice reduction that also accumulates R), and
+//      V -= H Q_old -- a block projection against the basis built so far;
+//   3. one CTA runs modified Gram-Schmidt with two passes over the panel's own
+//      new directions, row by row, decides rank (||v|| > tol * ||c_i||),
+//      normalises and appends accepted rows to Q.
+// In exact arithmetic this is the row-wise two-pass Gram-Schmidt of the
+// paper's construction (projections onto orthonormal directions commute);
+// the block passes against the old basis are what make it data-parallel.
+// The only host synchronisation is the read of the final rank r.
+//
+// Afterwards fp32 copies of Q and R are made for the caller, plus the
+// fp16 operand copies of the tensor-core kernels (unbiased dithered rounding
+// of the fp64 basis, see dither_half).
+
+#include <algorithm>
+#include <cmath>
+#include <vector>
+
+#include "gs_internal.h"
+
+namespace gs {
+namespace {
+
+constexpr int kPanel = 16;      // rows per panel
+constexpr int kDotTileQ = 16;   // basis rows per dot tile
+constexpr int kDotCols = 64;    // columns staged per step in the dot kernel
+constexpr int kUpdCols = 64;    // columns per CTA in the update kernel
+constexpr int kUpdJ = 128;      // coefficients staged per step in the update kernel
+
+__device__ unsigned g_err_build = 0;
+
+template <int NT>
+__device__ double block_sum(double v, double* sh) {
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    __syncthreads();  // protect sh from a previous use
+    if (l == 0) sh[w] = v;
+    __syncthreads();
+    double t = 0.0;
+    if (w == 0) {
+        t = l < NT / 32 ? sh[l] : 0.0;
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (l == 0) sh[32] = t;
+    }
+    __syncthreads();
+    return sh[32];
+}
+
+// 1. panel rows -> V (fp64), ||c_i||.  One CTA per panel row.
+__global__ void __launch_bounds__(256) k_panel_load(const float* __restrict__ C, long long ldc, int D,
+                                                     int p0, int normalize, double* __restrict__ V,
+                                                     double* __restrict__ cn) {
+    __shared__ double sh[33];
+    const int k = blockIdx.x;
+    const float* c = C + (size_t)(p0 + k) * ldc;
+    double* v = V + (size_t)k * D;
+    double ss = 0.0;
+    for (int d = threadIdx.x; d < D; d += 256) {
+        double x = (double)c[d];
+        v[d] = x;
+        ss += x * x;
+    }
+    double nrm = sqrt(block_sum<256>(ss, sh));
+    if (normalize && nrm > 0.0) {
+        const double sc = 1.0 / nrm;
+        ss = 0.0;
+        for (int d = threadIdx.x; d < D; d += 256) {
+            double x = v[d] * sc;
+            v[d] = x;
+            ss += x * x;
+        }
+        nrm = sqrt(block_sum<256>(ss, sh));
+    }
+    if (threadIdx.x == 0) cn[p0 + k] = nrm;
+}
+
+// 2a. partial dot products Hp[slice][k][j] = sum_{d in slice} V[k][d] Qw[j][d]
+//     for j < r0 (the rank at the start of this panel).  grid (q tiles, slices).
+__global__ void __launch_bounds__(256) k_panel_dots(const double* __restrict__ V,
+                                                     const double* __restrict__ Qw, int D, int bp,
+                                                     const int* __restrict__ r_start, int dslice,
+                                                     double* __restrict__ Hp, int ldh) {
+    const int r0 = *r_start;
+    const int j0 = blockIdx.x * kDotTileQ;
+    if (j0 >= r0) return;
+    const int d0 = blockIdx.y * dslice;
+    const int d1 = min(D, d0 + dslice);
+    __shared__ double sV[kPanel][kDotCols + 1];
+    __shared__ double sQ[kDotTileQ][kDotCols + 1];
+    const int ty = threadIdx.x / kDotTileQ;  // panel row
+    const int tx = threadIdx.x % kDotTileQ;  // basis row within the tile
+    double acc = 0.0;
+    for (int dd = d0; dd < d1; dd += kDotCols) {
+        for (int e = threadIdx.x; e < kPanel * kDotCols; e += 256) {
+            const int rr = e / kDotCols, cc = e % kDotCols;
+            const int d = dd + cc;
+            sV[rr][cc] = (rr < bp && d < d1) ? V[(size_t)rr * D + d] : 0.0;
+            sQ[rr][cc] = (j0 + rr < r0 && d < d1) ? Qw[(size_t)(j0 + rr) * D + d] : 0.0;
+        }
+        __syncthreads();
+#pragma unroll 16
+        for (int cc = 0; cc < kDotCols; ++cc) acc += sV[ty][cc] * sQ[tx][cc];
+        __syncthreads();
+    }
+    if (ty < bp && j0 + tx < r0) Hp[((size_t)blockIdx.y * kPanel + ty) * ldh + j0 + tx] = acc;
+}
+
+// 2b. H[k][j] = sum over slices; R64[p0+k][j] += H[k][j].
+__global__ void k_panel_reduce(const double* __restrict__ Hp, int nslices, int bp,
+                               const int* __restrict__ r_start, int ldh, double* __restrict__ H,
+                               double* __restrict__ R64, int ldr, int p0) {
+    const int r0 = *r_start;
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    const int k = (int)(idx / ldh), j = (int)(idx % ldh);
+    if (k >= bp || j >= r0) return;
+    double s = 0.0;
+    for (int t = 0; t < nslices; ++t) s += Hp[((size_t)t * kPanel + k) * ldh + j];
+    H[(size_t)k * ldh + j] = s;
+    R64[(size_t)(p0 + k) * ldr + j] += s;
+}
+
+// 2c. V[k][d] -= sum_{j < r0} H[k][j] Qw[j][d].  CTA = 64 columns x 4 row groups.
+__global__ void __launch_bounds__(256) k_panel_update(double* __restrict__ V,
+                                                       const double* __restrict__ Qw, int D, int bp,
+                                                       const int* __restrict__ r_start,
+                                                       const double* __restrict__ H, int ldh) {
+    const int r0 = *r_start;
+    if (r0 == 0) return;
+    __shared__ double sH[kPanel][kUpdJ];
+    const int d = blockIdx.x * kUpdCols + (threadIdx.x % kUpdCols);
+    const int kg = threadIdx.x / kUpdCols;  // 4 groups of 4 rows
+    double acc[4] = {0.0, 0.0, 0.0, 0.0};
+    for (int jc = 0; jc < r0; jc += kUpdJ) {
+        const int nj = min(kUpdJ, r0 - jc);
+        for (int e = threadIdx.x; e < kPanel * kUpdJ; e += 256) {
+            const int kk = e / kUpdJ, cc = e % kUpdJ;
+            sH[kk][cc] = (kk < bp && cc < nj) ? H[(size_t)kk * ldh + jc + cc] : 0.0;
+        }
+        __syncthreads();
+        if (d < D) {
+            for (int cc = 0; cc < nj; ++cc) {
+                const double q = Qw[(size_t)(jc + cc) * D + d];
+#pragma unroll
+                for (int t = 0; t < 4; ++t) acc[t] += sH[kg * 4 + t][cc] * q;
+            }
+        }
+        __syncthreads();
+    }
+    if (d < D) {
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+            const int k = kg * 4 + t;
+            if (k < bp) V[(size_t)k * D + d] -= acc[t];
+        }
+    }
+}
+
+// 3. modified Gram-Schmidt (two passes) inside the panel, rank decision,
+//    normalisation and append.  One CTA of 1024 threads; thread t owns the
+//    columns d = t, t + 1024, ... of every vector it touches.
+__global__ void __launch_bounds__(1024) k_panel_mgs(double* __restrict__ V, double* __restrict__ Qw,
+                                                     int D, int bp, int p0, double tau,
+                                                     const double* __restrict__ cn,
+                                                     double* __restrict__ R64, int ldr,
+                                                     int* __restrict__ r_dev, int rmax) {
+    __shared__ double sh[33];
+    const int r0 = *r_dev;
+    int r = r0;
+    for (int k = 0; k < bp; ++k) {
+        double* v = V + (size_t)k * D;
+        double* Rrow = R64 + (size_t)(p0 + k) * ldr;
+        for (int pass = 0; pass < 2; ++pass) {
+            for (int j = r0; j < r; ++j) {
+                const double* q = Qw + (size_t)j * D;
+                double part = 0.0;
+                for (int d = threadIdx.x; d < D; d += 1024) part += q[d] * v[d];
+                const double h = block_sum<1024>(part, sh);
+                for (int d = threadIdx.x; d < D; d += 1024) v[d] -= h * q[d];
+                if (threadIdx.x == 0) Rrow[j] += h;
+            }
+        }
+        double part = 0.0;
+        for (int d = threadIdx.x; d < D; d += 1024) part += v[d] * v[d];
+        const double nu = sqrt(block_sum<1024>(part, sh));
+        if (nu > tau * cn[p0 + k] && r < rmax) {
+            double* q = Qw + (size_t)r * D;
+            for (int d = threadIdx.x; d < D; d += 1024) q[d] = v[d] / nu;
+            if (threadIdx.x == 0) Rrow[r] = nu;
+            ++r;
+        }
+    }
+    if (threadIdx.x == 0) *r_dev = r;
+}
+
+// ----------------------------------------------------------------- finalisation
+__global__ void k_cast_rows(const double* __restrict__ src, long long lds, float* __restrict__ dst,
+                            long long ldd, int rows, int cols) {
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)rows * cols) return;
+    const int i = (int)(idx / cols), j = (int)(idx % cols);
+    dst[(size_t)i * ldd + j] = (float)src[(size_t)i * lds + j];
+}
+
+// rlen[i] = 1 + last nonzero column of R_i among the first r; chunk max per 32 rows
+__global__ void k_rlen(const double* __restrict__ R64, int ldr, int M, int r, int* __restrict__ rlen) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= M) return;
+    int last = 0;
+    for (int j = 0; j < r; ++j)
+        if (R64[(size_t)i * ldr + j] != 0.0) last = j + 1;
+    rlen[i] = last;
+}
+
+__global__ void k_rlen_chunk(const int* __restrict__ rlen, int M, int* __restrict__ out) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    if (c * 32 >= M) return;
+    int m = 0;
+    for (int i = c * 32; i < min(M, c * 32 + 32); ++i) m = max(m, rlen[i]);
+    out[c] = m;
+}
+
+// Counter-based 32-bit mixer (the "lowbias32" integer hash).
+__device__ __forceinline__ uint32_t mix32(uint32_t x) {
+    x ^= x >> 16;
+    x *= 0x7feb352du;
+    x ^= x >> 15;
+    x *= 0x846ca68bu;
+    x ^= x >> 16;
+    return x;
+}
+
+// Unbiased dithered (stochastic) rounding of a basis entry to fp16: round to
+// the fp16 neighbour below or above in magnitude with probability given by the
+// remainder, using a fixed hash of the element index.  The expected value is
+// the input, and the rounding errors of different elements are independent
+// even where the basis has few distinct magnitudes (the first basis vector of
+// a bipolar codebook is +-1/sqrt(D) everywhere), so in X Q^T they average out
+// over D instead of adding up coherently.  |q| <= 1, so no overflow.
+__device__ __forceinline__ __half dither_half(double qd, unsigned long long index) {
+    const float f = (float)qd;
+    const __half lo = __float2half_rz(f);
+    const float lof = __half2float(lo);
+    if (lof == f) return lo;
+    const __half hi = __ushort_as_half((unsigned short)(__half_as_ushort(lo) + 1));
+    const float hif = __half2float(hi);
+    const float frac = (f - lof) / (hif - lof);
+    const uint32_t hsh = mix32((uint32_t)index ^ mix32((uint32_t)(index >> 32) + 0x9e3779b9u));
+    const float u = (float)(hsh >> 8) * (1.0f / 16777216.0f);
+    return u < frac ? hi : lo;
+}
+
+// Q16[j][d] (r x ldq) and Q16t[d][j] (D x ldt) from Qw (fp64, r x D); zero padding.
+__global__ void k_q16(const double* __restrict__ Qw, int r, int D, __half* __restrict__ Q16, int ldq,
+                      __half* __restrict__ Q16t, int ldt) {
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)r * ldq) return;
+    const int j = (int)(idx / ldq), d = (int)(idx % ldq);
+    __half hv = __float2half(0.0f);
+    if (d < D) hv = dither_half(Qw[(size_t)j * D + d], (unsigned long long)j * D + d);
+    Q16[idx] = hv;
+    if (Q16t && d < D) Q16t[(size_t)d * ldt + j] = hv;
+}
+
+__global__ void k_zero_half(__half* p, long long n) {
+    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n) p[i] = __float2half(0.0f);
+}
+
+inline unsigned grid1(long long n, int b) { return (unsigned)((n + b - 1) / b); }
+
+struct DevBuf {
+    void* p = nullptr;
+    ~DevBuf() { if (p) cudaFree(p); }
+};
+
+}  // namespace
+
+unsigned take_device_error_build() {
+    unsigned v = 0, z = 0;
+    cudaMemcpyFromSymbol(&v, g_err_build, sizeof(v));
+    if (v) cudaMemcpyToSymbol(g_err_build, &z, sizeof(z));
+    return v;
+}
+
+#define GS_CK(x)                                                     \
+    do {                                                             \
+        cudaError_t e_ = (x);                                        \
+        if (e_ != cudaSuccess) {                                     \
+            return e_ == cudaErrorMemoryAllocation ? GS_ERR_NOMEM : GS_ERR_CUDA; \
+        }                                                            \
+    } while (0)
+
+gs_status build_basis(const float* C, int M, int D, int ldc, double tau, bool normalize,
+                      cudaStream_t s, gs_basis* h) {
+    const int rmax = std::min(M, D);
+    const int ldr = rmax;                       // R64 leading dimension
+    const int ldh = std::max(1, ((M + 15) / 16) * 16);  // >= any r0
+    const int dslice = std::max(kDotCols, ((D + 7) / 8 + kDotCols - 1) / kDotCols * kDotCols);
+    const int nslices = (D + dslice - 1) / dslice;
+
+    DevBuf bV, bQw, bR64, bH, bHp, bcn, br;
+    GS_CK(cudaMalloc(&bV.p, sizeof(double) * (size_t)kPanel * D));
+    GS_CK(cudaMalloc(&bQw.p, sizeof(double) * (size_t)rmax * D));
+    GS_CK(cudaMalloc(&bR64.p, sizeof(double) * (size_t)M * ldr));
+    GS_CK(cudaMalloc(&bH.p, sizeof(double) * (size_t)kPanel * ldh));
+    GS_CK(cudaMalloc(&bHp.p, sizeof(double) * (size_t)nslices * kPanel * ldh));
+    GS_CK(cudaMalloc(&bcn.p, sizeof(double) * (size_t)M));
+    GS_CK(cudaMalloc(&br.p, sizeof(int)));
+    double* V = (double*)bV.p;
+    double* Qw = (double*)bQw.p;
+    double* R64 = (double*)bR64.p;
+    double* H = (double*)bH.p;
+    double* Hp = (double*)bHp.p;
+    double* cn = (double*)bcn.p;
+    int* r_dev = (int*)br.p;
+    GS_CK(cudaMemsetAsync(R64, 0, sizeof(double) * (size_t)M * ldr, s));
+    GS_CK(cudaMemsetAsync(r_dev, 0, sizeof(int), s));
+
+    for (int p0 = 0; p0 < M; p0 += kPanel) {
+        const int bp = std::min(kPanel, M - p0);
+        k_panel_load<<<bp, 256, 0, s>>>(C, ldc, D, p0, normalize ? 1 : 0, V, cn);
+        if (p0 > 0) {
+            const int qt = (std::min(p0, rmax) + kDotTileQ - 1) / kDotTileQ;
+            for (int pass = 0; pass < 2; ++pass) {
+                k_panel_dots<<<dim3(qt, nslices), 256, 0, s>>>(V, Qw, D, bp, r_dev, dslice, Hp, ldh);
+                k_panel_reduce<<<grid1((long long)bp * ldh, 256), 256, 0, s>>>(Hp, nslices, bp, r_dev,
+                                                                                ldh, H, R64, ldr, p0);
+                k_panel_update<<<grid1(D, kUpdCols), 256, 0, s>>>(V, Qw, D, bp, r_dev, H, ldh);
+            }
+        }
+        k_panel_mgs<<<1, 1024, 0, s>>>(V, Qw, D, bp, p0, tau, cn, R64, ldr, r_dev, rmax);
+    }
+    GS_CK(cudaGetLastError());
+    int r = 0;
+    GS_CK(cudaMemcpyAsync(&r, r_dev, sizeof(int), cudaMemcpyDeviceToHost, s));
+    GS_CK(cudaStreamSynchronize(s));
+    h->M = M;
+    h->D = D;
+    h->r = r;
+    h->ldr = std::max(r, 1);
+
+    // user-visible fp32 results
+    GS_CK(cudaMalloc(&h->Q, sizeof(float) * (size_t)std::max(r, 1) * D));
+    GS_CK(cudaMalloc(&h->R, sizeof(float) * (size_t)M * h->ldr));
+    GS_CK(cudaMalloc(&h->cnorm, sizeof(float) * (size_t)M));
+    GS_CK(cudaMalloc(&h->rlen, sizeof(int) * (size_t)M));
+    GS_CK(cudaMalloc(&h->rlen_chunk, sizeof(int) * (size_t)((M + 31) / 32)));
+    GS_CK(cudaMemsetAsync(h->R, 0, sizeof(float) * (size_t)M * h->ldr, s));
+    if (r > 0) {
+        k_cast_rows<<<grid1((long long)r * D, 256), 256, 0, s>>>(Qw, D, h->Q, D, r, D);
+        k_cast_rows<<<grid1((long long)M * r, 256), 256, 0, s>>>(R64, ldr, h->R, h->ldr, M, r);
+    }
+    k_cast_rows<<<grid1(M, 256), 256, 0, s>>>(cn, 1, h->cnorm, 1, M, 1);
+    k_rlen<<<grid1(M, 128), 128, 0, s>>>(R64, ldr, M, r, h->rlen);
+    k_rlen_chunk<<<grid1((M + 31) / 32, 128), 128, 0, s>>>(h->rlen, M, h->rlen_chunk);
+
+    // tensor-core operand copies (fp16, dithered)
+    if (r > 0) {
+        h->ldq16 = (D + 7) / 8 * 8;
+        h->ldr16 = (r + 7) / 8 * 8;
+        GS_CK(cudaMalloc(&h->Q16, sizeof(__half) * (size_t)r * h->ldq16));
+        GS_CK(cudaMalloc(&h->Q16t, sizeof(__half) * (size_t)D * h->ldr16));
+        if (h->ldr16 != r)
+            k_zero_half<<<grid1((long long)D * h->ldr16, 256), 256, 0, s>>>(h->Q16t, (long long)D * h->ldr16);
+        k_q16<<<grid1((long long)r * h->ldq16, 256), 256, 0, s>>>(Qw, r, D, h->Q16, h->ldq16, h->Q16t,
+                                                                  h->ldr16);
+    }
+
+    // scratch for the chunked multi-kernel paths: rows x (r + M + 1) floats
+    const long long per_row = (long long)r + M + 1;
+    long long rows = std::max(256LL, (64LL << 20) / per_row);
+    rows = std::min(rows, 65536LL);
+    h->chunk_rows = rows;
+    h->scratch_floats = rows * per_row;
+    GS_CK(cudaMalloc(&h->scratch, sizeof(float) * (size_t)h->scratch_floats));
+    GS_CK(cudaGetLastError());
+    GS_CK(cudaStreamSynchronize(s));
+    return GS_OK;
+}
+
+}  // namespace gs

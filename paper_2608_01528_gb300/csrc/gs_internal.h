@@ -1,0 +1,104 @@
+// gs_internal.h -- host-side declarations shared by the library's translation units.
+//
+// Each .cu file owns its kernels; gs_api.cu validates arguments and calls the
+// launch functions declared here.  Nothing here is part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cuda_fp16.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "../../include/gramspace.h"
+
+struct gs_basis {
+    int device = 0;
+    int M = 0, D = 0, r = 0;
+    // user-visible results (fp32)
+    float* Q = nullptr;      // r x D, ld = D
+    float* R = nullptr;      // M x max(r,1), ld = ldr
+    int ldr = 1;
+    float* cnorm = nullptr;  // M
+    int* rlen = nullptr;     // M: 1 + index of the last nonzero of R_i (0 if none)
+    int* rlen_chunk = nullptr; // ceil(M/32): max rlen over each 32-row chunk of R
+    // tensor-core operand copies
+    __half* Q16 = nullptr;   // r x ldq16 fp16, dithered rounding of Q (K-major B of X Q^T)
+    int ldq16 = 0;
+    __half* Q16t = nullptr;  // D x ldr16 fp16, dithered rounding of Q^T (K-major B of T Q)
+    int ldr16 = 0;
+    CUtensorMap tmap_q16;    // box {64, 256} over Q16 (valid when r <= 256 and Q16 != null)
+    CUtensorMap tmap_q16t;   // box {64, 256} over Q16t
+    bool has_tmap_q16 = false, has_tmap_q16t = false;
+    // fused tensor-core similarity: zero-padded R (tc_mpad x tc_npad) and, per
+    // 16-codeword chunk, how many leading columns of R can be nonzero
+    float* tc_Rpad = nullptr;
+    int* tc_jlen16 = nullptr;
+    int tc_npad = 0, tc_mpad = 0;
+    // scratch for the multi-kernel paths (rows processed in chunks)
+    float* scratch = nullptr;
+    long long scratch_floats = 0;
+    long long chunk_rows = 0;
+};
+
+namespace gs {
+
+// ----------------------------------------------------------------- build (gs_build.cu)
+// Runs the fp64 panel Gram-Schmidt and fills every field of h except the
+// tensor maps.  Synchronises `s` once.
+gs_status build_basis(const float* C, int M, int D, int ldc, double tau, bool normalize,
+                      cudaStream_t s, gs_basis* h);
+
+// ----------------------------------------------------------------- SIMT kernels (gs_simt.cu)
+enum { MAT_F32 = 0, MAT_BF16 = 1 };
+
+// fused small-r project + similarity, one warp per query (r <= 32)
+cudaError_t launch_ps_warp(const float* X, long long N, int ldx, int D, const float* Q, int r,
+                           const float* R, int ldr, int M, const float* cnorm, int mode, float scale,
+                           float* Y, int ldy, float* S, int lds, int* argmax, float* maxval,
+                           cudaStream_t s);
+
+// C = alpha * A * op(B), batched over `batch` with element strides.
+//   A: m x k (lda), B: trans ? n x k : k x n (ldb); types MAT_F32 / MAT_BF16.
+//   rownorm/colnorm (optional): C[i][j] /= rownorm[i]*colnorm[j] (0 if product is 0)
+//   out type MAT_F32 / MAT_BF16.
+struct GemmArgs {
+    const void* A; int a_type; long long lda; long long a_bstride;
+    const void* B; int b_type; long long ldb; long long b_bstride; bool b_trans;
+    void* C; int c_type; long long ldc; long long c_bstride;
+    long long m; int n, k, batch;
+    float alpha;
+    const float* rownorm; const float* colnorm;
+    const int* b_rowlen;  // optional (b_trans only): row j of B is zero beyond b_rowlen[j]
+};
+cudaError_t launch_gemm_simt(const GemmArgs& g, cudaStream_t s);
+
+// per-row ||x||
+cudaError_t launch_rownorm(const float* X, long long N, int ldx, int D, float* out, cudaStream_t s);
+
+// per-row argmax / maxval over S (N x M); SOFTMAX mode rewrites the row in place.
+cudaError_t launch_row_finish(float* S, long long N, int M, int lds, bool softmax, int* argmax,
+                              float* maxval, cudaStream_t s);
+
+// row softmax in place over rows of length L (stride ld)
+cudaError_t launch_row_softmax(float* A, long long rows, int L, long long ld, cudaStream_t s);
+
+// ----------------------------------------------------------------- tensor-core kernels (gs_tc.cu)
+bool tc_available(int device);
+// creates the tensor maps of h's fp16 operand copies (after build_basis)
+gs_status tc_prepare(gs_basis* h);
+// fused project + similarity on tcgen05 (requires h->has_tmap_q16, r <= 256)
+cudaError_t launch_ps_tc(const gs_basis* h, const float* X, long long N, int ldx, int mode,
+                         float scale, float* Y, int ldy, float* S, int lds, int* argmax,
+                         float* maxval, cudaStream_t s);
+
+// ----------------------------------------------------------------- device error words
+// Each translation unit with kernels that can report device-side errors keeps
+// its own word; gs_stream_status reads and clears all of them.
+unsigned take_device_error_build();
+unsigned take_device_error_tc();
+
+}  // namespace gs
+
+#define GS_DEV_ERR_TIMEOUT 0x1u
+#define GS_DEV_ERR_RANGE 0x2u

@@ -1,0 +1,323 @@
+// gs_simt.cu -- fp32 CUDA-core kernels of the Gram-Space apply path.
+//
+// These kernels carry the small workloads (a handful of codewords, a few
+// hundred queries: launch-latency bound) and the precise fp32 path that any
+// shape can take (GS_PATH_SIMT).  The large-batch hot path is on tcgen05 in
+// gs_tc.cu.
+//
+//  k_ps_warp      fused project + similarity, one warp per query, r <= 32
+//                 (Sec. 3.1 t = U^T x; Sec. 2.2 similarity; Eq. 2-3)
+//  k_gemm         tiled fp32 GEMM with scale / cosine / bf16 epilogues; used for
+//                 Y = X Q^T, S = Y R^T, V = P R (Sec. 2.2 / 3.3), Xhat = T Q
+//                 (Sec. 3.1 / 3.3) and batched attention logits (Sec. 2.2)
+//  k_row_finish   argmax / maxval / softmax over each score row
+//  k_row_softmax  softmax over each attention row
+//  k_rownorm      full-D query norms for cosine scores
+
+#include <float.h>
+
+#include "gs_internal.h"
+
+namespace gs {
+namespace {
+
+__device__ __forceinline__ float warp_sum(float v) {
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+// (value, index) argmax across a warp: larger value wins, lower index on ties.
+__device__ __forceinline__ void warp_argmax(float& v, int& i) {
+    for (int o = 16; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(0xffffffffu, v, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, i, o);
+        if (ov > v || (ov == v && oi < i)) {
+            v = ov;
+            i = oi;
+        }
+    }
+}
+
+// ----------------------------------------------------------------- fused small-r kernel
+constexpr int kWarpR = 32;
+
+__global__ void __launch_bounds__(256) k_ps_warp(const float* __restrict__ X, long long N, int ldx,
+                                                  int D, const float* __restrict__ Q, int r,
+                                                  const float* __restrict__ R, int ldr, int M,
+                                                  const float* __restrict__ cnorm, int mode,
+                                                  float scale, float* __restrict__ Y, int ldy,
+                                                  float* __restrict__ S, int lds,
+                                                  int* __restrict__ argmax,
+                                                  float* __restrict__ maxval) {
+    const int lane = threadIdx.x & 31;
+    const long long n = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (n >= N) return;
+    const float* x = X + (size_t)n * ldx;
+    float y[kWarpR];
+#pragma unroll
+    for (int j = 0; j < kWarpR; ++j) y[j] = 0.f;
+    float xx = 0.f;
+    for (int d = lane; d < D; d += 32) {
+        const float xv = x[d];
+        xx = fmaf(xv, xv, xx);
+#pragma unroll
+        for (int j = 0; j < kWarpR; ++j)
+            if (j < r) y[j] = fmaf(xv, __ldg(Q + (size_t)j * D + d), y[j]);
+    }
+#pragma unroll
+    for (int j = 0; j < kWarpR; ++j)
+        if (j < r) y[j] = warp_sum(y[j]);
+    xx = warp_sum(xx);
+    if (Y) {
+        float mine = 0.f;
+#pragma unroll
+        for (int j = 0; j < kWarpR; ++j)
+            if (j == lane) mine = y[j];
+        if (lane < r) Y[(size_t)n * ldy + lane] = mine;
+    }
+    const float xnorm = sqrtf(xx);
+    // scores: lane handles codewords i = lane, lane + 32, ...
+    auto score = [&](int i) {
+        const float* Ri = R + (size_t)i * ldr;
+        float g = 0.f;
+#pragma unroll
+        for (int j = 0; j < kWarpR; ++j)
+            if (j < r) g = fmaf(y[j], __ldg(Ri + j), g);
+        g *= scale;
+        if (mode == GS_SCORE_COSINE) {
+            const float den = xnorm * cnorm[i];
+            g = den > 0.f ? g / den : 0.f;
+        }
+        return g;
+    };
+    float bv = -FLT_MAX;
+    int bi = 0x7fffffff;
+    for (int i = lane; i < M; i += 32) {
+        const float g = score(i);
+        if (g > bv) {
+            bv = g;
+            bi = i;
+        }
+        if (S && mode != GS_SCORE_SOFTMAX) S[(size_t)n * lds + i] = g;
+    }
+    warp_argmax(bv, bi);
+    if (bi == 0x7fffffff) bi = 0;
+    float outmax = bv;
+    if (mode == GS_SCORE_SOFTMAX) {
+        float z = 0.f;
+        for (int i = lane; i < M; i += 32) z += __expf(score(i) - bv);
+        z = warp_sum(z);
+        const float inv = 1.f / z;
+        if (S)
+            for (int i = lane; i < M; i += 32) S[(size_t)n * lds + i] = __expf(score(i) - bv) * inv;
+        outmax = inv;
+    }
+    if (lane == 0) {
+        if (argmax) argmax[n] = M > 0 ? bi : 0;
+        if (maxval) maxval[n] = M > 0 ? outmax : 0.f;
+    }
+}
+
+// ----------------------------------------------------------------- tiled GEMM
+constexpr int kTM = 64, kTN = 64, kTK = 16;
+
+template <int T>
+__device__ __forceinline__ float ld_elem(const void* p, long long i) {
+    if (T == MAT_F32) return __ldg((const float*)p + i);
+    return __bfloat162float(((const __nv_bfloat16*)p)[i]);
+}
+
+template <int TA, int TB, int TC, bool BT>
+__global__ void __launch_bounds__(256) k_gemm(GemmArgs g) {
+    __shared__ float As[kTK][kTM + 4];
+    __shared__ __align__(16) float Bs[kTK][kTN + 4];
+    const int tid = threadIdx.x;
+    const int tx = tid % 16, ty = tid / 16;
+    const long long m0 = (long long)blockIdx.y * kTM;
+    const int n0 = blockIdx.x * kTN;
+    const int b = blockIdx.z;
+    const char* Ab = (const char*)g.A + (size_t)b * g.a_bstride * (TA == MAT_F32 ? 4 : 2);
+    const char* Bb = (const char*)g.B + (size_t)b * g.b_bstride * (TB == MAT_F32 ? 4 : 2);
+    int kend = g.k;
+    if (BT && g.b_rowlen) {
+        // rows n0..n0+63 of B are zero beyond their row length: stop at the max
+        int mx = 0;
+        for (int j = tid; j < kTN; j += 256)
+            if (n0 + j < g.n) mx = max(mx, g.b_rowlen[n0 + j]);
+        for (int o = 16; o > 0; o >>= 1) mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        __shared__ int smx[8];
+        if ((tid & 31) == 0) smx[tid >> 5] = mx;
+        __syncthreads();
+        mx = 0;
+        for (int w = 0; w < 8; ++w) mx = max(mx, smx[w]);
+        kend = min(kend, mx);
+    }
+    float acc[4][4] = {};
+    for (int k0 = 0; k0 < kend; k0 += kTK) {
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+            const int e = tid + 256 * t;
+            const int row = e / kTK, kk = e % kTK;
+            const long long gm = m0 + row;
+            const int gk = k0 + kk;
+            As[kk][row] = (gm < g.m && gk < kend) ? ld_elem<TA>(Ab, gm * g.lda + gk) : 0.f;
+            if (BT) {
+                const int gn = n0 + row;
+                Bs[kk][row] = (gn < g.n && gk < kend) ? ld_elem<TB>(Bb, (long long)gn * g.ldb + gk) : 0.f;
+            } else {
+                const int kk2 = e / kTN, col = e % kTN;
+                const int gk2 = k0 + kk2, gn = n0 + col;
+                Bs[kk2][col] = (gn < g.n && gk2 < kend) ? ld_elem<TB>(Bb, (long long)gk2 * g.ldb + gn) : 0.f;
+            }
+        }
+        __syncthreads();
+#pragma unroll
+        for (int kk = 0; kk < kTK; ++kk) {
+            float a[4], bb[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
+            const float4 bv = *reinterpret_cast<const float4*>(&Bs[kk][tx * 4]);
+            bb[0] = bv.x; bb[1] = bv.y; bb[2] = bv.z; bb[3] = bv.w;
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], bb[j], acc[i][j]);
+        }
+        __syncthreads();
+    }
+    char* Cb = (char*)g.C + (size_t)b * g.c_bstride * (TC == MAT_F32 ? 4 : 2);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const long long gm = m0 + ty * 4 + i;
+        if (gm >= g.m) continue;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int gn = n0 + tx * 4 + j;
+            if (gn >= g.n) continue;
+            float v = g.alpha * acc[i][j];
+            if (g.rownorm) {
+                const float den = g.rownorm[gm] * g.colnorm[gn];
+                v = den > 0.f ? v / den : 0.f;
+            }
+            if (TC == MAT_F32) ((float*)Cb)[gm * g.ldc + gn] = v;
+            else ((__nv_bfloat16*)Cb)[gm * g.ldc + gn] = __float2bfloat16_rn(v);
+        }
+    }
+}
+
+// ----------------------------------------------------------------- row kernels
+__global__ void __launch_bounds__(256) k_row_finish(float* __restrict__ S, long long N, int M,
+                                                     int lds, int softmax, int* __restrict__ argmax,
+                                                     float* __restrict__ maxval) {
+    const int lane = threadIdx.x & 31;
+    const long long n = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (n >= N) return;
+    float* s = S + (size_t)n * lds;
+    float bv = -FLT_MAX;
+    int bi = 0x7fffffff;
+    for (int i = lane; i < M; i += 32) {
+        const float g = s[i];
+        if (g > bv) {
+            bv = g;
+            bi = i;
+        }
+    }
+    warp_argmax(bv, bi);
+    if (bi == 0x7fffffff) bi = 0;
+    float outmax = bv;
+    if (softmax) {
+        float z = 0.f;
+        for (int i = lane; i < M; i += 32) z += __expf(s[i] - bv);
+        z = warp_sum(z);
+        const float inv = 1.f / z;
+        for (int i = lane; i < M; i += 32) s[i] = __expf(s[i] - bv) * inv;
+        outmax = inv;
+    }
+    if (lane == 0) {
+        if (argmax) argmax[n] = M > 0 ? bi : 0;
+        if (maxval) maxval[n] = M > 0 ? outmax : 0.f;
+    }
+}
+
+__global__ void __launch_bounds__(256) k_row_softmax(float* __restrict__ A, long long rows, int L,
+                                                      long long ld) {
+    const int lane = threadIdx.x & 31;
+    const long long n = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (n >= rows) return;
+    float* a = A + (size_t)n * ld;
+    float mx = -FLT_MAX;
+    for (int i = lane; i < L; i += 32) mx = fmaxf(mx, a[i]);
+    mx = warp_max(mx);
+    float z = 0.f;
+    for (int i = lane; i < L; i += 32) z += __expf(a[i] - mx);
+    z = warp_sum(z);
+    const float inv = 1.f / z;
+    for (int i = lane; i < L; i += 32) a[i] = __expf(a[i] - mx) * inv;
+}
+
+__global__ void __launch_bounds__(256) k_rownorm(const float* __restrict__ X, long long N, int ldx,
+                                                  int D, float* __restrict__ out) {
+    const int lane = threadIdx.x & 31;
+    const long long n = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (n >= N) return;
+    const float* x = X + (size_t)n * ldx;
+    float s = 0.f;
+    for (int d = lane; d < D; d += 32) s = fmaf(x[d], x[d], s);
+    s = warp_sum(s);
+    if (lane == 0) out[n] = sqrtf(s);
+}
+
+inline unsigned rows_grid(long long n) { return (unsigned)((n + 7) / 8); }
+
+}  // namespace
+
+cudaError_t launch_ps_warp(const float* X, long long N, int ldx, int D, const float* Q, int r,
+                           const float* R, int ldr, int M, const float* cnorm, int mode, float scale,
+                           float* Y, int ldy, float* S, int lds, int* argmax, float* maxval,
+                           cudaStream_t s) {
+    k_ps_warp<<<rows_grid(N), 256, 0, s>>>(X, N, ldx, D, Q, r, R, ldr, M, cnorm, mode, scale, Y, ldy,
+                                           S, lds, argmax, maxval);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gemm_simt(const GemmArgs& g, cudaStream_t s) {
+    if (g.m <= 0 || g.n <= 0 || g.batch <= 0) return cudaSuccess;
+    dim3 grid((unsigned)((g.n + kTN - 1) / kTN), (unsigned)((g.m + kTM - 1) / kTM), (unsigned)g.batch);
+    if (grid.y > 65535u) return cudaErrorInvalidConfiguration;
+#define GS_GEMM_CASE(TA, TB, TC, BT)                                                        \
+    if (g.a_type == TA && g.b_type == TB && g.c_type == TC && g.b_trans == BT) {            \
+        k_gemm<TA, TB, TC, BT><<<grid, 256, 0, s>>>(g);                                     \
+        return cudaGetLastError();                                                          \
+    }
+    GS_GEMM_CASE(MAT_F32, MAT_F32, MAT_F32, true)
+    GS_GEMM_CASE(MAT_F32, MAT_F32, MAT_F32, false)
+    GS_GEMM_CASE(MAT_F32, MAT_F32, MAT_BF16, false)
+    GS_GEMM_CASE(MAT_BF16, MAT_F32, MAT_F32, false)
+    GS_GEMM_CASE(MAT_BF16, MAT_BF16, MAT_F32, true)
+#undef GS_GEMM_CASE
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_rownorm(const float* X, long long N, int ldx, int D, float* out, cudaStream_t s) {
+    if (N <= 0) return cudaSuccess;
+    k_rownorm<<<rows_grid(N), 256, 0, s>>>(X, N, ldx, D, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_row_finish(float* S, long long N, int M, int lds, bool softmax, int* argmax,
+                              float* maxval, cudaStream_t s) {
+    if (N <= 0) return cudaSuccess;
+    k_row_finish<<<rows_grid(N), 256, 0, s>>>(S, N, M, lds, softmax ? 1 : 0, argmax, maxval);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_row_softmax(float* A, long long rows, int L, long long ld, cudaStream_t s) {
+    if (rows <= 0) return cudaSuccess;
+    k_row_softmax<<<rows_grid(rows), 256, 0, s>>>(A, rows, L, ld);
+    return cudaGetLastError();
+}
+
+}  // namespace gs

@@ -1,0 +1,250 @@
+"""Thin Python binding of libgramspace.so (include/gramspace.h).
+
+Argument marshalling only: tensors are passed to the C ABI as raw device
+pointers, outputs are allocated with torch (device memory and streams are
+PyTorch's plumbing), and every step of the computation runs in the library's
+CUDA kernels.  There is no CPU fallback: if the library is not built, or no
+sm_103 device is present, calls raise.
+
+Names follow the C ABI: build_basis, project_similarity, prob_vectorize,
+reconstruct, attention_scores, stream_status.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "_build", "libgramspace.so")
+
+GS_OK, GS_ERR_INVALID_ARG, GS_ERR_ALIGNMENT, GS_ERR_SHAPE, GS_ERR_NOMEM = 0, 1, 2, 3, 4
+GS_ERR_CUDA, GS_ERR_TIMEOUT, GS_ERR_RANGE, GS_ERR_UNSUPPORTED = 5, 6, 7, 8
+GS_F32, GS_BF16 = 0, 1
+MODES = {"raw": 0, "cosine": 1, "softmax": 2}
+PATHS = {"auto": 0, "simt": 1, "tensor": 2}
+GS_BUILD_NORMALIZE_ROWS = 1
+
+# Every symbol include/gramspace.h declares (checked by the CPU tests).
+EXPORTS = ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_similarity",
+           "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores", "gs_stream_status",
+           "gs_status_string", "gs_version")
+
+
+class GramSpaceError(RuntimeError):
+    def __init__(self, status, where):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} ({status})")
+
+
+_lib = None
+
+
+def load_library(path=LIB_PATH):
+    """Loads (once) and returns the ctypes handle of libgramspace.so."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"libgramspace.so is not built ({path}); run __graft_entry__.build()")
+    L = ctypes.CDLL(path)
+    vp, ip, i64, f32, u32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_longlong, ctypes.c_float, ctypes.c_uint
+    L.gs_build_basis.argtypes = [vp, ip, ip, ip, f32, u32, vp, ctypes.POINTER(vp)]
+    L.gs_basis_info.argtypes = [vp, ctypes.POINTER(ip), ctypes.POINTER(ip), ctypes.POINTER(ip),
+                                ctypes.POINTER(vp), ctypes.POINTER(vp), ctypes.POINTER(vp)]
+    L.gs_basis_destroy.argtypes = [vp]
+    L.gs_project_similarity.argtypes = [vp, vp, i64, ip, ip, f32, u32, vp, ip, vp, ip, vp, vp, vp]
+    L.gs_prob_vectorize.argtypes = [vp, vp, i64, ip, vp, ip, ip, u32, vp]
+    L.gs_reconstruct.argtypes = [vp, vp, ip, i64, ip, vp, ip, u32, vp]
+    L.gs_attention_scores.argtypes = [vp, vp, ip, ip, ip, ip, ip, ip, f32, ip, vp, u32, vp]
+    L.gs_stream_status.argtypes = [vp]
+    L.gs_status_string.argtypes = [ip]
+    L.gs_status_string.restype = ctypes.c_char_p
+    L.gs_version.restype = ctypes.c_int
+    for name in ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_similarity",
+                 "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores", "gs_stream_status"):
+        getattr(L, name).restype = ctypes.c_int
+    _lib = L
+    return L
+
+
+def status_string(status):
+    return load_library().gs_status_string(int(status)).decode()
+
+
+def _check(status, where):
+    if status != GS_OK:
+        raise GramSpaceError(status, where)
+
+
+def _ptr(t):
+    return ctypes.c_void_p(t.data_ptr()) if t is not None else None
+
+
+def _stream(stream):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _ld(t):
+    if t.dim() != 2 or t.stride(1) != 1:
+        raise ValueError("expected a 2-D tensor with unit column stride")
+    return t.stride(0)
+
+
+def _dtype_code(t):
+    if t.dtype == torch.float32:
+        return GS_F32
+    if t.dtype == torch.bfloat16:
+        return GS_BF16
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+class _DevArray:
+    """__cuda_array_interface__ view of memory owned by a basis handle."""
+
+    def __init__(self, ptr, shape, typestr):
+        self.__cuda_array_interface__ = {"shape": tuple(shape), "typestr": typestr,
+                                         "data": (int(ptr or 0), False), "version": 3, "strides": None}
+
+
+class Basis:
+    """A built Gram-Space basis (owns the C handle): Q (r x D), R (M x r), cnorm (M)."""
+
+    def __init__(self, handle, device):
+        self._h = handle
+        self.device = device
+        L = load_library()
+        M, D, r = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+        q, rr, cn = ctypes.c_void_p(), ctypes.c_void_p(), ctypes.c_void_p()
+        _check(L.gs_basis_info(handle, ctypes.byref(M), ctypes.byref(D), ctypes.byref(r), ctypes.byref(q),
+                               ctypes.byref(rr), ctypes.byref(cn)), "gs_basis_info")
+        self.M, self.D, self.r = M.value, D.value, r.value
+        self._q, self._R, self._cn = q.value, rr.value, cn.value
+
+    @property
+    def handle(self):
+        if self._h is None:
+            raise RuntimeError("basis already destroyed")
+        return self._h
+
+    def _view(self, ptr, shape):
+        if 0 in shape:
+            return torch.zeros(shape, dtype=torch.float32, device=self.device)
+        with torch.cuda.device(self.device):
+            return torch.as_tensor(_DevArray(ptr, shape, "<f4"), device=self.device)
+
+    @property
+    def Q(self):
+        return self._view(self._q, (self.r, self.D))
+
+    @property
+    def R(self):
+        return self._view(self._R, (self.M, self.r))
+
+    @property
+    def cnorm(self):
+        return self._view(self._cn, (self.M,))
+
+    def destroy(self):
+        if self._h is not None:
+            load_library().gs_basis_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def build_basis(C, rank_tol=1e-6, normalize_rows=False, stream=None):
+    """Gram-Schmidt basis of the rows of C (M x D fp32 on the GPU); see gs_build_basis."""
+    if not C.is_cuda or C.dtype != torch.float32:
+        raise TypeError("C must be a float32 CUDA tensor")
+    L = load_library()
+    h = ctypes.c_void_p()
+    with torch.cuda.device(C.device):
+        st = L.gs_build_basis(_ptr(C), C.shape[0], C.shape[1], _ld(C), float(rank_tol),
+                              GS_BUILD_NORMALIZE_ROWS if normalize_rows else 0, _stream(stream),
+                              ctypes.byref(h))
+    _check(st, "gs_build_basis")
+    return Basis(h, C.device)
+
+
+def project_similarity(basis, X, mode="raw", scale=1.0, path="auto", want_Y=False, want_S=False,
+                       want_argmax=True, want_maxval=True, out=None, stream=None):
+    """Fused Y = X Q^T and scores against the codebook in Gram-loc; see gs_project_similarity.
+
+    Returns a dict with the requested outputs ("Y", "S", "argmax", "maxval").
+    `out` may supply preallocated output tensors under the same keys.
+    """
+    N = X.shape[0]
+    dev = X.device
+    out = dict(out or {})
+    if want_Y and "Y" not in out:
+        out["Y"] = torch.empty((N, basis.r), dtype=torch.float32, device=dev)
+    if want_S and "S" not in out:
+        out["S"] = torch.empty((N, basis.M), dtype=torch.float32, device=dev)
+    if want_argmax and "argmax" not in out:
+        out["argmax"] = torch.empty(N, dtype=torch.int32, device=dev)
+    if want_maxval and "maxval" not in out:
+        out["maxval"] = torch.empty(N, dtype=torch.float32, device=dev)
+    Y, S = out.get("Y"), out.get("S")
+    L = load_library()
+    with torch.cuda.device(dev):
+        st = L.gs_project_similarity(basis.handle, _ptr(X), N, _ld(X), MODES[mode], float(scale), PATHS[path],
+                                     _ptr(Y), _ld(Y) if Y is not None and Y.numel() else max(basis.r, 1),
+                                     _ptr(S), _ld(S) if S is not None and S.numel() else max(basis.M, 1),
+                                     _ptr(out.get("argmax")), _ptr(out.get("maxval")), _stream(stream))
+    _check(st, "gs_project_similarity")
+    return out
+
+
+def prob_vectorize(basis, P, dtype=torch.float32, path="auto", out=None, stream=None):
+    """V = P R (Gram-loc of P C); see gs_prob_vectorize."""
+    N = P.shape[0]
+    V = out if out is not None else torch.empty((N, basis.r), dtype=dtype, device=P.device)
+    L = load_library()
+    with torch.cuda.device(P.device):
+        st = L.gs_prob_vectorize(basis.handle, _ptr(P), N, _ld(P), _ptr(V), _dtype_code(V),
+                                 _ld(V) if V.numel() else max(basis.r, 1), PATHS[path], _stream(stream))
+    _check(st, "gs_prob_vectorize")
+    return V
+
+
+def reconstruct(basis, T, path="auto", out=None, stream=None):
+    """Xhat = T Q (x = U t); see gs_reconstruct."""
+    N = T.shape[0]
+    X = out if out is not None else torch.empty((N, basis.D), dtype=torch.float32, device=T.device)
+    L = load_library()
+    with torch.cuda.device(T.device):
+        st = L.gs_reconstruct(basis.handle, _ptr(T), _dtype_code(T), N, _ld(T) if T.numel() else max(basis.r, 1),
+                              _ptr(X), _ld(X), PATHS[path], _stream(stream))
+    _check(st, "gs_reconstruct")
+    return X
+
+
+def attention_scores(Yq, Yk, scale, apply_softmax=True, path="auto", out=None, stream=None):
+    """softmax_row(scale * Yq Yk^T) per sequence; Yq: B x Lq x r, Yk: B x Lk x r."""
+    B, Lq, r = Yq.shape
+    Lk = Yk.shape[1]
+    if Yk.shape[0] != B or Yk.shape[2] != r or Yq.dtype != Yk.dtype:
+        raise ValueError("Yq and Yk must agree in batch, width and dtype")
+    if not (Yq.is_contiguous() and Yk.is_contiguous()):
+        raise ValueError("Yq and Yk must be contiguous")
+    A = out if out is not None else torch.empty((B, Lq, Lk), dtype=torch.float32, device=Yq.device)
+    L = load_library()
+    with torch.cuda.device(Yq.device):
+        st = L.gs_attention_scores(_ptr(Yq), _ptr(Yk), _dtype_code(Yq), B, Lq, Lk, r, max(r, 1), float(scale),
+                                   1 if apply_softmax else 0, _ptr(A), PATHS[path], _stream(stream))
+    _check(st, "gs_attention_scores")
+    return A
+
+
+def stream_status(stream=None):
+    """Synchronises and raises GramSpaceError if the device recorded an error."""
+    L = load_library()
+    st = L.gs_stream_status(_stream(stream) if stream is not False else None)
+    _check(st, "gs_stream_status")

@@ -1,0 +1,58 @@
+"""Host-side checks of the C-ABI library that need no GPU: it loads, exports
+every symbol include/gramspace.h declares, and its status strings work."""
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "gramspace.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_01528_gb300 import build, gramspace
+    build.build()
+    return gramspace.load_library()
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"GS_API\s+[\w\s\*]*?\b(gs_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_five_operations():
+    names = declared_symbols()
+    for op in ("gs_build_basis", "gs_project_similarity", "gs_prob_vectorize", "gs_reconstruct",
+               "gs_attention_scores"):
+        assert op in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    from paper_2608_01528_gb300 import gramspace
+    names = declared_symbols()
+    assert sorted(gramspace.EXPORTS) == names
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_status_strings_and_version(lib):
+    from paper_2608_01528_gb300 import gramspace
+    assert gramspace.status_string(0) == "GS_OK"
+    assert gramspace.status_string(7) == "GS_ERR_RANGE"
+    assert gramspace.status_string(99) == "GS_ERR_UNKNOWN"
+    assert lib.gs_version() >= 100
+
+
+def test_host_side_argument_checks_need_no_device(lib):
+    """Invalid arguments are rejected on the host before any CUDA call."""
+    import ctypes
+    from paper_2608_01528_gb300 import gramspace as g
+    h = ctypes.c_void_p()
+    assert lib.gs_build_basis(None, 4, 4, 4, 1e-6, 0, None, None) == g.GS_ERR_INVALID_ARG
+    assert lib.gs_build_basis(None, 0, 4, 4, 1e-6, 0, None, ctypes.byref(h)) == g.GS_ERR_SHAPE
+    assert lib.gs_project_similarity(None, None, 1, 1, 0, 1.0, 0, None, 0, None, 0, None, None,
+                                     None) == g.GS_ERR_INVALID_ARG
+    assert lib.gs_attention_scores(None, None, 5, 1, 1, 1, 1, 1, 1.0, 1, None, 0, None) == g.GS_ERR_INVALID_ARG
+    assert lib.gs_attention_scores(None, None, 0, 1, 1, 1, 4, 2, 1.0, 1, None, 0, None) == g.GS_ERR_SHAPE
+    assert lib.gs_attention_scores(None, None, 0, 0, 4, 4, 4, 4, 1.0, 1, None, 0, None) == g.GS_OK

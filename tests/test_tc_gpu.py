@@ -1,0 +1,125 @@
+"""GPU parity of the tcgen05 fused project + similarity kernel against the oracle.
+
+Same bar as the fp32 paths: |S - S*| <= 1e-4 ||x|| ||c_i||, Y within 1e-4 ||x||,
+argmax bit-exact wherever the oracle's top-2 margin exceeds twice the score
+tolerance.  The kernel rounds X to fp16 (RN) and uses a dithered fp16 copy of
+Q with fp32 accumulation, then takes S = Y R^T in fp32.
+"""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from test_parity_gpu import TOL_S, check_scores, cuda, host
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def large_ref(orc):
+    C = synth.large_codebook()
+    return C, orc.build_basis(C)
+
+
+def test_tc_large_full_size(gs, orc, large_ref):
+    """The full large-batch workload on the tensor-core path: every argmax equals
+    its generating label; Y, S and maxval of a seeded sample of rows match the
+    oracle, and S of every row stays within the bound of the label score."""
+    C, (Qo, Ro, cno) = large_ref
+    w = synth.large()
+    b = gs.build_basis(cuda(C))
+    X = cuda(w["X"])
+    out = gs.project_similarity(b, X, path="tensor", want_S=True, want_Y=True)
+    gs.stream_status()
+    assert np.array_equal(out["argmax"].cpu().numpy(), w["labels"])
+    rows = np.sort(np.random.default_rng(11).choice(w["N"], 768, replace=False))
+    ref = orc.project_similarity(w["X"][rows], Qo, Ro, cno)
+    sub = {k: out[k][torch.from_numpy(rows).to(X.device)] for k in ("S", "Y", "argmax", "maxval")}
+    check_scores(sub, ref, w["X"][rows], cno)
+    xn = ref["xnorm"]
+    assert np.all(np.abs(host(sub["Y"]) - ref["Y"]) <= TOL_S * xn[:, None])
+    # every row: the label's score against the closed form <x, c_label>
+    lab = torch.from_numpy(w["labels"]).to(X.device)
+    s_lab = out["S"].gather(1, lab[:, None].long())[:, 0].double().cpu().numpy()
+    Xd = w["X"].astype(np.float64)
+    full = np.einsum("nd,nd->n", Xd, C[w["labels"]].astype(np.float64))
+    assert np.all(np.abs(s_lab - full) <= TOL_S * np.linalg.norm(Xd, axis=1) * np.sqrt(C.shape[1]))
+
+
+@pytest.mark.parametrize("mode,scale", [("raw", 1.0), ("raw", -0.5), ("cosine", 2.0), ("softmax", 1 / 90.0)])
+def test_tc_modes(gs, orc, large_ref, mode, scale):
+    C, (Qo, Ro, cno) = large_ref
+    w = synth.large(rows=(1000, 5096))
+    b = gs.build_basis(cuda(C))
+    out = gs.project_similarity(b, cuda(w["X"]), mode=mode, scale=scale, path="tensor", want_S=True)
+    gs.stream_status()
+    ref = orc.project_similarity(w["X"], Qo, Ro, cno, mode=getattr(orc, mode.upper()), scale=scale)
+    check_scores(out, ref, w["X"], cno, mode, scale)
+
+
+@pytest.mark.parametrize("N,M,D,ld", [(1, 40, 1000, 1000), (3, 40, 1000, 1000), (1000, 40, 1000, 1000),
+                                       (777, 40, 1002, 1004), (129, 256, 2048, 2048),
+                                       (4099, 100, 4096, 4100)])
+def test_tc_ragged(gs, orc, N, M, D, ld):
+    """Ragged batches (tiles of < 128 rows), D not a multiple of the 64-wide
+    K-block or of 4, r not a multiple of 16, leading dimension > D."""
+    rng = np.random.default_rng(N + M + D)
+    C = (rng.integers(0, 2, size=(M, D)) * 2 - 1).astype(np.float32)
+    X, _ = synth.noisy_rows(C, 5, 0, N, 1.0)
+    Xp = np.zeros((N, ld), np.float32)
+    Xp[:, :D] = X
+    Xp[:, D:] = np.nan  # padding must never be read
+    b = gs.build_basis(cuda(C))
+    Qo, Ro, cno = orc.build_basis(C)
+    Xd = cuda(Xp)[:, :D]
+    out = gs.project_similarity(b, Xd, path="tensor", want_S=True, want_Y=True)
+    gs.stream_status()
+    ref = orc.project_similarity(X, Qo, Ro, cno)
+    check_scores(out, ref, X, cno)
+    assert np.all(np.abs(host(out["Y"]) - ref["Y"]) <= TOL_S * ref["xnorm"][:, None])
+
+
+def test_tc_rank_deficient(gs, orc):
+    """Dependent codewords: R has rows that end early (lower echelon, r < M)."""
+    rng = np.random.default_rng(8)
+    ind = rng.integers(0, 2, size=(48, 3000)).astype(np.float32)
+    dep = np.stack([ind[3], ind[5] - ind[7], ind[0] + ind[1], ind[47]] * 4)
+    C = np.concatenate([ind[:20], dep, ind[20:]])[:64]
+    C = C[rng.permutation(64)]
+    b = gs.build_basis(cuda(C))
+    Qo, Ro, cno = orc.build_basis(C)
+    assert b.r == Qo.shape[0] < 64
+    X, _ = synth.noisy_rows(C, 6, 0, 2000, 1.0)
+    out = gs.project_similarity(b, cuda(X), path="tensor", want_S=True)
+    gs.stream_status()
+    check_scores(out, orc.project_similarity(X, Qo, Ro, cno), X, cno)
+
+
+def test_tc_auto_picks_tensor_and_matches_simt(gs, large_ref):
+    """The auto path and the fp32 SIMT path agree on argmax for the large batch."""
+    C, _ = large_ref
+    w = synth.large(rows=(0, 8192))
+    b = gs.build_basis(cuda(C))
+    X = cuda(w["X"])
+    a = gs.project_similarity(b, X, path="auto")
+    s = gs.project_similarity(b, X, path="simt")
+    assert torch.equal(a["argmax"], s["argmax"])
+    assert np.array_equal(a["argmax"].cpu().numpy(), w["labels"])
+
+
+def test_tc_range_error_is_reported(gs, large_ref):
+    """|x| beyond the fp16 range is caught by the kernel and reported on the
+    device word; the library stays usable afterwards."""
+    C, _ = large_ref
+    w = synth.large(rows=(0, 256))
+    b = gs.build_basis(cuda(C))
+    X = cuda(w["X"])
+    X[17, 3] = 1.0e5
+    gs.project_similarity(b, X, path="tensor")
+    with pytest.raises(gs.GramSpaceError) as ei:
+        gs.stream_status()
+    assert ei.value.status == gs.GS_ERR_RANGE
+    X[17, 3] = 0.0
+    o = gs.project_similarity(b, X, path="tensor")
+    gs.stream_status()
+    assert o["argmax"].shape[0] == 256
