@@ -44,6 +44,8 @@ def parse():
     p.add_argument("--path", default="auto", choices=["auto", "simt", "tensor"])
     p.add_argument("--no-rows", action="store_true", help="skip the per-row side measurements")
     p.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline leg")
+    p.add_argument("--rows", type=int, default=0,
+                   help="profiling only: use the first ROWS queries instead of all 65,536")
     return p.parse_args()
 
 
@@ -217,7 +219,7 @@ def main():
         dist.init_process_group("nccl", device_id=dev)
         pg = dist
 
-    w = synth.large()
+    w = synth.large(rows=(0, args.rows)) if args.rows else synth.large()
     N, D = w["X"].shape
     M = w["C"].shape[0]
     Xh = torch.from_numpy(w["X"]).pin_memory()
@@ -309,11 +311,15 @@ def main():
         rows = side_rows(gs, dev)
 
     if rank == 0:
+        if args.rows:
+            WL = WORKLOAD.replace("65536 queries", f"first {N} of 65536 queries (profiling subset)")
+        else:
+            WL = WORKLOAD
         line = {"metric": METRIC, "value": value, "unit": "queries/s", "n_gpus": ws, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": per_step_ms, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": "f16xf16->f32 (proj), f32 (scores)",
                 "data": "synthetic",
-                "config": {"workload": WORKLOAD, "N": N, "D": D, "M": M, "r": r, "path": args.path,
+                "config": {"workload": WL, "N": N, "D": D, "M": M, "r": r, "path": args.path,
                            "l2": "inputs (2 GiB) larger than L2; no flush", "parallelism": f"replicas x{ws}"},
                 "hbm_gbs": round(achieved, 1), "codebook_bytes_ratio": {
                     "coefficient_D_over_r": D / r, "total_MD_over_rD_plus_Mr": (M * D) / (r * D + M * r)},

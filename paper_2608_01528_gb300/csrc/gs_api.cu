@@ -53,8 +53,8 @@ void free_basis(gs_basis* h) {
     cudaFree(h->Q16);
     cudaFree(h->Q16t);
     cudaFree(h->scratch);
-    cudaFree(h->tc_Rpad);
-    cudaFree(h->tc_jlen16);
+    cudaFree(h->tc_Rh);
+    cudaFree(h->tc_Rl);
     delete h;
 }
 

@@ -30,10 +30,11 @@ struct gs_basis {
     CUtensorMap tmap_q16;    // box {64, 256} over Q16 (valid when r <= 256 and Q16 != null)
     CUtensorMap tmap_q16t;   // box {64, 256} over Q16t
     bool has_tmap_q16 = false, has_tmap_q16t = false;
-    // fused tensor-core similarity: zero-padded R (tc_mpad x tc_npad) and, per
-    // 16-codeword chunk, how many leading columns of R can be nonzero
-    float* tc_Rpad = nullptr;
-    int* tc_jlen16 = nullptr;
+    // fused tensor-core similarity: R split into two bf16 matrices (tc_mpad x
+    // tc_npad, zero padded), Rh = bf16(R) and Rl = bf16(R - Rh), with tensor maps
+    void* tc_Rh = nullptr;
+    void* tc_Rl = nullptr;
+    CUtensorMap tmap_rh, tmap_rl;
     int tc_npad = 0, tc_mpad = 0;
     // scratch for the multi-kernel paths (rows processed in chunks)
     float* scratch = nullptr;
@@ -87,7 +88,7 @@ cudaError_t launch_row_softmax(float* A, long long rows, int L, long long ld, cu
 bool tc_available(int device);
 // creates the tensor maps of h's fp16 operand copies (after build_basis)
 gs_status tc_prepare(gs_basis* h);
-// fused project + similarity on tcgen05 (requires h->has_tmap_q16, r <= 256)
+// fused project + similarity on tcgen05 (requires h->has_tmap_q16: r <= 256, M <= 256)
 cudaError_t launch_ps_tc(const gs_basis* h, const float* X, long long N, int ldx, int mode,
                          float scale, float* Y, int ldy, float* S, int lds, int* argmax,
                          float* maxval, cudaStream_t s);

@@ -1,32 +1,46 @@
 // gs_tc.cu -- tcgen05 (5th-generation tensor core) kernels for sm_103a.
 //
 // k_ps_tc: fused project + similarity for large query batches (paper Sec. 3.1
-// t = U^T x, Sec. 2.2 scaled dot-product similarity, Sec. 3.2 Eq. 2-3).
+// t = U^T x, Sec. 2.2 scaled dot-product similarity, Sec. 3.2 Eq. 2-3), for
+// bases with r <= 256 and codebooks with M <= 256.
 //
-//   GEMM1  Y = X Q^T   tcgen05.mma kind::f16, M = 128 queries, N = r (<= 256),
-//                      fp32 accumulator in TMEM (two 256-column buffers so the
-//                      epilogue of one tile overlaps the MMAs of the next).
-//                      A = X: fp32 in HBM, streamed once by 16 loader warps with
-//                      128-bit loads, rounded to fp16 (RN) and written straight
-//                      into the 128-byte-swizzled K-major layout the MMA reads.
+//   GEMM1  Y = X Q^T   tcgen05.mma kind::f16, M = 128 queries, N = r,
+//                      fp32 accumulator in TMEM columns [0, 256).
+//                      A = X: fp32 tiles streamed from HBM by TMA into a staging
+//                      ring (several 32 KB tiles in flight per SM), rounded to
+//                      fp16 (RN) by converter warps into the 128-byte-swizzled
+//                      K-major layout the MMA reads.
 //                      B = Q: the basis' fixed fp16 copy (dithered rounding, see
 //                      gs_build.cu), fetched per K-block by TMA (L2-resident).
-//   GEMM2  S = Y R^T   fp32 FMA on CUDA cores in the epilogue warps, reading Y
-//                      from TMEM with tcgen05.ld and skipping the zero tail of
-//                      each row of R (R is lower echelon).  The dominant terms of
-//                      S are single products Y_i R_ii, so this product needs fp32
-//                      rather than a single fp16/tf32 rounding.
-//   epilogue           scale / cosine (full-D ||x|| accumulated by the loaders
-//                      from the fp32 input) / online softmax, argmax (lowest index
-//                      on ties), maxval, optional Y and S stores.
+//   GEMM2  S = Y R^T   tcgen05.mma kind::f16 with bf16 operands split in two,
+//                      Y = Yh + Yl and R = Rh + Rl, S = Yh Rh + Yl Rh + Yh Rl
+//                      (relative error ~2^-16, fp32's exponent range), fp32
+//                      accumulator in TMEM columns [256, 512).  The epilogue
+//                      splits Y in place in TMEM (each 32-column fp32 chunk
+//                      becomes 16 columns of packed Yh and 16 of packed Yl), and
+//                      the MMA reads that A operand straight from TMEM; the Rh /
+//                      Rl tiles come through the same TMA ring as the Q tiles.
+//                      A single fp16/tf32 rounding would not do here: the
+//                      dominant terms of S are single products Y_i R_ii.
+//   epilogue           scale / cosine (full-D ||x|| accumulated by the
+//                      converters from the fp32 input) / online softmax, argmax
+//                      (lowest index on ties), maxval, optional Y and S stores.
+//
+// Why the X tiles go through TMA rather than through registers: a thread that
+// signals "A stage full" with an mbarrier arrive (a release) cannot complete
+// that arrive while its own prefetched global loads are still in flight, so a
+// register-prefetch loader serialises on one memory round trip per K-block.
+// With TMA the bytes in flight are the hardware's, and the converters' release
+// only orders shared-memory traffic.
 //
 // Work split: one persistent CTA per SM; each CTA takes a contiguous, balanced
 // range of rows and cuts it into tiles of at most 128 rows, so every CTA moves
-// the same number of bytes.  Warp roles:
-//   warps 0-3   epilogue (warp w reads TMEM lanes 32w..32w+31 = rows of the tile)
-//   warp  4     TMA producer of the Q tiles
-//   warp  5     TMEM allocator and MMA issuer (one elected lane)
-//   warps 6-17  X loaders / fp16 converters
+// the same number of bytes.  Warp roles (352 threads):
+//   warps 0-3    epilogue: warp w owns TMEM lanes 32w..32w+31 (rows of the tile)
+//   warp  4      TMA producer of the X tiles
+//   warp  5      TMEM allocator and MMA issuer (one elected lane)
+//   warp  6      TMA producer of the B operand tiles (Q per K-block, then Rh / Rl)
+//   warps 7-10   converters (fp32 -> fp16, row norms, range check)
 // Every wait on an mbarrier is bounded (wall-clock limit): on expiry the CTA
 // records GS_DEV_ERR_TIMEOUT, raises a CTA-wide abort flag so the other roles
 // leave their loops, waits (bounded) for its own TMA copies and MMAs to land,
@@ -35,6 +49,7 @@
 #include <float.h>
 
 #include <algorithm>
+#include <vector>
 
 #include "gs_internal.h"
 
@@ -43,19 +58,24 @@ namespace {
 
 __device__ unsigned g_err_tc = 0;
 
-constexpr int kBM = 128;           // queries per tile (MMA M)
-constexpr int kBK = 64;            // fp16 elements per K-block (one 128-byte row)
-constexpr int kStagesMax = 4;
+constexpr int kBM = 128;             // queries per tile (MMA M)
+constexpr int kBK = 64;              // K elements per block (fp16 A row = 128 B, fp32 staging row = 256 B)
 constexpr int kEpiWarps = 4;
-constexpr int kLoadWarps = 12;
-constexpr int kTmaWarp = 4;
+constexpr int kXWarp = 4;
 constexpr int kMmaWarp = 5;
-constexpr int kLoad0 = 6;
-constexpr int kThreads = (kLoad0 + kLoadWarps) * 32;  // 576
-constexpr int kRowGroups = kLoadWarps * 2;            // 24 rows per float4 column sweep
-constexpr int kRowsPerLoader = (kBM + kRowGroups - 1) / kRowGroups;  // 6
+constexpr int kBWarp = 6;
+constexpr int kCvt0 = 7;
+constexpr int kCvtWarps = 4;
+constexpr int kThreads = (kCvt0 + kCvtWarps) * 32;  // 352
+constexpr int kCvtThreads = kCvtWarps * 32;          // 128
+constexpr int kCvtRowStep = kCvtThreads / 16;        // 8 rows per sweep of the 16 float4 columns
+constexpr int kCvtRows = kBM / kCvtRowStep;          // 16 rows per converter thread
+constexpr int kXStageBytes = kBM * kBK * 4;          // 32 KB fp32 staging tile
+constexpr int kAStageBytes = kBM * kBK * 2;          // 16 KB fp16 operand tile
+constexpr int kBStageBytes = 256 * kBK * 2;          // 32 KB: up to 256 rows of one B operand K-block
+constexpr int kMaxSX = 4, kMaxSA = 2, kMaxSB = 4;
 constexpr int kTmemCols = 512;
-constexpr int kCwChunk = 16;       // codewords per epilogue accumulator chunk
+constexpr int kSCol = 256;           // first TMEM column of the score accumulator
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s
 
 // ----------------------------------------------------------------- PTX wrappers
@@ -133,9 +153,14 @@ __device__ __forceinline__ void tc_fence_before() {
 __device__ __forceinline__ void tc_fence_after() {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
-__device__ __forceinline__ uint64_t l2_evict_last_policy() {
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
     uint64_t p;
     asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
     return p;
 }
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
@@ -167,12 +192,37 @@ __device__ __forceinline__ void mma_f16_ss(uint32_t d_tmem, uint64_t a_desc, uin
         "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
+// D[tmem] (+)= A[tmem] * B[smem]^T, bf16 inputs, fp32 accumulate.
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
 // Arrives once on `bar` when every previously issued MMA of this thread has completed.
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                      smem_u32(bar))
                  : "memory");
 }
+// 16 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+          "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
 // 32 consecutive fp32 columns of this thread's TMEM lane.
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
     uint32_t r[32];
@@ -190,19 +240,22 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
-
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
-    uint32_t r[16];
+// Stores 16 consecutive 32-bit columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* v) {
     asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
-          "=r"(r[15])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
+        "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+        : "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() {
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+// Two bf16 values in one 32-bit word, the first in the low half.
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&v);
 }
 
 // Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
@@ -220,26 +273,31 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
 __host__ __device__ constexpr uint32_t idesc_f16_f32(int n) {
     return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
 }
+// The same with A = B = bf16 (atype = btype = 1).
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int n) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+}
 
+// ----------------------------------------------------------------- work split
 struct TileRange {
     long long row0;
     int nrows;
 };
 
-// Balanced contiguous row range of CTA c, cut into at most-128-row tiles.
+// Balanced contiguous row range of CTA c, cut into tiles of at most 128 rows.
 struct CtaRows {
     long long rb;
     long long rows;
     int ntiles;
     int tsize;
-    __device__ CtaRows(long long N, int G, int c) {
+    __host__ __device__ CtaRows(long long N, int G, int c) {
         const long long base = N / G, rem = N % G;
         rows = base + (c < rem ? 1 : 0);
         rb = (long long)c * base + (c < rem ? c : rem);
         ntiles = (int)((rows + kBM - 1) / kBM);
         tsize = ntiles ? (int)((rows + ntiles - 1) / ntiles) : 0;
     }
-    __device__ TileRange tile(int t) const {
+    __host__ __device__ TileRange tile(int t) const {
         TileRange tr;
         tr.row0 = rb + (long long)t * tsize;
         const long long left = rb + rows - tr.row0;
@@ -249,11 +307,10 @@ struct CtaRows {
 };
 
 struct PsParams {
-    const float* X;
     long long N;
-    int ldx, D, r, npad, M, mpad, nkb, stages;
-    const float* Rpad;      // mpad x npad fp32, zero padded copy of R
-    const int* jlen16;      // per 16-codeword chunk: columns of R that can be nonzero
+    int D, r, npad, M, mpad, nkb, nkr;
+    int sx, sa, sb;         // ring depths: fp32 X staging, fp16 A, B operand tiles
+    int box_rows;           // rows of each X TMA box (>= every tile's rows)
     const float* cnorm;     // M
     int mode;
     float scale;
@@ -265,248 +322,311 @@ struct PsParams {
     float* maxval;
 };
 
-struct Smem {
-    uint64_t a_full[kStagesMax], b_full[kStagesMax], empty[kStagesMax];
-    uint64_t y_full[2], y_empty[2], xn_full[2], xn_empty[2], mma_done;
+struct Ctl {
+    uint64_t x_full[kMaxSX], x_empty[kMaxSX];
+    uint64_t a_full[kMaxSA], a_empty[kMaxSA];
+    uint64_t b_full[kMaxSB], b_empty[kMaxSB];
+    uint64_t y_full, ysplit_full, s_full, s_empty, gemm2_done;
+    uint64_t xn_full[2], xn_empty[2];
+    uint64_t mma_done;
     float xn[2][kBM];
     uint32_t tmem_base;
     int abort_flag;
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
-    k_ps_tc(const __grid_constant__ CUtensorMap tmap_q, const PsParams p) {
+    k_ps_tc(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_q,
+            const __grid_constant__ CUtensorMap tmap_rh, const __grid_constant__ CUtensorMap tmap_rl,
+            const PsParams p) {
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte aligned operand area (SW128 atoms), control block after it
     const uint32_t raw = smem_u32(smem_raw);
     uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
-    const int S = p.stages;
-    const uint32_t a_bytes = kBM * 128;
-    const uint32_t b_bytes = (uint32_t)p.npad * 128;
-    uint8_t* A = base;
-    uint8_t* B = base + (size_t)S * a_bytes;
-    Smem& sm = *reinterpret_cast<Smem*>(B + (size_t)S * b_bytes);
-    volatile int* abort_flag = &sm.abort_flag;
+    uint8_t* Xs = base;
+    uint8_t* As = Xs + (size_t)p.sx * kXStageBytes;
+    uint8_t* Bs = As + (size_t)p.sa * kAStageBytes;
+    Ctl& c = *reinterpret_cast<Ctl*>(Bs + (size_t)p.sb * kBStageBytes);
+    volatile int* abort_flag = &c.abort_flag;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const CtaRows cr(p.N, gridDim.x, blockIdx.x);
-    const int total_it = cr.ntiles * p.nkb;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < S; ++s) {
-            mbar_init(&sm.a_full[s], kLoadWarps);
-            mbar_init(&sm.b_full[s], 1);
-            mbar_init(&sm.empty[s], 1);
+        for (int s = 0; s < p.sx; ++s) {
+            mbar_init(&c.x_full[s], 1);
+            mbar_init(&c.x_empty[s], kCvtWarps);
         }
+        for (int s = 0; s < p.sa; ++s) {
+            mbar_init(&c.a_full[s], kCvtWarps);
+            mbar_init(&c.a_empty[s], 1);
+        }
+        for (int s = 0; s < p.sb; ++s) {
+            mbar_init(&c.b_full[s], 1);
+            mbar_init(&c.b_empty[s], 1);
+        }
+        mbar_init(&c.y_full, 1);
+        mbar_init(&c.ysplit_full, kEpiWarps);
+        mbar_init(&c.s_full, 1);
+        mbar_init(&c.s_empty, kEpiWarps);
+        mbar_init(&c.gemm2_done, 1);
         for (int b = 0; b < 2; ++b) {
-            mbar_init(&sm.y_full[b], 1);
-            mbar_init(&sm.y_empty[b], kEpiWarps);
-            mbar_init(&sm.xn_full[b], kLoadWarps);
-            mbar_init(&sm.xn_empty[b], kEpiWarps);
+            mbar_init(&c.xn_full[b], kCvtWarps);
+            mbar_init(&c.xn_empty[b], kEpiWarps);
         }
-        mbar_init(&sm.mma_done, 1);
-        sm.abort_flag = 0;
+        mbar_init(&c.mma_done, 1);
+        c.abort_flag = 0;
         fence_barrier_init();
     }
     if (warp == kMmaWarp) {
-        tmem_alloc(&sm.tmem_base, kTmemCols);
+        tmem_alloc(&c.tmem_base, kTmemCols);
         tmem_relinquish();
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tmem = sm.tmem_base;
+    const uint32_t tmem = c.tmem_base;
 
-    if (warp == kTmaWarp) {
-        // ------------------------------------------------------------- Q tiles via TMA
+    if (warp == kXWarp) {
+        // ------------------------------------------------------------- X tiles via TMA
         if (lane == 0) {
-            const uint64_t pol = l2_evict_last_policy();
+            const uint64_t pol = l2_policy_evict_first();
+            const uint32_t bytes = (uint32_t)p.box_rows * kBK * 4;
             int it = 0;
-            for (; it < total_it; ++it) {
-                const int s = it % S;
-                const uint32_t ph = (uint32_t)(it / S) & 1u;
-                if (!mbar_wait(&sm.empty[s], ph ^ 1u, abort_flag)) break;
-                mbar_arrive_expect_tx(&sm.b_full[s], b_bytes);
-                tma_load_2d(B + (size_t)s * b_bytes, &tmap_q, &sm.b_full[s], (it % p.nkb) * kBK, 0, pol);
+            bool ok = true;
+            for (int t = 0; t < cr.ntiles && ok; ++t) {
+                const TileRange tr = cr.tile(t);
+                for (int kb = 0; kb < p.nkb; ++kb, ++it) {
+                    const int s = it % p.sx;
+                    if (!mbar_wait(&c.x_empty[s], ((uint32_t)(it / p.sx) & 1u) ^ 1u, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&c.x_full[s], bytes);
+                    tma_load_2d(Xs + (size_t)s * kXStageBytes, &tmap_x, &c.x_full[s], kb * kBK, (int)tr.row0, pol);
+                }
             }
-            // make sure every copy this thread started has landed before the CTA exits
-            for (int j = std::max(0, it - S); j < it; ++j)
-                mbar_drain(&sm.b_full[j % S], (uint32_t)(j / S) & 1u);
+            // every copy this thread started lands before the CTA can exit
+            for (int j = std::max(0, it - p.sx); j < it; ++j) mbar_drain(&c.x_full[j % p.sx], (uint32_t)(j / p.sx) & 1u);
+        }
+    } else if (warp == kBWarp) {
+        // ------------------------------------------------------------- B operand tiles via TMA:
+        // per tile, nkb Q tiles (GEMM1), then nkr pairs of Rh / Rl tiles (GEMM2)
+        if (lane == 0) {
+            const uint64_t pol = l2_policy_evict_last();
+            const uint32_t qbytes = (uint32_t)p.npad * kBK * 2, rbytes = (uint32_t)p.mpad * kBK * 2;
+            const int per_tile = p.nkb + 2 * p.nkr;
+            const int total = cr.ntiles * per_tile;
+            int it = 0;
+            for (; it < total; ++it) {
+                const int s = it % p.sb;
+                if (!mbar_wait(&c.b_empty[s], ((uint32_t)(it / p.sb) & 1u) ^ 1u, abort_flag)) break;
+                const int k = it % per_tile;
+                uint8_t* dst = Bs + (size_t)s * kBStageBytes;
+                if (k < p.nkb) {
+                    mbar_arrive_expect_tx(&c.b_full[s], qbytes);
+                    tma_load_2d(dst, &tmap_q, &c.b_full[s], k * kBK, 0, pol);
+                } else {
+                    const int kr = (k - p.nkb) >> 1;
+                    mbar_arrive_expect_tx(&c.b_full[s], rbytes);
+                    tma_load_2d(dst, ((k - p.nkb) & 1) ? &tmap_rl : &tmap_rh, &c.b_full[s], kr * kBK, 0, pol);
+                }
+            }
+            for (int j = std::max(0, it - p.sb); j < it; ++j) mbar_drain(&c.b_full[j % p.sb], (uint32_t)(j / p.sb) & 1u);
         }
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------- MMA issue
         if (lane == 0) {
-            const uint32_t idesc = idesc_f16_f32(p.npad);
-            int it = 0;
+            const uint32_t idesc1 = idesc_f16_f32(p.npad);
+            const uint32_t idesc2 = idesc_bf16_f32(p.mpad);
+            const uint32_t y_tmem = tmem, s_tmem = tmem + kSCol;
+            int ia = 0, ib = 0;
             bool ok = true;
             for (int t = 0; t < cr.ntiles && ok; ++t) {
-                const int b = t & 1;
-                if (!mbar_wait(&sm.y_empty[b], ((uint32_t)(t >> 1) & 1u) ^ 1u, abort_flag)) break;
-                tc_fence_after();
-                const uint32_t d_tmem = tmem + (uint32_t)(b * 256);
-                for (int kb = 0; kb < p.nkb; ++kb, ++it) {
-                    const int s = it % S;
-                    const uint32_t ph = (uint32_t)(it / S) & 1u;
-                    if (!mbar_wait(&sm.a_full[s], ph, abort_flag) || !mbar_wait(&sm.b_full[s], ph, abort_flag)) {
+                const uint32_t pt = (uint32_t)t & 1u;
+                // GEMM1: Y = X Q^T into columns [0, npad)
+                for (int kb = 0; kb < p.nkb; ++kb, ++ia, ++ib) {
+                    const int sa = ia % p.sa, sb = ib % p.sb;
+                    if (!mbar_wait(&c.a_full[sa], (uint32_t)(ia / p.sa) & 1u, abort_flag) ||
+                        !mbar_wait(&c.b_full[sb], (uint32_t)(ib / p.sb) & 1u, abort_flag)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint64_t ad = sdesc_sw128(smem_u32(A + (size_t)s * a_bytes));
-                    const uint64_t bd = sdesc_sw128(smem_u32(B + (size_t)s * b_bytes));
+                    const uint64_t ad = sdesc_sw128(smem_u32(As + (size_t)sa * kAStageBytes));
+                    const uint64_t bd = sdesc_sw128(smem_u32(Bs + (size_t)sb * kBStageBytes));
 #pragma unroll
                     for (int k = 0; k < kBK / 16; ++k)
-                        mma_f16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
+                        mma_f16_ss(y_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc1,
                                    (kb | k) != 0 ? 1u : 0u);
-                    mma_commit(&sm.empty[s]);
+                    mma_commit(&c.a_empty[sa]);
+                    mma_commit(&c.b_empty[sb]);
                 }
-                if (ok) mma_commit(&sm.y_full[b]);
+                if (!ok) break;
+                mma_commit(&c.y_full);
+                // GEMM2: S = Yh Rh + Yl Rh + Yh Rl into columns [256, 256 + mpad), once the
+                // epilogue has split Y in place and released the previous tile's S
+                if (!mbar_wait(&c.ysplit_full, pt, abort_flag) || !mbar_wait(&c.s_empty, pt ^ 1u, abort_flag)) break;
+                tc_fence_after();
+                for (int kr = 0; kr < p.nkr; ++kr, ib += 2) {
+                    const int sh = ib % p.sb, sl = (ib + 1) % p.sb;
+                    if (!mbar_wait(&c.b_full[sh], (uint32_t)(ib / p.sb) & 1u, abort_flag) ||
+                        !mbar_wait(&c.b_full[sl], (uint32_t)((ib + 1) / p.sb) & 1u, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint64_t rh = sdesc_sw128(smem_u32(Bs + (size_t)sh * kBStageBytes));
+                    const uint64_t rl = sdesc_sw128(smem_u32(Bs + (size_t)sl * kBStageBytes));
+#pragma unroll
+                    for (int k = 0; k < kBK / 16; ++k) {
+                        // r columns [64 kr + 16 k, +16): chunk of 32 = (4 kr + k) / 2, half = k & 1
+                        const int kk = 4 * kr + k;
+                        const uint32_t a_hi = y_tmem + (uint32_t)(32 * (kk >> 1) + 8 * (kk & 1));
+                        const uint32_t a_lo = a_hi + 16;
+                        mma_bf16_ts(s_tmem, a_hi, rh + (uint64_t)(2 * k), idesc2, (kr | k) != 0 ? 1u : 0u);
+                        mma_bf16_ts(s_tmem, a_lo, rh + (uint64_t)(2 * k), idesc2, 1u);
+                        mma_bf16_ts(s_tmem, a_hi, rl + (uint64_t)(2 * k), idesc2, 1u);
+                    }
+                    mma_commit(&c.b_empty[sh]);
+                    mma_commit(&c.b_empty[sl]);
+                }
+                if (!ok) break;
+                mma_commit(&c.s_full);
+                // the next tile's GEMM1 overwrites the columns GEMM2 reads: wait for it to finish
+                mma_commit(&c.gemm2_done);
+                if (!mbar_wait(&c.gemm2_done, pt, abort_flag)) break;
+                tc_fence_after();
             }
             // all MMAs issued by this thread complete before TMEM is released
-            mma_commit(&sm.mma_done);
-            mbar_drain(&sm.mma_done, 0);
+            mma_commit(&c.mma_done);
+            mbar_drain(&c.mma_done, 0);
         }
-    } else if (warp >= kLoad0) {
-        // ------------------------------------------------------------- X loaders
-        const int l = threadIdx.x - kLoad0 * 32;  // 0..383
-        // thread l covers float4 column c4 = l % 16 of rows l/16 + 24u (u < 6, row < 128)
-        float nrm[kRowsPerLoader];
+    } else if (warp >= kCvt0) {
+        // ------------------------------------------------------------- converters
+        const int l = threadIdx.x - kCvt0 * 32;  // 0..127
+        const int c4 = l & 15;                   // float4 column of the 64-wide K-block
+        const int rbase = l >> 4;                // rows rbase + 8u, u < 16
+        float nrm[kCvtRows];
 #pragma unroll
-        for (int u = 0; u < kRowsPerLoader; ++u) nrm[u] = 0.f;
+        for (int u = 0; u < kCvtRows; ++u) nrm[u] = 0.f;
         float amax = 0.f;
-        float4 cur[kRowsPerLoader], nxt[kRowsPerLoader];
-        const int c4 = l & 15;
-        auto fetch = [&](int it, float4* v) {
-            const int t = it / p.nkb, kb = it % p.nkb;
+        int it = 0;
+        bool ok = true;
+        for (int t = 0; t < cr.ntiles && ok; ++t) {
             const TileRange tr = cr.tile(t);
-            const int col = kb * kBK + c4 * 4;
-#pragma unroll
-            for (int u = 0; u < kRowsPerLoader; ++u) {
-                const int row = (l >> 4) + kRowGroups * u;
-                float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (row < tr.nrows) {
-                    const float* src = p.X + (size_t)(tr.row0 + row) * p.ldx + col;
-                    if (col + 3 < p.D) {
-                        x = __ldcs(reinterpret_cast<const float4*>(src));
-                    } else if (col < p.D) {
-                        x.x = src[0];
-                        if (col + 1 < p.D) x.y = src[1];
-                        if (col + 2 < p.D) x.z = src[2];
-                    }
+            const int b = t & 1;
+            for (int kb = 0; kb < p.nkb; ++kb, ++it) {
+                const int sx = it % p.sx, sa = it % p.sa;
+                if (!mbar_wait_warp(&c.x_full[sx], (uint32_t)(it / p.sx) & 1u, abort_flag) ||
+                    !mbar_wait_warp(&c.a_empty[sa], ((uint32_t)(it / p.sa) & 1u) ^ 1u, abort_flag)) {
+                    ok = false;
+                    break;
                 }
-                v[u] = x;
-            }
-        };
-        if (total_it > 0) fetch(0, cur);
-        for (int it = 0; it < total_it; ++it) {
-            if (it + 1 < total_it) fetch(it + 1, nxt);
-            const int s = it % S;
-            const uint32_t ph = (uint32_t)(it / S) & 1u;
-            if (!mbar_wait_warp(&sm.empty[s], ph ^ 1u, abort_flag)) break;
-            uint8_t* At = A + (size_t)s * a_bytes;
+                const uint8_t* Xt = Xs + (size_t)sx * kXStageBytes;
+                uint8_t* At = As + (size_t)sa * kAStageBytes;
 #pragma unroll
-            for (int u = 0; u < kRowsPerLoader; ++u) {
-                const int row = (l >> 4) + kRowGroups * u;
-                if (row >= kBM) break;
-                const float4 x = cur[u];
-                nrm[u] = fmaf(x.x, x.x, fmaf(x.y, x.y, fmaf(x.z, x.z, fmaf(x.w, x.w, nrm[u]))));
-                amax = fmaxf(amax, fmaxf(fmaxf(fabsf(x.x), fabsf(x.y)), fmaxf(fabsf(x.z), fabsf(x.w))));
-                const __half2 h0 = __floats2half2_rn(x.x, x.y);
-                const __half2 h1 = __floats2half2_rn(x.z, x.w);
-                uint2 pk;
-                pk.x = *reinterpret_cast<const uint32_t*>(&h0);
-                pk.y = *reinterpret_cast<const uint32_t*>(&h1);
-                const int chunk = (c4 >> 1) ^ (row & 7);
-                *reinterpret_cast<uint2*>(At + row * 128 + chunk * 16 + (c4 & 1) * 8) = pk;
-            }
-            fence_proxy_async();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sm.a_full[s]);
-#pragma unroll
-            for (int u = 0; u < kRowsPerLoader; ++u) cur[u] = nxt[u];
-            if (it % p.nkb == p.nkb - 1) {
-                // tile finished: ||x||^2 of this thread's rows -> shared, for cosine scores
-                const int t = it / p.nkb, b = t & 1;
-#pragma unroll
-                for (int u = 0; u < kRowsPerLoader; ++u) {
-                    float v = nrm[u];
-                    v += __shfl_xor_sync(0xffffffffu, v, 8);
-                    v += __shfl_xor_sync(0xffffffffu, v, 4);
-                    v += __shfl_xor_sync(0xffffffffu, v, 2);
-                    v += __shfl_xor_sync(0xffffffffu, v, 1);
-                    nrm[u] = v;
+                for (int u = 0; u < kCvtRows; ++u) {
+                    const int row = rbase + kCvtRowStep * u;
+                    float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (row < tr.nrows) x = *reinterpret_cast<const float4*>(Xt + row * (kBK * 4) + c4 * 16);
+                    nrm[u] = fmaf(x.x, x.x, fmaf(x.y, x.y, fmaf(x.z, x.z, fmaf(x.w, x.w, nrm[u]))));
+                    amax = fmaxf(amax, fmaxf(fmaxf(fabsf(x.x), fabsf(x.y)), fmaxf(fabsf(x.z), fabsf(x.w))));
+                    const __half2 h0 = __floats2half2_rn(x.x, x.y);
+                    const __half2 h1 = __floats2half2_rn(x.z, x.w);
+                    uint2 pk;
+                    pk.x = *reinterpret_cast<const uint32_t*>(&h0);
+                    pk.y = *reinterpret_cast<const uint32_t*>(&h1);
+                    const int chunk = (c4 >> 1) ^ (row & 7);
+                    *reinterpret_cast<uint2*>(At + row * 128 + chunk * 16 + (c4 & 1) * 8) = pk;
                 }
-                if (!mbar_wait_warp(&sm.xn_empty[b], ((uint32_t)(t >> 1) & 1u) ^ 1u, abort_flag)) break;
-                if ((lane & 15) == 0) {
-#pragma unroll
-                    for (int u = 0; u < kRowsPerLoader; ++u) {
-                        const int row = (l >> 4) + kRowGroups * u;
-                        if (row < kBM) sm.xn[b][row] = nrm[u];
-                    }
-                }
+                fence_proxy_async();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&sm.xn_full[b]);
-#pragma unroll
-                for (int u = 0; u < kRowsPerLoader; ++u) nrm[u] = 0.f;
+                if (lane == 0) {
+                    mbar_arrive(&c.a_full[sa]);
+                    mbar_arrive(&c.x_empty[sx]);
+                }
             }
+            if (!ok) break;
+            // tile finished: ||x||^2 of each row -> shared, for cosine scores
+#pragma unroll
+            for (int u = 0; u < kCvtRows; ++u) {
+                float v = nrm[u];
+                v += __shfl_xor_sync(0xffffffffu, v, 8);
+                v += __shfl_xor_sync(0xffffffffu, v, 4);
+                v += __shfl_xor_sync(0xffffffffu, v, 2);
+                v += __shfl_xor_sync(0xffffffffu, v, 1);
+                nrm[u] = v;
+            }
+            if (!mbar_wait_warp(&c.xn_empty[b], ((uint32_t)(t >> 1) & 1u) ^ 1u, abort_flag)) break;
+            if ((lane & 15) == 0) {
+#pragma unroll
+                for (int u = 0; u < kCvtRows; ++u) c.xn[b][rbase + kCvtRowStep * u] = nrm[u];
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&c.xn_full[b]);
+#pragma unroll
+            for (int u = 0; u < kCvtRows; ++u) nrm[u] = 0.f;
         }
         if (amax > 65504.f) atomicOr(&g_err_tc, GS_DEV_ERR_RANGE);
     } else {
         // ------------------------------------------------------------- epilogue (warps 0-3)
         const int i = threadIdx.x;  // row within the tile = TMEM lane
         const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        const uint32_t ty = tmem + lane_base, ts = tmem + lane_base + kSCol;
         for (int t = 0; t < cr.ntiles; ++t) {
+            const uint32_t pt = (uint32_t)t & 1u;
             const int b = t & 1;
-            const uint32_t ph = (uint32_t)(t >> 1) & 1u;
-            if (!mbar_wait_warp(&sm.y_full[b], ph, abort_flag)) break;
+            if (!mbar_wait_warp(&c.y_full, pt, abort_flag)) break;
             tc_fence_after();
-            if (!mbar_wait_warp(&sm.xn_full[b], ph, abort_flag)) break;
-            const float xnorm = sqrtf(sm.xn[b][i]);
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sm.xn_empty[b]);
             const TileRange tr = cr.tile(t);
             const bool valid = i < tr.nrows;
             const long long row = tr.row0 + i;
-            const uint32_t tb = tmem + lane_base + (uint32_t)(b * 256);
-            float y[32];
-            if (p.Y) {
-                for (int jc = 0; jc < p.npad; jc += 32) {
-                    tmem_ld32(tb + (uint32_t)jc, y);
-                    if (valid) {
-                        float* dst = p.Y + (size_t)row * p.ldy + jc;
+            // split Y in place: chunk of 32 fp32 columns -> 16 columns bf16(Y) + 16 columns bf16(Y - bf16(Y))
+            for (int jc = 0; jc < p.npad; jc += 32) {
+                float y[32];
+                tmem_ld32(ty + (uint32_t)jc, y);
+                // columns past npad were never written by GEMM1: make them exact zeros
 #pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (jc + j < p.r) dst[j] = y[j];
-                    }
+                for (int j = 0; j < 32; ++j)
+                    if (jc + j >= p.npad) y[j] = 0.f;
+                if (p.Y && valid) {
+                    float* dst = p.Y + (size_t)row * p.ldy + jc;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (jc + j < p.r) dst[j] = y[j];
                 }
+                uint32_t hi[16], lo[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                    const float a = y[2 * j], bb = y[2 * j + 1];
+                    const float ah = __bfloat162float(__float2bfloat16_rn(a));
+                    const float bh = __bfloat162float(__float2bfloat16_rn(bb));
+                    hi[j] = pack_bf16(ah, bh);
+                    lo[j] = pack_bf16(a - ah, bb - bh);
+                }
+                tmem_st16(ty + (uint32_t)jc, hi);
+                tmem_st16(ty + (uint32_t)(jc + 16), lo);
             }
+            tmem_wait_st();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&c.ysplit_full);
+            if (!mbar_wait_warp(&c.xn_full[b], (uint32_t)(t >> 1) & 1u, abort_flag)) break;
+            const float xnorm = sqrtf(c.xn[b][i]);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&c.xn_empty[b]);
+            if (!mbar_wait_warp(&c.s_full, pt, abort_flag)) break;
+            tc_fence_after();
             float best = -FLT_MAX, run_max = -FLT_MAX, run_sum = 0.f;
             int besti = 0;
-            for (int ic = 0; ic < p.mpad; ic += kCwChunk) {
-                float acc[kCwChunk];
+            for (int ic = 0; ic < p.mpad; ic += 16) {
+                float sv[16];
+                tmem_ld16(ts + (uint32_t)ic, sv);
 #pragma unroll
-                for (int q = 0; q < kCwChunk; ++q) acc[q] = 0.f;
-                const int jl = p.jlen16[ic / kCwChunk];
-                for (int jc = 0; jc < jl; jc += 16) {
-                    float y16[16];
-                    tmem_ld16(tb + (uint32_t)jc, y16);
-#pragma unroll
-                    for (int q = 0; q < kCwChunk; ++q) {
-                        const float4* Rq = reinterpret_cast<const float4*>(p.Rpad + (size_t)(ic + q) * p.npad + jc);
-#pragma unroll
-                        for (int j4 = 0; j4 < 4; ++j4) {
-                            const float4 rv = __ldg(Rq + j4);
-                            acc[q] = fmaf(y16[4 * j4 + 0], rv.x, acc[q]);
-                            acc[q] = fmaf(y16[4 * j4 + 1], rv.y, acc[q]);
-                            acc[q] = fmaf(y16[4 * j4 + 2], rv.z, acc[q]);
-                            acc[q] = fmaf(y16[4 * j4 + 3], rv.w, acc[q]);
-                        }
-                    }
-                }
-#pragma unroll
-                for (int q = 0; q < kCwChunk; ++q) {
-                    const int ci = ic + q;
+                for (int j = 0; j < 16; ++j) {
+                    const int ci = ic + j;
                     if (ci >= p.M) break;
-                    float g = p.scale * acc[q];
+                    float g = p.scale * sv[j];
                     if (p.mode == GS_SCORE_COSINE) {
                         const float den = xnorm * p.cnorm[ci];
                         g = den > 0.f ? g / den : 0.f;
@@ -525,7 +645,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&sm.y_empty[b]);
+            if (lane == 0) mbar_arrive(&c.s_empty);
             if (!valid) continue;
             float outmax = best;
             if (p.mode == GS_SCORE_SOFTMAX) {
@@ -557,46 +677,40 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
 EncodeTiledFn encode_fn() {
     static EncodeTiledFn fn = nullptr;
     if (!fn) {
-        void* p = nullptr;
+        void* ptr = nullptr;
         cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
                 cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
-            fn = (EncodeTiledFn)p;
+            fn = (EncodeTiledFn)ptr;
     }
     return fn;
 }
 
-// 2-D fp16 tensor map over a row-major (rows x cols, ld elements) matrix with a
-// {64, box_rows} box and 128-byte swizzle; out-of-range elements read as zero.
-bool make_tmap_f16(CUtensorMap* m, const void* ptr, int rows, int cols, int ld, int box_rows) {
+// 2-D tensor map over a row-major (rows x cols, ld elements) matrix with a
+// {box_cols, box_rows} box; out-of-range elements read as zero.
+bool make_tmap_2d(CUtensorMap* m, CUtensorMapDataType dt, int esize, const void* ptr, long long rows, int cols,
+                  long long ld, int box_cols, int box_rows, CUtensorMapSwizzle sw) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
-    cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
+    cuuint64_t strides[1] = {(cuuint64_t)ld * esize};
+    cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    return fn(m, dt, 2, const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-__global__ void k_pad_r(const float* __restrict__ R, int M, int r, int ldr, float* __restrict__ Rp, int mpad,
-                        int npad) {
+// R (M x r fp32) -> Rh = bf16(R), Rl = bf16(R - Rh), both mpad x npad, zero padded.
+__global__ void k_split_r(const float* __restrict__ R, int M, int r, int ldr, __nv_bfloat16* __restrict__ Rh,
+                          __nv_bfloat16* __restrict__ Rl, int mpad, int npad) {
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= (long long)mpad * npad) return;
     const int i = (int)(idx / npad), j = (int)(idx % npad);
-    Rp[idx] = (i < M && j < r) ? R[(size_t)i * ldr + j] : 0.f;
-}
-
-// Per 16-codeword chunk: the leading columns of R (rounded up to the epilogue's
-// 16-column step, never past npad) that hold any nonzero coefficient.
-__global__ void k_jlen16(const int* __restrict__ rlen, int M, int nchunks, int npad, int* __restrict__ out) {
-    const int c = blockIdx.x * blockDim.x + threadIdx.x;
-    if (c >= nchunks) return;
-    int m = 0;
-    for (int i = c * kCwChunk; i < min(M, c * kCwChunk + kCwChunk); ++i) m = max(m, rlen[i]);
-    out[c] = min((m + 15) / 16 * 16, npad);
+    const float v = (i < M && j < r) ? R[(size_t)i * ldr + j] : 0.f;
+    const __nv_bfloat16 hv = __float2bfloat16_rn(v);
+    Rh[idx] = hv;
+    Rl[idx] = __float2bfloat16_rn(v - __bfloat162float(hv));
 }
 
 int num_sms(int dev) {
@@ -605,14 +719,24 @@ int num_sms(int dev) {
     return n > 0 ? n : 1;
 }
 
-size_t ps_smem_bytes(int npad, int stages) {
-    return 1024 + (size_t)stages * (kBM * 128 + (size_t)npad * 128) + sizeof(Smem);
+struct Rings {
+    int sx, sa, sb;
+};
+
+size_t ps_smem_bytes(Rings g) {
+    return 1024 + (size_t)g.sx * kXStageBytes + (size_t)g.sa * kAStageBytes + (size_t)g.sb * kBStageBytes +
+           sizeof(Ctl);
 }
 
-int ps_stages(int npad) {
-    for (int s = kStagesMax; s >= 2; --s)
-        if (ps_smem_bytes(npad, s) <= 227 * 1024) return s;
-    return 2;
+// deepest X staging ring that fits next to two A stages and two or more B stages
+Rings ps_rings() {
+    const size_t cap = 227 * 1024;
+    for (int sx = kMaxSX; sx >= 2; --sx)
+        for (int sb = kMaxSB; sb >= 2; --sb) {
+            Rings g{sx, kMaxSA, sb};
+            if (ps_smem_bytes(g) <= cap) return g;
+        }
+    return Rings{2, 2, 2};
 }
 
 }  // namespace
@@ -632,20 +756,27 @@ bool tc_available(int device) {
 }
 
 gs_status tc_prepare(gs_basis* h) {
-    if (h->r < 1 || h->r > 256) return GS_OK;  // no tensor-core similarity kernel for this basis
+    // the fused kernel keeps Y (r <= 256 columns) and S (M <= 256 columns) in TMEM
+    if (h->r < 1 || h->r > 256 || h->M > 256) return GS_OK;
     const int npad = (h->r + 15) / 16 * 16;
-    const int mpad = (h->M + kCwChunk - 1) / kCwChunk * kCwChunk;
-    if (cudaMalloc(&h->tc_Rpad, sizeof(float) * (size_t)mpad * npad) != cudaSuccess) return GS_ERR_NOMEM;
-    if (cudaMalloc(&h->tc_jlen16, sizeof(int) * (size_t)(mpad / kCwChunk)) != cudaSuccess) return GS_ERR_NOMEM;
-    k_pad_r<<<(unsigned)(((long long)mpad * npad + 255) / 256), 256>>>(h->R, h->M, h->r, h->ldr, h->tc_Rpad, mpad,
-                                                                       npad);
-    k_jlen16<<<(mpad / kCwChunk + 127) / 128, 128>>>(h->rlen, h->M, mpad / kCwChunk, npad, h->tc_jlen16);
+    const int mpad = (h->M + 15) / 16 * 16;
+    const size_t n = (size_t)mpad * npad;
+    if (cudaMalloc(&h->tc_Rh, sizeof(__nv_bfloat16) * n) != cudaSuccess) return GS_ERR_NOMEM;
+    if (cudaMalloc(&h->tc_Rl, sizeof(__nv_bfloat16) * n) != cudaSuccess) return GS_ERR_NOMEM;
+    k_split_r<<<(unsigned)((n + 255) / 256), 256>>>(h->R, h->M, h->r, h->ldr, (__nv_bfloat16*)h->tc_Rh,
+                                                    (__nv_bfloat16*)h->tc_Rl, mpad, npad);
     if (cudaGetLastError() != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) return GS_ERR_CUDA;
-    if (!make_tmap_f16(&h->tmap_q16, h->Q16, h->r, h->D, h->ldq16, npad)) return GS_ERR_CUDA;
+    if (!make_tmap_2d(&h->tmap_q16, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, h->Q16, h->r, h->D, h->ldq16, kBK, npad,
+                      CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_tmap_2d(&h->tmap_rh, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, h->tc_Rh, mpad, npad, npad, kBK, mpad,
+                      CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_tmap_2d(&h->tmap_rl, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, h->tc_Rl, mpad, npad, npad, kBK, mpad,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+        return GS_ERR_CUDA;
     h->tc_npad = npad;
     h->tc_mpad = mpad;
-    if (cudaFuncSetAttribute(k_ps_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)ps_smem_bytes(npad, ps_stages(npad))) != cudaSuccess)
+    if (cudaFuncSetAttribute(k_ps_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ps_smem_bytes(ps_rings())) !=
+        cudaSuccess)
         return GS_ERR_CUDA;
     // the fused kernel needs all of its threads resident in one CTA; otherwise the
     // basis simply has no tensor-core similarity path
@@ -658,19 +789,29 @@ gs_status tc_prepare(gs_basis* h) {
 cudaError_t launch_ps_tc(const gs_basis* h, const float* X, long long N, int ldx, int mode, float scale, float* Y,
                          int ldy, float* S, int lds, int* argmax, float* maxval, cudaStream_t s) {
     if (!h->has_tmap_q16) return cudaErrorNotSupported;
+    const long long tiles = (N + kBM - 1) / kBM;
+    const int grid = (int)std::min<long long>(num_sms(h->device), tiles);
+    // the X box must cover the largest tile of any CTA (CTAs differ by one row)
+    int box_rows = 1;
+    for (int cta : {0, grid - 1}) box_rows = std::max(box_rows, CtaRows(N, grid, cta).tsize);
+    CUtensorMap tmx;
+    if (!make_tmap_2d(&tmx, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, X, N, h->D, ldx, kBK, box_rows,
+                      CU_TENSOR_MAP_SWIZZLE_NONE))
+        return cudaErrorInvalidValue;
+    const Rings g = ps_rings();
     PsParams p;
-    p.X = X;
     p.N = N;
-    p.ldx = ldx;
     p.D = h->D;
     p.r = h->r;
     p.npad = h->tc_npad;
     p.M = h->M;
     p.mpad = h->tc_mpad;
     p.nkb = (h->D + kBK - 1) / kBK;
-    p.stages = ps_stages(p.npad);
-    p.Rpad = h->tc_Rpad;
-    p.jlen16 = h->tc_jlen16;
+    p.nkr = (h->tc_npad + kBK - 1) / kBK;
+    p.sx = g.sx;
+    p.sa = g.sa;
+    p.sb = g.sb;
+    p.box_rows = box_rows;
     p.cnorm = h->cnorm;
     p.mode = mode;
     p.scale = scale;
@@ -680,9 +821,7 @@ cudaError_t launch_ps_tc(const gs_basis* h, const float* X, long long N, int ldx
     p.lds = lds;
     p.argmax = argmax;
     p.maxval = maxval;
-    const long long tiles = (N + kBM - 1) / kBM;
-    const int grid = (int)std::min<long long>(num_sms(h->device), tiles);
-    k_ps_tc<<<grid, kThreads, ps_smem_bytes(p.npad, p.stages), s>>>(h->tmap_q16, p);
+    k_ps_tc<<<grid, kThreads, ps_smem_bytes(g), s>>>(tmx, h->tmap_q16, h->tmap_rh, h->tmap_rl, p);
     return cudaGetLastError();
 }
 
