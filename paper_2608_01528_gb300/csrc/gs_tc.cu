@@ -16,8 +16,8 @@
 //                      Y = Yh + Yl and R = Rh + Rl, S = Yh Rh + Yl Rh + Yh Rl
 //                      (relative error ~2^-16, fp32's exponent range), fp32
 //                      accumulator in TMEM columns [256, 512).  The epilogue
-//                      splits Y in place in TMEM (each 32-column fp32 chunk
-//                      becomes 16 columns of packed Yh and 16 of packed Yl), and
+//                      splits Y in place in TMEM (each 16-column fp32 chunk
+//                      becomes 8 columns of packed Yh and 8 of packed Yl), and
 //                      the MMA reads that A operand straight from TMEM; the Rh /
 //                      Rl tiles come through the same TMA ring as the Q tiles.
 //                      A single fp16/tf32 rounding would not do here: the
@@ -35,12 +35,13 @@
 //
 // Work split: one persistent CTA per SM; each CTA takes a contiguous, balanced
 // range of rows and cuts it into tiles of at most 128 rows, so every CTA moves
-// the same number of bytes.  Warp roles (352 threads):
+// the same number of bytes.  Warp roles (480 threads):
 //   warps 0-3    epilogue: warp w owns TMEM lanes 32w..32w+31 (rows of the tile)
 //   warp  4      TMA producer of the X tiles
 //   warp  5      TMEM allocator and MMA issuer (one elected lane)
 //   warp  6      TMA producer of the B operand tiles (Q per K-block, then Rh / Rl)
-//   warps 7-10   converters (fp32 -> fp16, row norms, range check)
+//   warps 7-14   converters (fp32 -> fp16, row norms, range check), two groups of
+//                four warps taking alternate K-blocks so two blocks convert at once
 // Every wait on an mbarrier is bounded (wall-clock limit): on expiry the CTA
 // records GS_DEV_ERR_TIMEOUT, raises a CTA-wide abort flag so the other roles
 // leave their loops, waits (bounded) for its own TMA copies and MMAs to land,
@@ -65,9 +66,11 @@ constexpr int kXWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kBWarp = 6;
 constexpr int kCvt0 = 7;
-constexpr int kCvtWarps = 4;
-constexpr int kThreads = (kCvt0 + kCvtWarps) * 32;  // 352
-constexpr int kCvtThreads = kCvtWarps * 32;          // 128
+constexpr int kCvtGroups = 2;        // converter groups take alternate K-blocks
+constexpr int kCvtGroupWarps = 4;
+constexpr int kCvtWarps = kCvtGroups * kCvtGroupWarps;
+constexpr int kThreads = (kCvt0 + kCvtWarps) * 32;  // 480
+constexpr int kCvtThreads = kCvtGroupWarps * 32;     // 128 per group
 constexpr int kCvtRowStep = kCvtThreads / 16;        // 8 rows per sweep of the 16 float4 columns
 constexpr int kCvtRows = kBM / kCvtRowStep;          // 16 rows per converter thread
 constexpr int kXStageBytes = kBM * kBK * 4;          // 32 KB fp32 staging tile
@@ -249,6 +252,12 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* v) {
         "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
         : "memory");
 }
+// Stores 8 consecutive 32-bit columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t* v) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(v[0]),
+                 "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+                 : "memory");
+}
 __device__ __forceinline__ void tmem_wait_st() {
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
@@ -329,7 +338,7 @@ struct Ctl {
     uint64_t y_full, ysplit_full, s_full, s_empty, gemm2_done;
     uint64_t xn_full[2], xn_empty[2];
     uint64_t mma_done;
-    float xn[2][kBM];
+    float xn[2][kCvtGroups][kBM];
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -354,10 +363,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < p.sx; ++s) {
             mbar_init(&c.x_full[s], 1);
-            mbar_init(&c.x_empty[s], kCvtWarps);
+            mbar_init(&c.x_empty[s], kCvtGroupWarps);
         }
         for (int s = 0; s < p.sa; ++s) {
-            mbar_init(&c.a_full[s], kCvtWarps);
+            mbar_init(&c.a_full[s], kCvtGroupWarps);
             mbar_init(&c.a_empty[s], 1);
         }
         for (int s = 0; s < p.sb; ++s) {
@@ -479,10 +488,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint64_t rl = sdesc_sw128(smem_u32(Bs + (size_t)sl * kBStageBytes));
 #pragma unroll
                     for (int k = 0; k < kBK / 16; ++k) {
-                        // r columns [64 kr + 16 k, +16): chunk of 32 = (4 kr + k) / 2, half = k & 1
+                        // r columns [64 kr + 16 k, +16) were split into TMEM columns
+                        // [16 kk, 16 kk + 8) (Yh) and [16 kk + 8, 16 kk + 16) (Yl), kk = 4 kr + k
                         const int kk = 4 * kr + k;
-                        const uint32_t a_hi = y_tmem + (uint32_t)(32 * (kk >> 1) + 8 * (kk & 1));
-                        const uint32_t a_lo = a_hi + 16;
+                        if (16 * kk >= p.npad) break;  // past r: no split columns there
+                        const uint32_t a_hi = y_tmem + (uint32_t)(16 * kk);
+                        const uint32_t a_lo = a_hi + 8;
                         mma_bf16_ts(s_tmem, a_hi, rh + (uint64_t)(2 * k), idesc2, (kr | k) != 0 ? 1u : 0u);
                         mma_bf16_ts(s_tmem, a_lo, rh + (uint64_t)(2 * k), idesc2, 1u);
                         mma_bf16_ts(s_tmem, a_hi, rl + (uint64_t)(2 * k), idesc2, 1u);
@@ -503,9 +514,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp >= kCvt0) {
         // ------------------------------------------------------------- converters
-        const int l = threadIdx.x - kCvt0 * 32;  // 0..127
+        const int g = (warp - kCvt0) / kCvtGroupWarps;           // group: K-blocks with it % 2 == g
+        const int l = threadIdx.x - (kCvt0 + g * kCvtGroupWarps) * 32;  // 0..127 within the group
         const int c4 = l & 15;                   // float4 column of the 64-wide K-block
         const int rbase = l >> 4;                // rows rbase + 8u, u < 16
+        const bool want_norm = p.mode == GS_SCORE_COSINE;
         float nrm[kCvtRows];
 #pragma unroll
         for (int u = 0; u < kCvtRows; ++u) nrm[u] = 0.f;
@@ -516,6 +529,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const TileRange tr = cr.tile(t);
             const int b = t & 1;
             for (int kb = 0; kb < p.nkb; ++kb, ++it) {
+                if ((it & 1) != g) continue;
                 const int sx = it % p.sx, sa = it % p.sa;
                 if (!mbar_wait_warp(&c.x_full[sx], (uint32_t)(it / p.sx) & 1u, abort_flag) ||
                     !mbar_wait_warp(&c.a_empty[sa], ((uint32_t)(it / p.sa) & 1u) ^ 1u, abort_flag)) {
@@ -529,7 +543,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int row = rbase + kCvtRowStep * u;
                     float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
                     if (row < tr.nrows) x = *reinterpret_cast<const float4*>(Xt + row * (kBK * 4) + c4 * 16);
-                    nrm[u] = fmaf(x.x, x.x, fmaf(x.y, x.y, fmaf(x.z, x.z, fmaf(x.w, x.w, nrm[u]))));
+                    if (want_norm) nrm[u] = fmaf(x.x, x.x, fmaf(x.y, x.y, fmaf(x.z, x.z, fmaf(x.w, x.w, nrm[u]))));
                     amax = fmaxf(amax, fmaxf(fmaxf(fabsf(x.x), fabsf(x.y)), fmaxf(fabsf(x.z), fabsf(x.w))));
                     const __half2 h0 = __floats2half2_rn(x.x, x.y);
                     const __half2 h1 = __floats2half2_rn(x.z, x.w);
@@ -547,7 +561,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             if (!ok) break;
-            // tile finished: ||x||^2 of each row -> shared, for cosine scores
+            // tile finished: this group's part of ||x||^2 of each row -> shared, for cosine scores
 #pragma unroll
             for (int u = 0; u < kCvtRows; ++u) {
                 float v = nrm[u];
@@ -560,7 +574,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!mbar_wait_warp(&c.xn_empty[b], ((uint32_t)(t >> 1) & 1u) ^ 1u, abort_flag)) break;
             if ((lane & 15) == 0) {
 #pragma unroll
-                for (int u = 0; u < kCvtRows; ++u) c.xn[b][rbase + kCvtRowStep * u] = nrm[u];
+                for (int u = 0; u < kCvtRows; ++u) c.xn[b][g][rbase + kCvtRowStep * u] = nrm[u];
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(&c.xn_full[b]);
@@ -581,38 +595,34 @@ __global__ void __launch_bounds__(kThreads, 1)
             const TileRange tr = cr.tile(t);
             const bool valid = i < tr.nrows;
             const long long row = tr.row0 + i;
-            // split Y in place: chunk of 32 fp32 columns -> 16 columns bf16(Y) + 16 columns bf16(Y - bf16(Y))
-            for (int jc = 0; jc < p.npad; jc += 32) {
-                float y[32];
-                tmem_ld32(ty + (uint32_t)jc, y);
-                // columns past npad were never written by GEMM1: make them exact zeros
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    if (jc + j >= p.npad) y[j] = 0.f;
+            // split Y in place: chunk of 16 fp32 columns -> 8 columns bf16(Y) + 8 columns bf16(Y - bf16(Y))
+            for (int jc = 0; jc < p.npad; jc += 16) {
+                float y[16];
+                tmem_ld16(ty + (uint32_t)jc, y);
                 if (p.Y && valid) {
                     float* dst = p.Y + (size_t)row * p.ldy + jc;
 #pragma unroll
-                    for (int j = 0; j < 32; ++j)
+                    for (int j = 0; j < 16; ++j)
                         if (jc + j < p.r) dst[j] = y[j];
                 }
-                uint32_t hi[16], lo[16];
+                uint32_t hi[8], lo[8];
 #pragma unroll
-                for (int j = 0; j < 16; ++j) {
+                for (int j = 0; j < 8; ++j) {
                     const float a = y[2 * j], bb = y[2 * j + 1];
                     const float ah = __bfloat162float(__float2bfloat16_rn(a));
                     const float bh = __bfloat162float(__float2bfloat16_rn(bb));
                     hi[j] = pack_bf16(ah, bh);
                     lo[j] = pack_bf16(a - ah, bb - bh);
                 }
-                tmem_st16(ty + (uint32_t)jc, hi);
-                tmem_st16(ty + (uint32_t)(jc + 16), lo);
+                tmem_st8(ty + (uint32_t)jc, hi);
+                tmem_st8(ty + (uint32_t)(jc + 8), lo);
             }
             tmem_wait_st();
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&c.ysplit_full);
             if (!mbar_wait_warp(&c.xn_full[b], (uint32_t)(t >> 1) & 1u, abort_flag)) break;
-            const float xnorm = sqrtf(c.xn[b][i]);
+            const float xnorm = sqrtf(c.xn[b][0][i] + c.xn[b][1][i]);
             __syncwarp();
             if (lane == 0) mbar_arrive(&c.xn_empty[b]);
             if (!mbar_wait_warp(&c.s_full, pt, abort_flag)) break;
