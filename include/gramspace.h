@@ -171,6 +171,30 @@ GS_API gs_status gs_attention_scores(const void* Yq, const void* Yk, int in_dtyp
                               unsigned flags, void* stream);
 
 /*
+ * Project + similarity that allocates nothing (the paper has no counterpart;
+ * this is a deployment variant).  For callers that cannot call cudaMalloc:
+ * code running under a CUDA graph capture that forbids allocation, plugins
+ * confined to a host framework's fixed device-memory budget, integrations whose
+ * own allocator owns all device memory.  No basis handle is needed: the caller
+ * passes the basis it holds, Q (r x D fp32, ld = D), R (M x r fp32, ld = r)
+ * and cnorm (M fp32, only read for GS_SCORE_COSINE), plus X (N x D fp32,
+ * ld = ldx) and receives argmax and/or maxval (N each; either may be NULL, not
+ * both).  Scores are computed like gs_project_similarity with GS_PATH_SIMT
+ * (fp32 CUDA cores, any value range).
+ * Scratch lives in a fixed 16 MiB device array inside the library (held by
+ * every GPU that loads it until exit), processed in chunks of rows; a problem
+ * with r + M + 1 > 4,194,304 is rejected with GS_ERR_SHAPE.  The first call on
+ * a device looks up that array's device address (cudaGetSymbolAddress) with
+ * the device current, so make that first call before any stream capture.  All
+ * calls on a device share the array: calls that overlap on the GPU race.
+ * Errors: GS_ERR_INVALID_ARG, GS_ERR_SHAPE, GS_ERR_CUDA, GS_ERR_UNSUPPORTED.
+ */
+GS_API gs_status gs_project_similarity_static(const float* Q, int r, int D, const float* R, int M,
+                                              const float* cnorm, const float* X, long long N, int ldx,
+                                              int mode, float scale, int* argmax, float* maxval,
+                                              void* stream);
+
+/*
  * Synchronises `stream` (NULL = the whole device) and returns the first error
  * the device recorded since the last call (GS_ERR_TIMEOUT, GS_ERR_RANGE), or
  * GS_ERR_CUDA if the stream itself failed; clears the recorded word.

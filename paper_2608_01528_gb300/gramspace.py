@@ -29,7 +29,7 @@ GS_BUILD_NORMALIZE_ROWS = 1
 # Every symbol include/gramspace.h declares (checked by the CPU tests).
 EXPORTS = ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_similarity",
            "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores", "gs_stream_status",
-           "gs_status_string", "gs_version")
+           "gs_status_string", "gs_version", "gs_project_similarity_static")
 
 
 class GramSpaceError(RuntimeError):
@@ -59,6 +59,8 @@ def load_library(path=LIB_PATH):
     L.gs_reconstruct.argtypes = [vp, vp, ip, i64, ip, vp, ip, u32, vp]
     L.gs_attention_scores.argtypes = [vp, vp, ip, ip, ip, ip, ip, ip, f32, ip, vp, u32, vp]
     L.gs_stream_status.argtypes = [vp]
+    L.gs_project_similarity_static.argtypes = [vp, ip, ip, vp, ip, vp, vp, i64, ip, ip, f32, vp, vp, vp]
+    L.gs_project_similarity_static.restype = ctypes.c_int
     L.gs_status_string.argtypes = [ip]
     L.gs_status_string.restype = ctypes.c_char_p
     L.gs_version.restype = ctypes.c_int
@@ -241,6 +243,30 @@ def attention_scores(Yq, Yk, scale, apply_softmax=True, path="auto", out=None, s
                                    1 if apply_softmax else 0, _ptr(A), PATHS[path], _stream(stream))
     _check(st, "gs_attention_scores")
     return A
+
+
+def project_similarity_static(Q, R, cnorm, X, mode="raw", scale=1.0, want_argmax=True, want_maxval=True,
+                              out=None, stream=None):
+    """Project + similarity from a caller-held basis without any device allocation by the
+    library; see gs_project_similarity_static.  Q: r x D, R: M x r, cnorm: M (fp32, CUDA)."""
+    N = X.shape[0]
+    r, D = Q.shape
+    M = R.shape[0]
+    out = dict(out or {})
+    if want_argmax and "argmax" not in out:
+        out["argmax"] = torch.empty(N, dtype=torch.int32, device=X.device)
+    if want_maxval and "maxval" not in out:
+        out["maxval"] = torch.empty(N, dtype=torch.float32, device=X.device)
+    for t in (Q, R):
+        if t.numel() and not t.is_contiguous():
+            raise ValueError("Q and R must be contiguous")
+    L = load_library()
+    with torch.cuda.device(X.device):
+        st = L.gs_project_similarity_static(_ptr(Q) if Q.numel() else None, r, D, _ptr(R) if R.numel() else None,
+                                            M, _ptr(cnorm), _ptr(X), N, _ld(X), MODES[mode], float(scale),
+                                            _ptr(out.get("argmax")), _ptr(out.get("maxval")), _stream(stream))
+    _check(st, "gs_project_similarity_static")
+    return out
 
 
 def stream_status(stream=None):
