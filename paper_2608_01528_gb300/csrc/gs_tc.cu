@@ -338,7 +338,7 @@ struct Ctl {
     uint64_t y_full, ysplit_full, s_full, s_empty, gemm2_done;
     uint64_t xn_full[2], xn_empty[2];
     uint64_t mma_done;
-    float xn[2][kCvtGroups][kBM];
+    float xn[2][kBM];  // ||x||^2 per row, both converter groups add into it
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -384,6 +384,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         mbar_init(&c.mma_done, 1);
         c.abort_flag = 0;
+        for (int j = 0; j < 2 * kBM; ++j) (&c.xn[0][0])[j] = 0.f;
         fence_barrier_init();
     }
     if (warp == kMmaWarp) {
@@ -561,7 +562,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             if (!ok) break;
-            // tile finished: this group's part of ||x||^2 of each row -> shared, for cosine scores
+            // tile finished: this group's part of ||x||^2 of each row is added into shared memory
 #pragma unroll
             for (int u = 0; u < kCvtRows; ++u) {
                 float v = nrm[u];
@@ -572,9 +573,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 nrm[u] = v;
             }
             if (!mbar_wait_warp(&c.xn_empty[b], ((uint32_t)(t >> 1) & 1u) ^ 1u, abort_flag)) break;
-            if ((lane & 15) == 0) {
+            if (want_norm && (lane & 15) == 0) {
 #pragma unroll
-                for (int u = 0; u < kCvtRows; ++u) c.xn[b][g][rbase + kCvtRowStep * u] = nrm[u];
+                for (int u = 0; u < kCvtRows; ++u) atomicAdd(&c.xn[b][rbase + kCvtRowStep * u], nrm[u]);
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(&c.xn_full[b]);
@@ -622,7 +623,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(&c.ysplit_full);
             if (!mbar_wait_warp(&c.xn_full[b], (uint32_t)(t >> 1) & 1u, abort_flag)) break;
-            const float xnorm = sqrtf(c.xn[b][0][i] + c.xn[b][1][i]);
+            const float xnorm = sqrtf(c.xn[b][i]);
+            c.xn[b][i] = 0.f;  // ready for the tile after next (both groups add into it)
             __syncwarp();
             if (lane == 0) mbar_arrive(&c.xn_empty[b]);
             if (!mbar_wait_warp(&c.s_full, pt, abort_flag)) break;
