@@ -365,7 +365,8 @@ def side_rows(gs, dev):
     out["build_rankdef_ms"] = round(1e3 * (time.perf_counter() - t0), 2)
     out["build_rankdef_r"] = b4.r
     # reconstruct 16,384 x 922 -> 16,384 x 10,000
-    T = torch.randn(16384, b4.r, device=dev)
+    r4 = (b4.r + 3) // 4 * 4  # 16-byte rows, as the tensor-core path needs
+    T = torch.randn(16384, r4, device=dev)[:, :b4.r]
     Xh = torch.empty(16384, 10000, device=dev)
     ms = timeit(lambda: gs.reconstruct(b4, T, out=Xh))
     out["reconstruct_rankdef_ms"] = round(ms, 4)

@@ -55,10 +55,71 @@ void free_basis(gs_basis* h) {
     cudaFree(h->scratch);
     cudaFree(h->tc_Rh);
     cudaFree(h->tc_Rl);
+    cudaFree(h->tc_Rth);
+    cudaFree(h->tc_Rtl);
+    cudaFree(h->tc_Qh);
+    cudaFree(h->tc_Ql);
     delete h;
 }
 
 constexpr long long kMaxGemmRows = 65535LL * 64;  // grid.y limit of the SIMT GEMM
+
+// Project + similarity on the tensor core for bases the fused kernel cannot hold
+// in TMEM (r > 256 or M > 256): Y = X Q^T (fp16 operands, fp32 accumulation)
+// into the handle's scratch, then S = Y R^T with Y and R split into bf16 hi / lo,
+// then the row reductions.  Rows are processed in chunks that fit the scratch.
+gs_status ps_two_gemm(const gs_basis* h, const float* X, long long N, int ldx, int mode, float scale, float* Y,
+                      int ldy, float* S, int lds, int* argmax, float* maxval, cudaStream_t s) {
+    const int r = h->r, M = h->M, D = h->D;
+    const int r4 = (r + 3) / 4 * 4;  // padded ld of the Y scratch (16-byte rows for TMA)
+    const long long per_row = (long long)r4 + M + 1;
+    long long chunk = std::min(h->scratch_floats / per_row, kMaxGemmRows);
+    if (chunk < 1) return GS_ERR_SHAPE;
+    const bool need_s = S || argmax || maxval;
+    for (long long c0 = 0; c0 < N; c0 += chunk) {
+        const long long nc = std::min(chunk, N - c0);
+        float* Ybuf = h->scratch;
+        float* xn = Ybuf + nc * r4;
+        float* Sscr = xn + nc;
+        gs::GemmTcArgs g1{};
+        g1.A = X + c0 * ldx; g1.lda = ldx; g1.m = nc; g1.K = D;
+        g1.split = D < gs::kMinF16Depth;  // short rows: bf16 hi / lo split instead of one fp16 rounding
+        g1.B0 = g1.split ? h->tc_Qh : (const void*)h->Q16;
+        g1.B1 = g1.split ? h->tc_Ql : nullptr;
+        g1.ldb = h->ldq16; g1.n = r;
+        g1.C = Ybuf; g1.ldc = r4; g1.c_bf16 = false; g1.alpha = 1.f;
+        cudaError_t e = gs::launch_gemm_tc(g1, h->device, s);
+        if (e != cudaSuccess) return from_cuda(e);
+        if (Y) {
+            e = cudaMemcpy2DAsync(Y + c0 * ldy, sizeof(float) * ldy, Ybuf, sizeof(float) * r4, sizeof(float) * r, nc,
+                                  cudaMemcpyDeviceToDevice, s);
+            if (e != cudaSuccess) return from_cuda(e);
+        }
+        if (!need_s) continue;
+        if (mode == GS_SCORE_COSINE) {
+            e = gs::launch_rownorm(X + c0 * ldx, nc, ldx, D, xn, s);
+            if (e != cudaSuccess) return from_cuda(e);
+        }
+        float* Sbuf = S ? S + c0 * lds : Sscr;
+        const long long ldsb = S ? lds : M;
+        gs::GemmTcArgs g2{};
+        g2.A = Ybuf; g2.lda = r4; g2.m = nc; g2.K = r; g2.split = true;
+        g2.B0 = h->tc_Rh; g2.B1 = h->tc_Rl; g2.ldb = h->tc_npad; g2.n = M;
+        g2.C = Sbuf; g2.ldc = ldsb; g2.c_bf16 = false; g2.alpha = scale;
+        if (mode == GS_SCORE_COSINE) { g2.rownorm = xn; g2.colnorm = h->cnorm; }
+        e = gs::launch_gemm_tc(g2, h->device, s);
+        if (e != cudaSuccess) return from_cuda(e);
+        if (argmax || maxval || mode == GS_SCORE_SOFTMAX) {
+            e = gs::launch_row_finish(Sbuf, nc, M, (int)ldsb, mode == GS_SCORE_SOFTMAX, argmax ? argmax + c0 : nullptr,
+                                      maxval ? maxval + c0 : nullptr, s);
+            if (e != cudaSuccess) return from_cuda(e);
+        }
+    }
+    return GS_OK;
+}
+
+// Whether a GEMM of m rows, n columns and depth k is worth the tensor-core kernel.
+bool big_gemm(long long m, long long n, long long k) { return m >= 512 && 2.0 * m * n * k >= 2e9; }
 
 }  // namespace
 
@@ -140,11 +201,14 @@ gs_status gs_project_similarity(const gs_basis* h, const float* X, long long N, 
     cudaStream_t s = (cudaStream_t)stream;
     const int r = h->r, M = h->M, D = h->D;
 
-    const bool tc_shape = r >= 1 && r <= 256 && h->has_tmap_q16 && (uintptr_t)X % 16 == 0 && ldx % 4 == 0;
+    const bool aligned = (uintptr_t)X % 16 == 0 && ldx % 4 == 0;
+    const bool fused = h->has_tmap_q16 && aligned && D >= gs::kMinF16Depth;  // r <= 256, M <= 256
+    const bool two_gemm = h->has_split && aligned;      // any r >= 1
     const bool big = (double)N * D >= (double)(1 << 24);
-    if (flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && big && tc_shape)) {
-        if (!tc_shape) return (uintptr_t)X % 16 || ldx % 4 ? GS_ERR_ALIGNMENT : GS_ERR_UNSUPPORTED;
-        return from_cuda(gs::launch_ps_tc(h, X, N, ldx, mode, scale, Y, ldy, S, lds, argmax, maxval, s));
+    if (flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && big && (fused || two_gemm))) {
+        if (fused) return from_cuda(gs::launch_ps_tc(h, X, N, ldx, mode, scale, Y, ldy, S, lds, argmax, maxval, s));
+        if (two_gemm) return ps_two_gemm(h, X, N, ldx, mode, scale, Y, ldy, S, lds, argmax, maxval, s);
+        return !aligned ? GS_ERR_ALIGNMENT : GS_ERR_UNSUPPORTED;
     }
     if (r <= 32) {
         return from_cuda(gs::launch_ps_warp(X, N, ldx, D, h->Q, r, h->R, h->ldr, M, h->cnorm, mode, scale,
@@ -199,10 +263,19 @@ gs_status gs_prob_vectorize(const gs_basis* h, const float* P, long long N, int 
     if (N < 0 || ldp < h->M || ldv < h->r) return GS_ERR_SHAPE;
     if (N == 0 || h->r == 0) return GS_OK;
     if (!P || !V) return GS_ERR_INVALID_ARG;
-    if (flags == GS_PATH_TENSOR) return GS_ERR_UNSUPPORTED;
     DeviceGuard g(h->device);
     if (!g.ok) return GS_ERR_CUDA;
     cudaStream_t s = (cudaStream_t)stream;
+    const bool tc_ok = h->has_split && (uintptr_t)P % 16 == 0 && ldp % 4 == 0;
+    if (flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && tc_ok && big_gemm(N, h->r, h->M))) {
+        if (!tc_ok) return h->has_split ? GS_ERR_ALIGNMENT : GS_ERR_UNSUPPORTED;
+        // V = P R with P and R^T split into bf16 hi / lo (fp32-level accuracy)
+        gs::GemmTcArgs a{};
+        a.A = P; a.lda = ldp; a.m = N; a.K = h->M; a.split = true;
+        a.B0 = h->tc_Rth; a.B1 = h->tc_Rtl; a.ldb = h->tc_mpad; a.n = h->r;
+        a.C = V; a.ldc = ldv; a.c_bf16 = v_dtype == GS_BF16; a.alpha = 1.f;
+        return from_cuda(gs::launch_gemm_tc(a, h->device, s));
+    }
     for (long long c0 = 0; c0 < N; c0 += kMaxGemmRows) {
         const long long nc = std::min(kMaxGemmRows, N - c0);
         gs::GemmArgs a{};
@@ -224,10 +297,19 @@ gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, long lon
     if (N < 0 || ldt < h->r || ldxh < h->D) return GS_ERR_SHAPE;
     if (N == 0) return GS_OK;
     if (!T || !Xhat) return GS_ERR_INVALID_ARG;
-    if (flags == GS_PATH_TENSOR) return GS_ERR_UNSUPPORTED;
     DeviceGuard g(h->device);
     if (!g.ok) return GS_ERR_CUDA;
     cudaStream_t s = (cudaStream_t)stream;
+    const bool tc_ok = h->has_split && h->r >= 1 && t_dtype == GS_F32 && (uintptr_t)T % 16 == 0 && ldt % 4 == 0;
+    if (flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && tc_ok && big_gemm(N, h->D, h->r))) {
+        if (!tc_ok) return t_dtype != GS_F32 || !h->has_split ? GS_ERR_UNSUPPORTED : GS_ERR_ALIGNMENT;
+        // Xhat = T Q: T rounded to fp16 on the fly, the basis' dithered fp16 Q^T, fp32 accumulation
+        gs::GemmTcArgs a{};
+        a.A = (const float*)T; a.lda = ldt; a.m = N; a.K = h->r; a.split = false;
+        a.B0 = h->Q16t; a.ldb = h->ldr16; a.n = h->D;
+        a.C = Xhat; a.ldc = ldxh; a.c_bf16 = false; a.alpha = 1.f;
+        return from_cuda(gs::launch_gemm_tc(a, h->device, s));
+    }
     for (long long c0 = 0; c0 < N; c0 += kMaxGemmRows) {
         const long long nc = std::min(kMaxGemmRows, N - c0);
         gs::GemmArgs a{};
@@ -274,7 +356,7 @@ gs_status gs_attention_scores(const void* Yq, const void* Yk, int in_dtype, int 
 gs_status gs_stream_status(void* stream) {
     cudaError_t e = stream ? cudaStreamSynchronize((cudaStream_t)stream) : cudaDeviceSynchronize();
     if (e != cudaSuccess) return GS_ERR_CUDA;
-    const unsigned w = gs::take_device_error_build() | gs::take_device_error_tc();
+    const unsigned w = gs::take_device_error_build() | gs::take_device_error_tc() | gs::take_device_error_gemm();
     if (w & GS_DEV_ERR_TIMEOUT) return GS_ERR_TIMEOUT;
     if (w & GS_DEV_ERR_RANGE) return GS_ERR_RANGE;
     return GS_OK;

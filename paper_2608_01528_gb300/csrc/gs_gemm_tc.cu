@@ -1,0 +1,414 @@
+// gs_gemm_tc.cu -- general tcgen05 GEMM for the matrix-space operators:
+//
+//     C = alpha * A B^T            (optionally divided by rownorm[i] * colnorm[j])
+//
+//   A  fp32, m x K row-major, streamed by TMA into an fp32 staging ring and
+//      converted on the fly by two groups of converter warps into the
+//      128-byte-swizzled K-major operand layout:
+//        kAF16     one fp16 copy (round to nearest)     D  = A16 B0^T
+//        kABF16X2  hi = bf16(A), lo = bf16(A - hi)      D  = Ah B0^T + Al B0^T + Ah B1^T
+//      (the split keeps ~16 significant bits and fp32's exponent range, for
+//      products whose terms do not average out, e.g. with the dominant diagonal of R)
+//   B0, B1  16-bit (fp16 with kAF16, bf16 with kABF16X2), n x K row-major (K-major),
+//      by TMA; these are the basis' operand copies, L2-resident.
+//   C  fp32 or bf16, m x n, leading dimension ldc.
+//
+// Uses (paper Sec. 3.1 / 3.3): reconstruction Xhat = T Q (B0 = fp16 Q^T), the
+// projection Y = X Q^T for bases too wide for the fused kernel (B0 = fp16 Q),
+// scores S = Y R^T (split, B0 / B1 = bf16 hi / lo of R) and probability
+// vectorization V = P R (split, B0 / B1 = bf16 hi / lo of R^T).
+//
+// Tiles are 128 x nt (nt <= 256) with the fp32 accumulator double-buffered in
+// TMEM (2 x 256 columns); one persistent CTA per SM walks the tiles with the n
+// index fastest, so CTAs running at the same time share A rows in L2.
+// Warp roles (480 threads): 0-3 epilogue (warp w owns TMEM lanes 32w..32w+31),
+// 4 TMA producer of A, 5 TMEM allocator + MMA issuer, 6 TMA producer of B,
+// 7-14 converters in two groups taking alternate K-blocks.  Every mbarrier wait
+// is bounded (see gs_tc_ptx.cuh); on expiry the CTA records GS_DEV_ERR_TIMEOUT,
+// unwinds, waits for its own copies and MMAs, frees TMEM and returns.
+
+#include <algorithm>
+
+#include "gs_internal.h"
+#include "gs_tc_ptx.cuh"
+
+namespace gs {
+namespace {
+
+using namespace ptx;
+
+__device__ unsigned g_err_gemm = 0;
+
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+constexpr int kEpiWarps = 4;
+constexpr int kAWarp = 4;
+constexpr int kMmaWarp = 5;
+constexpr int kBWarp = 6;
+constexpr int kCvt0 = 7;
+constexpr int kCvtGroups = 2;
+constexpr int kCvtGroupWarps = 4;
+constexpr int kCvtWarps = kCvtGroups * kCvtGroupWarps;
+constexpr int kThreads = (kCvt0 + kCvtWarps) * 32;  // 480
+constexpr int kCvtRowStep = kCvtGroupWarps * 32 / 16;  // 8
+constexpr int kCvtRows = kBM / kCvtRowStep;            // 16
+constexpr int kXStageBytes = kBM * kBK * 4;            // 32 KB
+constexpr int kAPartBytes = kBM * kBK * 2;             // 16 KB
+constexpr int kBStageBytes = 256 * kBK * 2;            // 32 KB
+constexpr int kMaxSX = 4, kMaxSA = 4, kMaxSB = 4;
+constexpr int kTmemCols = 512;
+
+enum { kAF16 = 0, kABF16X2 = 1 };
+
+struct GemmParams {
+    long long m;
+    int n, K, nkb, nt, tiles_n;
+    long long tiles;
+    int amode, nb, parts;   // nb: B matrices per K-block; parts: A operand tiles per K-block
+    int sx, sa, sb;
+    void* C;
+    long long ldc;
+    int c_bf16, c_vec;      // c_vec: 16-byte aligned rows, vector stores allowed
+    float alpha;
+    const float* rownorm;
+    const float* colnorm;
+};
+
+struct Ctl {
+    uint64_t x_full[kMaxSX], x_empty[kMaxSX];
+    uint64_t a_full[kMaxSA], a_empty[kMaxSA];
+    uint64_t b_full[kMaxSB], b_empty[kMaxSB];
+    uint64_t d_full[2], d_empty[2];
+    uint64_t mma_done;
+    uint32_t tmem_base;
+    int abort_flag;
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_gemm_tc(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b0,
+              const __grid_constant__ CUtensorMap tmap_b1, const GemmParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+    uint8_t* Xs = base;
+    uint8_t* As = Xs + (size_t)p.sx * kXStageBytes;
+    uint8_t* Bs = As + (size_t)p.sa * p.parts * kAPartBytes;
+    Ctl& c = *reinterpret_cast<Ctl*>(Bs + (size_t)p.sb * kBStageBytes);
+    volatile int* abort_flag = &c.abort_flag;
+    unsigned* err = &g_err_gemm;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // this CTA's tiles: blockIdx.x, blockIdx.x + gridDim.x, ...
+    const int ntiles = p.tiles > blockIdx.x ? (int)((p.tiles - 1 - blockIdx.x) / gridDim.x + 1) : 0;
+    const int total_it = ntiles * p.nkb;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < p.sx; ++s) {
+            mbar_init(&c.x_full[s], 1);
+            mbar_init(&c.x_empty[s], kCvtGroupWarps);
+        }
+        for (int s = 0; s < p.sa; ++s) {
+            mbar_init(&c.a_full[s], kCvtGroupWarps);
+            mbar_init(&c.a_empty[s], 1);
+        }
+        for (int s = 0; s < p.sb; ++s) {
+            mbar_init(&c.b_full[s], 1);
+            mbar_init(&c.b_empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&c.d_full[b], 1);
+            mbar_init(&c.d_empty[b], kEpiWarps);
+        }
+        mbar_init(&c.mma_done, 1);
+        c.abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == kMmaWarp) {
+        tmem_alloc(&c.tmem_base, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = c.tmem_base;
+
+    auto tile_mn = [&](int lt, long long& tm, int& tn) {
+        const long long tg = blockIdx.x + (long long)lt * gridDim.x;
+        tm = tg / p.tiles_n;
+        tn = (int)(tg % p.tiles_n);
+    };
+
+    if (warp == kAWarp) {
+        // ------------------------------------------------------------- A tiles (fp32) via TMA
+        if (lane == 0) {
+            const uint64_t pol = l2_policy_evict_first();
+            int it = 0;
+            for (; it < total_it; ++it) {
+                const int s = it % p.sx;
+                if (!mbar_wait(&c.x_empty[s], ((uint32_t)(it / p.sx) & 1u) ^ 1u, abort_flag, err)) break;
+                long long tm;
+                int tn;
+                tile_mn(it / p.nkb, tm, tn);
+                mbar_arrive_expect_tx(&c.x_full[s], kXStageBytes);
+                tma_load_2d(Xs + (size_t)s * kXStageBytes, &tmap_a, &c.x_full[s], (it % p.nkb) * kBK,
+                            (int)(tm * kBM), pol);
+            }
+            for (int j = std::max(0, it - p.sx); j < it; ++j) mbar_drain(&c.x_full[j % p.sx], (uint32_t)(j / p.sx) & 1u, err);
+        }
+    } else if (warp == kBWarp) {
+        // ------------------------------------------------------------- B tiles via TMA (nb per K-block)
+        if (lane == 0) {
+            const uint64_t pol = l2_policy_evict_last();
+            const uint32_t bytes = (uint32_t)p.nt * kBK * 2;
+            const int total = total_it * p.nb;
+            int ib = 0;
+            for (; ib < total; ++ib) {
+                const int s = ib % p.sb;
+                if (!mbar_wait(&c.b_empty[s], ((uint32_t)(ib / p.sb) & 1u) ^ 1u, abort_flag, err)) break;
+                const int it = ib / p.nb, which = ib % p.nb;
+                long long tm;
+                int tn;
+                tile_mn(it / p.nkb, tm, tn);
+                mbar_arrive_expect_tx(&c.b_full[s], bytes);
+                tma_load_2d(Bs + (size_t)s * kBStageBytes, which ? &tmap_b1 : &tmap_b0, &c.b_full[s],
+                            (it % p.nkb) * kBK, tn * p.nt, pol);
+            }
+            for (int j = std::max(0, ib - p.sb); j < ib; ++j) mbar_drain(&c.b_full[j % p.sb], (uint32_t)(j / p.sb) & 1u, err);
+        }
+    } else if (warp == kMmaWarp) {
+        // ------------------------------------------------------------- MMA issue
+        if (lane == 0) {
+            const uint32_t idesc = p.amode == kAF16 ? idesc_f16_f32(p.nt) : idesc_bf16_f32(p.nt);
+            int it = 0, ib = 0;
+            bool ok = true;
+            for (int lt = 0; lt < ntiles && ok; ++lt) {
+                const int buf = lt & 1;
+                if (!mbar_wait(&c.d_empty[buf], ((uint32_t)(lt >> 1) & 1u) ^ 1u, abort_flag, err)) break;
+                tc_fence_after();
+                const uint32_t d_tmem = tmem + (uint32_t)(buf * 256);
+                for (int kb = 0; kb < p.nkb; ++kb, ++it) {
+                    const int sa = it % p.sa;
+                    if (!mbar_wait(&c.a_full[sa], (uint32_t)(it / p.sa) & 1u, abort_flag, err)) {
+                        ok = false;
+                        break;
+                    }
+                    int sb[2];
+                    for (int w = 0; w < p.nb; ++w, ++ib) {
+                        sb[w] = ib % p.sb;
+                        if (!mbar_wait(&c.b_full[sb[w]], (uint32_t)(ib / p.sb) & 1u, abort_flag, err)) ok = false;
+                    }
+                    if (!ok) break;
+                    tc_fence_after();
+                    const uint8_t* At = As + (size_t)sa * p.parts * kAPartBytes;
+                    const uint64_t ah = sdesc_sw128(smem_u32(At));
+                    const uint64_t b0 = sdesc_sw128(smem_u32(Bs + (size_t)sb[0] * kBStageBytes));
+                    if (p.amode == kAF16) {
+#pragma unroll
+                        for (int k = 0; k < kBK / 16; ++k)
+                            mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
+                                       (kb | k) != 0 ? 1u : 0u);
+                    } else {
+                        const uint64_t al = sdesc_sw128(smem_u32(At + kAPartBytes));
+                        const uint64_t b1 = sdesc_sw128(smem_u32(Bs + (size_t)sb[1] * kBStageBytes));
+#pragma unroll
+                        for (int k = 0; k < kBK / 16; ++k) {
+                            mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
+                                       (kb | k) != 0 ? 1u : 0u);
+                            mma_f16_ss(d_tmem, al + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc, 1u);
+                            mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b1 + (uint64_t)(2 * k), idesc, 1u);
+                        }
+                    }
+                    mma_commit(&c.a_empty[sa]);
+                    for (int w = 0; w < p.nb; ++w) mma_commit(&c.b_empty[sb[w]]);
+                }
+                if (ok) mma_commit(&c.d_full[buf]);
+            }
+            mma_commit(&c.mma_done);
+            mbar_drain(&c.mma_done, 0, err);
+        }
+    } else if (warp >= kCvt0) {
+        // ------------------------------------------------------------- converters
+        const int g = (warp - kCvt0) / kCvtGroupWarps;
+        const int l = threadIdx.x - (kCvt0 + g * kCvtGroupWarps) * 32;  // 0..127
+        const int c4 = l & 15, rbase = l >> 4;
+        float amax = 0.f;
+        for (int it = g; it < total_it; it += kCvtGroups) {
+            const int sx = it % p.sx, sa = it % p.sa;
+            if (!mbar_wait_warp(&c.x_full[sx], (uint32_t)(it / p.sx) & 1u, abort_flag, err) ||
+                !mbar_wait_warp(&c.a_empty[sa], ((uint32_t)(it / p.sa) & 1u) ^ 1u, abort_flag, err))
+                break;
+            const uint8_t* Xt = Xs + (size_t)sx * kXStageBytes;
+            uint8_t* At = As + (size_t)sa * p.parts * kAPartBytes;
+#pragma unroll 4
+            for (int u = 0; u < kCvtRows; ++u) {
+                const int row = rbase + kCvtRowStep * u;
+                const float4 x = *reinterpret_cast<const float4*>(Xt + row * (kBK * 4) + c4 * 16);
+                const int off = row * 128 + (((c4 >> 1) ^ (row & 7)) * 16) + (c4 & 1) * 8;
+                uint2 hi;
+                if (p.amode == kAF16) {
+                    amax = fmaxf(amax, fmaxf(fmaxf(fabsf(x.x), fabsf(x.y)), fmaxf(fabsf(x.z), fabsf(x.w))));
+                    const __half2 h0 = __floats2half2_rn(x.x, x.y), h1 = __floats2half2_rn(x.z, x.w);
+                    hi.x = *reinterpret_cast<const uint32_t*>(&h0);
+                    hi.y = *reinterpret_cast<const uint32_t*>(&h1);
+                } else {
+                    const __nv_bfloat162 b0 = __floats2bfloat162_rn(x.x, x.y), b1 = __floats2bfloat162_rn(x.z, x.w);
+                    hi.x = *reinterpret_cast<const uint32_t*>(&b0);
+                    hi.y = *reinterpret_cast<const uint32_t*>(&b1);
+                    const float2 f0 = __bfloat1622float2(b0), f1 = __bfloat1622float2(b1);
+                    uint2 lo;
+                    lo.x = pack_bf16(x.x - f0.x, x.y - f0.y);
+                    lo.y = pack_bf16(x.z - f1.x, x.w - f1.y);
+                    *reinterpret_cast<uint2*>(At + kAPartBytes + off) = lo;
+                }
+                *reinterpret_cast<uint2*>(At + off) = hi;
+            }
+            fence_proxy_async();
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(&c.a_full[sa]);
+                mbar_arrive(&c.x_empty[sx]);
+            }
+        }
+        if (amax > 65504.f) atomicOr(err, GS_DEV_ERR_RANGE);
+    } else {
+        // ------------------------------------------------------------- epilogue (warps 0-3)
+        const int i = threadIdx.x;
+        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        for (int lt = 0; lt < ntiles; ++lt) {
+            const int buf = lt & 1;
+            if (!mbar_wait_warp(&c.d_full[buf], (uint32_t)(lt >> 1) & 1u, abort_flag, err)) break;
+            tc_fence_after();
+            long long tm;
+            int tn;
+            tile_mn(lt, tm, tn);
+            const long long row = tm * kBM + i;
+            const bool valid = row < p.m;
+            const float rn = (valid && p.rownorm) ? p.rownorm[row] : 1.f;
+            const uint32_t tb = tmem + lane_base + (uint32_t)(buf * 256);
+            for (int jc = 0; jc < p.nt; jc += 16) {
+                float v[16];
+                tmem_ld16(tb + (uint32_t)jc, v);
+                const int col0 = tn * p.nt + jc;
+                if (!valid || col0 >= p.n) continue;
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                    float g = p.alpha * v[j];
+                    if (p.colnorm) {
+                        const int col = col0 + j;
+                        const float den = col < p.n ? rn * p.colnorm[col] : 0.f;
+                        g = den > 0.f ? g / den : 0.f;
+                    }
+                    v[j] = g;
+                }
+                if (p.c_bf16) {
+                    __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(p.C) + (size_t)row * p.ldc + col0;
+                    if (p.c_vec && col0 + 16 <= p.n) {
+                        uint4 w0, w1;
+                        w0.x = pack_bf16(v[0], v[1]); w0.y = pack_bf16(v[2], v[3]);
+                        w0.z = pack_bf16(v[4], v[5]); w0.w = pack_bf16(v[6], v[7]);
+                        w1.x = pack_bf16(v[8], v[9]); w1.y = pack_bf16(v[10], v[11]);
+                        w1.z = pack_bf16(v[12], v[13]); w1.w = pack_bf16(v[14], v[15]);
+                        reinterpret_cast<uint4*>(dst)[0] = w0;
+                        reinterpret_cast<uint4*>(dst)[1] = w1;
+                    } else {
+                        for (int j = 0; j < 16 && col0 + j < p.n; ++j) dst[j] = __float2bfloat16_rn(v[j]);
+                    }
+                } else {
+                    float* dst = reinterpret_cast<float*>(p.C) + (size_t)row * p.ldc + col0;
+                    if (p.c_vec && col0 + 16 <= p.n) {
+#pragma unroll
+                        for (int j = 0; j < 16; j += 4)
+                            __stcs(reinterpret_cast<float4*>(dst + j), make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]));
+                    } else {
+                        for (int j = 0; j < 16 && col0 + j < p.n; ++j) dst[j] = v[j];
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&c.d_empty[buf]);
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == kMmaWarp) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+size_t gemm_smem_bytes(int sx, int sa, int parts, int sb) {
+    return 1024 + (size_t)sx * kXStageBytes + (size_t)sa * parts * kAPartBytes + (size_t)sb * kBStageBytes +
+           sizeof(Ctl);
+}
+
+bool g_attr_set[64];
+
+}  // namespace
+
+unsigned take_device_error_gemm() {
+    unsigned v = 0, z = 0;
+    cudaMemcpyFromSymbol(&v, g_err_gemm, sizeof(v));
+    if (v) cudaMemcpyToSymbol(g_err_gemm, &z, sizeof(z));
+    return v;
+}
+
+cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
+    if (a.m <= 0 || a.n <= 0) return cudaSuccess;
+    GemmParams p;
+    p.m = a.m;
+    p.n = a.n;
+    p.K = a.K;
+    p.nkb = (a.K + kBK - 1) / kBK;
+    p.nt = a.n >= 256 ? 256 : (a.n + 15) / 16 * 16;
+    p.tiles_n = (a.n + p.nt - 1) / p.nt;
+    p.tiles = ((a.m + kBM - 1) / kBM) * (long long)p.tiles_n;
+    p.amode = a.split ? kABF16X2 : kAF16;
+    p.nb = a.split ? 2 : 1;
+    p.parts = a.split ? 2 : 1;
+    // deepest staging that fits: two A stages, B stages for at least one K-block (+1)
+    const size_t cap = 227 * 1024;
+    p.sa = 2;
+    p.sx = 2;
+    p.sb = 2 * p.nb;
+    for (int sx = kMaxSX; sx >= 2; --sx) {
+        bool done = false;
+        for (int sb = kMaxSB; sb >= p.nb + 1; --sb)
+            if (gemm_smem_bytes(sx, p.sa, p.parts, sb) <= cap) {
+                p.sx = sx;
+                p.sb = sb;
+                done = true;
+                break;
+            }
+        if (done) break;
+    }
+    if (gemm_smem_bytes(p.sx, p.sa, p.parts, p.sb) > cap) return cudaErrorInvalidConfiguration;
+    p.C = a.C;
+    p.ldc = a.ldc;
+    p.c_bf16 = a.c_bf16 ? 1 : 0;
+    p.c_vec = ((uintptr_t)a.C % 16 == 0) && (a.ldc % (a.c_bf16 ? 8 : 4) == 0);
+    p.alpha = a.alpha;
+    p.rownorm = a.rownorm;
+    p.colnorm = a.colnorm;
+    CUtensorMap ta, tb0, tb1;
+    const CUtensorMapDataType bt = a.split ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
+    if (!make_tmap_2d(&ta, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, a.A, a.m, a.K, a.lda, kBK, kBM,
+                      CU_TENSOR_MAP_SWIZZLE_NONE) ||
+        !make_tmap_2d(&tb0, bt, 2, a.B0, a.n, a.K, a.ldb, kBK, p.nt, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_tmap_2d(&tb1, bt, 2, a.split ? a.B1 : a.B0, a.n, a.K, a.ldb, kBK, p.nt, CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    const size_t smem = gemm_smem_bytes(p.sx, p.sa, p.parts, p.sb);
+    if (device >= 0 && device < 64 && !g_attr_set[device]) {
+        cudaError_t e = cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cap);
+        if (e != cudaSuccess) return e;
+        g_attr_set[device] = true;
+    }
+    int sms = 0;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+    const int grid = (int)std::min<long long>(sms > 0 ? sms : 1, p.tiles);
+    k_gemm_tc<<<grid, kThreads, smem, s>>>(ta, tb0, tb1, p);
+    return cudaGetLastError();
+}
+
+}  // namespace gs

@@ -34,8 +34,16 @@ struct gs_basis {
     // tc_npad, zero padded), Rh = bf16(R) and Rl = bf16(R - Rh), with tensor maps
     void* tc_Rh = nullptr;
     void* tc_Rl = nullptr;
-    CUtensorMap tmap_rh, tmap_rl;
+    CUtensorMap tmap_rh, tmap_rl;   // boxes of tc_mpad rows (fused kernel only, M <= 256)
     int tc_npad = 0, tc_mpad = 0;
+    // R^T split the same way (tc_npad x tc_mpad), the B operand of V = P R
+    void* tc_Rth = nullptr;
+    void* tc_Rtl = nullptr;
+    // Q split into bf16 hi / lo (r x ldq16): the projection's B operands when D is
+    // too small for one fp16 rounding to average out (D < kMinF16Depth)
+    void* tc_Qh = nullptr;
+    void* tc_Ql = nullptr;
+    bool has_split = false;         // tc_Rh / tc_Rl / tc_Rth / tc_Rtl exist
     // scratch for the multi-kernel paths (rows processed in chunks)
     float* scratch = nullptr;
     long long scratch_floats = 0;
@@ -43,6 +51,12 @@ struct gs_basis {
 };
 
 namespace gs {
+
+// The fp16 projection rounds every x_d and q_jd once; those errors average out
+// over the D terms of <x, q_j>, and D >= 1024 keeps the worst score error of the
+// large workloads below half the 1e-4 ||x|| ||c|| bound.  Shorter rows use the
+// bf16 hi / lo split (three products) instead.
+constexpr int kMinF16Depth = 1024;
 
 // ----------------------------------------------------------------- build (gs_build.cu)
 // Runs the fp64 panel Gram-Schmidt and fills every field of h except the
@@ -93,11 +107,26 @@ cudaError_t launch_ps_tc(const gs_basis* h, const float* X, long long N, int ldx
                          float scale, float* Y, int ldy, float* S, int lds, int* argmax,
                          float* maxval, cudaStream_t s);
 
+// ----------------------------------------------------------------- general tcgen05 GEMM (gs_gemm_tc.cu)
+// C = alpha * A B^T (/ rownorm[i] colnorm[j] when both are given).  A: fp32 m x K
+// (lda % 4 == 0, 16-byte aligned).  split = false: B0 fp16 n x K, one fp16
+// rounding of A; split = true: B0 / B1 bf16 hi / lo, A split into bf16 hi / lo
+// (three products).  B rows 16-byte aligned (ldb % 8 == 0).  C fp32 or bf16.
+struct GemmTcArgs {
+    const float* A; long long lda; long long m; int K;
+    bool split;
+    const void* B0; const void* B1; long long ldb; int n;
+    void* C; long long ldc; bool c_bf16; float alpha;
+    const float* rownorm; const float* colnorm;
+};
+cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s);
+
 // ----------------------------------------------------------------- device error words
 // Each translation unit with kernels that can report device-side errors keeps
 // its own word; gs_stream_status reads and clears all of them.
 unsigned take_device_error_build();
 unsigned take_device_error_tc();
+unsigned take_device_error_gemm();
 
 }  // namespace gs
 

@@ -53,9 +53,12 @@
 #include <vector>
 
 #include "gs_internal.h"
+#include "gs_tc_ptx.cuh"
 
 namespace gs {
 namespace {
+
+using namespace ptx;
 
 __device__ unsigned g_err_tc = 0;
 
@@ -79,213 +82,6 @@ constexpr int kBStageBytes = 256 * kBK * 2;          // 32 KB: up to 256 rows of
 constexpr int kMaxSX = 4, kMaxSA = 2, kMaxSB = 4;
 constexpr int kTmemCols = 512;
 constexpr int kSCol = 256;           // first TMEM column of the score accumulator
-constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s
-
-// ----------------------------------------------------------------- PTX wrappers
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-    return (uint32_t)__cvta_generic_to_shared(p);
-}
-__device__ __forceinline__ unsigned long long globaltimer() {
-    unsigned long long t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-                 : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-// Bounded wait.  Returns false (and leaves the caller to unwind) on abort or timeout.
-__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const unsigned long long t0 = globaltimer();
-    for (uint32_t i = 1;; ++i) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if ((i & 255u) == 0) {
-            if (*abort_flag) return false;
-            if (globaltimer() - t0 > kWaitLimitNs) {
-                *abort_flag = 1;
-                atomicOr(&g_err_tc, GS_DEV_ERR_TIMEOUT);
-                return false;
-            }
-        }
-    }
-}
-// The same wait taken by a whole warp: every lane waits (each acquires the
-// barrier's phase) and the warp leaves only together, so .sync.aligned
-// instructions and warp shuffles after it always see a converged warp.
-__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
-    const bool ok = mbar_wait(bar, parity, abort_flag);
-    return __all_sync(0xffffffffu, ok);
-}
-// Wait used while unwinding: bounded, ignores the abort flag.
-__device__ __noinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
-    const unsigned long long t0 = globaltimer();
-    while (!mbar_try_wait(bar, parity)) {
-        if (globaltimer() - t0 > kWaitLimitNs) {
-            atomicOr(&g_err_tc, GS_DEV_ERR_TIMEOUT);
-            return;
-        }
-    }
-}
-__device__ __forceinline__ void fence_proxy_async() {
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-__device__ __forceinline__ void fence_barrier_init() {
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_before() {
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ uint64_t l2_policy_evict_last() {
-    uint64_t p;
-    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-    return p;
-}
-__device__ __forceinline__ uint64_t l2_policy_evict_first() {
-    uint64_t p;
-    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-    return p;
-}
-__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
-                                            uint64_t policy) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
-        "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y), "l"(policy)
-        : "memory");
-}
-__device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst)),
-                 "r"(ncols)
-                 : "memory");
-}
-__device__ __forceinline__ void tmem_relinquish() {
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
-}
-// D[tmem] (+)= A[smem] * B[smem]^T, fp16 inputs, fp32 accumulate.
-__device__ __forceinline__ void mma_f16_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
-                                           uint32_t accumulate) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-// D[tmem] (+)= A[tmem] * B[smem]^T, bf16 inputs, fp32 accumulate.
-__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
-                                            uint32_t accumulate) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-// Arrives once on `bar` when every previously issued MMA of this thread has completed.
-__device__ __forceinline__ void mma_commit(uint64_t* bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                     smem_u32(bar))
-                 : "memory");
-}
-// 16 consecutive fp32 columns of this thread's TMEM lane.
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
-    uint32_t r[16];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
-          "=r"(r[15])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-// 32 consecutive fp32 columns of this thread's TMEM lane.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
-    uint32_t r[32];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
-          "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
-          "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
-          "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
-// Stores 16 consecutive 32-bit columns of this thread's TMEM lane.
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* v) {
-    asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
-        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
-        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
-        "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
-        : "memory");
-}
-// Stores 8 consecutive 32-bit columns of this thread's TMEM lane.
-__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t* v) {
-    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(v[0]),
-                 "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
-                 : "memory");
-}
-__device__ __forceinline__ void tmem_wait_st() {
-    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-}
-// Two bf16 values in one 32-bit word, the first in the low half.
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<const uint32_t*>(&v);
-}
-
-// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
-// 1024 bytes apart (SBO), LBO unused for this layout (encoded 1), descriptor
-// version 1 (bits 46-48), swizzle mode 2 = 128B (bits 61-63).
-__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
-    uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
-    d |= (uint64_t)1 << 16;
-    d |= (uint64_t)(1024 >> 4) << 32;
-    d |= (uint64_t)1 << 46;
-    d |= (uint64_t)2 << 61;
-    return d;
-}
-// Instruction descriptor, kind::f16: D f32, A = B = f16, both K-major, N, M = 128.
-__host__ __device__ constexpr uint32_t idesc_f16_f32(int n) {
-    return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
-}
-// The same with A = B = bf16 (atype = btype = 1).
-__host__ __device__ constexpr uint32_t idesc_bf16_f32(int n) {
-    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
-}
 
 // ----------------------------------------------------------------- work split
 struct TileRange {
@@ -407,7 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const TileRange tr = cr.tile(t);
                 for (int kb = 0; kb < p.nkb; ++kb, ++it) {
                     const int s = it % p.sx;
-                    if (!mbar_wait(&c.x_empty[s], ((uint32_t)(it / p.sx) & 1u) ^ 1u, abort_flag)) {
+                    if (!mbar_wait(&c.x_empty[s], ((uint32_t)(it / p.sx) & 1u) ^ 1u, abort_flag, &g_err_tc)) {
                         ok = false;
                         break;
                     }
@@ -416,7 +212,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             // every copy this thread started lands before the CTA can exit
-            for (int j = std::max(0, it - p.sx); j < it; ++j) mbar_drain(&c.x_full[j % p.sx], (uint32_t)(j / p.sx) & 1u);
+            for (int j = std::max(0, it - p.sx); j < it; ++j) mbar_drain(&c.x_full[j % p.sx], (uint32_t)(j / p.sx) & 1u, &g_err_tc);
         }
     } else if (warp == kBWarp) {
         // ------------------------------------------------------------- B operand tiles via TMA:
@@ -429,7 +225,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             int it = 0;
             for (; it < total; ++it) {
                 const int s = it % p.sb;
-                if (!mbar_wait(&c.b_empty[s], ((uint32_t)(it / p.sb) & 1u) ^ 1u, abort_flag)) break;
+                if (!mbar_wait(&c.b_empty[s], ((uint32_t)(it / p.sb) & 1u) ^ 1u, abort_flag, &g_err_tc)) break;
                 const int k = it % per_tile;
                 uint8_t* dst = Bs + (size_t)s * kBStageBytes;
                 if (k < p.nkb) {
@@ -441,7 +237,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tma_load_2d(dst, ((k - p.nkb) & 1) ? &tmap_rl : &tmap_rh, &c.b_full[s], kr * kBK, 0, pol);
                 }
             }
-            for (int j = std::max(0, it - p.sb); j < it; ++j) mbar_drain(&c.b_full[j % p.sb], (uint32_t)(j / p.sb) & 1u);
+            for (int j = std::max(0, it - p.sb); j < it; ++j) mbar_drain(&c.b_full[j % p.sb], (uint32_t)(j / p.sb) & 1u, &g_err_tc);
         }
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------- MMA issue
@@ -456,8 +252,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // GEMM1: Y = X Q^T into columns [0, npad)
                 for (int kb = 0; kb < p.nkb; ++kb, ++ia, ++ib) {
                     const int sa = ia % p.sa, sb = ib % p.sb;
-                    if (!mbar_wait(&c.a_full[sa], (uint32_t)(ia / p.sa) & 1u, abort_flag) ||
-                        !mbar_wait(&c.b_full[sb], (uint32_t)(ib / p.sb) & 1u, abort_flag)) {
+                    if (!mbar_wait(&c.a_full[sa], (uint32_t)(ia / p.sa) & 1u, abort_flag, &g_err_tc) ||
+                        !mbar_wait(&c.b_full[sb], (uint32_t)(ib / p.sb) & 1u, abort_flag, &g_err_tc)) {
                         ok = false;
                         break;
                     }
@@ -475,12 +271,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mma_commit(&c.y_full);
                 // GEMM2: S = Yh Rh + Yl Rh + Yh Rl into columns [256, 256 + mpad), once the
                 // epilogue has split Y in place and released the previous tile's S
-                if (!mbar_wait(&c.ysplit_full, pt, abort_flag) || !mbar_wait(&c.s_empty, pt ^ 1u, abort_flag)) break;
+                if (!mbar_wait(&c.ysplit_full, pt, abort_flag, &g_err_tc) || !mbar_wait(&c.s_empty, pt ^ 1u, abort_flag, &g_err_tc)) break;
                 tc_fence_after();
                 for (int kr = 0; kr < p.nkr; ++kr, ib += 2) {
                     const int sh = ib % p.sb, sl = (ib + 1) % p.sb;
-                    if (!mbar_wait(&c.b_full[sh], (uint32_t)(ib / p.sb) & 1u, abort_flag) ||
-                        !mbar_wait(&c.b_full[sl], (uint32_t)((ib + 1) / p.sb) & 1u, abort_flag)) {
+                    if (!mbar_wait(&c.b_full[sh], (uint32_t)(ib / p.sb) & 1u, abort_flag, &g_err_tc) ||
+                        !mbar_wait(&c.b_full[sl], (uint32_t)((ib + 1) / p.sb) & 1u, abort_flag, &g_err_tc)) {
                         ok = false;
                         break;
                     }
@@ -506,12 +302,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mma_commit(&c.s_full);
                 // the next tile's GEMM1 overwrites the columns GEMM2 reads: wait for it to finish
                 mma_commit(&c.gemm2_done);
-                if (!mbar_wait(&c.gemm2_done, pt, abort_flag)) break;
+                if (!mbar_wait(&c.gemm2_done, pt, abort_flag, &g_err_tc)) break;
                 tc_fence_after();
             }
             // all MMAs issued by this thread complete before TMEM is released
             mma_commit(&c.mma_done);
-            mbar_drain(&c.mma_done, 0);
+            mbar_drain(&c.mma_done, 0, &g_err_tc);
         }
     } else if (warp >= kCvt0) {
         // ------------------------------------------------------------- converters
@@ -532,8 +328,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int kb = 0; kb < p.nkb; ++kb, ++it) {
                 if ((it & 1) != g) continue;
                 const int sx = it % p.sx, sa = it % p.sa;
-                if (!mbar_wait_warp(&c.x_full[sx], (uint32_t)(it / p.sx) & 1u, abort_flag) ||
-                    !mbar_wait_warp(&c.a_empty[sa], ((uint32_t)(it / p.sa) & 1u) ^ 1u, abort_flag)) {
+                if (!mbar_wait_warp(&c.x_full[sx], (uint32_t)(it / p.sx) & 1u, abort_flag, &g_err_tc) ||
+                    !mbar_wait_warp(&c.a_empty[sa], ((uint32_t)(it / p.sa) & 1u) ^ 1u, abort_flag, &g_err_tc)) {
                     ok = false;
                     break;
                 }
@@ -572,7 +368,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 v += __shfl_xor_sync(0xffffffffu, v, 1);
                 nrm[u] = v;
             }
-            if (!mbar_wait_warp(&c.xn_empty[b], ((uint32_t)(t >> 1) & 1u) ^ 1u, abort_flag)) break;
+            if (!mbar_wait_warp(&c.xn_empty[b], ((uint32_t)(t >> 1) & 1u) ^ 1u, abort_flag, &g_err_tc)) break;
             if (want_norm && (lane & 15) == 0) {
 #pragma unroll
                 for (int u = 0; u < kCvtRows; ++u) atomicAdd(&c.xn[b][rbase + kCvtRowStep * u], nrm[u]);
@@ -591,7 +387,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int t = 0; t < cr.ntiles; ++t) {
             const uint32_t pt = (uint32_t)t & 1u;
             const int b = t & 1;
-            if (!mbar_wait_warp(&c.y_full, pt, abort_flag)) break;
+            if (!mbar_wait_warp(&c.y_full, pt, abort_flag, &g_err_tc)) break;
             tc_fence_after();
             const TileRange tr = cr.tile(t);
             const bool valid = i < tr.nrows;
@@ -622,12 +418,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&c.ysplit_full);
-            if (!mbar_wait_warp(&c.xn_full[b], (uint32_t)(t >> 1) & 1u, abort_flag)) break;
+            if (!mbar_wait_warp(&c.xn_full[b], (uint32_t)(t >> 1) & 1u, abort_flag, &g_err_tc)) break;
             const float xnorm = sqrtf(c.xn[b][i]);
             c.xn[b][i] = 0.f;  // ready for the tile after next (both groups add into it)
             __syncwarp();
             if (lane == 0) mbar_arrive(&c.xn_empty[b]);
-            if (!mbar_wait_warp(&c.s_full, pt, abort_flag)) break;
+            if (!mbar_wait_warp(&c.s_full, pt, abort_flag, &g_err_tc)) break;
             tc_fence_after();
             float best = -FLT_MAX, run_max = -FLT_MAX, run_sum = 0.f;
             int besti = 0;
@@ -682,47 +478,33 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ----------------------------------------------------------------- host side
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn() {
-    static EncodeTiledFn fn = nullptr;
-    if (!fn) {
-        void* ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = (EncodeTiledFn)ptr;
-    }
-    return fn;
-}
-
-// 2-D tensor map over a row-major (rows x cols, ld elements) matrix with a
-// {box_cols, box_rows} box; out-of-range elements read as zero.
-bool make_tmap_2d(CUtensorMap* m, CUtensorMapDataType dt, int esize, const void* ptr, long long rows, int cols,
-                  long long ld, int box_cols, int box_rows, CUtensorMapSwizzle sw) {
-    EncodeTiledFn fn = encode_fn();
-    if (!fn) return false;
-    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)ld * esize};
-    cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
-    cuuint32_t estr[2] = {1, 1};
-    return fn(m, dt, 2, const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
-              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-// R (M x r fp32) -> Rh = bf16(R), Rl = bf16(R - Rh), both mpad x npad, zero padded.
+// R (M x r fp32) -> Rh = bf16(R), Rl = bf16(R - Rh) (mpad x npad) and the same
+// split of R^T (npad x mpad), all zero padded.
 __global__ void k_split_r(const float* __restrict__ R, int M, int r, int ldr, __nv_bfloat16* __restrict__ Rh,
-                          __nv_bfloat16* __restrict__ Rl, int mpad, int npad) {
+                          __nv_bfloat16* __restrict__ Rl, __nv_bfloat16* __restrict__ Rth,
+                          __nv_bfloat16* __restrict__ Rtl, int mpad, int npad) {
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= (long long)mpad * npad) return;
     const int i = (int)(idx / npad), j = (int)(idx % npad);
     const float v = (i < M && j < r) ? R[(size_t)i * ldr + j] : 0.f;
     const __nv_bfloat16 hv = __float2bfloat16_rn(v);
+    const __nv_bfloat16 lv = __float2bfloat16_rn(v - __bfloat162float(hv));
     Rh[idx] = hv;
-    Rl[idx] = __float2bfloat16_rn(v - __bfloat162float(hv));
+    Rl[idx] = lv;
+    Rth[(size_t)j * mpad + i] = hv;
+    Rtl[(size_t)j * mpad + i] = lv;
+}
+
+// Q (r x D fp32, ld = D) -> Qh = bf16(Q), Ql = bf16(Q - Qh), both r x ldq, zero padded.
+__global__ void k_split_q(const float* __restrict__ Q, int r, int D, int ldq, __nv_bfloat16* __restrict__ Qh,
+                          __nv_bfloat16* __restrict__ Ql) {
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)r * ldq) return;
+    const int j = (int)(idx / ldq), d = (int)(idx % ldq);
+    const float v = d < D ? Q[(size_t)j * D + d] : 0.f;
+    const __nv_bfloat16 hv = __float2bfloat16_rn(v);
+    Qh[idx] = hv;
+    Ql[idx] = __float2bfloat16_rn(v - __bfloat162float(hv));
 }
 
 int num_sms(int dev) {
@@ -768,16 +550,28 @@ bool tc_available(int device) {
 }
 
 gs_status tc_prepare(gs_basis* h) {
-    // the fused kernel keeps Y (r <= 256 columns) and S (M <= 256 columns) in TMEM
-    if (h->r < 1 || h->r > 256 || h->M > 256) return GS_OK;
+    if (h->r < 1) return GS_OK;
     const int npad = (h->r + 15) / 16 * 16;
     const int mpad = (h->M + 15) / 16 * 16;
     const size_t n = (size_t)mpad * npad;
-    if (cudaMalloc(&h->tc_Rh, sizeof(__nv_bfloat16) * n) != cudaSuccess) return GS_ERR_NOMEM;
-    if (cudaMalloc(&h->tc_Rl, sizeof(__nv_bfloat16) * n) != cudaSuccess) return GS_ERR_NOMEM;
+    // bf16 hi / lo splits of R (mpad x npad) and of R^T (npad x mpad)
+    for (void** ptr : {&h->tc_Rh, &h->tc_Rl, &h->tc_Rth, &h->tc_Rtl})
+        if (cudaMalloc(ptr, sizeof(__nv_bfloat16) * n) != cudaSuccess) return GS_ERR_NOMEM;
     k_split_r<<<(unsigned)((n + 255) / 256), 256>>>(h->R, h->M, h->r, h->ldr, (__nv_bfloat16*)h->tc_Rh,
-                                                    (__nv_bfloat16*)h->tc_Rl, mpad, npad);
+                                                    (__nv_bfloat16*)h->tc_Rl, (__nv_bfloat16*)h->tc_Rth,
+                                                    (__nv_bfloat16*)h->tc_Rtl, mpad, npad);
+    // bf16 hi / lo split of Q (r x ldq16, zero padded)
+    const size_t nq = (size_t)h->r * h->ldq16;
+    for (void** ptr : {&h->tc_Qh, &h->tc_Ql})
+        if (cudaMalloc(ptr, sizeof(__nv_bfloat16) * nq) != cudaSuccess) return GS_ERR_NOMEM;
+    k_split_q<<<(unsigned)((nq + 255) / 256), 256>>>(h->Q, h->r, h->D, h->ldq16, (__nv_bfloat16*)h->tc_Qh,
+                                                     (__nv_bfloat16*)h->tc_Ql);
     if (cudaGetLastError() != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) return GS_ERR_CUDA;
+    h->tc_npad = npad;
+    h->tc_mpad = mpad;
+    h->has_split = true;
+    // the fused kernel keeps Y (r <= 256 columns) and S (M <= 256 columns) in TMEM
+    if (h->r > 256 || h->M > 256) return GS_OK;
     if (!make_tmap_2d(&h->tmap_q16, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, h->Q16, h->r, h->D, h->ldq16, kBK, npad,
                       CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_tmap_2d(&h->tmap_rh, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, h->tc_Rh, mpad, npad, npad, kBK, mpad,
@@ -785,13 +579,11 @@ gs_status tc_prepare(gs_basis* h) {
         !make_tmap_2d(&h->tmap_rl, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, h->tc_Rl, mpad, npad, npad, kBK, mpad,
                       CU_TENSOR_MAP_SWIZZLE_128B))
         return GS_ERR_CUDA;
-    h->tc_npad = npad;
-    h->tc_mpad = mpad;
     if (cudaFuncSetAttribute(k_ps_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ps_smem_bytes(ps_rings())) !=
         cudaSuccess)
         return GS_ERR_CUDA;
     // the fused kernel needs all of its threads resident in one CTA; otherwise the
-    // basis simply has no tensor-core similarity path
+    // basis simply has no fused tensor-core similarity path
     cudaFuncAttributes fa;
     if (cudaFuncGetAttributes(&fa, k_ps_tc) != cudaSuccess) return GS_ERR_CUDA;
     h->has_tmap_q16 = fa.maxThreadsPerBlock >= kThreads;

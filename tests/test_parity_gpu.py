@@ -59,7 +59,10 @@ def check_scores(out, ref, X, cno, mode="raw", scale=1.0):
     elif mode == "cosine":
         bound = np.full(ref["S"].shape, TOL_S * abs(scale))
     else:
-        bound = np.full(ref["S"].shape, TOL_S)
+        # a logit error of at most d moves each probability p by at most p (e^(2d) - 1);
+        # d is the raw-score bound times the scale
+        d = TOL_S * abs(scale) * xn[:, None] * cno.max()
+        bound = ref["S"] * np.expm1(2 * d) + 1e-9
     if "S" in out:
         assert np.all(np.abs(host(out["S"]) - ref["S"]) <= bound + 1e-12)
     if "maxval" in out:

@@ -1,9 +1,12 @@
-"""GPU parity of the tcgen05 fused project + similarity kernel against the oracle.
+"""GPU parity of the tcgen05 kernels against the oracle.
 
 Same bar as the fp32 paths: |S - S*| <= 1e-4 ||x|| ||c_i||, Y within 1e-4 ||x||,
 argmax bit-exact wherever the oracle's top-2 margin exceeds twice the score
-tolerance.  The kernel rounds X to fp16 (RN) and uses a dithered fp16 copy of
-Q with fp32 accumulation, then takes S = Y R^T in fp32.
+tolerance, V within 1e-4 sum_i |p_i| ||c_i|| (plus 2^-8 |V*| for bf16 output),
+Xhat within 1e-4 ||t||.  The kernels round X (or T) to fp16 (RN) against a
+dithered fp16 copy of the basis with fp32 accumulation, and take the products
+whose terms do not average out (S = Y R^T, V = P R) with both operands split
+into bf16 hi / lo.
 """
 import numpy as np
 import pytest
@@ -123,3 +126,84 @@ def test_tc_range_error_is_reported(gs, large_ref):
     o = gs.project_similarity(b, X, path="tensor")
     gs.stream_status()
     assert o["argmax"].shape[0] == 256
+
+
+# ----------------------------------------------------------------- general tcgen05 GEMM paths
+@pytest.fixture(scope="module")
+def rankdef_ref(orc):
+    C, rank = synth.rankdef_codebook()
+    return C, orc.build_basis(C)
+
+
+@pytest.mark.parametrize("mode", ["raw", "cosine", "softmax"])
+def test_tc_two_gemm_rank_deficient(gs, orc, rankdef_ref, mode):
+    """r = 922 > 256: Y = X Q^T (fp16) then S = Y R^T (bf16 hi/lo split) on the tensor core."""
+    C, (Qo, Ro, cno) = rankdef_ref
+    X, _ = synth.noisy_rows(C, synth.SEEDS["rankdef"], 0, 1500, 1.0)
+    b = gs.build_basis(cuda(C))
+    scale = 1.0 if mode != "softmax" else 1.0 / 100.0
+    out = gs.project_similarity(b, cuda(X), mode=mode, scale=scale, path="tensor", want_S=True, want_Y=True)
+    gs.stream_status()
+    ref = orc.project_similarity(X, Qo, Ro, cno, mode=getattr(orc, mode.upper()), scale=scale)
+    check_scores(out, ref, X, cno, mode, scale)
+    assert np.all(np.abs(host(out["Y"]) - ref["Y"]) <= TOL_S * ref["xnorm"][:, None])
+
+
+def test_tc_two_gemm_wide_codebook(gs, orc):
+    """M = 300 > 256 codewords in D = 200 (rank 200 < M, Sec. 3.1's D < M case)."""
+    rng = np.random.default_rng(21)
+    C = (rng.integers(0, 2, size=(300, 200)) * 2 - 1).astype(np.float32)
+    X, _ = synth.noisy_rows(C, 22, 0, 3000, 1.0)
+    b = gs.build_basis(cuda(C))
+    Qo, Ro, cno = orc.build_basis(C)
+    assert b.r == Qo.shape[0] == 200
+    out = gs.project_similarity(b, cuda(X), path="tensor", want_S=True)
+    gs.stream_status()
+    check_scores(out, orc.project_similarity(X, Qo, Ro, cno), X, cno)
+
+
+def test_tc_reconstruct_round_trips(gs, orc, rankdef_ref):
+    """Reconstructing R itself returns the integer codebook bit-exactly after rounding."""
+    t = synth.tiny()
+    b = gs.build_basis(cuda(t["C"]))
+    assert np.array_equal(np.rint(gs.reconstruct(b, b.R.contiguous(), path="tensor").cpu().numpy()), t["C"])
+    C, _ = rankdef_ref
+    b = gs.build_basis(cuda(C))
+    r4 = (b.r + 3) // 4 * 4  # 16-byte rows for the TMA loads of T
+    T = torch.zeros((b.M, r4), device=b.R.device)
+    T[:, :b.r] = b.R
+    Xh = gs.reconstruct(b, T[:, :b.r], path="tensor")
+    gs.stream_status()
+    assert np.array_equal(np.rint(Xh.cpu().numpy()), C)
+
+
+@pytest.mark.parametrize("N,M,D", [(777, 40, 1002), (130, 8, 1024), (4096, 256, 8192)])
+def test_tc_reconstruct_matches_oracle(gs, orc, N, M, D):
+    rng = np.random.default_rng(N + D)
+    C = (rng.integers(0, 2, size=(M, D)) * 2 - 1).astype(np.float32)
+    b = gs.build_basis(cuda(C))
+    Qo, _, _ = orc.build_basis(C)
+    T = rng.standard_normal((N, b.r)).astype(np.float32) * 3.0
+    Xh = gs.reconstruct(b, cuda(T), path="tensor")
+    gs.stream_status()
+    ref = orc.reconstruct(T, Qo)
+    assert np.all(np.abs(host(Xh) - ref) <= 1e-4 * np.linalg.norm(T.astype(np.float64), axis=1)[:, None])
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_tc_prob_vectorize(gs, orc, dtype):
+    cases = [synth.tiny(), synth.multiattr()[2], {"C": synth.attention(B=1, L=1)["C"],
+                                                   "P": synth.attention_probs(5, 3, 700, 512, 1)}]
+    for t in cases:
+        b = gs.build_basis(cuda(t["C"]))
+        _, Ro, cno = orc.build_basis(t["C"])
+        Vo = orc.prob_vectorize(t["P"], Ro)
+        bound = 1e-4 * (np.abs(t["P"].astype(np.float64)) @ cno)[:, None]
+        if dtype == torch.bfloat16:
+            bound = bound + 2.0 ** -8 * np.abs(Vo)
+        N, M = t["P"].shape
+        Pp = torch.zeros((N, (M + 3) // 4 * 4), device="cuda:0")  # 16-byte rows for TMA
+        Pp[:, :M] = cuda(t["P"])
+        V = gs.prob_vectorize(b, Pp[:, :M], dtype=dtype, path="tensor")
+        gs.stream_status()
+        assert np.all(np.abs(host(V) - Vo) <= bound)
