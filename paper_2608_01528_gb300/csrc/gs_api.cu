@@ -333,11 +333,16 @@ gs_status gs_attention_scores(const void* Yq, const void* Yk, int in_dtype, int 
     if ((long long)B * Lq * Lk == 0) return GS_OK;
     if (!Yq || !Yk || !A) return GS_ERR_INVALID_ARG;
     if (B > 65535 || Lq > kMaxGemmRows) return GS_ERR_SHAPE;
-    if (flags == GS_PATH_TENSOR) return GS_ERR_UNSUPPORTED;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return GS_ERR_CUDA;
     if (!device_supported(dev)) return GS_ERR_UNSUPPORTED;
     cudaStream_t s = (cudaStream_t)stream;
+    const bool tc_ok = in_dtype == GS_BF16 && gs::tc_available(dev) && gs::attn_tc_supported(r, ldy, Yq, Yk);
+    const bool big = (double)B * Lq * Lk * r >= (double)(1 << 26);
+    if (flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && tc_ok && big)) {
+        if (!tc_ok) return in_dtype != GS_BF16 || r > 512 ? GS_ERR_UNSUPPORTED : GS_ERR_ALIGNMENT;
+        return from_cuda(gs::launch_attn_tc(Yq, Yk, B, Lq, Lk, r, ldy, scale, apply_softmax != 0, A, dev, s));
+    }
     gs::GemmArgs a{};
     const int t = in_dtype == GS_F32 ? gs::MAT_F32 : gs::MAT_BF16;
     a.A = Yq; a.a_type = t; a.lda = ldy; a.a_bstride = (long long)Lq * ldy;
@@ -356,7 +361,8 @@ gs_status gs_attention_scores(const void* Yq, const void* Yk, int in_dtype, int 
 gs_status gs_stream_status(void* stream) {
     cudaError_t e = stream ? cudaStreamSynchronize((cudaStream_t)stream) : cudaDeviceSynchronize();
     if (e != cudaSuccess) return GS_ERR_CUDA;
-    const unsigned w = gs::take_device_error_build() | gs::take_device_error_tc() | gs::take_device_error_gemm();
+    const unsigned w = gs::take_device_error_build() | gs::take_device_error_tc() | gs::take_device_error_gemm() |
+                       gs::take_device_error_attn();
     if (w & GS_DEV_ERR_TIMEOUT) return GS_ERR_TIMEOUT;
     if (w & GS_DEV_ERR_RANGE) return GS_ERR_RANGE;
     return GS_OK;

@@ -1,0 +1,323 @@
+// gs_attn_tc.cu -- attention scores between compressed vectors on tcgen05
+// (paper Sec. 2.2 attention score; Sec. 3.2: scores that use matrix
+// multiplication are preserved on Gram-loc):
+//
+//     A[b] = softmax_row(scale * Yq[b] Yk[b]^T)      (or the scaled logits)
+//
+// Yq: B x Lq x r bf16, Yk: B x Lk x r bf16 (row stride ld, r <= 512), A: fp32.
+//
+// One persistent CTA per SM walks work items (sequence b, 128-query tile).  The
+// query tile (128 x r bf16, up to 128 KB) stays resident in shared memory for
+// the whole item, in K-blocks of 64 that are released one by one, so the next
+// item's tile streams in while the current item's last MMAs run.  Key tiles
+// (256 keys x 64) stream through a TMA ring.  Logits accumulate in fp32 in TMEM,
+// double-buffered over units of 256 keys.  The row softmax needs every key, so
+// each item runs two passes over its key tiles: pass 1 keeps an online row max
+// and sum of exponentials; pass 2 recomputes the logits and writes
+// exp(scale s - max) / sum.  The logits never go to HBM; the price is twice the
+// MMA work (the tensor pipe has the headroom: the output write bounds it).
+//
+// Warp roles (224 threads): 0-3 epilogue (warp w owns TMEM lanes 32w..+31 =
+// query rows), 4 TMA producer of query K-blocks, 5 TMEM allocator + MMA issuer,
+// 6 TMA producer of key tiles.  Every mbarrier wait is bounded.
+
+#include <float.h>
+
+#include <algorithm>
+
+#include "gs_internal.h"
+#include "gs_tc_ptx.cuh"
+
+namespace gs {
+namespace {
+
+using namespace ptx;
+
+__device__ unsigned g_err_attn = 0;
+
+constexpr int kBM = 128;          // queries per item
+constexpr int kBN = 256;          // keys per unit
+constexpr int kBK = 64;           // r per K-block (128 bytes of bf16)
+constexpr int kMaxKB = 8;         // r <= 512
+constexpr int kQBlockBytes = kBM * kBK * 2;   // 16 KB
+constexpr int kKStageBytes = kBN * kBK * 2;   // 32 KB
+constexpr int kKStages = 3;
+constexpr int kEpiWarps = 4;
+constexpr int kQWarp = 4, kMmaWarp = 5, kKWarp = 6;
+constexpr int kThreads = 7 * 32;
+constexpr int kTmemCols = 512;
+
+struct AttnParams {
+    int B, Lq, Lk, r, nkb;
+    int qtiles, ntiles;      // query tiles per sequence, key tiles per sequence
+    int passes;              // 2 with the row softmax, 1 for plain scaled logits
+    float scale;
+    float* A;                // B x Lq x Lk
+    int a_vec;               // 16-byte aligned rows (Lk % 4 == 0 and A aligned)
+};
+
+struct Ctl {
+    uint64_t q_full[kMaxKB], q_empty[kMaxKB];
+    uint64_t k_full[kKStages], k_empty[kKStages];
+    uint64_t d_full[2], d_empty[2];
+    uint64_t mma_done;
+    uint32_t tmem_base;
+    int abort_flag;
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_attn_tc(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
+              const AttnParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+    uint8_t* Qs = base;                                 // kMaxKB x 16 KB
+    uint8_t* Ks = Qs + (size_t)kMaxKB * kQBlockBytes;   // kKStages x 32 KB
+    Ctl& c = *reinterpret_cast<Ctl*>(Ks + (size_t)kKStages * kKStageBytes);
+    volatile int* abort_flag = &c.abort_flag;
+    unsigned* err = &g_err_attn;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const long long items = (long long)p.B * p.qtiles;
+    const int nitems = items > blockIdx.x ? (int)((items - 1 - blockIdx.x) / gridDim.x + 1) : 0;
+    const int units_per_item = p.passes * p.ntiles;
+
+    if (threadIdx.x == 0) {
+        for (int k = 0; k < kMaxKB; ++k) {
+            mbar_init(&c.q_full[k], 1);
+            mbar_init(&c.q_empty[k], 1);
+        }
+        for (int s = 0; s < kKStages; ++s) {
+            mbar_init(&c.k_full[s], 1);
+            mbar_init(&c.k_empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&c.d_full[b], 1);
+            mbar_init(&c.d_empty[b], kEpiWarps);
+        }
+        mbar_init(&c.mma_done, 1);
+        c.abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == kMmaWarp) {
+        tmem_alloc(&c.tmem_base, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = c.tmem_base;
+
+    auto item_bq = [&](int li, int& b, int& qt) {
+        const long long ig = blockIdx.x + (long long)li * gridDim.x;
+        b = (int)(ig / p.qtiles);
+        qt = (int)(ig % p.qtiles);
+    };
+
+    if (warp == kQWarp) {
+        // ------------------------------------------------------------- query K-blocks via TMA
+        if (lane == 0) {
+            const uint64_t pol = l2_policy_evict_first();
+            int li = 0;
+            bool ok = true;
+            for (; li < nitems && ok; ++li) {
+                int b, qt;
+                item_bq(li, b, qt);
+                const uint32_t ph = ((uint32_t)li & 1u) ^ 1u;
+                for (int k = 0; k < p.nkb; ++k) {
+                    if (!mbar_wait(&c.q_empty[k], ph, abort_flag, err)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&c.q_full[k], kQBlockBytes);
+                    tma_load_2d(Qs + (size_t)k * kQBlockBytes, &tmap_q, &c.q_full[k], k * kBK,
+                                b * p.Lq + qt * kBM, pol);
+                }
+            }
+            // the last item's (possibly partial) loads land before the CTA exits
+            if (li > 0)
+                for (int k = 0; k < p.nkb; ++k) mbar_drain(&c.q_full[k], (uint32_t)(li - 1) & 1u, err);
+        }
+    } else if (warp == kKWarp) {
+        // ------------------------------------------------------------- key tiles via TMA
+        if (lane == 0) {
+            const uint64_t pol = l2_policy_evict_last();
+            const int total = nitems * units_per_item * p.nkb;
+            int it = 0;
+            for (; it < total; ++it) {
+                const int s = it % kKStages;
+                if (!mbar_wait(&c.k_empty[s], ((uint32_t)(it / kKStages) & 1u) ^ 1u, abort_flag, err)) break;
+                const int kb = it % p.nkb;
+                const int unit = (it / p.nkb) % units_per_item;
+                const int li = it / (p.nkb * units_per_item);
+                int b, qt;
+                item_bq(li, b, qt);
+                const int nt = unit % p.ntiles;
+                mbar_arrive_expect_tx(&c.k_full[s], kKStageBytes);
+                tma_load_2d(Ks + (size_t)s * kKStageBytes, &tmap_k, &c.k_full[s], kb * kBK, b * p.Lk + nt * kBN, pol);
+            }
+            for (int j = std::max(0, it - kKStages); j < it; ++j)
+                mbar_drain(&c.k_full[j % kKStages], (uint32_t)(j / kKStages) & 1u, err);
+        }
+    } else if (warp == kMmaWarp) {
+        // ------------------------------------------------------------- MMA issue
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(kBN);
+            int it = 0, gu = 0;
+            bool ok = true;
+            for (int li = 0; li < nitems && ok; ++li) {
+                const uint32_t qph = (uint32_t)li & 1u;
+                for (int u = 0; u < units_per_item && ok; ++u, ++gu) {
+                    const int buf = gu & 1;
+                    if (!mbar_wait(&c.d_empty[buf], ((uint32_t)(gu >> 1) & 1u) ^ 1u, abort_flag, err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t d_tmem = tmem + (uint32_t)(buf * kBN);
+                    for (int kb = 0; kb < p.nkb; ++kb, ++it) {
+                        const int s = it % kKStages;
+                        if ((u == 0 && !mbar_wait(&c.q_full[kb], qph, abort_flag, err)) ||
+                            !mbar_wait(&c.k_full[s], (uint32_t)(it / kKStages) & 1u, abort_flag, err)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint64_t ad = sdesc_sw128(smem_u32(Qs + (size_t)kb * kQBlockBytes));
+                        const uint64_t bd = sdesc_sw128(smem_u32(Ks + (size_t)s * kKStageBytes));
+#pragma unroll
+                        for (int k = 0; k < kBK / 16; ++k)
+                            mma_f16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
+                                       (kb | k) != 0 ? 1u : 0u);
+                        mma_commit(&c.k_empty[s]);
+                        // the item's last unit releases each query K-block as soon as it has used it
+                        if (u == units_per_item - 1) mma_commit(&c.q_empty[kb]);
+                    }
+                    if (ok) mma_commit(&c.d_full[buf]);
+                }
+            }
+            mma_commit(&c.mma_done);
+            mbar_drain(&c.mma_done, 0, err);
+        }
+    } else if (warp < kEpiWarps) {
+        // ------------------------------------------------------------- epilogue
+        const int i = threadIdx.x;  // query row within the item
+        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        int gu = 0;
+        for (int li = 0; li < nitems; ++li) {
+            int b, qt;
+            item_bq(li, b, qt);
+            const int q = qt * kBM + i;
+            const bool valid = q < p.Lq;
+            float* arow = p.A + ((size_t)b * p.Lq + (valid ? q : 0)) * p.Lk;
+            float m = -FLT_MAX, l = 0.f;
+            bool ok = true;
+            for (int u = 0; u < units_per_item; ++u, ++gu) {
+                const int buf = gu & 1;
+                if (!mbar_wait_warp(&c.d_full[buf], (uint32_t)(gu >> 1) & 1u, abort_flag, err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const int nt = u % p.ntiles;
+                const bool stats = p.passes == 2 && u < p.ntiles;
+                const float inv = l > 0.f ? 1.f / l : 0.f;
+                const uint32_t tb = tmem + lane_base + (uint32_t)(buf * kBN);
+                for (int jc = 0; jc < kBN; jc += 16) {
+                    float v[16];
+                    tmem_ld16(tb + (uint32_t)jc, v);
+                    const int k0 = nt * kBN + jc;
+                    if (!valid || k0 >= p.Lk) continue;
+                    const int nv = min(16, p.Lk - k0);
+                    if (stats) {
+                        float cm = m;
+#pragma unroll
+                        for (int j = 0; j < 16; ++j)
+                            if (j < nv) cm = fmaxf(cm, p.scale * v[j]);
+                        float add = 0.f;
+#pragma unroll
+                        for (int j = 0; j < 16; ++j)
+                            if (j < nv) add += __expf(p.scale * v[j] - cm);
+                        l = l * __expf(m - cm) + add;
+                        m = cm;
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 16; ++j)
+                            v[j] = p.passes == 2 ? __expf(p.scale * v[j] - m) * inv : p.scale * v[j];
+                        float* dst = arow + k0;
+                        if (p.a_vec && nv == 16) {
+#pragma unroll
+                            for (int j = 0; j < 16; j += 4)
+                                __stcs(reinterpret_cast<float4*>(dst + j), make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]));
+                        } else {
+                            for (int j = 0; j < nv; ++j) dst[j] = v[j];
+                        }
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&c.d_empty[buf]);
+            }
+            if (!ok) break;
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == kMmaWarp) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+constexpr size_t kSmemBytes = 1024 + (size_t)kMaxKB * kQBlockBytes + (size_t)kKStages * kKStageBytes + sizeof(Ctl);
+
+bool g_attr_set[64];
+
+}  // namespace
+
+unsigned take_device_error_attn() {
+    unsigned v = 0, z = 0;
+    cudaMemcpyFromSymbol(&v, g_err_attn, sizeof(v));
+    if (v) cudaMemcpyToSymbol(g_err_attn, &z, sizeof(z));
+    return v;
+}
+
+bool attn_tc_supported(int r, long long ldy, const void* Yq, const void* Yk) {
+    return r >= 1 && r <= kMaxKB * kBK && ldy % 8 == 0 && (uintptr_t)Yq % 16 == 0 && (uintptr_t)Yk % 16 == 0;
+}
+
+cudaError_t launch_attn_tc(const void* Yq, const void* Yk, int B, int Lq, int Lk, int r, long long ldy, float scale,
+                           bool softmax, float* A, int device, cudaStream_t s) {
+    AttnParams p;
+    p.B = B;
+    p.Lq = Lq;
+    p.Lk = Lk;
+    p.r = r;
+    p.nkb = (r + kBK - 1) / kBK;
+    p.qtiles = (Lq + kBM - 1) / kBM;
+    p.ntiles = (Lk + kBN - 1) / kBN;
+    p.passes = softmax ? 2 : 1;
+    p.scale = scale;
+    p.A = A;
+    p.a_vec = ((uintptr_t)A % 16 == 0) && (Lk % 4 == 0);
+    CUtensorMap tq, tk;
+    if (!make_tmap_2d(&tq, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, Yq, (long long)B * Lq, r, ldy, kBK, kBM,
+                      CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_tmap_2d(&tk, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, Yk, (long long)B * Lk, r, ldy, kBK, kBN,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    if (device >= 0 && device < 64 && !g_attr_set[device]) {
+        cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+        if (e != cudaSuccess) return e;
+        g_attr_set[device] = true;
+    }
+    int sms = 0;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+    const long long items = (long long)B * p.qtiles;
+    const int grid = (int)std::min<long long>(sms > 0 ? sms : 1, items);
+    k_attn_tc<<<grid, kThreads, kSmemBytes, s>>>(tq, tk, p);
+    return cudaGetLastError();
+}
+
+}  // namespace gs

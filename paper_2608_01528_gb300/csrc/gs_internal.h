@@ -121,12 +121,19 @@ struct GemmTcArgs {
 };
 cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s);
 
+// ----------------------------------------------------------------- attention scores on tcgen05 (gs_attn_tc.cu)
+// bf16 Yq (B x Lq x r) and Yk (B x Lk x r), row stride ldy; fp32 A (B x Lq x Lk, dense).
+bool attn_tc_supported(int r, long long ldy, const void* Yq, const void* Yk);
+cudaError_t launch_attn_tc(const void* Yq, const void* Yk, int B, int Lq, int Lk, int r, long long ldy, float scale,
+                           bool softmax, float* A, int device, cudaStream_t s);
+
 // ----------------------------------------------------------------- device error words
 // Each translation unit with kernels that can report device-side errors keeps
 // its own word; gs_stream_status reads and clears all of them.
 unsigned take_device_error_build();
 unsigned take_device_error_tc();
 unsigned take_device_error_gemm();
+unsigned take_device_error_attn();
 
 }  // namespace gs
 

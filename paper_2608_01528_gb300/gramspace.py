@@ -235,7 +235,7 @@ def attention_scores(Yq, Yk, scale, apply_softmax=True, path="auto", out=None, s
     if Yk.shape[0] != B or Yk.shape[2] != r or Yq.dtype != Yk.dtype:
         raise ValueError("Yq and Yk must agree in batch, width and dtype")
     if not (Yq.is_contiguous() and Yk.is_contiguous()):
-        raise ValueError("Yq and Yk must be contiguous")
+        raise ValueError("Yq and Yk must be contiguous (row stride r)")
     A = out if out is not None else torch.empty((B, Lq, Lk), dtype=torch.float32, device=Yq.device)
     L = load_library()
     with torch.cuda.device(Yq.device):

@@ -207,3 +207,35 @@ def test_tc_prob_vectorize(gs, orc, dtype):
         V = gs.prob_vectorize(b, Pp[:, :M], dtype=dtype, path="tensor")
         gs.stream_status()
         assert np.all(np.abs(host(V) - Vo) <= bound)
+
+
+# ----------------------------------------------------------------- attention on tcgen05
+@pytest.fixture(scope="module")
+def attn_R(orc):
+    return orc.build_basis(synth.attention(B=1, L=1)["C"])[1]
+
+
+def _attn_inputs(orc, R, B, Lq, Lk, seed=5):
+    """Compressed query / key vectors V = P R from the oracle, rounded to bf16."""
+    Vq = orc.prob_vectorize(synth.attention_probs(seed, B, Lq, 512, 1), R).astype(np.float32)
+    Vk = orc.prob_vectorize(synth.attention_probs(seed, B, Lk, 512, 2), R).astype(np.float32)
+    tq = torch.from_numpy(Vq).to("cuda:0").to(torch.bfloat16).reshape(B, Lq, -1).contiguous()
+    tk = torch.from_numpy(Vk).to("cuda:0").to(torch.bfloat16).reshape(B, Lk, -1).contiguous()
+    return tq, tk
+
+
+@pytest.mark.parametrize("B,Lq,Lk", [(3, 40, 40), (2, 300, 700), (1, 128, 256), (2, 1024, 1024)])
+def test_tc_attention(gs, orc, attn_R, B, Lq, Lk):
+    """bf16 compressed vectors (r = 512), fp32 accumulation, row softmax over all keys
+    in two passes; against the oracle run on the same bf16 inputs."""
+    tq, tk = _attn_inputs(orc, attn_R, B, Lq, Lk)
+    scale = 1.0 / 64.0
+    A = gs.attention_scores(tq, tk, scale, path="tensor")
+    L = gs.attention_scores(tq, tk, scale, apply_softmax=False, path="tensor")
+    gs.stream_status()
+    q64, k64 = tq.double().cpu().numpy(), tk.double().cpu().numpy()
+    ref = orc.attention(q64, k64, B, Lq, Lk, scale)
+    refl = orc.attention(q64, k64, B, Lq, Lk, scale, apply_softmax=False)
+    assert (np.abs(host(A) - ref) / ref).max() <= 2e-2
+    assert np.allclose(host(A).sum(axis=2), 1.0, atol=1e-4)
+    assert np.abs(host(L) - refl).max() <= 1e-4 * np.abs(refl).max()
