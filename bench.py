@@ -46,6 +46,8 @@ def parse():
     p.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline leg")
     p.add_argument("--rows", type=int, default=0,
                    help="profiling only: use the first ROWS queries instead of all 65,536")
+    p.add_argument("--rows-only", action="store_true",
+                   help="profiling only: run just the per-row side measurements and print them")
     return p.parse_args()
 
 
@@ -201,6 +203,12 @@ def main():
         run_reference(args)
         return
     ws, rank, local = dist_env()
+    if args.rows_only:
+        import torch
+        from paper_2608_01528_gb300 import gramspace as gs
+        torch.cuda.set_device(local)
+        print(json.dumps({"rows": side_rows(gs, torch.device("cuda", local))}), flush=True)
+        return
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu:
         # the oracle leg runs before CUDA is touched (no forked workers after GPU init)
@@ -338,9 +346,12 @@ def main():
 
 
 def side_rows(gs, dev):
-    """One timed measurement per other hot-path row (small, HBM-resident inputs)."""
+    """One timed measurement per other hot-path row (inputs resident in HBM), each
+    with its roofline: algorithmic bytes or flops per launch over the measured time,
+    against MEASURED_PEAKS.json (HBM copy GB/s; bf16 dense TFLOP/s, which fp16 matches)."""
     import torch
     import synth
+    peaks = load_peaks()
     out = {}
 
     def timeit(fn, reps=10):
@@ -355,36 +366,46 @@ def side_rows(gs, dev):
         torch.cuda.synchronize()
         return a.elapsed_time(b) / reps
 
-    # build (init-time) on the rank-deficient binary codebook
+    def roof(ms, nbytes, flops, bound):
+        sec = ms / 1e3
+        d = {"ms": round(ms, 4), "gbs": round(nbytes / sec / 1e9, 1), "tflops": round(flops / sec / 1e12, 1),
+             "bound": bound}
+        d["frac"] = round(d["gbs"] / peaks["hbm_gbs"] if bound == "hbm" else d["tflops"] / peaks["bf16_tflops"], 4)
+        return d
+
+    # basis build (init-time, not rooflined) on the rank-deficient binary codebook
     C4, _ = synth.rankdef_codebook()
     C4d = torch.from_numpy(C4).to(dev)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     b4 = gs.build_basis(C4d)
     torch.cuda.synchronize()
-    out["build_rankdef_ms"] = round(1e3 * (time.perf_counter() - t0), 2)
-    out["build_rankdef_r"] = b4.r
-    # reconstruct 16,384 x 922 -> 16,384 x 10,000
+    out["build_rankdef"] = {"ms": round(1e3 * (time.perf_counter() - t0), 2), "r": b4.r}
     r4 = (b4.r + 3) // 4 * 4  # 16-byte rows, as the tensor-core path needs
+    # project + similarity with r = 922 > 256 (two tensor-core GEMMs), 16,384 queries
+    X4 = torch.from_numpy(synth.rankdef()["X"]).to(dev)
+    am = torch.empty(X4.shape[0], dtype=torch.int32, device=dev)
+    mv = torch.empty(X4.shape[0], device=dev)
+    ms = timeit(lambda: gs.project_similarity(b4, X4, out={"argmax": am, "maxval": mv}))
+    N4, D4 = X4.shape
+    out["project_similarity_rankdef"] = roof(ms, N4 * D4 * 4, 2 * N4 * D4 * b4.r + 2 * N4 * b4.r * b4.M, "tensor")
+    del X4
+    # reconstruct 16,384 x 922 -> 16,384 x 10,000
     T = torch.randn(16384, r4, device=dev)[:, :b4.r]
     Xh = torch.empty(16384, 10000, device=dev)
     ms = timeit(lambda: gs.reconstruct(b4, T, out=Xh))
-    out["reconstruct_rankdef_ms"] = round(ms, 4)
-    out["reconstruct_rankdef_gflops"] = round(2 * 16384 * b4.r * 10000 / (ms / 1e3) / 1e9, 1)
-    # prob-vectorize + attention on the attention workload (64 x 1024, r = 512)
+    out["reconstruct_rankdef"] = roof(ms, 16384 * (b4.r + 10000) * 4, 2 * 16384 * b4.r * 10000, "tensor")
+    # prob-vectorize + attention on the attention workload (64 x 1024 tokens, r = 512)
     a = synth.attention()
     b5 = gs.build_basis(torch.from_numpy(a["C"]).to(dev))
     Pq = torch.from_numpy(a["Pq"]).to(dev)
     Vq = torch.empty(Pq.shape[0], b5.r, dtype=torch.bfloat16, device=dev)
     ms = timeit(lambda: gs.prob_vectorize(b5, Pq, out=Vq))
-    out["probvec_attention_ms"] = round(ms, 4)
-    out["probvec_attention_gbs"] = round((Pq.numel() * 4 + Vq.numel() * 2) / (ms / 1e3) / 1e9, 1)
+    out["probvec_attention"] = roof(ms, Pq.numel() * 4 + Vq.numel() * 2, 2 * Pq.shape[0] * b5.M * b5.r, "hbm")
     V3 = Vq.reshape(64, 1024, -1)
     A = torch.empty(64, 1024, 1024, device=dev)
     ms = timeit(lambda: gs.attention_scores(V3, V3, 1 / 64.0, out=A))
-    out["attention_ms"] = round(ms, 4)
-    out["attention_gbs"] = round((2 * V3.numel() * 2 + A.numel() * 4) / (ms / 1e3) / 1e9, 1)
-    out["attention_tflops"] = round(2 * 64 * 1024 * 1024 * b5.r / (ms / 1e3) / 1e12, 1)
+    out["attention"] = roof(ms, 2 * V3.numel() * 2 + A.numel() * 4, 2 * 64 * 1024 * 1024 * b5.r, "hbm")
     del b4, b5
     return out
 

@@ -53,7 +53,7 @@ struct AttnParams {
     int passes;              // 2 with the row softmax, 1 for plain scaled logits
     float scale;
     float* A;                // B x Lq x Lk
-    int a_vec;               // 16-byte aligned rows (Lk % 4 == 0 and A aligned)
+    int a_vec;               // rows aligned for two-element stores (Lk even, A 8-byte aligned)
 };
 
 struct Ctl {
@@ -201,15 +201,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp < kEpiWarps) {
         // ------------------------------------------------------------- epilogue
-        const int i = threadIdx.x;  // query row within the item
+        // Statistics pass: TMEM read one row per thread (32x32b), online max / sum.
+        // Writing pass: TMEM read in the 16x256b pattern (a quad of threads holds 8
+        // consecutive keys of one row, so stores write whole sectors); each row's
+        // max and sum come by shuffle from the thread that owned the row.
+        const int i = threadIdx.x;  // query row within the item (statistics pass)
         const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
         int gu = 0;
         for (int li = 0; li < nitems; ++li) {
             int b, qt;
             item_bq(li, b, qt);
-            const int q = qt * kBM + i;
-            const bool valid = q < p.Lq;
-            float* arow = p.A + ((size_t)b * p.Lq + (valid ? q : 0)) * p.Lk;
+            const bool valid = qt * kBM + i < p.Lq;
             float m = -FLT_MAX, l = 0.f;
             bool ok = true;
             for (int u = 0; u < units_per_item; ++u, ++gu) {
@@ -220,16 +222,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_after();
                 const int nt = u % p.ntiles;
-                const bool stats = p.passes == 2 && u < p.ntiles;
-                const float inv = l > 0.f ? 1.f / l : 0.f;
-                const uint32_t tb = tmem + lane_base + (uint32_t)(buf * kBN);
-                for (int jc = 0; jc < kBN; jc += 16) {
-                    float v[16];
-                    tmem_ld16(tb + (uint32_t)jc, v);
-                    const int k0 = nt * kBN + jc;
-                    if (!valid || k0 >= p.Lk) continue;
-                    const int nv = min(16, p.Lk - k0);
-                    if (stats) {
+                if (p.passes == 2 && u < p.ntiles) {
+                    const uint32_t tb = tmem + lane_base + (uint32_t)(buf * kBN);
+                    for (int jc = 0; jc < kBN; jc += 16) {
+                        float v[16];
+                        tmem_ld16(tb + (uint32_t)jc, v);
+                        const int k0 = nt * kBN + jc;
+                        if (!valid || k0 >= p.Lk) continue;
+                        const int nv = min(16, p.Lk - k0);
                         float cm = m;
 #pragma unroll
                         for (int j = 0; j < 16; ++j)
@@ -240,17 +240,45 @@ __global__ void __launch_bounds__(kThreads, 1)
                             if (j < nv) add += __expf(p.scale * v[j] - cm);
                         l = l * __expf(m - cm) + add;
                         m = cm;
-                    } else {
+                    }
+                } else {
+                    for (int half = 0; half < 2; ++half) {
+                        const int r0 = half * 16 + (lane >> 2);  // rows r0 and r0 + 8 of this warp
+                        const float m0 = __shfl_sync(0xffffffffu, m, r0), l0 = __shfl_sync(0xffffffffu, l, r0);
+                        const float m1 = __shfl_sync(0xffffffffu, m, r0 + 8), l1 = __shfl_sync(0xffffffffu, l, r0 + 8);
+                        const float mh[2] = {m0, m1};
+                        const float ih[2] = {l0 > 0.f ? 1.f / l0 : 0.f, l1 > 0.f ? 1.f / l1 : 0.f};
+                        int qrow[2];
+                        float* arow[2];
 #pragma unroll
-                        for (int j = 0; j < 16; ++j)
-                            v[j] = p.passes == 2 ? __expf(p.scale * v[j] - m) * inv : p.scale * v[j];
-                        float* dst = arow + k0;
-                        if (p.a_vec && nv == 16) {
+                        for (int h = 0; h < 2; ++h) {
+                            qrow[h] = qt * kBM + warp * 32 + r0 + 8 * h;
+                            arow[h] = p.A + ((size_t)b * p.Lq + (qrow[h] < p.Lq ? qrow[h] : 0)) * p.Lk;
+                        }
+                        const uint32_t tb = tmem + ((uint32_t)(warp * 32 + half * 16) << 16) + (uint32_t)(buf * kBN);
+                        for (int jc = 0; jc < kBN; jc += 32) {
+                            float v[16];
+                            tmem_ld16x256b_x4(tb + (uint32_t)jc, v);
 #pragma unroll
-                            for (int j = 0; j < 16; j += 4)
-                                __stcs(reinterpret_cast<float4*>(dst + j), make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]));
-                        } else {
-                            for (int j = 0; j < nv; ++j) dst[j] = v[j];
+                            for (int j = 0; j < 4; ++j) {
+                                const int key = nt * kBN + jc + 8 * j + 2 * (lane & 3);
+#pragma unroll
+                                for (int h = 0; h < 2; ++h) {
+                                    if (qrow[h] >= p.Lq || key >= p.Lk) continue;
+                                    float a0 = p.scale * v[4 * j + 2 * h], a1 = p.scale * v[4 * j + 2 * h + 1];
+                                    if (p.passes == 2) {
+                                        a0 = __expf(a0 - mh[h]) * ih[h];
+                                        a1 = __expf(a1 - mh[h]) * ih[h];
+                                    }
+                                    float* dst = arow[h] + key;
+                                    if (p.a_vec && key + 1 < p.Lk) {
+                                        __stcs(reinterpret_cast<float2*>(dst), make_float2(a0, a1));
+                                    } else {
+                                        dst[0] = a0;
+                                        if (key + 1 < p.Lk) dst[1] = a1;
+                                    }
+                                }
+                            }
                         }
                     }
                 }
@@ -300,7 +328,7 @@ cudaError_t launch_attn_tc(const void* Yq, const void* Yk, int B, int Lq, int Lk
     p.passes = softmax ? 2 : 1;
     p.scale = scale;
     p.A = A;
-    p.a_vec = ((uintptr_t)A % 16 == 0) && (Lk % 4 == 0);
+    p.a_vec = ((uintptr_t)A % 8 == 0) && (Lk % 2 == 0);
     CUtensorMap tq, tk;
     if (!make_tmap_2d(&tq, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, Yq, (long long)B * Lq, r, ldy, kBK, kBM,
                       CU_TENSOR_MAP_SWIZZLE_128B) ||

@@ -68,7 +68,7 @@ struct GemmParams {
     int sx, sa, sb;
     void* C;
     long long ldc;
-    int c_bf16, c_vec;      // c_vec: 16-byte aligned rows, vector stores allowed
+    int c_bf16, c_vec;      // c_vec: rows aligned for two-element stores
     float alpha;
     const float* rownorm;
     const float* colnorm;
@@ -272,8 +272,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (amax > 65504.f) atomicOr(err, GS_DEV_ERR_RANGE);
     } else {
         // ------------------------------------------------------------- epilogue (warps 0-3)
-        const int i = threadIdx.x;
-        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        // TMEM is read in the 16x256b pattern so that each store writes whole sectors:
+        // thread t holds rows (t/4) and (t/4 + 8) of a 16-lane half, 8 columns per quad.
         for (int lt = 0; lt < ntiles; ++lt) {
             const int buf = lt & 1;
             if (!mbar_wait_warp(&c.d_full[buf], (uint32_t)(lt >> 1) & 1u, abort_flag, err)) break;
@@ -281,46 +281,48 @@ __global__ void __launch_bounds__(kThreads, 1)
             long long tm;
             int tn;
             tile_mn(lt, tm, tn);
-            const long long row = tm * kBM + i;
-            const bool valid = row < p.m;
-            const float rn = (valid && p.rownorm) ? p.rownorm[row] : 1.f;
-            const uint32_t tb = tmem + lane_base + (uint32_t)(buf * 256);
-            for (int jc = 0; jc < p.nt; jc += 16) {
-                float v[16];
-                tmem_ld16(tb + (uint32_t)jc, v);
-                const int col0 = tn * p.nt + jc;
-                if (!valid || col0 >= p.n) continue;
+            for (int half = 0; half < 2; ++half) {
+                const int lrow = warp * 32 + half * 16;
+                const uint32_t tb = tmem + ((uint32_t)lrow << 16) + (uint32_t)(buf * 256);
+                const long long row[2] = {tm * kBM + lrow + (lane >> 2), tm * kBM + lrow + (lane >> 2) + 8};
+                float rn[2];
 #pragma unroll
-                for (int j = 0; j < 16; ++j) {
-                    float g = p.alpha * v[j];
-                    if (p.colnorm) {
-                        const int col = col0 + j;
-                        const float den = col < p.n ? rn * p.colnorm[col] : 0.f;
-                        g = den > 0.f ? g / den : 0.f;
-                    }
-                    v[j] = g;
-                }
-                if (p.c_bf16) {
-                    __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(p.C) + (size_t)row * p.ldc + col0;
-                    if (p.c_vec && col0 + 16 <= p.n) {
-                        uint4 w0, w1;
-                        w0.x = pack_bf16(v[0], v[1]); w0.y = pack_bf16(v[2], v[3]);
-                        w0.z = pack_bf16(v[4], v[5]); w0.w = pack_bf16(v[6], v[7]);
-                        w1.x = pack_bf16(v[8], v[9]); w1.y = pack_bf16(v[10], v[11]);
-                        w1.z = pack_bf16(v[12], v[13]); w1.w = pack_bf16(v[14], v[15]);
-                        reinterpret_cast<uint4*>(dst)[0] = w0;
-                        reinterpret_cast<uint4*>(dst)[1] = w1;
-                    } else {
-                        for (int j = 0; j < 16 && col0 + j < p.n; ++j) dst[j] = __float2bfloat16_rn(v[j]);
-                    }
-                } else {
-                    float* dst = reinterpret_cast<float*>(p.C) + (size_t)row * p.ldc + col0;
-                    if (p.c_vec && col0 + 16 <= p.n) {
+                for (int h = 0; h < 2; ++h) rn[h] = (p.rownorm && row[h] < p.m) ? p.rownorm[row[h]] : 1.f;
+                for (int jc = 0; jc < p.nt; jc += 32) {
+                    float v[16];
+                    tmem_ld16x256b_x4(tb + (uint32_t)jc, v);
 #pragma unroll
-                        for (int j = 0; j < 16; j += 4)
-                            __stcs(reinterpret_cast<float4*>(dst + j), make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]));
-                    } else {
-                        for (int j = 0; j < 16 && col0 + j < p.n; ++j) dst[j] = v[j];
+                    for (int j = 0; j < 4; ++j) {
+                        const int col = tn * p.nt + jc + 8 * j + 2 * (lane & 3);
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            if (row[h] >= p.m || col >= p.n) continue;
+                            float g0 = p.alpha * v[4 * j + 2 * h], g1 = p.alpha * v[4 * j + 2 * h + 1];
+                            if (p.colnorm) {
+                                const float d0 = rn[h] * p.colnorm[col];
+                                const float d1 = col + 1 < p.n ? rn[h] * p.colnorm[col + 1] : 0.f;
+                                g0 = d0 > 0.f ? g0 / d0 : 0.f;
+                                g1 = d1 > 0.f ? g1 / d1 : 0.f;
+                            }
+                            const size_t off = (size_t)row[h] * p.ldc + col;
+                            if (p.c_bf16) {
+                                __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(p.C) + off;
+                                if (p.c_vec && col + 1 < p.n) {
+                                    *reinterpret_cast<uint32_t*>(dst) = pack_bf16(g0, g1);
+                                } else {
+                                    dst[0] = __float2bfloat16_rn(g0);
+                                    if (col + 1 < p.n) dst[1] = __float2bfloat16_rn(g1);
+                                }
+                            } else {
+                                float* dst = reinterpret_cast<float*>(p.C) + off;
+                                if (p.c_vec && col + 1 < p.n) {
+                                    __stcs(reinterpret_cast<float2*>(dst), make_float2(g0, g1));
+                                } else {
+                                    dst[0] = g0;
+                                    if (col + 1 < p.n) dst[1] = g1;
+                                }
+                            }
+                        }
                     }
                 }
             }
@@ -361,7 +363,7 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     p.n = a.n;
     p.K = a.K;
     p.nkb = (a.K + kBK - 1) / kBK;
-    p.nt = a.n >= 256 ? 256 : (a.n + 15) / 16 * 16;
+    p.nt = a.n >= 256 ? 256 : (a.n + 31) / 32 * 32;
     p.tiles_n = (a.n + p.nt - 1) / p.nt;
     p.tiles = ((a.m + kBM - 1) / kBM) * (long long)p.tiles_n;
     p.amode = a.split ? kABF16X2 : kAF16;
@@ -387,7 +389,7 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     p.C = a.C;
     p.ldc = a.ldc;
     p.c_bf16 = a.c_bf16 ? 1 : 0;
-    p.c_vec = ((uintptr_t)a.C % 16 == 0) && (a.ldc % (a.c_bf16 ? 8 : 4) == 0);
+    p.c_vec = ((uintptr_t)a.C % (a.c_bf16 ? 4 : 8) == 0) && (a.ldc % 2 == 0);
     p.alpha = a.alpha;
     p.rownorm = a.rownorm;
     p.colnorm = a.colnorm;
