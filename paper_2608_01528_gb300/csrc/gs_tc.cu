@@ -76,10 +76,9 @@ constexpr int kThreads = (kCvt0 + kCvtWarps) * 32;  // 480
 constexpr int kCvtThreads = kCvtGroupWarps * 32;     // 128 per group
 constexpr int kCvtRowStep = kCvtThreads / 16;        // 8 rows per sweep of the 16 float4 columns
 constexpr int kCvtRows = kBM / kCvtRowStep;          // 16 rows per converter thread
-constexpr int kXStageBytes = kBM * kBK * 4;          // 32 KB fp32 staging tile
 constexpr int kAStageBytes = kBM * kBK * 2;          // 16 KB fp16 operand tile
 constexpr int kBStageBytes = 256 * kBK * 2;          // 32 KB: up to 256 rows of one B operand K-block
-constexpr int kMaxSX = 4, kMaxSA = 2, kMaxSB = 4;
+constexpr int kMaxSX = 6, kMaxSA = 2, kMaxSB = 4;
 constexpr int kTmemCols = 512;
 constexpr int kSCol = 256;           // first TMEM column of the score accumulator
 
@@ -116,6 +115,7 @@ struct PsParams {
     int D, r, npad, M, mpad, nkb, nkr;
     int sx, sa, sb;         // ring depths: fp32 X staging, fp16 A, B operand tiles
     int box_rows;           // rows of each X TMA box (>= every tile's rows)
+    int xstage;             // bytes between X staging tiles (box_rows x 256, 1 KB aligned)
     const float* cnorm;     // M
     int mode;
     float scale;
@@ -148,7 +148,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t raw = smem_u32(smem_raw);
     uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
     uint8_t* Xs = base;
-    uint8_t* As = Xs + (size_t)p.sx * kXStageBytes;
+    uint8_t* As = Xs + (size_t)p.sx * p.xstage;
     uint8_t* Bs = As + (size_t)p.sa * kAStageBytes;
     Ctl& c = *reinterpret_cast<Ctl*>(Bs + (size_t)p.sb * kBStageBytes);
     volatile int* abort_flag = &c.abort_flag;
@@ -198,17 +198,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint64_t pol = l2_policy_evict_first();
             const uint32_t bytes = (uint32_t)p.box_rows * kBK * 4;
             int it = 0;
+            RingPos xs;
             bool ok = true;
             for (int t = 0; t < cr.ntiles && ok; ++t) {
                 const TileRange tr = cr.tile(t);
-                for (int kb = 0; kb < p.nkb; ++kb, ++it) {
-                    const int s = it % p.sx;
-                    if (!mbar_wait(&c.x_empty[s], ((uint32_t)(it / p.sx) & 1u) ^ 1u, abort_flag, &g_err_tc)) {
+                for (int kb = 0; kb < p.nkb; ++kb, ++it, xs.next(p.sx)) {
+                    if (!mbar_wait_1t(&c.x_empty[xs.idx], xs.phase ^ 1u, abort_flag, &g_err_tc)) {
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(&c.x_full[s], bytes);
-                    tma_load_2d(Xs + (size_t)s * kXStageBytes, &tmap_x, &c.x_full[s], kb * kBK, (int)tr.row0, pol);
+                    mbar_arrive_expect_tx(&c.x_full[xs.idx], bytes);
+                    tma_load_2d(Xs + (size_t)xs.idx * p.xstage, &tmap_x, &c.x_full[xs.idx], kb * kBK, (int)tr.row0,
+                                pol);
                 }
             }
             // every copy this thread started lands before the CTA can exit
@@ -223,10 +224,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int per_tile = p.nkb + 2 * p.nkr;
             const int total = cr.ntiles * per_tile;
             int it = 0;
-            for (; it < total; ++it) {
-                const int s = it % p.sb;
-                if (!mbar_wait(&c.b_empty[s], ((uint32_t)(it / p.sb) & 1u) ^ 1u, abort_flag, &g_err_tc)) break;
-                const int k = it % per_tile;
+            RingPos bs;
+            for (int k = 0; it < total; ++it, bs.next(p.sb), k = k + 1 == per_tile ? 0 : k + 1) {
+                const int s = bs.idx;
+                if (!mbar_wait_1t(&c.b_empty[s], bs.phase ^ 1u, abort_flag, &g_err_tc)) break;
                 uint8_t* dst = Bs + (size_t)s * kBStageBytes;
                 if (k < p.nkb) {
                     mbar_arrive_expect_tx(&c.b_full[s], qbytes);
@@ -245,15 +246,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t idesc1 = idesc_f16_f32(p.npad);
             const uint32_t idesc2 = idesc_bf16_f32(p.mpad);
             const uint32_t y_tmem = tmem, s_tmem = tmem + kSCol;
-            int ia = 0, ib = 0;
+            RingPos ra, rb;
             bool ok = true;
             for (int t = 0; t < cr.ntiles && ok; ++t) {
                 const uint32_t pt = (uint32_t)t & 1u;
                 // GEMM1: Y = X Q^T into columns [0, npad)
-                for (int kb = 0; kb < p.nkb; ++kb, ++ia, ++ib) {
-                    const int sa = ia % p.sa, sb = ib % p.sb;
-                    if (!mbar_wait(&c.a_full[sa], (uint32_t)(ia / p.sa) & 1u, abort_flag, &g_err_tc) ||
-                        !mbar_wait(&c.b_full[sb], (uint32_t)(ib / p.sb) & 1u, abort_flag, &g_err_tc)) {
+                for (int kb = 0; kb < p.nkb; ++kb, ra.next(p.sa), rb.next(p.sb)) {
+                    const int sa = ra.idx, sb = rb.idx;
+                    if (!mbar_wait_1t(&c.a_full[sa], ra.phase, abort_flag, &g_err_tc) ||
+                        !mbar_wait_1t(&c.b_full[sb], rb.phase, abort_flag, &g_err_tc)) {
                         ok = false;
                         break;
                     }
@@ -271,12 +272,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mma_commit(&c.y_full);
                 // GEMM2: S = Yh Rh + Yl Rh + Yh Rl into columns [256, 256 + mpad), once the
                 // epilogue has split Y in place and released the previous tile's S
-                if (!mbar_wait(&c.ysplit_full, pt, abort_flag, &g_err_tc) || !mbar_wait(&c.s_empty, pt ^ 1u, abort_flag, &g_err_tc)) break;
+                if (!mbar_wait_1t(&c.ysplit_full, pt, abort_flag, &g_err_tc) || !mbar_wait_1t(&c.s_empty, pt ^ 1u, abort_flag, &g_err_tc)) break;
                 tc_fence_after();
-                for (int kr = 0; kr < p.nkr; ++kr, ib += 2) {
-                    const int sh = ib % p.sb, sl = (ib + 1) % p.sb;
-                    if (!mbar_wait(&c.b_full[sh], (uint32_t)(ib / p.sb) & 1u, abort_flag, &g_err_tc) ||
-                        !mbar_wait(&c.b_full[sl], (uint32_t)((ib + 1) / p.sb) & 1u, abort_flag, &g_err_tc)) {
+                for (int kr = 0; kr < p.nkr; ++kr) {
+                    const int sh = rb.idx;
+                    const uint32_t ph = rb.phase;
+                    rb.next(p.sb);
+                    const int sl = rb.idx;
+                    const uint32_t pl = rb.phase;
+                    rb.next(p.sb);
+                    if (!mbar_wait_1t(&c.b_full[sh], ph, abort_flag, &g_err_tc) ||
+                        !mbar_wait_1t(&c.b_full[sl], pl, abort_flag, &g_err_tc)) {
                         ok = false;
                         break;
                     }
@@ -302,7 +308,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mma_commit(&c.s_full);
                 // the next tile's GEMM1 overwrites the columns GEMM2 reads: wait for it to finish
                 mma_commit(&c.gemm2_done);
-                if (!mbar_wait(&c.gemm2_done, pt, abort_flag, &g_err_tc)) break;
+                if (!mbar_wait_1t(&c.gemm2_done, pt, abort_flag, &g_err_tc)) break;
                 tc_fence_after();
             }
             // all MMAs issued by this thread complete before TMEM is released
@@ -321,19 +327,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int u = 0; u < kCvtRows; ++u) nrm[u] = 0.f;
         float amax = 0.f;
         int it = 0;
+        RingPos rx, ra;  // every K-block advances both rings; this group takes those with it % 2 == g
         bool ok = true;
         for (int t = 0; t < cr.ntiles && ok; ++t) {
             const TileRange tr = cr.tile(t);
             const int b = t & 1;
-            for (int kb = 0; kb < p.nkb; ++kb, ++it) {
+            for (int kb = 0; kb < p.nkb; ++kb, ++it, rx.next(p.sx), ra.next(p.sa)) {
                 if ((it & 1) != g) continue;
-                const int sx = it % p.sx, sa = it % p.sa;
-                if (!mbar_wait_warp(&c.x_full[sx], (uint32_t)(it / p.sx) & 1u, abort_flag, &g_err_tc) ||
-                    !mbar_wait_warp(&c.a_empty[sa], ((uint32_t)(it / p.sa) & 1u) ^ 1u, abort_flag, &g_err_tc)) {
+                const int sx = rx.idx, sa = ra.idx;
+                if (!mbar_wait_warp(&c.x_full[sx], rx.phase, abort_flag, &g_err_tc) ||
+                    !mbar_wait_warp(&c.a_empty[sa], ra.phase ^ 1u, abort_flag, &g_err_tc)) {
                     ok = false;
                     break;
                 }
-                const uint8_t* Xt = Xs + (size_t)sx * kXStageBytes;
+                const uint8_t* Xt = Xs + (size_t)sx * p.xstage;
                 uint8_t* At = As + (size_t)sa * kAStageBytes;
 #pragma unroll
                 for (int u = 0; u < kCvtRows; ++u) {
@@ -517,20 +524,30 @@ struct Rings {
     int sx, sa, sb;
 };
 
-size_t ps_smem_bytes(Rings g) {
-    return 1024 + (size_t)g.sx * kXStageBytes + (size_t)g.sa * kAStageBytes + (size_t)g.sb * kBStageBytes +
-           sizeof(Ctl);
+constexpr size_t kSmemCap = 227 * 1024;
+
+// bytes between fp32 X staging tiles of `box_rows` rows (SW128 operand areas follow: 1 KB aligned)
+int ps_xstage(int box_rows) { return (box_rows * kBK * 4 + 1023) / 1024 * 1024; }
+
+size_t ps_smem_bytes(Rings g, int xstage) {
+    return 1024 + (size_t)g.sx * xstage + (size_t)g.sa * kAStageBytes + (size_t)g.sb * kBStageBytes + sizeof(Ctl);
 }
 
-// deepest X staging ring that fits next to two A stages and two or more B stages
-Rings ps_rings() {
-    const size_t cap = 227 * 1024;
-    for (int sx = kMaxSX; sx >= 2; --sx)
+// Ring depths for X boxes of `box_rows` rows: the deepest X ring that fits, then the
+// deepest B ring.  The X depth must be even.  The two converter groups take alternate
+// K-blocks, so with an even depth every X stage belongs to one group, which waits on its
+// phases in order.  With an odd depth a stage alternates between the groups: one group
+// can reach the stage two phases on while the other group's load into it is still in
+// flight (TMA loads may land out of order), and the parity test would then pass on the
+// stage's older, completed phase and hand over stale data.
+Rings ps_rings(int box_rows) {
+    const int xs = ps_xstage(box_rows);
+    for (int sx = kMaxSX; sx >= 2; sx -= 2)
         for (int sb = kMaxSB; sb >= 2; --sb) {
             Rings g{sx, kMaxSA, sb};
-            if (ps_smem_bytes(g) <= cap) return g;
+            if (ps_smem_bytes(g, xs) <= kSmemCap) return g;
         }
-    return Rings{2, 2, 2};
+    return Rings{2, kMaxSA, 2};
 }
 
 }  // namespace
@@ -579,7 +596,7 @@ gs_status tc_prepare(gs_basis* h) {
         !make_tmap_2d(&h->tmap_rl, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, h->tc_Rl, mpad, npad, npad, kBK, mpad,
                       CU_TENSOR_MAP_SWIZZLE_128B))
         return GS_ERR_CUDA;
-    if (cudaFuncSetAttribute(k_ps_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ps_smem_bytes(ps_rings())) !=
+    if (cudaFuncSetAttribute(k_ps_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemCap) !=
         cudaSuccess)
         return GS_ERR_CUDA;
     // the fused kernel needs all of its threads resident in one CTA; otherwise the
@@ -602,7 +619,8 @@ cudaError_t launch_ps_tc(const gs_basis* h, const float* X, long long N, int ldx
     if (!make_tmap_2d(&tmx, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, X, N, h->D, ldx, kBK, box_rows,
                       CU_TENSOR_MAP_SWIZZLE_NONE))
         return cudaErrorInvalidValue;
-    const Rings g = ps_rings();
+    const Rings g = ps_rings(box_rows);
+    if (g.sx % kCvtGroups != 0 || g.sa % kCvtGroups != 0) return cudaErrorInvalidConfiguration;
     PsParams p;
     p.N = N;
     p.D = h->D;
@@ -616,6 +634,7 @@ cudaError_t launch_ps_tc(const gs_basis* h, const float* X, long long N, int ldx
     p.sa = g.sa;
     p.sb = g.sb;
     p.box_rows = box_rows;
+    p.xstage = ps_xstage(box_rows);
     p.cnorm = h->cnorm;
     p.mode = mode;
     p.scale = scale;
@@ -625,7 +644,7 @@ cudaError_t launch_ps_tc(const gs_basis* h, const float* X, long long N, int ldx
     p.lds = lds;
     p.argmax = argmax;
     p.maxval = maxval;
-    k_ps_tc<<<grid, kThreads, ps_smem_bytes(g), s>>>(tmx, h->tmap_q16, h->tmap_rh, h->tmap_rl, p);
+    k_ps_tc<<<grid, kThreads, ps_smem_bytes(g, p.xstage), s>>>(tmx, h->tmap_q16, h->tmap_rh, h->tmap_rl, p);
     return cudaGetLastError();
 }
 

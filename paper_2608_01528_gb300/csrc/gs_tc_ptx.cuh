@@ -64,6 +64,27 @@ static __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, vo
         }
     }
 }
+// The same bounded wait for a thread that runs alone (lane 0 of a producer or MMA
+// warp): a phase that has already completed costs one inline try_wait instead of a
+// call, which matters in issue loops that take two or three waits per K-block.
+// Warp-wide waits keep the call, so that every lane leaves through one return point.
+static __device__ __forceinline__ bool mbar_wait_1t(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                             unsigned* err_word) {
+    if (mbar_try_wait(bar, parity)) return true;
+    return mbar_wait(bar, parity, abort_flag, err_word);
+}
+// Position in a ring of mbarrier-guarded stages: slot index and the parity of its
+// current phase, advanced without integer division.
+struct RingPos {
+    int idx = 0;
+    uint32_t phase = 0;
+    __device__ __forceinline__ void next(int depth) {
+        if (++idx == depth) {
+            idx = 0;
+            phase ^= 1u;
+        }
+    }
+};
 // The same wait taken by a whole warp: every lane waits (each acquires the
 // barrier's phase) and the warp leaves only together, so .sync.aligned
 // instructions and warp shuffles after it always see a converged warp.
@@ -180,6 +201,23 @@ static __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+// 16 TMEM lanes x 32 columns in the 16x256b pattern: with t = lane id, v[4j], v[4j+1]
+// are lane (t/4), columns 8j + 2(t%4) and +1, and v[4j+2], v[4j+3] are lane (t/4 + 8),
+// the same columns (j = 0..3).  Four consecutive threads hold 8 consecutive columns of
+// one row, so stores from this layout write whole 32-byte sectors.
+static __device__ __forceinline__ void tmem_ld16x256b_x4(uint32_t taddr, float* v) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x256b.x4.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+          "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 // Stores 16 consecutive 32-bit columns of this thread's TMEM lane.
 static __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* v) {
