@@ -125,7 +125,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 item_bq(li, b, qt);
                 const uint32_t ph = ((uint32_t)li & 1u) ^ 1u;
                 for (int k = 0; k < p.nkb; ++k) {
-                    if (!mbar_wait(&c.q_empty[k], ph, abort_flag, err)) {
+                    if (!mbar_wait_1t(&c.q_empty[k], ph, abort_flag, err)) {
                         ok = false;
                         break;
                     }
@@ -144,17 +144,24 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint64_t pol = l2_policy_evict_last();
             const int total = nitems * units_per_item * p.nkb;
             int it = 0;
-            for (; it < total; ++it) {
-                const int s = it % kKStages;
-                if (!mbar_wait(&c.k_empty[s], ((uint32_t)(it / kKStages) & 1u) ^ 1u, abort_flag, err)) break;
-                const int kb = it % p.nkb;
-                const int unit = (it / p.nkb) % units_per_item;
-                const int li = it / (p.nkb * units_per_item);
-                int b, qt;
-                item_bq(li, b, qt);
-                const int nt = unit % p.ntiles;
+            RingPos ks;
+            int b = 0, qt = 0;
+            for (int kb = 0, unit = 0, nt = 0, li = 0; it < total; ++it, ks.next(kKStages)) {
+                const int s = ks.idx;
+                if (!mbar_wait_1t(&c.k_empty[s], ks.phase ^ 1u, abort_flag, err)) break;
+                if (kb == 0 && unit == 0) item_bq(li, b, qt);
                 mbar_arrive_expect_tx(&c.k_full[s], kKStageBytes);
                 tma_load_2d(Ks + (size_t)s * kKStageBytes, &tmap_k, &c.k_full[s], kb * kBK, b * p.Lk + nt * kBN, pol);
+                // next (item, unit, K-block); units run over the key tiles once per pass
+                if (++kb == p.nkb) {
+                    kb = 0;
+                    if (++nt == p.ntiles) nt = 0;
+                    if (++unit == units_per_item) {
+                        unit = 0;
+                        nt = 0;
+                        ++li;
+                    }
+                }
             }
             for (int j = std::max(0, it - kKStages); j < it; ++j)
                 mbar_drain(&c.k_full[j % kKStages], (uint32_t)(j / kKStages) & 1u, err);
@@ -163,22 +170,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------------- MMA issue
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16_f32(kBN);
-            int it = 0, gu = 0;
+            int gu = 0;
+            RingPos ks;
             bool ok = true;
             for (int li = 0; li < nitems && ok; ++li) {
                 const uint32_t qph = (uint32_t)li & 1u;
                 for (int u = 0; u < units_per_item && ok; ++u, ++gu) {
                     const int buf = gu & 1;
-                    if (!mbar_wait(&c.d_empty[buf], ((uint32_t)(gu >> 1) & 1u) ^ 1u, abort_flag, err)) {
+                    if (!mbar_wait_1t(&c.d_empty[buf], ((uint32_t)(gu >> 1) & 1u) ^ 1u, abort_flag, err)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
                     const uint32_t d_tmem = tmem + (uint32_t)(buf * kBN);
-                    for (int kb = 0; kb < p.nkb; ++kb, ++it) {
-                        const int s = it % kKStages;
-                        if ((u == 0 && !mbar_wait(&c.q_full[kb], qph, abort_flag, err)) ||
-                            !mbar_wait(&c.k_full[s], (uint32_t)(it / kKStages) & 1u, abort_flag, err)) {
+                    for (int kb = 0; kb < p.nkb; ++kb, ks.next(kKStages)) {
+                        const int s = ks.idx;
+                        if ((u == 0 && !mbar_wait_1t(&c.q_full[kb], qph, abort_flag, err)) ||
+                            !mbar_wait_1t(&c.k_full[s], ks.phase, abort_flag, err)) {
                             ok = false;
                             break;
                         }

@@ -143,15 +143,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             const uint64_t pol = l2_policy_evict_first();
             int it = 0;
-            for (; it < total_it; ++it) {
-                const int s = it % p.sx;
-                if (!mbar_wait(&c.x_empty[s], ((uint32_t)(it / p.sx) & 1u) ^ 1u, abort_flag, err)) break;
-                long long tm;
-                int tn;
-                tile_mn(it / p.nkb, tm, tn);
+            RingPos xs;
+            long long tm = 0;
+            int tn = 0;
+            for (int kb = 0, lt = 0; it < total_it; ++it, xs.next(p.sx)) {
+                const int s = xs.idx;
+                if (!mbar_wait_1t(&c.x_empty[s], xs.phase ^ 1u, abort_flag, err)) break;
+                if (kb == 0) tile_mn(lt, tm, tn);
                 mbar_arrive_expect_tx(&c.x_full[s], kXStageBytes);
-                tma_load_2d(Xs + (size_t)s * kXStageBytes, &tmap_a, &c.x_full[s], (it % p.nkb) * kBK,
-                            (int)(tm * kBM), pol);
+                tma_load_2d(Xs + (size_t)s * kXStageBytes, &tmap_a, &c.x_full[s], kb * kBK, (int)(tm * kBM), pol);
+                if (++kb == p.nkb) {
+                    kb = 0;
+                    ++lt;
+                }
             }
             for (int j = std::max(0, it - p.sx); j < it; ++j) mbar_drain(&c.x_full[j % p.sx], (uint32_t)(j / p.sx) & 1u, err);
         }
@@ -162,16 +166,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t bytes = (uint32_t)p.nt * kBK * 2;
             const int total = total_it * p.nb;
             int ib = 0;
-            for (; ib < total; ++ib) {
-                const int s = ib % p.sb;
-                if (!mbar_wait(&c.b_empty[s], ((uint32_t)(ib / p.sb) & 1u) ^ 1u, abort_flag, err)) break;
-                const int it = ib / p.nb, which = ib % p.nb;
-                long long tm;
-                int tn;
-                tile_mn(it / p.nkb, tm, tn);
+            RingPos bs;
+            long long tm = 0;
+            int tn = 0;
+            for (int which = 0, kb = 0, lt = 0; ib < total; ++ib, bs.next(p.sb)) {
+                const int s = bs.idx;
+                if (!mbar_wait_1t(&c.b_empty[s], bs.phase ^ 1u, abort_flag, err)) break;
+                if (kb == 0 && which == 0) tile_mn(lt, tm, tn);
                 mbar_arrive_expect_tx(&c.b_full[s], bytes);
-                tma_load_2d(Bs + (size_t)s * kBStageBytes, which ? &tmap_b1 : &tmap_b0, &c.b_full[s],
-                            (it % p.nkb) * kBK, tn * p.nt, pol);
+                tma_load_2d(Bs + (size_t)s * kBStageBytes, which ? &tmap_b1 : &tmap_b0, &c.b_full[s], kb * kBK,
+                            tn * p.nt, pol);
+                if (++which == p.nb) {
+                    which = 0;
+                    if (++kb == p.nkb) {
+                        kb = 0;
+                        ++lt;
+                    }
+                }
             }
             for (int j = std::max(0, ib - p.sb); j < ib; ++j) mbar_drain(&c.b_full[j % p.sb], (uint32_t)(j / p.sb) & 1u, err);
         }
@@ -179,29 +190,33 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------------- MMA issue
         if (lane == 0) {
             const uint32_t idesc = p.amode == kAF16 ? idesc_f16_f32(p.nt) : idesc_bf16_f32(p.nt);
-            int it = 0, ib = 0;
+            RingPos ra, rb;
             bool ok = true;
             for (int lt = 0; lt < ntiles && ok; ++lt) {
                 const int buf = lt & 1;
-                if (!mbar_wait(&c.d_empty[buf], ((uint32_t)(lt >> 1) & 1u) ^ 1u, abort_flag, err)) break;
+                if (!mbar_wait_1t(&c.d_empty[buf], ((uint32_t)(lt >> 1) & 1u) ^ 1u, abort_flag, err)) break;
                 tc_fence_after();
                 const uint32_t d_tmem = tmem + (uint32_t)(buf * 256);
-                for (int kb = 0; kb < p.nkb; ++kb, ++it) {
-                    const int sa = it % p.sa;
-                    if (!mbar_wait(&c.a_full[sa], (uint32_t)(it / p.sa) & 1u, abort_flag, err)) {
+                for (int kb = 0; kb < p.nkb; ++kb, ra.next(p.sa)) {
+                    const int sa = ra.idx;
+                    if (!mbar_wait_1t(&c.a_full[sa], ra.phase, abort_flag, err)) {
                         ok = false;
                         break;
                     }
-                    int sb[2];
-                    for (int w = 0; w < p.nb; ++w, ++ib) {
-                        sb[w] = ib % p.sb;
-                        if (!mbar_wait(&c.b_full[sb[w]], (uint32_t)(ib / p.sb) & 1u, abort_flag, err)) ok = false;
+                    const int sb0 = rb.idx;
+                    if (!mbar_wait_1t(&c.b_full[sb0], rb.phase, abort_flag, err)) ok = false;
+                    rb.next(p.sb);
+                    int sb1 = sb0;
+                    if (p.nb == 2) {
+                        sb1 = rb.idx;
+                        if (ok && !mbar_wait_1t(&c.b_full[sb1], rb.phase, abort_flag, err)) ok = false;
+                        rb.next(p.sb);
                     }
                     if (!ok) break;
                     tc_fence_after();
                     const uint8_t* At = As + (size_t)sa * p.parts * kAPartBytes;
                     const uint64_t ah = sdesc_sw128(smem_u32(At));
-                    const uint64_t b0 = sdesc_sw128(smem_u32(Bs + (size_t)sb[0] * kBStageBytes));
+                    const uint64_t b0 = sdesc_sw128(smem_u32(Bs + (size_t)sb0 * kBStageBytes));
                     if (p.amode == kAF16) {
 #pragma unroll
                         for (int k = 0; k < kBK / 16; ++k)
@@ -209,7 +224,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                        (kb | k) != 0 ? 1u : 0u);
                     } else {
                         const uint64_t al = sdesc_sw128(smem_u32(At + kAPartBytes));
-                        const uint64_t b1 = sdesc_sw128(smem_u32(Bs + (size_t)sb[1] * kBStageBytes));
+                        const uint64_t b1 = sdesc_sw128(smem_u32(Bs + (size_t)sb1 * kBStageBytes));
 #pragma unroll
                         for (int k = 0; k < kBK / 16; ++k) {
                             mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
@@ -219,7 +234,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     }
                     mma_commit(&c.a_empty[sa]);
-                    for (int w = 0; w < p.nb; ++w) mma_commit(&c.b_empty[sb[w]]);
+                    mma_commit(&c.b_empty[sb0]);
+                    if (p.nb == 2) mma_commit(&c.b_empty[sb1]);
                 }
                 if (ok) mma_commit(&c.d_full[buf]);
             }
@@ -232,11 +248,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int l = threadIdx.x - (kCvt0 + g * kCvtGroupWarps) * 32;  // 0..127
         const int c4 = l & 15, rbase = l >> 4;
         float amax = 0.f;
+        // ring positions of K-block g, then advanced by the two groups' K-blocks each step
+        RingPos rx, ra;
+        for (int j = 0; j < g; ++j) {
+            rx.next(p.sx);
+            ra.next(p.sa);
+        }
         for (int it = g; it < total_it; it += kCvtGroups) {
-            const int sx = it % p.sx, sa = it % p.sa;
-            if (!mbar_wait_warp(&c.x_full[sx], (uint32_t)(it / p.sx) & 1u, abort_flag, err) ||
-                !mbar_wait_warp(&c.a_empty[sa], ((uint32_t)(it / p.sa) & 1u) ^ 1u, abort_flag, err))
+            const int sx = rx.idx, sa = ra.idx;
+            if (!mbar_wait_warp(&c.x_full[sx], rx.phase, abort_flag, err) ||
+                !mbar_wait_warp(&c.a_empty[sa], ra.phase ^ 1u, abort_flag, err))
                 break;
+            for (int j = 0; j < kCvtGroups; ++j) {
+                rx.next(p.sx);
+                ra.next(p.sa);
+            }
             const uint8_t* Xt = Xs + (size_t)sx * kXStageBytes;
             uint8_t* At = As + (size_t)sa * p.parts * kAPartBytes;
 #pragma unroll 4
@@ -369,12 +395,15 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     p.amode = a.split ? kABF16X2 : kAF16;
     p.nb = a.split ? 2 : 1;
     p.parts = a.split ? 2 : 1;
-    // deepest staging that fits: two A stages, B stages for at least one K-block (+1)
+    // deepest staging that fits: two A stages, B stages for at least one K-block (+1).
+    // The X depth stays even: the two converter groups take alternate K-blocks, and with
+    // an even depth each X stage belongs to one group, which waits on its phases in order
+    // (on an odd-depth ring a group could pass a parity test on a stage's older phase).
     const size_t cap = 227 * 1024;
     p.sa = 2;
     p.sx = 2;
     p.sb = 2 * p.nb;
-    for (int sx = kMaxSX; sx >= 2; --sx) {
+    for (int sx = kMaxSX / 2 * 2; sx >= 2; sx -= 2) {
         bool done = false;
         for (int sb = kMaxSB; sb >= p.nb + 1; --sb)
             if (gemm_smem_bytes(sx, p.sa, p.parts, sb) <= cap) {

@@ -399,27 +399,36 @@ __global__ void __launch_bounds__(kThreads, 1)
             const TileRange tr = cr.tile(t);
             const bool valid = i < tr.nrows;
             const long long row = tr.row0 + i;
-            // split Y in place: chunk of 16 fp32 columns -> 8 columns bf16(Y) + 8 columns bf16(Y - bf16(Y))
-            for (int jc = 0; jc < p.npad; jc += 16) {
-                float y[16];
-                tmem_ld16(ty + (uint32_t)jc, y);
+            // split Y in place: chunk of 16 fp32 columns -> 8 columns bf16(Y) + 8 columns
+            // bf16(Y - bf16(Y)).  This runs between GEMM1 and GEMM2 of the tile, with the
+            // tensor pipe idle, so columns are read 32 at a time (one TMEM load wait each).
+            for (int jc = 0; jc < p.npad; jc += 32) {
+                const int w = p.npad - jc >= 32 ? 32 : 16;
+                float y[32];
+                if (w == 32)
+                    tmem_ld32(ty + (uint32_t)jc, y);
+                else
+                    tmem_ld16(ty + (uint32_t)jc, y);
                 if (p.Y && valid) {
                     float* dst = p.Y + (size_t)row * p.ldy + jc;
 #pragma unroll
-                    for (int j = 0; j < 16; ++j)
-                        if (jc + j < p.r) dst[j] = y[j];
+                    for (int j = 0; j < 32; ++j)
+                        if (j < w && jc + j < p.r) dst[j] = y[j];
                 }
-                uint32_t hi[8], lo[8];
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    const float a = y[2 * j], bb = y[2 * j + 1];
-                    const float ah = __bfloat162float(__float2bfloat16_rn(a));
-                    const float bh = __bfloat162float(__float2bfloat16_rn(bb));
-                    hi[j] = pack_bf16(ah, bh);
-                    lo[j] = pack_bf16(a - ah, bb - bh);
+                for (int h = 0; h < 2; ++h) {
+                    if (h * 16 >= w) break;
+                    uint32_t hl[16];  // 8 columns of packed hi, then 8 of packed lo
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const float a = y[16 * h + 2 * j], bb = y[16 * h + 2 * j + 1];
+                        const float ah = __bfloat162float(__float2bfloat16_rn(a));
+                        const float bh = __bfloat162float(__float2bfloat16_rn(bb));
+                        hl[j] = pack_bf16(ah, bh);
+                        hl[8 + j] = pack_bf16(a - ah, bb - bh);
+                    }
+                    tmem_st16(ty + (uint32_t)(jc + 16 * h), hl);
                 }
-                tmem_st8(ty + (uint32_t)jc, hi);
-                tmem_st8(ty + (uint32_t)(jc + 8), lo);
             }
             tmem_wait_st();
             tc_fence_before();
