@@ -34,7 +34,10 @@ struct gs_basis {
     // tc_npad, zero padded), Rh = bf16(R) and Rl = bf16(R - Rh), with tensor maps
     void* tc_Rh = nullptr;
     void* tc_Rl = nullptr;
-    CUtensorMap tmap_rh, tmap_rl;   // boxes of tc_mpad rows (fused kernel only, M <= 256)
+    CUtensorMap tmap_rh, tmap_rl;   // boxes of tc_half_rows rows (fused kernel only, M <= 256)
+    // the fused kernel runs S = Y R^T in halves of tc_half_rows codewords (min(tc_mpad, 128));
+    // R is lower echelon, so half h needs only its first tc_nkr_half[h] K-blocks of 64
+    int tc_nh = 0, tc_half_rows = 0, tc_nkr_half[2] = {0, 0};
     int tc_npad = 0, tc_mpad = 0;
     // R^T split the same way (tc_npad x tc_mpad), the B operand of V = P R
     void* tc_Rth = nullptr;

@@ -18,8 +18,13 @@
 //                      accumulator in TMEM columns [256, 512).  The epilogue
 //                      splits Y in place in TMEM (each 16-column fp32 chunk
 //                      becomes 8 columns of packed Yh and 8 of packed Yl), and
-//                      the MMA reads that A operand straight from TMEM; the Rh /
-//                      Rl tiles come through the same TMA ring as the Q tiles.
+//                      the MMA reads that A operand straight from TMEM.  S runs
+//                      in halves of up to 128 codewords; one B-ring slot holds
+//                      one K-block of both Rh and Rl of a half, so each slot is
+//                      consumed on its own and the next one loads meanwhile.
+//                      Gram-Schmidt leaves R lower echelon (codeword i has no
+//                      component past the basis vectors built before it), so a
+//                      half stops at the K-block holding its last nonzero.
 //                      A single fp16/tf32 rounding would not do here: the
 //                      dominant terms of S are single products Y_i R_ii.
 //   epilogue           scale / cosine (full-D ||x|| accumulated by the
@@ -80,6 +85,7 @@ constexpr int kAStageBytes = kBM * kBK * 2;          // 16 KB fp16 operand tile
 constexpr int kBStageBytes = 256 * kBK * 2;          // 32 KB: up to 256 rows of one B operand K-block
 constexpr int kMaxSX = 6, kMaxSA = 2, kMaxSB = 4;
 constexpr int kTmemCols = 512;
+constexpr int kMaxKR = 4;            // K-blocks of 64 in r <= 256
 constexpr int kSCol = 256;           // first TMEM column of the score accumulator
 
 // ----------------------------------------------------------------- work split
@@ -112,7 +118,8 @@ struct CtaRows {
 
 struct PsParams {
     long long N;
-    int D, r, npad, M, mpad, nkb, nkr;
+    int D, r, npad, M, mpad, nkb;
+    int nh, half_rows, nkr_h[2];  // GEMM2: halves of codewords, K-blocks of R each half needs
     int sx, sa, sb;         // ring depths: fp32 X staging, fp16 A, B operand tiles
     int box_rows;           // rows of each X TMA box (>= every tile's rows)
     int xstage;             // bytes between X staging tiles (box_rows x 256, 1 KB aligned)
@@ -131,7 +138,8 @@ struct Ctl {
     uint64_t x_full[kMaxSX], x_empty[kMaxSX];
     uint64_t a_full[kMaxSA], a_empty[kMaxSA];
     uint64_t b_full[kMaxSB], b_empty[kMaxSB];
-    uint64_t y_full, ysplit_full, s_full, s_empty, gemm2_done;
+    uint64_t y_full, s_full, s_empty, gemm2_done;
+    uint64_t ysplit[kMaxKR];  // Y columns [64 k, 64 k + 64) split in TMEM (GEMM2 K-block k may start)
     uint64_t xn_full[2], xn_empty[2];
     uint64_t mma_done;
     float xn[2][kBM];  // ||x||^2 per row, both converter groups add into it
@@ -170,7 +178,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&c.b_empty[s], 1);
         }
         mbar_init(&c.y_full, 1);
-        mbar_init(&c.ysplit_full, kEpiWarps);
+        for (int k = 0; k < kMaxKR; ++k) mbar_init(&c.ysplit[k], kEpiWarps);
         mbar_init(&c.s_full, 1);
         mbar_init(&c.s_empty, kEpiWarps);
         mbar_init(&c.gemm2_done, 1);
@@ -217,11 +225,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp == kBWarp) {
         // ------------------------------------------------------------- B operand tiles via TMA:
-        // per tile, nkb Q tiles (GEMM1), then nkr pairs of Rh / Rl tiles (GEMM2)
+        // per tile, nkb Q tiles (GEMM1), then per half of the codewords its K-blocks of
+        // Rh and Rl, both in one slot (GEMM2)
         if (lane == 0) {
             const uint64_t pol = l2_policy_evict_last();
-            const uint32_t qbytes = (uint32_t)p.npad * kBK * 2, rbytes = (uint32_t)p.mpad * kBK * 2;
-            const int per_tile = p.nkb + 2 * p.nkr;
+            const uint32_t qbytes = (uint32_t)p.npad * kBK * 2, rbytes = 2u * (uint32_t)p.half_rows * kBK * 2;
+            const uint32_t rl_off = (uint32_t)p.half_rows * kBK * 2;  // Rl after Rh in the slot
+            const int per_tile = p.nkb + p.nkr_h[0] + p.nkr_h[1];
             const int total = cr.ntiles * per_tile;
             int it = 0;
             RingPos bs;
@@ -233,9 +243,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mbar_arrive_expect_tx(&c.b_full[s], qbytes);
                     tma_load_2d(dst, &tmap_q, &c.b_full[s], k * kBK, 0, pol);
                 } else {
-                    const int kr = (k - p.nkb) >> 1;
+                    const int j = k - p.nkb;
+                    const int h = j < p.nkr_h[0] ? 0 : 1;
+                    const int kr = h ? j - p.nkr_h[0] : j;
                     mbar_arrive_expect_tx(&c.b_full[s], rbytes);
-                    tma_load_2d(dst, ((k - p.nkb) & 1) ? &tmap_rl : &tmap_rh, &c.b_full[s], kr * kBK, 0, pol);
+                    tma_load_2d(dst, &tmap_rh, &c.b_full[s], kr * kBK, h * p.half_rows, pol);
+                    tma_load_2d(dst + rl_off, &tmap_rl, &c.b_full[s], kr * kBK, h * p.half_rows, pol);
                 }
             }
             for (int j = std::max(0, it - p.sb); j < it; ++j) mbar_drain(&c.b_full[j % p.sb], (uint32_t)(j / p.sb) & 1u, &g_err_tc);
@@ -244,7 +257,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------------- MMA issue
         if (lane == 0) {
             const uint32_t idesc1 = idesc_f16_f32(p.npad);
-            const uint32_t idesc2 = idesc_bf16_f32(p.mpad);
+            const uint32_t idesc2 = idesc_bf16_f32(p.half_rows);
             const uint32_t y_tmem = tmem, s_tmem = tmem + kSCol;
             RingPos ra, rb;
             bool ok = true;
@@ -272,37 +285,36 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mma_commit(&c.y_full);
                 // GEMM2: S = Yh Rh + Yl Rh + Yh Rl into columns [256, 256 + mpad), once the
                 // epilogue has split Y in place and released the previous tile's S
-                if (!mbar_wait_1t(&c.ysplit_full, pt, abort_flag, &g_err_tc) || !mbar_wait_1t(&c.s_empty, pt ^ 1u, abort_flag, &g_err_tc)) break;
-                tc_fence_after();
-                for (int kr = 0; kr < p.nkr; ++kr) {
-                    const int sh = rb.idx;
-                    const uint32_t ph = rb.phase;
-                    rb.next(p.sb);
-                    const int sl = rb.idx;
-                    const uint32_t pl = rb.phase;
-                    rb.next(p.sb);
-                    if (!mbar_wait_1t(&c.b_full[sh], ph, abort_flag, &g_err_tc) ||
-                        !mbar_wait_1t(&c.b_full[sl], pl, abort_flag, &g_err_tc)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint64_t rh = sdesc_sw128(smem_u32(Bs + (size_t)sh * kBStageBytes));
-                    const uint64_t rl = sdesc_sw128(smem_u32(Bs + (size_t)sl * kBStageBytes));
+                if (!mbar_wait_1t(&c.s_empty, pt ^ 1u, abort_flag, &g_err_tc)) break;
+                int nsplit = 0;  // K-blocks of Y known to be split; the epilogue signals each one
+                for (int h = 0; h < p.nh && ok; ++h) {
+                    const uint32_t s_half = s_tmem + (uint32_t)(h * p.half_rows);
+                    for (int kr = 0; kr < p.nkr_h[h]; ++kr, rb.next(p.sb)) {
+                        for (; nsplit <= kr && ok; ++nsplit)
+                            ok = mbar_wait_1t(&c.ysplit[nsplit], pt, abort_flag, &g_err_tc);
+                        const int sr = rb.idx;
+                        if (!ok || !mbar_wait_1t(&c.b_full[sr], rb.phase, abort_flag, &g_err_tc)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t rs = smem_u32(Bs + (size_t)sr * kBStageBytes);
+                        const uint64_t rh = sdesc_sw128(rs);
+                        const uint64_t rl = sdesc_sw128(rs + (uint32_t)p.half_rows * kBK * 2);
 #pragma unroll
-                    for (int k = 0; k < kBK / 16; ++k) {
-                        // r columns [64 kr + 16 k, +16) were split into TMEM columns
-                        // [16 kk, 16 kk + 8) (Yh) and [16 kk + 8, 16 kk + 16) (Yl), kk = 4 kr + k
-                        const int kk = 4 * kr + k;
-                        if (16 * kk >= p.npad) break;  // past r: no split columns there
-                        const uint32_t a_hi = y_tmem + (uint32_t)(16 * kk);
-                        const uint32_t a_lo = a_hi + 8;
-                        mma_bf16_ts(s_tmem, a_hi, rh + (uint64_t)(2 * k), idesc2, (kr | k) != 0 ? 1u : 0u);
-                        mma_bf16_ts(s_tmem, a_lo, rh + (uint64_t)(2 * k), idesc2, 1u);
-                        mma_bf16_ts(s_tmem, a_hi, rl + (uint64_t)(2 * k), idesc2, 1u);
+                        for (int k = 0; k < kBK / 16; ++k) {
+                            // r columns [64 kr + 16 k, +16) were split into TMEM columns
+                            // [16 kk, 16 kk + 8) (Yh) and [16 kk + 8, 16 kk + 16) (Yl), kk = 4 kr + k
+                            const int kk = 4 * kr + k;
+                            if (16 * kk >= p.npad) break;  // past r: no split columns there
+                            const uint32_t a_hi = y_tmem + (uint32_t)(16 * kk);
+                            const uint32_t a_lo = a_hi + 8;
+                            mma_bf16_ts(s_half, a_hi, rh + (uint64_t)(2 * k), idesc2, (kr | k) != 0 ? 1u : 0u);
+                            mma_bf16_ts(s_half, a_lo, rh + (uint64_t)(2 * k), idesc2, 1u);
+                            mma_bf16_ts(s_half, a_hi, rl + (uint64_t)(2 * k), idesc2, 1u);
+                        }
+                        mma_commit(&c.b_empty[sr]);
                     }
-                    mma_commit(&c.b_empty[sh]);
-                    mma_commit(&c.b_empty[sl]);
                 }
                 if (!ok) break;
                 mma_commit(&c.s_full);
@@ -400,8 +412,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool valid = i < tr.nrows;
             const long long row = tr.row0 + i;
             // split Y in place: chunk of 16 fp32 columns -> 8 columns bf16(Y) + 8 columns
-            // bf16(Y - bf16(Y)).  This runs between GEMM1 and GEMM2 of the tile, with the
-            // tensor pipe idle, so columns are read 32 at a time (one TMEM load wait each).
+            // bf16(Y - bf16(Y)), read 32 columns per TMEM load wait.  Each finished K-block
+            // of 64 columns is signalled on its own, so GEMM2 starts on it while the rest
+            // of Y is still being split.
             for (int jc = 0; jc < p.npad; jc += 32) {
                 const int w = p.npad - jc >= 32 ? 32 : 16;
                 float y[32];
@@ -429,11 +442,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     tmem_st16(ty + (uint32_t)(jc + 16 * h), hl);
                 }
+                if (((jc + 32) & 63) == 0 || jc + 32 >= p.npad) {  // K-block jc / 64 is split
+                    tmem_wait_st();
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&c.ysplit[jc >> 6]);
+                }
             }
-            tmem_wait_st();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&c.ysplit_full);
             if (!mbar_wait_warp(&c.xn_full[b], (uint32_t)(t >> 1) & 1u, abort_flag, &g_err_tc)) break;
             const float xnorm = sqrtf(c.xn[b][i]);
             c.xn[b][i] = 0.f;  // ready for the tile after next (both groups add into it)
@@ -446,6 +461,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int ic = 0; ic < p.mpad; ic += 16) {
                 float sv[16];
                 tmem_ld16(ts + (uint32_t)ic, sv);
+                if (p.nkr_h[ic >= p.half_rows ? 1 : 0] == 0) {  // a half with no nonzero R: S = 0
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) sv[j] = 0.f;
+                }
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {
                     const int ci = ic + j;
@@ -598,12 +617,26 @@ gs_status tc_prepare(gs_basis* h) {
     h->has_split = true;
     // the fused kernel keeps Y (r <= 256 columns) and S (M <= 256 columns) in TMEM
     if (h->r > 256 || h->M > 256) return GS_OK;
+    // GEMM2 halves: up to 128 codewords each; K-blocks per half from the last nonzero of R
+    h->tc_half_rows = mpad > 128 ? 128 : mpad;
+    h->tc_nh = (mpad + h->tc_half_rows - 1) / h->tc_half_rows;
+    {
+        std::vector<int> rl((size_t)h->M);
+        if (cudaMemcpy(rl.data(), h->rlen, sizeof(int) * (size_t)h->M, cudaMemcpyDeviceToHost) != cudaSuccess)
+            return GS_ERR_CUDA;
+        for (int hh = 0; hh < 2; ++hh) {
+            int last = 0;
+            for (int i = hh * h->tc_half_rows; hh < h->tc_nh && i < std::min(h->M, (hh + 1) * h->tc_half_rows); ++i)
+                last = std::max(last, rl[(size_t)i]);
+            h->tc_nkr_half[hh] = (last + kBK - 1) / kBK;
+        }
+    }
     if (!make_tmap_2d(&h->tmap_q16, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, h->Q16, h->r, h->D, h->ldq16, kBK, npad,
                       CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_tmap_2d(&h->tmap_rh, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, h->tc_Rh, mpad, npad, npad, kBK, mpad,
-                      CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_tmap_2d(&h->tmap_rl, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, h->tc_Rl, mpad, npad, npad, kBK, mpad,
-                      CU_TENSOR_MAP_SWIZZLE_128B))
+        !make_tmap_2d(&h->tmap_rh, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, h->tc_Rh, mpad, npad, npad, kBK,
+                      h->tc_half_rows, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_tmap_2d(&h->tmap_rl, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, h->tc_Rl, mpad, npad, npad, kBK,
+                      h->tc_half_rows, CU_TENSOR_MAP_SWIZZLE_128B))
         return GS_ERR_CUDA;
     if (cudaFuncSetAttribute(k_ps_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemCap) !=
         cudaSuccess)
@@ -638,7 +671,10 @@ cudaError_t launch_ps_tc(const gs_basis* h, const float* X, long long N, int ldx
     p.M = h->M;
     p.mpad = h->tc_mpad;
     p.nkb = (h->D + kBK - 1) / kBK;
-    p.nkr = (h->tc_npad + kBK - 1) / kBK;
+    p.nh = h->tc_nh;
+    p.half_rows = h->tc_half_rows;
+    p.nkr_h[0] = h->tc_nkr_half[0];
+    p.nkr_h[1] = h->tc_nkr_half[1];
     p.sx = g.sx;
     p.sa = g.sa;
     p.sb = g.sb;
