@@ -17,9 +17,11 @@
 // exp(scale s - max) / sum.  The logits never go to HBM; the price is twice the
 // MMA work (the tensor pipe has the headroom: the output write bounds it).
 //
-// Warp roles (224 threads): 0-3 epilogue (warp w owns TMEM lanes 32w..+31 =
-// query rows), 4 TMA producer of query K-blocks, 5 TMEM allocator + MMA issuer,
-// 6 TMA producer of key tiles.  Every mbarrier wait is bounded.
+// Warp roles (352 threads): 0-7 epilogue (warp w reads TMEM lanes 32 (w % 4)..+31 =
+// query rows, and keys [128 (w / 4), +128) of each 256-key unit; the two warps of a
+// lane quadrant merge their row statistics between the passes through shared
+// memory), 8 TMA producer of query K-blocks, 9 TMEM allocator + MMA issuer, 10 TMA
+// producer of key tiles.  Every mbarrier wait is bounded.
 
 #include <float.h>
 
@@ -42,9 +44,9 @@ constexpr int kMaxKB = 8;         // r <= 512
 constexpr int kQBlockBytes = kBM * kBK * 2;   // 16 KB
 constexpr int kKStageBytes = kBN * kBK * 2;   // 32 KB
 constexpr int kKStages = 3;
-constexpr int kEpiWarps = 4;
-constexpr int kQWarp = 4, kMmaWarp = 5, kKWarp = 6;
-constexpr int kThreads = 7 * 32;
+constexpr int kEpiWarps = 8;        // two per TMEM lane quadrant, each half of the keys of a unit
+constexpr int kQWarp = 8, kMmaWarp = 9, kKWarp = 10;
+constexpr int kThreads = 11 * 32;
 constexpr int kTmemCols = 512;
 
 struct AttnParams {
@@ -60,7 +62,9 @@ struct Ctl {
     uint64_t q_full[kMaxKB], q_empty[kMaxKB];
     uint64_t k_full[kKStages], k_empty[kKStages];
     uint64_t d_full[2], d_empty[2];
+    uint64_t st_part, st_merged;  // row statistics: second key half posted / merged result posted
     uint64_t mma_done;
+    float st_m[kBM], st_l[kBM];   // per query row: max and sum of exponentials being merged
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -95,6 +99,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&c.d_full[b], 1);
             mbar_init(&c.d_empty[b], kEpiWarps);
         }
+        mbar_init(&c.st_part, kEpiWarps / 2);
+        mbar_init(&c.st_merged, kEpiWarps / 2);
         mbar_init(&c.mma_done, 1);
         c.abort_flag = 0;
         fence_barrier_init();
@@ -209,12 +215,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp < kEpiWarps) {
         // ------------------------------------------------------------- epilogue
-        // Statistics pass: TMEM read one row per thread (32x32b), online max / sum.
+        // Statistics pass: TMEM read one row per thread (32x32b), online max / sum over
+        // this warp's half of the keys; the halves are merged before the writing pass.
         // Writing pass: TMEM read in the 16x256b pattern (a quad of threads holds 8
         // consecutive keys of one row, so stores write whole sectors); each row's
         // max and sum come by shuffle from the thread that owned the row.
-        const int i = threadIdx.x;  // query row within the item (statistics pass)
-        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        const int quad = warp & 3, kh = warp >> 2;  // lane quadrant, key half of each unit
+        const int i = quad * 32 + lane;             // query row within the item (statistics pass)
+        const int c0 = kh * (kBN / 2);              // first column of this warp's key half
+        const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
         int gu = 0;
         for (int li = 0; li < nitems; ++li) {
             int b, qt;
@@ -230,9 +239,38 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_after();
                 const int nt = u % p.ntiles;
+                if (p.passes == 2 && u == p.ntiles) {
+                    // merge the two key halves' statistics of each row (max, rescaled sums)
+                    const uint32_t ph = (uint32_t)li & 1u;
+                    if (kh == 1) {
+                        c.st_m[i] = m;
+                        c.st_l[i] = l;
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&c.st_part);
+                        if (!mbar_wait_warp(&c.st_merged, ph, abort_flag, err)) {
+                            ok = false;
+                            break;
+                        }
+                        m = c.st_m[i];
+                        l = c.st_l[i];
+                    } else {
+                        if (!mbar_wait_warp(&c.st_part, ph, abort_flag, err)) {
+                            ok = false;
+                            break;
+                        }
+                        const float m1 = c.st_m[i], l1 = c.st_l[i];
+                        const float mm = fmaxf(m, m1);
+                        l = l * __expf(m - mm) + l1 * __expf(m1 - mm);
+                        m = mm;
+                        c.st_m[i] = m;
+                        c.st_l[i] = l;
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&c.st_merged);
+                    }
+                }
                 if (p.passes == 2 && u < p.ntiles) {
                     const uint32_t tb = tmem + lane_base + (uint32_t)(buf * kBN);
-                    for (int jc = 0; jc < kBN; jc += 16) {
+                    for (int jc = c0; jc < c0 + kBN / 2; jc += 16) {
                         float v[16];
                         tmem_ld16(tb + (uint32_t)jc, v);
                         const int k0 = nt * kBN + jc;
@@ -260,11 +298,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                         float* arow[2];
 #pragma unroll
                         for (int h = 0; h < 2; ++h) {
-                            qrow[h] = qt * kBM + warp * 32 + r0 + 8 * h;
+                            qrow[h] = qt * kBM + quad * 32 + r0 + 8 * h;
                             arow[h] = p.A + ((size_t)b * p.Lq + (qrow[h] < p.Lq ? qrow[h] : 0)) * p.Lk;
                         }
-                        const uint32_t tb = tmem + ((uint32_t)(warp * 32 + half * 16) << 16) + (uint32_t)(buf * kBN);
-                        for (int jc = 0; jc < kBN; jc += 32) {
+                        const uint32_t tb = tmem + ((uint32_t)(quad * 32 + half * 16) << 16) + (uint32_t)(buf * kBN);
+                        for (int jc = c0; jc < c0 + kBN / 2; jc += 32) {
                             float v[16];
                             tmem_ld16x256b_x4(tb + (uint32_t)jc, v);
 #pragma unroll
@@ -307,6 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 constexpr size_t kSmemBytes = 1024 + (size_t)kMaxKB * kQBlockBytes + (size_t)kKStages * kKStageBytes + sizeof(Ctl);
+static_assert(kSmemBytes <= 227 * 1024, "attention kernel shared memory exceeds the per-CTA limit");
 
 bool g_attr_set[64];
 
