@@ -25,10 +25,14 @@
  *  - Errors that only the device can see (a bounded wait that ran out, an
  *    input outside a fast path's numeric range) set a per-device error word;
  *    gs_stream_status() synchronises the stream and returns and clears it.
- *  - Only gs_build_basis (and gs_basis_reserve_host_staging) allocate device
- *    memory; the other calls allocate nothing.  N = 0 is a valid no-op.
+ *  - Only gs_build_basis allocates device memory; the other calls allocate
+ *    nothing.  N = 0 is a valid no-op.
  *  - All functions are callable from any host thread; a gs_basis must not be
- *    destroyed while work that uses it is in flight.
+ *    destroyed while work that uses it is in flight.  Some paths keep
+ *    intermediate results in a scratch area owned by the gs_basis (the two-GEMM
+ *    similarity for bases the fused kernel cannot hold, the tensor-core
+ *    reconstruct), so calls on one gs_basis that may run at the same time on
+ *    the GPU (different streams) must be ordered by the caller.
  */
 #ifndef GRAMSPACE_H
 #define GRAMSPACE_H

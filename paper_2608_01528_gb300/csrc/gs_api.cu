@@ -303,12 +303,25 @@ gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, long lon
     const bool tc_ok = h->has_split && h->r >= 1 && t_dtype == GS_F32 && (uintptr_t)T % 16 == 0 && ldt % 4 == 0;
     if (flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && tc_ok && big_gemm(N, h->D, h->r))) {
         if (!tc_ok) return t_dtype != GS_F32 || !h->has_split ? GS_ERR_UNSUPPORTED : GS_ERR_ALIGNMENT;
-        // Xhat = T Q: T rounded to fp16 on the fly, the basis' dithered fp16 Q^T, fp32 accumulation
-        gs::GemmTcArgs a{};
-        a.A = (const float*)T; a.lda = ldt; a.m = N; a.K = h->r; a.split = false;
-        a.B0 = h->Q16t; a.ldb = h->ldr16; a.n = h->D;
-        a.C = Xhat; a.ldc = ldxh; a.c_bf16 = false; a.alpha = 1.f;
-        return from_cuda(gs::launch_gemm_tc(a, h->device, s));
+        // Xhat = T Q: T rounded once to fp16 into the handle's scratch (every column tile of
+        // Xhat re-reads it), the basis' dithered fp16 Q^T, fp32 accumulation; rows in chunks
+        // that fit the scratch
+        const int ld16 = (h->r + 7) / 8 * 8;  // 16-byte rows for TMA
+        const long long chunk = std::min(h->scratch_floats * 2 / ld16, kMaxGemmRows) / 128 * 128;
+        if (chunk < 128) return GS_ERR_SHAPE;
+        for (long long c0 = 0; c0 < N; c0 += chunk) {
+            const long long nc = std::min(chunk, N - c0);
+            const float* Tc = (const float*)T + (size_t)c0 * ldt;
+            gs_status st = from_cuda(gs::launch_round_f16(Tc, ldt, nc, h->r, h->scratch, ld16, s));
+            if (st != GS_OK) return st;
+            gs::GemmTcArgs a{};
+            a.A = h->scratch; a.lda = ld16; a.m = nc; a.K = h->r; a.split = false; a.a_half = true;
+            a.B0 = h->Q16t; a.ldb = h->ldr16; a.n = h->D;
+            a.C = Xhat + (size_t)c0 * ldxh; a.ldc = ldxh; a.c_bf16 = false; a.alpha = 1.f;
+            st = from_cuda(gs::launch_gemm_tc(a, h->device, s));
+            if (st != GS_OK) return st;
+        }
+        return GS_OK;
     }
     for (long long c0 = 0; c0 < N; c0 += kMaxGemmRows) {
         const long long nc = std::min(kMaxGemmRows, N - c0);

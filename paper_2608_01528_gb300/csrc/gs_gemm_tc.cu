@@ -2,18 +2,23 @@
 //
 //     C = alpha * A B^T            (optionally divided by rownorm[i] * colnorm[j])
 //
-//   A  fp32, m x K row-major, streamed by TMA into an fp32 staging ring and
-//      converted on the fly by two groups of converter warps into the
-//      128-byte-swizzled K-major operand layout:
-//        kAF16     one fp16 copy (round to nearest)     D  = A16 B0^T
-//        kABF16X2  hi = bf16(A), lo = bf16(A - hi)      D  = Ah B0^T + Al B0^T + Ah B1^T
-//      (the split keeps ~16 significant bits and fp32's exponent range, for
-//      products whose terms do not average out, e.g. with the dominant diagonal of R)
-//   B0, B1  16-bit (fp16 with kAF16, bf16 with kABF16X2), n x K row-major (K-major),
-//      by TMA; these are the basis' operand copies, L2-resident.
+//   A  m x K row-major, in one of three modes:
+//        kAF16     fp32, rounded to fp16 (RN) on the fly   D  = A16 B0^T
+//        kABF16X2  fp32, hi = bf16(A), lo = bf16(A - hi)   D  = Ah B0^T + Al B0^T + Ah B1^T
+//        kAF16T    fp16 already (rounded once by the caller) D = A16 B0^T
+//      In the first two, TMA streams fp32 tiles into a staging ring and two groups
+//      of converter warps write the 128-byte-swizzled K-major operand layout (the
+//      split keeps ~16 significant bits and fp32's exponent range, for products
+//      whose terms do not average out, e.g. with the dominant diagonal of R).  In
+//      kAF16T, TMA writes that layout itself, straight into the A stages: for an A
+//      that every N tile re-reads (reconstruct: T against 40 column tiles of Q),
+//      rounding it once halves its L2 traffic and frees the converters and the
+//      staging ring's shared memory for deeper A and B rings.
+//   B0, B1  16-bit (fp16 with kAF16 / kAF16T, bf16 with kABF16X2), n x K row-major
+//      (K-major), by TMA; these are the basis' operand copies, L2-resident.
 //   C  fp32 or bf16, m x n, leading dimension ldc.
 //
-// Uses (paper Sec. 3.1 / 3.3): reconstruction Xhat = T Q (B0 = fp16 Q^T), the
+// Uses (paper Sec. 3.1 / 3.3): reconstruction Xhat = T Q (kAF16T, B0 = fp16 Q^T), the
 // projection Y = X Q^T for bases too wide for the fused kernel (B0 = fp16 Q),
 // scores S = Y R^T (split, B0 / B1 = bf16 hi / lo of R) and probability
 // vectorization V = P R (split, B0 / B1 = bf16 hi / lo of R^T).
@@ -21,7 +26,9 @@
 // Tiles are 128 x nt (nt <= 256) with the fp32 accumulator double-buffered in
 // TMEM (2 x 256 columns); one persistent CTA per SM walks the tiles with the n
 // index fastest, so CTAs running at the same time share A rows in L2.
-// Warp roles (480 threads): 0-3 epilogue (warp w owns TMEM lanes 32w..32w+31),
+// Warp roles (608 threads): 0-3 and 15-18 epilogue (warp w reads TMEM lanes
+// 32 (w % 4)..+31; the two warps of a lane quadrant take alternate 32-column chunks,
+// so output-heavy products like reconstruct are not held up by the stores),
 // 4 TMA producer of A, 5 TMEM allocator + MMA issuer, 6 TMA producer of B,
 // 7-14 converters in two groups taking alternate K-blocks.  Every mbarrier wait
 // is bounded (see gs_tc_ptx.cuh); on expiry the CTA records GS_DEV_ERR_TIMEOUT,
@@ -49,7 +56,11 @@ constexpr int kCvt0 = 7;
 constexpr int kCvtGroups = 2;
 constexpr int kCvtGroupWarps = 4;
 constexpr int kCvtWarps = kCvtGroups * kCvtGroupWarps;
-constexpr int kThreads = (kCvt0 + kCvtWarps) * 32;  // 480
+constexpr int kEpi2 = kCvt0 + kCvtWarps;               // second epilogue group: warps 15-18
+constexpr int kEpiWarpsTotal = 2 * kEpiWarps;
+constexpr int kThreads = (kEpi2 + kEpiWarps) * 32;       // 608
+// 19 warps: one sub-partition holds 5, so a thread may use at most 65536 / 4 / (5 * 32) = 102
+// registers (allocated in steps of 8: 96)
 constexpr int kCvtRowStep = kCvtGroupWarps * 32 / 16;  // 8
 constexpr int kCvtRows = kBM / kCvtRowStep;            // 16
 constexpr int kXStageBytes = kBM * kBK * 4;            // 32 KB
@@ -58,7 +69,10 @@ constexpr int kBStageBytes = 256 * kBK * 2;            // 32 KB
 constexpr int kMaxSX = 4, kMaxSA = 4, kMaxSB = 4;
 constexpr int kTmemCols = 512;
 
-enum { kAF16 = 0, kABF16X2 = 1 };
+// A operand modes: fp32 rounded to fp16 by the converters; fp32 split into bf16 hi / lo by
+// the converters (three products with B hi / lo); fp16 already, loaded by TMA straight into
+// the A stages (no staging ring, no converters).
+enum { kAF16 = 0, kABF16X2 = 1, kAF16T = 2 };
 
 struct GemmParams {
     long long m;
@@ -84,7 +98,7 @@ struct Ctl {
     int abort_flag;
 };
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see kThreads)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b0,
               const __grid_constant__ CUtensorMap tmap_b1, const GemmParams p) {
     extern __shared__ uint8_t smem_raw[];
@@ -108,7 +122,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&c.x_empty[s], kCvtGroupWarps);
         }
         for (int s = 0; s < p.sa; ++s) {
-            mbar_init(&c.a_full[s], kCvtGroupWarps);
+            mbar_init(&c.a_full[s], p.amode == kAF16T ? 1 : kCvtGroupWarps);
             mbar_init(&c.a_empty[s], 1);
         }
         for (int s = 0; s < p.sb; ++s) {
@@ -117,7 +131,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&c.d_full[b], 1);
-            mbar_init(&c.d_empty[b], kEpiWarps);
+            mbar_init(&c.d_empty[b], kEpiWarpsTotal);
         }
         mbar_init(&c.mma_done, 1);
         c.abort_flag = 0;
@@ -138,7 +152,29 @@ __global__ void __launch_bounds__(kThreads, 1)
         tn = (int)(tg % p.tiles_n);
     };
 
-    if (warp == kAWarp) {
+    if (warp == kAWarp && p.amode == kAF16T) {
+        // ------------------------------------------------------------- A tiles (fp16) via TMA
+        // straight into the swizzled A stages the MMA reads
+        if (lane == 0) {
+            const uint64_t pol = l2_policy_evict_last();  // each row block is read once per N tile
+            int it = 0;
+            RingPos as;
+            long long tm = 0;
+            int tn = 0;
+            for (int kb = 0, lt = 0; it < total_it; ++it, as.next(p.sa)) {
+                const int s = as.idx;
+                if (!mbar_wait_1t(&c.a_empty[s], as.phase ^ 1u, abort_flag, err)) break;
+                if (kb == 0) tile_mn(lt, tm, tn);
+                mbar_arrive_expect_tx(&c.a_full[s], kAPartBytes);
+                tma_load_2d(As + (size_t)s * kAPartBytes, &tmap_a, &c.a_full[s], kb * kBK, (int)(tm * kBM), pol);
+                if (++kb == p.nkb) {
+                    kb = 0;
+                    ++lt;
+                }
+            }
+            for (int j = std::max(0, it - p.sa); j < it; ++j) mbar_drain(&c.a_full[j % p.sa], (uint32_t)(j / p.sa) & 1u, err);
+        }
+    } else if (warp == kAWarp) {
         // ------------------------------------------------------------- A tiles (fp32) via TMA
         if (lane == 0) {
             const uint64_t pol = l2_policy_evict_first();
@@ -189,7 +225,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------- MMA issue
         if (lane == 0) {
-            const uint32_t idesc = p.amode == kAF16 ? idesc_f16_f32(p.nt) : idesc_bf16_f32(p.nt);
+            const uint32_t idesc = p.amode == kABF16X2 ? idesc_bf16_f32(p.nt) : idesc_f16_f32(p.nt);
             RingPos ra, rb;
             bool ok = true;
             for (int lt = 0; lt < ntiles && ok; ++lt) {
@@ -217,7 +253,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint8_t* At = As + (size_t)sa * p.parts * kAPartBytes;
                     const uint64_t ah = sdesc_sw128(smem_u32(At));
                     const uint64_t b0 = sdesc_sw128(smem_u32(Bs + (size_t)sb0 * kBStageBytes));
-                    if (p.amode == kAF16) {
+                    if (p.amode != kABF16X2) {
 #pragma unroll
                         for (int k = 0; k < kBK / 16; ++k)
                             mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
@@ -242,7 +278,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_commit(&c.mma_done);
             mbar_drain(&c.mma_done, 0, err);
         }
-    } else if (warp >= kCvt0) {
+    } else if (warp >= kCvt0 && warp < kEpi2) {
         // ------------------------------------------------------------- converters
         const int g = (warp - kCvt0) / kCvtGroupWarps;
         const int l = threadIdx.x - (kCvt0 + g * kCvtGroupWarps) * 32;  // 0..127
@@ -254,7 +290,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             rx.next(p.sx);
             ra.next(p.sa);
         }
-        for (int it = g; it < total_it; it += kCvtGroups) {
+        for (int it = g; p.amode != kAF16T && it < total_it; it += kCvtGroups) {
             const int sx = rx.idx, sa = ra.idx;
             if (!mbar_wait_warp(&c.x_full[sx], rx.phase, abort_flag, err) ||
                 !mbar_wait_warp(&c.a_empty[sa], ra.phase ^ 1u, abort_flag, err))
@@ -297,9 +333,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (amax > 65504.f) atomicOr(err, GS_DEV_ERR_RANGE);
     } else {
-        // ------------------------------------------------------------- epilogue (warps 0-3)
+        // ------------------------------------------------------------- epilogue (warps 0-3, 15-18)
         // TMEM is read in the 16x256b pattern so that each store writes whole sectors:
         // thread t holds rows (t/4) and (t/4 + 8) of a 16-lane half, 8 columns per quad.
+        const int quad = warp & 3, kh = warp >= kEpi2 ? 1 : 0;  // lane quadrant, column chunks
         for (int lt = 0; lt < ntiles; ++lt) {
             const int buf = lt & 1;
             if (!mbar_wait_warp(&c.d_full[buf], (uint32_t)(lt >> 1) & 1u, abort_flag, err)) break;
@@ -308,13 +345,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             int tn;
             tile_mn(lt, tm, tn);
             for (int half = 0; half < 2; ++half) {
-                const int lrow = warp * 32 + half * 16;
+                const int lrow = quad * 32 + half * 16;
                 const uint32_t tb = tmem + ((uint32_t)lrow << 16) + (uint32_t)(buf * 256);
                 const long long row[2] = {tm * kBM + lrow + (lane >> 2), tm * kBM + lrow + (lane >> 2) + 8};
                 float rn[2];
 #pragma unroll
                 for (int h = 0; h < 2; ++h) rn[h] = (p.rownorm && row[h] < p.m) ? p.rownorm[row[h]] : 1.f;
-                for (int jc = 0; jc < p.nt; jc += 32) {
+                for (int jc = 32 * kh; jc < p.nt; jc += 64) {
                     float v[16];
                     tmem_ld16x256b_x4(tb + (uint32_t)jc, v);
 #pragma unroll
@@ -373,6 +410,37 @@ size_t gemm_smem_bytes(int sx, int sa, int parts, int sb) {
 
 bool g_attr_set[64];
 
+// fp32 rows -> fp16 (RN), four columns per thread (X 16-byte aligned, ldx % 4 == 0;
+// out rows 8-byte aligned); values beyond the fp16 range are flagged
+__global__ void k_round_f16(const float* __restrict__ X, long long ldx, long long rows, int cols,
+                            __half* __restrict__ out, long long ldo) {
+    const int c4n = (cols + 3) / 4;
+    const long long total = rows * c4n;
+    float amax = 0.f;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        const long long row = i / c4n;
+        const int c = (int)(i - row * c4n) * 4;
+        const float* src = X + row * ldx + c;
+        __half* dst = out + row * ldo + c;
+        if (c + 4 <= cols) {
+            const float4 v = *reinterpret_cast<const float4*>(src);
+            amax = fmaxf(amax, fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w))));
+            const __half2 h0 = __floats2half2_rn(v.x, v.y), h1 = __floats2half2_rn(v.z, v.w);
+            uint2 pk;
+            pk.x = *reinterpret_cast<const uint32_t*>(&h0);
+            pk.y = *reinterpret_cast<const uint32_t*>(&h1);
+            *reinterpret_cast<uint2*>(dst) = pk;
+        } else {
+            for (int j = 0; c + j < cols; ++j) {
+                amax = fmaxf(amax, fabsf(src[j]));
+                dst[j] = __float2half_rn(src[j]);
+            }
+        }
+    }
+    if (amax > 65504.f) atomicOr(&g_err_gemm, GS_DEV_ERR_RANGE);
+}
+
 }  // namespace
 
 unsigned take_device_error_gemm() {
@@ -392,9 +460,10 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     p.nt = a.n >= 256 ? 256 : (a.n + 31) / 32 * 32;
     p.tiles_n = (a.n + p.nt - 1) / p.nt;
     p.tiles = ((a.m + kBM - 1) / kBM) * (long long)p.tiles_n;
-    p.amode = a.split ? kABF16X2 : kAF16;
+    p.amode = a.a_half ? kAF16T : a.split ? kABF16X2 : kAF16;
     p.nb = a.split ? 2 : 1;
     p.parts = a.split ? 2 : 1;
+    if (a.a_half && a.split) return cudaErrorInvalidValue;
     // deepest staging that fits: two A stages, B stages for at least one K-block (+1).
     // The X depth stays even: the two converter groups take alternate K-blocks, and with
     // an even depth each X stage belongs to one group, which waits on its phases in order
@@ -414,6 +483,11 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
             }
         if (done) break;
     }
+    if (p.amode == kAF16T) {  // no staging ring: the deepest A and B rings that fit
+        p.sx = 0;
+        p.sa = kMaxSA;
+        p.sb = kMaxSB;
+    }
     if (gemm_smem_bytes(p.sx, p.sa, p.parts, p.sb) > cap) return cudaErrorInvalidConfiguration;
     p.C = a.C;
     p.ldc = a.ldc;
@@ -424,8 +498,11 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     p.colnorm = a.colnorm;
     CUtensorMap ta, tb0, tb1;
     const CUtensorMapDataType bt = a.split ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
-    if (!make_tmap_2d(&ta, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, a.A, a.m, a.K, a.lda, kBK, kBM,
-                      CU_TENSOR_MAP_SWIZZLE_NONE) ||
+    const bool ta_ok = a.a_half ? make_tmap_2d(&ta, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, a.A, a.m, a.K, a.lda, kBK,
+                                               kBM, CU_TENSOR_MAP_SWIZZLE_128B)
+                                : make_tmap_2d(&ta, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, a.A, a.m, a.K, a.lda, kBK,
+                                               kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
+    if (!ta_ok ||
         !make_tmap_2d(&tb0, bt, 2, a.B0, a.n, a.K, a.ldb, kBK, p.nt, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_tmap_2d(&tb1, bt, 2, a.split ? a.B1 : a.B0, a.n, a.K, a.ldb, kBK, p.nt, CU_TENSOR_MAP_SWIZZLE_128B))
         return cudaErrorInvalidValue;
@@ -439,6 +516,19 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
     const int grid = (int)std::min<long long>(sms > 0 ? sms : 1, p.tiles);
     k_gemm_tc<<<grid, kThreads, smem, s>>>(ta, tb0, tb1, p);
+    return cudaGetLastError();
+}
+
+}  // namespace gs
+
+namespace gs {
+
+cudaError_t launch_round_f16(const float* X, long long ldx, long long rows, int cols, void* out, long long ldo,
+                             cudaStream_t s) {
+    if (rows <= 0 || cols <= 0) return cudaSuccess;
+    const long long work = rows * ((cols + 3) / 4);
+    const int grid = (int)std::min<long long>((work + 255) / 256, 152LL * 8);
+    k_round_f16<<<grid, 256, 0, s>>>(X, ldx, rows, cols, static_cast<__half*>(out), ldo);
     return cudaGetLastError();
 }
 

@@ -116,13 +116,17 @@ cudaError_t launch_ps_tc(const gs_basis* h, const float* X, long long N, int ldx
 // rounding of A; split = true: B0 / B1 bf16 hi / lo, A split into bf16 hi / lo
 // (three products).  B rows 16-byte aligned (ldb % 8 == 0).  C fp32 or bf16.
 struct GemmTcArgs {
-    const float* A; long long lda; long long m; int K;
+    const void* A; long long lda; long long m; int K;
     bool split;
+    bool a_half;    // A already fp16 (lda in halves, multiple of 8): TMA feeds the MMA directly
     const void* B0; const void* B1; long long ldb; int n;
     void* C; long long ldc; bool c_bf16; float alpha;
     const float* rownorm; const float* colnorm;
 };
 cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s);
+// fp32 rows -> fp16 (RN), for the fp16-A GEMM; values beyond the fp16 range set GS_DEV_ERR_RANGE
+cudaError_t launch_round_f16(const float* X, long long ldx, long long rows, int cols, void* out, long long ldo,
+                             cudaStream_t s);
 
 // ----------------------------------------------------------------- attention scores on tcgen05 (gs_attn_tc.cu)
 // bf16 Yq (B x Lq x r) and Yk (B x Lk x r), row stride ldy; fp32 A (B x Lq x Lk, dense).
