@@ -165,6 +165,22 @@ def cpu_baseline(seconds=10.0):
             "seconds": round(dt, 3)}
 
 
+def max_over_ranks(ms, pg, device):
+    """The slowest rank's time (every rank's timed region must end before the job's does);
+    `pg` is torch.distributed (any backend) or None for one process."""
+    if pg is None:
+        return float(ms)
+    import torch
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(units_per_rank, world, steps, ms):
+    """Whole-job units per second: every rank processes its own `units_per_rank` per step."""
+    return units_per_rank * world * steps / (ms / 1e3)
+
+
 def run_reference(args):
     ws, rank, _ = dist_env()
     if rank != 0:
@@ -265,14 +281,10 @@ def main():
             step()
         e1.record(stream)
         barrier()
-    ms = e0.elapsed_time(e1)
-    if pg is not None:
-        t = torch.tensor([ms], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(e0.elapsed_time(e1), pg, dev)
     gs.stream_status()
     per_step_ms = ms / args.steps
-    value = N * ws * args.steps / (ms / 1e3)
+    value = job_throughput(N, ws, args.steps, ms)
 
     # end to end through the same API: pinned host queries in, argmax/maxval out
     amh = torch.empty(N, dtype=torch.int32).pin_memory()
@@ -294,12 +306,8 @@ def main():
         step_e2e()
     f1.record(stream)
     barrier()
-    ms_e2e = f0.elapsed_time(f1)
-    if pg is not None:
-        t = torch.tensor([ms_e2e], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        ms_e2e = float(t.item())
-    e2e = {"value": N * ws * ke / (ms_e2e / 1e3), "unit": "queries/s",
+    ms_e2e = max_over_ranks(f0.elapsed_time(f1), pg, dev)
+    e2e = {"value": job_throughput(N, ws, ke, ms_e2e), "unit": "queries/s",
            "h2d_bytes_per_step": N * D * 4, "d2h_bytes_per_step": N * 8}
     ok = ok and bool(np.array_equal(amh.numpy(), w["labels"]))
 
