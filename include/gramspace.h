@@ -31,8 +31,9 @@
  *    destroyed while work that uses it is in flight.  Some paths keep
  *    intermediate results in a scratch area owned by the gs_basis (the two-GEMM
  *    similarity for bases the fused kernel cannot hold, the tensor-core
- *    reconstruct), so calls on one gs_basis that may run at the same time on
- *    the GPU (different streams) must be ordered by the caller.
+ *    reconstruct, gs_similarity_coeffs), so calls on one gs_basis that may run
+ *    at the same time on the GPU (different streams) must be ordered by the
+ *    caller.
  */
 #ifndef GRAMSPACE_H
 #define GRAMSPACE_H
@@ -139,6 +140,28 @@ GS_API gs_status gs_basis_destroy(gs_basis* h);
 GS_API gs_status gs_project_similarity(const gs_basis* h, const float* X, long long N, int ldx,
                                 int mode, float scale, unsigned flags, float* Y, int ldy,
                                 float* S, int lds, int* argmax, float* maxval, void* stream);
+
+/*
+ * Similarity of queries given by their Gram-loc coordinates (Sec. 3.2, Eq. 2:
+ * inner products between vectors in span(C) equal those of their Gram-loc
+ * coordinates; Sec. 2.2 scaled dot-product similarity).  This is the lookup that
+ * never touches a D-dimensional vector: its cost does not grow with D (the
+ * "compressed" row of the paper's latency-versus-dimension table).
+ *
+ * Y: N x r fp32 Gram-loc queries (ld = ldy >= r), e.g. V from gs_prob_vectorize
+ * or Y from gs_project_similarity.  S = scale * Y R^T (N x M); COSINE divides by
+ * ||y_n|| (equal to ||x_n|| for x in span(C), Eq. 3) and ||c_i||; SOFTMAX as in
+ * gs_project_similarity.  Outputs S (ld = lds), argmax, maxval as in
+ * gs_project_similarity; at least one must be non-NULL.  Y may be NULL only when
+ * r = 0 (every score is then 0).
+ * Tensor-core path (GS_PATH_AUTO for large N·M·r): Y and R split into bf16 hi /
+ * lo, three products, fp32 accumulation (~2^-16 relative); needs Y 16-byte
+ * aligned and ldy % 4 == 0.  Otherwise fp32 CUDA cores.  Uses the basis'
+ * scratch for cosine norms and, when S is NULL, for the scores.
+ */
+GS_API gs_status gs_similarity_coeffs(const gs_basis* h, const float* Y, long long N, int ldy, int mode,
+                                      float scale, unsigned flags, float* S, int lds, int* argmax,
+                                      float* maxval, void* stream);
 
 /*
  * Probability vectorization on Gram-loc (Sec. 2.2: weighted sum of codewords

@@ -256,6 +256,66 @@ gs_status gs_project_similarity(const gs_basis* h, const float* X, long long N, 
     return GS_OK;
 }
 
+gs_status gs_similarity_coeffs(const gs_basis* h, const float* Y, long long N, int ldy, int mode, float scale,
+                               unsigned flags, float* S, int lds, int* argmax, float* maxval, void* stream) {
+    if (!h || !valid_path(flags)) return GS_ERR_INVALID_ARG;
+    if (mode < GS_SCORE_RAW || mode > GS_SCORE_SOFTMAX || !isfinite(scale)) return GS_ERR_INVALID_ARG;
+    if (N < 0 || ldy < h->r || ldy < 1 || (S && lds < h->M)) return GS_ERR_SHAPE;
+    if (N == 0) return GS_OK;
+    if (!S && !argmax && !maxval) return GS_ERR_INVALID_ARG;
+    if (!Y && h->r > 0) return GS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    if (!g.ok) return GS_ERR_CUDA;
+    cudaStream_t s = (cudaStream_t)stream;
+    const int r = h->r, M = h->M;
+    const bool tc_ok = h->has_split && r >= 1 && (uintptr_t)Y % 16 == 0 && ldy % 4 == 0;
+    const bool tensor = flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && tc_ok && big_gemm(N, M, r));
+    if (tensor && !tc_ok) return h->has_split && r >= 1 ? GS_ERR_ALIGNMENT : GS_ERR_UNSUPPORTED;
+    // scratch per row: ||y|| (cosine) and the score row when S is not an output
+    const long long per_row = (mode == GS_SCORE_COSINE ? 1 : 0) + (S ? 0 : M);
+    const long long chunk = std::min(per_row ? h->scratch_floats / per_row : N, kMaxGemmRows);
+    if (chunk < 1) return GS_ERR_SHAPE;
+    for (long long c0 = 0; c0 < N; c0 += chunk) {
+        const long long nc = std::min(chunk, N - c0);
+        const float* Yc = Y ? Y + c0 * ldy : nullptr;
+        float* xn = nullptr;
+        float* scr = h->scratch;
+        if (mode == GS_SCORE_COSINE) {  // ||y|| = ||x|| for x in span(C) (Eq. 3)
+            xn = scr;
+            scr += nc;
+            cudaError_t e = gs::launch_rownorm(Yc, nc, ldy, r, xn, s);
+            if (e != cudaSuccess) return from_cuda(e);
+        }
+        float* Sbuf = S ? S + c0 * lds : scr;
+        const long long ldsb = S ? lds : M;
+        cudaError_t e;
+        if (tensor) {
+            // S = Yh Rh^T + Yl Rh^T + Yh Rl^T (bf16 hi / lo split, fp32 accumulation)
+            gs::GemmTcArgs a{};
+            a.A = Yc; a.lda = ldy; a.m = nc; a.K = r; a.split = true;
+            a.B0 = h->tc_Rh; a.B1 = h->tc_Rl; a.ldb = h->tc_npad; a.n = M;
+            a.C = Sbuf; a.ldc = ldsb; a.c_bf16 = false; a.alpha = scale;
+            if (xn) { a.rownorm = xn; a.colnorm = h->cnorm; }
+            e = gs::launch_gemm_tc(a, h->device, s);
+        } else {
+            gs::GemmArgs b{};
+            b.A = Yc ? (const void*)Yc : (const void*)h->scratch; b.a_type = gs::MAT_F32; b.lda = ldy;
+            b.B = h->R; b.b_type = gs::MAT_F32; b.ldb = h->ldr; b.b_trans = true; b.b_rowlen = h->rlen;
+            b.C = Sbuf; b.c_type = gs::MAT_F32; b.ldc = ldsb;
+            b.m = nc; b.n = M; b.k = r; b.batch = 1; b.alpha = scale;
+            if (xn) { b.rownorm = xn; b.colnorm = h->cnorm; }
+            e = gs::launch_gemm_simt(b, s);
+        }
+        if (e != cudaSuccess) return from_cuda(e);
+        if (argmax || maxval || mode == GS_SCORE_SOFTMAX) {
+            e = gs::launch_row_finish(Sbuf, nc, M, (int)ldsb, mode == GS_SCORE_SOFTMAX, argmax ? argmax + c0 : nullptr,
+                                      maxval ? maxval + c0 : nullptr, s);
+            if (e != cudaSuccess) return from_cuda(e);
+        }
+    }
+    return GS_OK;
+}
+
 gs_status gs_prob_vectorize(const gs_basis* h, const float* P, long long N, int ldp, void* V, int v_dtype,
                             int ldv, unsigned flags, void* stream) {
     if (!h || !valid_path(flags)) return GS_ERR_INVALID_ARG;

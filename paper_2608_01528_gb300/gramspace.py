@@ -29,7 +29,7 @@ GS_BUILD_NORMALIZE_ROWS = 1
 # Every symbol include/gramspace.h declares (checked by the CPU tests).
 EXPORTS = ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_similarity",
            "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores", "gs_stream_status",
-           "gs_status_string", "gs_version", "gs_project_similarity_static")
+           "gs_status_string", "gs_version", "gs_project_similarity_static", "gs_similarity_coeffs")
 
 
 class GramSpaceError(RuntimeError):
@@ -55,6 +55,7 @@ def load_library(path=LIB_PATH):
                                 ctypes.POINTER(vp), ctypes.POINTER(vp), ctypes.POINTER(vp)]
     L.gs_basis_destroy.argtypes = [vp]
     L.gs_project_similarity.argtypes = [vp, vp, i64, ip, ip, f32, u32, vp, ip, vp, ip, vp, vp, vp]
+    L.gs_similarity_coeffs.argtypes = [vp, vp, i64, ip, ip, f32, u32, vp, ip, vp, vp, vp]
     L.gs_prob_vectorize.argtypes = [vp, vp, i64, ip, vp, ip, ip, u32, vp]
     L.gs_reconstruct.argtypes = [vp, vp, ip, i64, ip, vp, ip, u32, vp]
     L.gs_attention_scores.argtypes = [vp, vp, ip, ip, ip, ip, ip, ip, f32, ip, vp, u32, vp]
@@ -65,7 +66,8 @@ def load_library(path=LIB_PATH):
     L.gs_status_string.restype = ctypes.c_char_p
     L.gs_version.restype = ctypes.c_int
     for name in ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_similarity",
-                 "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores", "gs_stream_status"):
+                 "gs_similarity_coeffs", "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores",
+                 "gs_stream_status"):
         getattr(L, name).restype = ctypes.c_int
     _lib = L
     return L
@@ -201,6 +203,30 @@ def project_similarity(basis, X, mode="raw", scale=1.0, path="auto", want_Y=Fals
                                      _ptr(S), _ld(S) if S is not None and S.numel() else max(basis.M, 1),
                                      _ptr(out.get("argmax")), _ptr(out.get("maxval")), _stream(stream))
     _check(st, "gs_project_similarity")
+    return out
+
+
+def similarity_coeffs(basis, Y, mode="raw", scale=1.0, path="auto", want_S=False, want_argmax=True,
+                      want_maxval=True, out=None, stream=None):
+    """Scores of Gram-loc queries Y (N x r fp32) against the codebook, S = Y R^T; see
+    gs_similarity_coeffs.  Returns a dict with the requested outputs ("S", "argmax", "maxval")."""
+    N = Y.shape[0]
+    dev = Y.device
+    out = dict(out or {})
+    if want_S and "S" not in out:
+        out["S"] = torch.empty((N, basis.M), dtype=torch.float32, device=dev)
+    if want_argmax and "argmax" not in out:
+        out["argmax"] = torch.empty(N, dtype=torch.int32, device=dev)
+    if want_maxval and "maxval" not in out:
+        out["maxval"] = torch.empty(N, dtype=torch.float32, device=dev)
+    S = out.get("S")
+    L = load_library()
+    with torch.cuda.device(dev):
+        st = L.gs_similarity_coeffs(basis.handle, _ptr(Y) if Y.numel() else None, N,
+                                    _ld(Y) if Y.numel() else max(basis.r, 1), MODES[mode], float(scale),
+                                    PATHS[path], _ptr(S), _ld(S) if S is not None and S.numel() else max(basis.M, 1),
+                                    _ptr(out.get("argmax")), _ptr(out.get("maxval")), _stream(stream))
+    _check(st, "gs_similarity_coeffs")
     return out
 
 
