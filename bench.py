@@ -415,7 +415,58 @@ def side_rows(gs, dev):
     ms = timeit(lambda: gs.attention_scores(V3, V3, 1 / 64.0, out=A))
     out["attention"] = roof(ms, 2 * V3.numel() * 2 + A.numel() * 4, 2 * 64 * 1024 * 1024 * b5.r, "hbm")
     del b4, b5
+    out["lookup_sweep"] = lookup_sweep(gs, dev)
     return out
+
+
+def lookup_sweep(gs, dev, reps=50):
+    """Similarity-lookup latency across the original dimension D (M = 40, 1,024 lookups per
+    batch): uncompressed X Cᵀ + argmax (torch.matmul, fp32: the paper's "original"), the
+    compressed lookup on Gram-loc queries (gs_similarity_coeffs: S = Y Rᵀ, no D-dimensional
+    work), and projection + compressed scoring from the D-dimensional queries
+    (gs_project_similarity).  Single-call latency: events around one call issued to an idle
+    stream, median of `reps` calls (host issue time included, as in a lookup)."""
+    import torch
+    import synth
+
+    def latency(fn):
+        for _ in range(5):
+            fn()
+        torch.cuda.synchronize()
+        s = torch.cuda.current_stream()
+        ts = []
+        for _ in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(s)
+            fn()
+            b.record(s)
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b) * 1e3)
+        return round(statistics.median(ts), 1)
+
+    res = {"M": 40, "lookups_per_batch": 1024, "unit": "us per batch", "D": [], "original_xct": [],
+           "compressed_coeffs": [], "project_then_compressed": [], "argmax_agree": True}
+    for D in synth.SWEEP_D:
+        w = synth.sweep(D)
+        C = torch.from_numpy(w["C"]).to(dev)
+        X = torch.from_numpy(w["X"]).to(dev)
+        b = gs.build_basis(C)
+        Y = gs.project_similarity(b, X, want_Y=True, want_argmax=False, want_maxval=False)["Y"]
+        am = torch.empty(X.shape[0], dtype=torch.int32, device=dev)
+        mv = torch.empty(X.shape[0], device=dev)
+        CT = C.t().contiguous()
+        t_orig = latency(lambda: torch.matmul(X, CT).argmax(dim=1))
+        t_comp = latency(lambda: gs.similarity_coeffs(b, Y, out={"argmax": am, "maxval": mv}))
+        t_proj = latency(lambda: gs.project_similarity(b, X, out={"argmax": am, "maxval": mv}))
+        gs.similarity_coeffs(b, Y, out={"argmax": am, "maxval": mv})
+        agree = bool(torch.equal(am.long(), torch.matmul(X, CT).argmax(dim=1)))
+        res["D"].append(D)
+        res["original_xct"].append(t_orig)
+        res["compressed_coeffs"].append(t_comp)
+        res["project_then_compressed"].append(t_proj)
+        res["argmax_agree"] = res["argmax_agree"] and agree
+        del b
+    return res
 
 
 if __name__ == "__main__":

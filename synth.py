@@ -33,7 +33,8 @@ import numpy as np
 
 BLOCK = 256
 SEEDS = {"tiny": 20260001, "multiattr": 20260002, "large": 20260003,
-         "rankdef": 20260004, "attention": 20260005}
+         "rankdef": 20260004, "attention": 20260005, "sweep": 20260006}
+SWEEP_D = (256, 512, 1024, 2048, 4096, 8192)
 MULTIATTR_M = (5, 6, 10, 9)
 
 
@@ -150,3 +151,12 @@ def attention(seed=SEEDS["attention"], M=512, D=4096, B=64, L=1024):
     Pq = attention_probs(seed, B, L, M, 1)
     Pk = attention_probs(seed, B, L, M, 101)
     return {"C": C, "Pq": Pq, "Pk": Pk, "B": B, "L": L, "D": D}
+
+
+def sweep(D, seed=SEEDS["sweep"], M=40, N=1024, sigma=0.5):
+    """Lookup-latency sweep over the original dimension: a bipolar global codebook of
+    M = 40 attribute vectors (the paper's memory-model example) at dimension D, and a
+    batch of N random attribute lookups x = c_k + N(0, sigma^2)."""
+    C = bipolar(_rng(seed, 0, D), M, D)
+    X, L = noisy_rows(C, seed + D, 0, N, sigma)
+    return {"C": C, "X": X, "labels": L, "D": D}
