@@ -118,6 +118,17 @@ gs_status ps_two_gemm(const gs_basis* h, const float* X, long long N, int ldx, i
     return GS_OK;
 }
 
+// K chunks for the fp32 GEMM of m x n outputs over depth k: enough 64 x 64 tiles x chunks to
+// give every SM about two blocks, chunks of at least 512.
+int gemm_ksplit(long long m, int n, int k, int dev) {
+    int sms = 0;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const long long tiles = ((m + 63) / 64) * ((n + 63) / 64);
+    const long long want = (2LL * std::max(sms, 1) + tiles - 1) / tiles;
+    const long long most = std::max(1, k / 512);
+    return (int)std::max(1LL, std::min(want, most));
+}
+
 // Whether a GEMM of m rows, n columns and depth k is worth the tensor-core kernel.
 bool big_gemm(long long m, long long n, long long k) { return m >= 512 && 2.0 * m * n * k >= 2e9; }
 
@@ -234,6 +245,13 @@ gs_status gs_project_similarity(const gs_basis* h, const float* X, long long N, 
         a.B = h->Q; a.b_type = gs::MAT_F32; a.ldb = D; a.b_trans = true;
         a.C = Ybuf; a.c_type = gs::MAT_F32; a.ldc = ldyb;
         a.m = nc; a.n = r; a.k = D; a.batch = 1; a.alpha = 1.f;
+        // few output tiles (a small batch against a narrow basis): cut D into chunks so that
+        // every SM gets work, partial sums added into Y (zeroed first)
+        a.ksplit = gemm_ksplit(nc, r, D, h->device);
+        if (a.ksplit > 1) {
+            cudaError_t e = cudaMemset2DAsync(Ybuf, sizeof(float) * ldyb, 0, sizeof(float) * r, nc, s);
+            if (e != cudaSuccess) return from_cuda(e);
+        }
         cudaError_t e = gs::launch_gemm_simt(a, s);
         if (e != cudaSuccess) return from_cuda(e);
         if (!S && !argmax && !maxval) continue;

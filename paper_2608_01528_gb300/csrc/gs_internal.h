@@ -88,6 +88,9 @@ struct GemmArgs {
     float alpha;
     const float* rownorm; const float* colnorm;
     const int* b_rowlen;  // optional (b_trans only): row j of B is zero beyond b_rowlen[j]
+    int ksplit;           // > 1 (batch 1, fp32 C only): K is cut into ksplit chunks, one per
+                          // grid z index, whose partial tiles are added into C atomically;
+                          // C must hold zeros before the launch
 };
 cudaError_t launch_gemm_simt(const GemmArgs& g, cudaStream_t s);
 

@@ -138,7 +138,8 @@ __global__ void __launch_bounds__(256) k_gemm(GemmArgs g) {
     const int tx = tid % 16, ty = tid / 16;
     const long long m0 = (long long)blockIdx.y * kTM;
     const int n0 = blockIdx.x * kTN;
-    const int b = blockIdx.z;
+    const bool split = g.ksplit > 1;
+    const int b = split ? 0 : blockIdx.z;
     const char* Ab = (const char*)g.A + (size_t)b * g.a_bstride * (TA == MAT_F32 ? 4 : 2);
     const char* Bb = (const char*)g.B + (size_t)b * g.b_bstride * (TB == MAT_F32 ? 4 : 2);
     int kend = g.k;
@@ -155,8 +156,14 @@ __global__ void __launch_bounds__(256) k_gemm(GemmArgs g) {
         for (int w = 0; w < 8; ++w) mx = max(mx, smx[w]);
         kend = min(kend, mx);
     }
+    int kbeg = 0;
+    if (split) {  // this block's chunk of K (chunks are whole kTK steps)
+        const int chunk = ((g.k + g.ksplit - 1) / g.ksplit + kTK - 1) / kTK * kTK;
+        kbeg = blockIdx.z * chunk;
+        kend = min(kend, kbeg + chunk);
+    }
     float acc[4][4] = {};
-    for (int k0 = 0; k0 < kend; k0 += kTK) {
+    for (int k0 = kbeg; k0 < kend; k0 += kTK) {
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
             const int e = tid + 256 * t;
@@ -202,8 +209,12 @@ __global__ void __launch_bounds__(256) k_gemm(GemmArgs g) {
                 const float den = g.rownorm[gm] * g.colnorm[gn];
                 v = den > 0.f ? v / den : 0.f;
             }
-            if (TC == MAT_F32) ((float*)Cb)[gm * g.ldc + gn] = v;
-            else ((__nv_bfloat16*)Cb)[gm * g.ldc + gn] = __float2bfloat16_rn(v);
+            if (TC == MAT_F32) {
+                if (split) atomicAdd((float*)Cb + gm * g.ldc + gn, v);
+                else ((float*)Cb)[gm * g.ldc + gn] = v;
+            } else {
+                ((__nv_bfloat16*)Cb)[gm * g.ldc + gn] = __float2bfloat16_rn(v);
+            }
         }
     }
 }
@@ -285,7 +296,9 @@ cudaError_t launch_ps_warp(const float* X, long long N, int ldx, int D, const fl
 
 cudaError_t launch_gemm_simt(const GemmArgs& g, cudaStream_t s) {
     if (g.m <= 0 || g.n <= 0 || g.batch <= 0) return cudaSuccess;
-    dim3 grid((unsigned)((g.n + kTN - 1) / kTN), (unsigned)((g.m + kTM - 1) / kTM), (unsigned)g.batch);
+    if (g.ksplit > 1 && (g.batch != 1 || g.c_type != MAT_F32)) return cudaErrorInvalidValue;
+    dim3 grid((unsigned)((g.n + kTN - 1) / kTN), (unsigned)((g.m + kTM - 1) / kTM),
+              (unsigned)(g.ksplit > 1 ? g.ksplit : g.batch));
     if (grid.y > 65535u) return cudaErrorInvalidConfiguration;
 #define GS_GEMM_CASE(TA, TB, TC, BT)                                                        \
     if (g.a_type == TA && g.b_type == TB && g.c_type == TC && g.b_trans == BT) {            \
