@@ -229,6 +229,18 @@ GS_API gs_status gs_project_similarity_static(const float* Q, int r, int D, cons
 GS_API gs_status gs_stream_status(void* stream);
 
 /* Static, human-readable name of a status code. */
+/*
+ * Self-test of the device-side failure detection (the paper has no counterpart:
+ * this checks the library's own machinery).  Every wait of the tensor-core
+ * kernels on a pipeline barrier is bounded (2 s); when one runs out the kernel
+ * records a timeout in the device error word, unwinds and returns, so the CUDA
+ * context stays usable.  This call enqueues one block on `stream` whose single
+ * thread waits, through that same bounded wait, on a barrier that nothing will
+ * ever complete: about 2 s later gs_stream_status() on that stream returns
+ * GS_ERR_TIMEOUT.  Returns GS_ERR_UNSUPPORTED on devices other than sm_103.
+ */
+GS_API gs_status gs_selftest_wait_timeout(void* stream);
+
 GS_API const char* gs_status_string(gs_status s);
 
 /* Library version, major*10000 + minor*100 + patch. */

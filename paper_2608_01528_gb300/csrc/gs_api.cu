@@ -449,6 +449,13 @@ gs_status gs_attention_scores(const void* Yq, const void* Yk, int in_dtype, int 
     return GS_OK;
 }
 
+gs_status gs_selftest_wait_timeout(void* stream) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return GS_ERR_CUDA;
+    if (!device_supported(dev)) return GS_ERR_UNSUPPORTED;
+    return from_cuda(gs::launch_wait_selftest((cudaStream_t)stream));
+}
+
 gs_status gs_stream_status(void* stream) {
     cudaError_t e = stream ? cudaStreamSynchronize((cudaStream_t)stream) : cudaDeviceSynchronize();
     if (e != cudaSuccess) return GS_ERR_CUDA;

@@ -142,6 +142,8 @@ cudaError_t launch_attn_tc(const void* Yq, const void* Yk, int B, int Lq, int Lk
 // its own word; gs_stream_status reads and clears all of them.
 unsigned take_device_error_build();
 unsigned take_device_error_tc();
+// one block whose wait on a never-completed mbarrier runs out (failure-detection self-test)
+cudaError_t launch_wait_selftest(cudaStream_t s);
 unsigned take_device_error_gemm();
 unsigned take_device_error_attn();
 

@@ -580,6 +580,28 @@ Rings ps_rings(int box_rows) {
 
 }  // namespace
 
+namespace {
+// Self-test of the bounded waits: one thread waits, through the same mbar_wait the
+// tensor-core kernels use, on an mbarrier that nothing ever arrives on.  The wait gives up
+// after its limit, records GS_DEV_ERR_TIMEOUT in this file's device word and returns.
+__global__ void k_wait_selftest() {
+    __shared__ uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        abort_flag = 0;
+        fence_barrier_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) mbar_wait(&bar, 0u, &abort_flag, &g_err_tc);  // phase 0 never completes
+}
+}  // namespace
+
+cudaError_t launch_wait_selftest(cudaStream_t s) {
+    k_wait_selftest<<<1, 32, 0, s>>>();
+    return cudaGetLastError();
+}
+
 unsigned take_device_error_tc() {
     unsigned v = 0, z = 0;
     cudaMemcpyFromSymbol(&v, g_err_tc, sizeof(v));

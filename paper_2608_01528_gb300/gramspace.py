@@ -29,7 +29,8 @@ GS_BUILD_NORMALIZE_ROWS = 1
 # Every symbol include/gramspace.h declares (checked by the CPU tests).
 EXPORTS = ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_similarity",
            "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores", "gs_stream_status",
-           "gs_status_string", "gs_version", "gs_project_similarity_static", "gs_similarity_coeffs")
+           "gs_status_string", "gs_version", "gs_project_similarity_static", "gs_similarity_coeffs",
+           "gs_selftest_wait_timeout")
 
 
 class GramSpaceError(RuntimeError):
@@ -60,6 +61,7 @@ def load_library(path=LIB_PATH):
     L.gs_reconstruct.argtypes = [vp, vp, ip, i64, ip, vp, ip, u32, vp]
     L.gs_attention_scores.argtypes = [vp, vp, ip, ip, ip, ip, ip, ip, f32, ip, vp, u32, vp]
     L.gs_stream_status.argtypes = [vp]
+    L.gs_selftest_wait_timeout.argtypes = [vp]
     L.gs_project_similarity_static.argtypes = [vp, ip, ip, vp, ip, vp, vp, i64, ip, ip, f32, vp, vp, vp]
     L.gs_project_similarity_static.restype = ctypes.c_int
     L.gs_status_string.argtypes = [ip]
@@ -67,7 +69,7 @@ def load_library(path=LIB_PATH):
     L.gs_version.restype = ctypes.c_int
     for name in ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_similarity",
                  "gs_similarity_coeffs", "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores",
-                 "gs_stream_status"):
+                 "gs_stream_status", "gs_selftest_wait_timeout"):
         getattr(L, name).restype = ctypes.c_int
     _lib = L
     return L
@@ -300,3 +302,9 @@ def stream_status(stream=None):
     L = load_library()
     st = L.gs_stream_status(_stream(stream) if stream is not False else None)
     _check(st, "gs_stream_status")
+
+
+def selftest_wait_timeout(stream=None):
+    """Enqueue a block whose bounded wait runs out (~2 s); see gs_selftest_wait_timeout.
+    stream_status() afterwards raises GramSpaceError with GS_ERR_TIMEOUT."""
+    _check(load_library().gs_selftest_wait_timeout(_stream(stream)), "gs_selftest_wait_timeout")
