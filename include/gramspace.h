@@ -115,6 +115,24 @@ GS_API gs_status gs_build_basis(const float* C, int M, int D, int ldc, float ran
 GS_API gs_status gs_basis_info(const gs_basis* h, int* M, int* D, int* r, const float** Q,
                         const float** R, const float** cnorm);
 
+/*
+ * Restores a handle from a basis saved earlier: the checkpoint / restore of the
+ * state gs_build_basis computes once at initialisation (Sec. 3.3), without
+ * running Gram-Schmidt again.  Save what gs_basis_info returns (Q, R, cnorm,
+ * with r, M, D) and pass it back here: every result of the restored handle then
+ * equals the original's bit for bit (its fp16 / bf16 operand copies are derived
+ * from the same fp32 values).
+ *   Q      r x D fp32, ld = ldq >= D (may be NULL when r = 0)
+ *   R      M x r fp32, ld = ldr >= r (may be NULL when r = 0)
+ *   cnorm  M fp32 codeword norms, or NULL to use ||R_i|| (equal to ||c_i||
+ *          because C = R Q with orthonormal Q)
+ * Device pointers owned by the caller; the handle keeps its own copies.  The
+ * rows of Q are taken as orthonormal and R as lower echelon (as a build leaves
+ * them); neither is re-checked.  Synchronises `stream` before returning.
+ */
+GS_API gs_status gs_basis_import(const float* Q, int r, int D, int ldq, const float* R, int M, int ldr,
+                                 const float* cnorm, void* stream, gs_basis** out);
+
 /* Releases a handle and its device memory (synchronises its device first). */
 GS_API gs_status gs_basis_destroy(gs_basis* h);
 

@@ -177,6 +177,29 @@ gs_status gs_build_basis(const float* C, int M, int D, int ldc, float rank_tol, 
     return GS_OK;
 }
 
+gs_status gs_basis_import(const float* Q, int r, int D, int ldq, const float* R, int M, int ldr,
+                          const float* cnorm, void* stream, gs_basis** out) {
+    if (!out) return GS_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (M < 1 || D < 1 || r < 0 || r > std::min(M, D)) return GS_ERR_SHAPE;
+    if (r > 0 && (ldq < D || ldr < r)) return GS_ERR_SHAPE;
+    if (r > 0 && (!Q || !R)) return GS_ERR_INVALID_ARG;
+    if (((uintptr_t)Q | (uintptr_t)R | (uintptr_t)cnorm) % sizeof(float)) return GS_ERR_ALIGNMENT;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return GS_ERR_CUDA;
+    if (!device_supported(dev)) return GS_ERR_UNSUPPORTED;
+    gs_basis* h = new gs_basis();
+    h->device = dev;
+    gs_status st = gs::import_basis(Q, ldq, R, ldr, cnorm, M, D, r, (cudaStream_t)stream, h);
+    if (st == GS_OK && gs::tc_available(dev)) st = gs::tc_prepare(h);
+    if (st != GS_OK) {
+        free_basis(h);
+        return st;
+    }
+    *out = h;
+    return GS_OK;
+}
+
 gs_status gs_basis_info(const gs_basis* h, int* M, int* D, int* r, const float** Q, const float** R,
                         const float** cnorm) {
     if (!h) return GS_ERR_INVALID_ARG;
@@ -246,11 +269,13 @@ gs_status gs_project_similarity(const gs_basis* h, const float* X, long long N, 
         a.C = Ybuf; a.c_type = gs::MAT_F32; a.ldc = ldyb;
         a.m = nc; a.n = r; a.k = D; a.batch = 1; a.alpha = 1.f;
         // few output tiles (a small batch against a narrow basis): cut D into chunks so that
-        // every SM gets work, partial sums added into Y (zeroed first)
-        a.ksplit = gemm_ksplit(nc, r, D, h->device);
-        if (a.ksplit > 1) {
-            cudaError_t e = cudaMemset2DAsync(Ybuf, sizeof(float) * ldyb, 0, sizeof(float) * r, nc, s);
-            if (e != cudaSuccess) return from_cuda(e);
+        // every SM gets work; the partial products go to the scratch after Y and the norms
+        // (the score rows are written there only later) and are summed in a fixed order
+        {
+            const long long used = (long long)(scr - h->scratch);
+            const long long room = (h->scratch_floats - used) / std::max(1LL, nc * r);
+            a.ksplit = (int)std::min<long long>(gemm_ksplit(nc, r, D, h->device), room);
+            a.kpart = a.ksplit > 1 ? scr : nullptr;
         }
         cudaError_t e = gs::launch_gemm_simt(a, s);
         if (e != cudaSuccess) return from_cuda(e);

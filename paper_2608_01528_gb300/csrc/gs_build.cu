@@ -276,6 +276,24 @@ __global__ void k_zero_half(__half* p, long long n) {
 
 inline unsigned grid1(long long n, int b) { return (unsigned)((n + b - 1) / b); }
 
+// fp32 rows (ld lds) -> fp64 rows (ld ldd)
+__global__ void k_widen_rows(const float* __restrict__ src, long long lds, double* __restrict__ dst,
+                             long long ldd, int rows, int cols) {
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)rows * cols) return;
+    const int i = (int)(idx / cols), j = (int)(idx % cols);
+    dst[(size_t)i * ldd + j] = (double)src[(size_t)i * lds + j];
+}
+
+// ||R_i|| in fp64, one thread per row (C = R Q with orthonormal Q, so this is ||c_i||)
+__global__ void k_row_norms64(const double* __restrict__ R64, int ldr, int M, int r, double* __restrict__ cn) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= M) return;
+    double ss = 0.0;
+    for (int j = 0; j < r; ++j) ss += R64[(size_t)i * ldr + j] * R64[(size_t)i * ldr + j];
+    cn[i] = sqrt(ss);
+}
+
 struct DevBuf {
     void* p = nullptr;
     ~DevBuf() { if (p) cudaFree(p); }
@@ -297,6 +315,9 @@ unsigned take_device_error_build() {
             return e_ == cudaErrorMemoryAllocation ? GS_ERR_NOMEM : GS_ERR_CUDA; \
         }                                                            \
     } while (0)
+
+gs_status finalize_basis(const double* Qw, const double* R64, int ldr, const double* cn, int M, int D, int r,
+                         cudaStream_t s, gs_basis* h);
 
 gs_status build_basis(const float* C, int M, int D, int ldc, double tau, bool normalize,
                       cudaStream_t s, gs_basis* h) {
@@ -342,6 +363,13 @@ gs_status build_basis(const float* C, int M, int D, int ldc, double tau, bool no
     int r = 0;
     GS_CK(cudaMemcpyAsync(&r, r_dev, sizeof(int), cudaMemcpyDeviceToHost, s));
     GS_CK(cudaStreamSynchronize(s));
+    return finalize_basis(Qw, R64, ldr, cn, M, D, r, s, h);
+}
+
+// Everything a handle holds besides the fp64 factorisation: fp32 Q, R and norms for the
+// caller, R's echelon lengths, the fp16 operand copies (dithered) and the chunk scratch.
+gs_status finalize_basis(const double* Qw, const double* R64, int ldr, const double* cn, int M, int D, int r,
+                         cudaStream_t s, gs_basis* h) {
     h->M = M;
     h->D = D;
     h->r = r;
@@ -384,6 +412,33 @@ gs_status build_basis(const float* C, int M, int D, int ldc, double tau, bool no
     GS_CK(cudaGetLastError());
     GS_CK(cudaStreamSynchronize(s));
     return GS_OK;
+}
+
+}  // namespace gs
+
+namespace gs {
+
+gs_status import_basis(const float* Q, int ldq, const float* R, int ldr_in, const float* cnorm, int M, int D,
+                       int r, cudaStream_t s, gs_basis* h) {
+    const int ldr = std::max(r, 1);
+    DevBuf bQw, bR64, bcn;
+    GS_CK(cudaMalloc(&bQw.p, sizeof(double) * (size_t)std::max(r, 1) * D));
+    GS_CK(cudaMalloc(&bR64.p, sizeof(double) * (size_t)M * ldr));
+    GS_CK(cudaMalloc(&bcn.p, sizeof(double) * (size_t)M));
+    double* Qw = (double*)bQw.p;
+    double* R64 = (double*)bR64.p;
+    double* cn = (double*)bcn.p;
+    GS_CK(cudaMemsetAsync(R64, 0, sizeof(double) * (size_t)M * ldr, s));
+    if (r > 0) {
+        k_widen_rows<<<grid1((long long)r * D, 256), 256, 0, s>>>(Q, ldq, Qw, D, r, D);
+        k_widen_rows<<<grid1((long long)M * r, 256), 256, 0, s>>>(R, ldr_in, R64, ldr, M, r);
+    }
+    if (cnorm)
+        k_widen_rows<<<grid1(M, 256), 256, 0, s>>>(cnorm, 1, cn, 1, M, 1);
+    else
+        k_row_norms64<<<grid1(M, 128), 128, 0, s>>>(R64, ldr, M, r, cn);
+    GS_CK(cudaGetLastError());
+    return finalize_basis(Qw, R64, ldr, cn, M, D, r, s, h);
 }
 
 }  // namespace gs

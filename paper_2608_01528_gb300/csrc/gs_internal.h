@@ -66,6 +66,9 @@ constexpr int kMinF16Depth = 1024;
 // tensor maps.  Synchronises `s` once.
 gs_status build_basis(const float* C, int M, int D, int ldc, double tau, bool normalize,
                       cudaStream_t s, gs_basis* h);
+// a handle from a saved basis (fp32 Q r x D, R M x r, optional norms), same finalisation as a build
+gs_status import_basis(const float* Q, int ldq, const float* R, int ldr_in, const float* cnorm, int M, int D,
+                       int r, cudaStream_t s, gs_basis* h);
 
 // ----------------------------------------------------------------- SIMT kernels (gs_simt.cu)
 enum { MAT_F32 = 0, MAT_BF16 = 1 };
@@ -89,8 +92,10 @@ struct GemmArgs {
     const float* rownorm; const float* colnorm;
     const int* b_rowlen;  // optional (b_trans only): row j of B is zero beyond b_rowlen[j]
     int ksplit;           // > 1 (batch 1, fp32 C only): K is cut into ksplit chunks, one per
-                          // grid z index, whose partial tiles are added into C atomically;
-                          // C must hold zeros before the launch
+                          // grid z index; each chunk's m x n partial product goes to kpart
+                          // (ksplit x m x n floats, caller's workspace) and a second kernel
+                          // sums the chunks in a fixed order into C (deterministic)
+    float* kpart;
 };
 cudaError_t launch_gemm_simt(const GemmArgs& g, cudaStream_t s);
 

@@ -210,13 +210,23 @@ __global__ void __launch_bounds__(256) k_gemm(GemmArgs g) {
                 v = den > 0.f ? v / den : 0.f;
             }
             if (TC == MAT_F32) {
-                if (split) atomicAdd((float*)Cb + gm * g.ldc + gn, v);
+                if (split) g.kpart[((size_t)blockIdx.z * g.m + gm) * g.n + gn] = v;
                 else ((float*)Cb)[gm * g.ldc + gn] = v;
             } else {
                 ((__nv_bfloat16*)Cb)[gm * g.ldc + gn] = __float2bfloat16_rn(v);
             }
         }
     }
+}
+
+// C[i][j] = sum over z (in order) of part[z][i][j]: the split-K partials of k_gemm
+__global__ void k_ksum(const float* __restrict__ part, int ks, long long m, int n, float* __restrict__ C,
+                       long long ldc) {
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= m * n) return;
+    float s = 0.f;
+    for (int z = 0; z < ks; ++z) s += part[(size_t)z * m * n + idx];
+    C[(idx / n) * ldc + idx % n] = s;
 }
 
 // ----------------------------------------------------------------- row kernels
@@ -296,13 +306,18 @@ cudaError_t launch_ps_warp(const float* X, long long N, int ldx, int D, const fl
 
 cudaError_t launch_gemm_simt(const GemmArgs& g, cudaStream_t s) {
     if (g.m <= 0 || g.n <= 0 || g.batch <= 0) return cudaSuccess;
-    if (g.ksplit > 1 && (g.batch != 1 || g.c_type != MAT_F32)) return cudaErrorInvalidValue;
+    if (g.ksplit > 1 && (g.batch != 1 || g.c_type != MAT_F32 || !g.kpart)) return cudaErrorInvalidValue;
     dim3 grid((unsigned)((g.n + kTN - 1) / kTN), (unsigned)((g.m + kTM - 1) / kTM),
               (unsigned)(g.ksplit > 1 ? g.ksplit : g.batch));
     if (grid.y > 65535u) return cudaErrorInvalidConfiguration;
 #define GS_GEMM_CASE(TA, TB, TC, BT)                                                        \
     if (g.a_type == TA && g.b_type == TB && g.c_type == TC && g.b_trans == BT) {            \
         k_gemm<TA, TB, TC, BT><<<grid, 256, 0, s>>>(g);                                     \
+        if (g.ksplit > 1) {                                                                 \
+            const long long mn = g.m * g.n;                                                 \
+            k_ksum<<<(unsigned)((mn + 255) / 256), 256, 0, s>>>(g.kpart, g.ksplit, g.m, g.n, \
+                                                                 (float*)g.C, g.ldc);       \
+        }                                                                                   \
         return cudaGetLastError();                                                          \
     }
     GS_GEMM_CASE(MAT_F32, MAT_F32, MAT_F32, true)

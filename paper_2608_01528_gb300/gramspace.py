@@ -30,7 +30,7 @@ GS_BUILD_NORMALIZE_ROWS = 1
 EXPORTS = ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_similarity",
            "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores", "gs_stream_status",
            "gs_status_string", "gs_version", "gs_project_similarity_static", "gs_similarity_coeffs",
-           "gs_selftest_wait_timeout")
+           "gs_selftest_wait_timeout", "gs_basis_import")
 
 
 class GramSpaceError(RuntimeError):
@@ -55,6 +55,7 @@ def load_library(path=LIB_PATH):
     L.gs_basis_info.argtypes = [vp, ctypes.POINTER(ip), ctypes.POINTER(ip), ctypes.POINTER(ip),
                                 ctypes.POINTER(vp), ctypes.POINTER(vp), ctypes.POINTER(vp)]
     L.gs_basis_destroy.argtypes = [vp]
+    L.gs_basis_import.argtypes = [vp, ip, ip, ip, vp, ip, ip, vp, vp, ctypes.POINTER(vp)]
     L.gs_project_similarity.argtypes = [vp, vp, i64, ip, ip, f32, u32, vp, ip, vp, ip, vp, vp, vp]
     L.gs_similarity_coeffs.argtypes = [vp, vp, i64, ip, ip, f32, u32, vp, ip, vp, vp, vp]
     L.gs_prob_vectorize.argtypes = [vp, vp, i64, ip, vp, ip, ip, u32, vp]
@@ -69,7 +70,7 @@ def load_library(path=LIB_PATH):
     L.gs_version.restype = ctypes.c_int
     for name in ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_similarity",
                  "gs_similarity_coeffs", "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores",
-                 "gs_stream_status", "gs_selftest_wait_timeout"):
+                 "gs_stream_status", "gs_selftest_wait_timeout", "gs_basis_import"):
         getattr(L, name).restype = ctypes.c_int
     _lib = L
     return L
@@ -177,6 +178,23 @@ def build_basis(C, rank_tol=1e-6, normalize_rows=False, stream=None):
                               ctypes.byref(h))
     _check(st, "gs_build_basis")
     return Basis(h, C.device)
+
+
+def import_basis(Q, R, cnorm=None, stream=None):
+    """Restore a basis saved from Basis.Q / Basis.R / Basis.cnorm (fp32 CUDA tensors, Q: r x D,
+    R: M x r); see gs_basis_import.  The restored basis gives bit-identical results."""
+    for t in (Q, R) + ((cnorm,) if cnorm is not None else ()):
+        if not t.is_cuda or t.dtype != torch.float32:
+            raise TypeError("Q, R and cnorm must be float32 CUDA tensors")
+    r, D = Q.shape
+    M = R.shape[0]
+    L = load_library()
+    h = ctypes.c_void_p()
+    with torch.cuda.device(R.device):
+        st = L.gs_basis_import(_ptr(Q) if r else None, r, D, _ld(Q) if r else D, _ptr(R) if r else None, M,
+                               _ld(R) if r else 1, _ptr(cnorm), _stream(stream), ctypes.byref(h))
+    _check(st, "gs_basis_import")
+    return Basis(h, R.device)
 
 
 def project_similarity(basis, X, mode="raw", scale=1.0, path="auto", want_Y=False, want_S=False,
