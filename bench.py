@@ -69,15 +69,24 @@ def load_peaks():
         return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "src": "fallback"}
 
 
+def kernel_source_sha(kernel_file, kernel_name):
+    """sha256 of one kernel's device source: from its __global__ declaration to the
+    file's host-side section marker (edits elsewhere in the file leave it unchanged)."""
+    src = open(os.path.join(ROOT, "paper_2608_01528_gb300", "csrc", kernel_file)).read()
+    start = src.index(f"\n    {kernel_name}(")
+    start = src.rindex("__global__", 0, start)
+    end = src.index("// ----------------------------------------------------------------- host side", start)
+    return hashlib.sha256(src[start:end].encode()).hexdigest()
+
+
 def traffic_record(kernel_file, key):
     """DRAM traffic per launch from a committed ncu summary, valid only while the
-    kernel source is unchanged (sha256 recorded next to the number)."""
+    kernel's source is unchanged (sha256 of that source recorded next to the number)."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f)[key]
-        src = os.path.join(ROOT, "paper_2608_01528_gb300", "csrc", kernel_file)
-        h = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        h = kernel_source_sha(kernel_file, key.split("/")[0])
         return rec["bytes_per_launch"] if rec.get("source_sha256") == h else None
     except Exception:
         return None
