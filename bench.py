@@ -107,16 +107,15 @@ class ClockSampler:
         try:
             self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={q}",
-                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=self.file, stderr=subprocess.DEVNULL)
-            time.sleep(0.3)
+            time.sleep(0.1)
         except Exception:
             self.proc = None
         return self
 
     def __exit__(self, *a):
         if self.proc is not None:
-            time.sleep(0.2)
             self.proc.terminate()
             try:
                 self.proc.wait(timeout=5)
@@ -148,7 +147,9 @@ class ClockSampler:
         if not sm:
             return None
         self._summary = {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
-                         "samples": len(sm)}
+                         "samples": len(sm),
+                         "window": "every 50 ms over the timed steps and 0.4 s / 0.3 s of the same step "
+                                   "just before / after them"}
         return self._summary
 
 
@@ -282,14 +283,26 @@ def main():
             pg.barrier()
         torch.cuda.synchronize()
 
+    def load(seconds):
+        # untimed steps around the timed ones: the timed region itself lasts milliseconds,
+        # nvidia-smi samples every 50 ms, so the samples are taken with the GPU under this
+        # same load just before, during and just after it
+        t_end = time.perf_counter() + seconds
+        while time.perf_counter() < t_end:
+            for _ in range(16):
+                step()
+            torch.cuda.synchronize()
+
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clk:
+        load(0.4)
         barrier()
         e0.record(stream)
         for _ in range(args.steps):
             step()
         e1.record(stream)
         barrier()
+        load(0.3)
     ms = max_over_ranks(e0.elapsed_time(e1), pg, dev)
     gs.stream_status()
     per_step_ms = ms / args.steps
