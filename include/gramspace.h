@@ -25,8 +25,9 @@
  *  - Errors that only the device can see (a bounded wait that ran out, an
  *    input outside a fast path's numeric range) set a per-device error word;
  *    gs_stream_status() synchronises the stream and returns and clears it.
- *  - Only gs_build_basis allocates device memory; the other calls allocate
- *    nothing.  N = 0 is a valid no-op.
+ *  - Only gs_build_basis, gs_basis_import and gs_basis_reserve_staging
+ *    allocate device memory; the other calls allocate nothing.  N = 0 is a
+ *    valid no-op.
  *  - All functions are callable from any host thread; a gs_basis must not be
  *    destroyed while work that uses it is in flight.  Some paths keep
  *    intermediate results in a scratch area owned by the gs_basis (the two-GEMM
@@ -158,6 +159,36 @@ GS_API gs_status gs_basis_destroy(gs_basis* h);
 GS_API gs_status gs_project_similarity(const gs_basis* h, const float* X, long long N, int ldx,
                                 int mode, float scale, unsigned flags, float* Y, int ldy,
                                 float* S, int lds, int* argmax, float* maxval, void* stream);
+
+/*
+ * Device staging for gs_project_similarity_host, owned by the handle: two slots,
+ * each holding `rows` queries of the basis' dimension D (fp32) and their argmax /
+ * maxval (2 x rows x (4 D + 8) bytes), plus a copy stream and five events.
+ * rows = 0 releases it (gs_basis_destroy releases it too); a new call replaces
+ * the old staging.  Reserve it once, outside any timed or latency-critical code:
+ * besides the two builds this is the only call that allocates.  Must not be
+ * called while work that uses the staging is in flight.
+ */
+GS_API gs_status gs_basis_reserve_staging(gs_basis* h, long long rows);
+
+/*
+ * Project + similarity from HOST memory (Sec. 3.1 / 2.2, as gs_project_similarity
+ * with Y and S not returned): X is N x D fp32 in host memory (ld = ldx >= D),
+ * argmax / maxval are host arrays of N (either may be NULL, not both).  The
+ * queries go through the staging (gs_basis_reserve_staging) in chunks of its
+ * rows, alternating between its two slots: chunk i is copied in on the handle's
+ * copy stream while chunk i - 1 is scored on `stream`, and each chunk's results
+ * are copied back on `stream`.  The work starts after what is already enqueued on
+ * `stream`, and work enqueued on `stream` after the call starts after all of it.
+ * The call returns before the work finishes: X must stay unchanged and the host
+ * arrays valid until then.  Use page-locked host memory (cudaHostAlloc, torch
+ * pin_memory) for the copies to run asynchronously at the link's rate.
+ * Returns GS_ERR_INVALID_ARG when no staging has been reserved.  The staging is
+ * shared by every call on the handle: calls on different streams must be ordered.
+ */
+GS_API gs_status gs_project_similarity_host(const gs_basis* h, const float* X, long long N, int ldx, int mode,
+                                            float scale, unsigned flags, int* argmax, float* maxval,
+                                            void* stream);
 
 /*
  * Similarity of queries given by their Gram-loc coordinates (Sec. 3.2, Eq. 2:

@@ -43,6 +43,21 @@ bool valid_path(unsigned flags) {
     return flags == GS_PATH_AUTO || flags == GS_PATH_SIMT || flags == GS_PATH_TENSOR;
 }
 
+void release_staging(gs_basis* h) {
+    cudaFree(h->stage_x);
+    cudaFree(h->stage_am);
+    cudaFree(h->stage_mv);
+    if (h->stage_copy) cudaStreamDestroy(h->stage_copy);
+    cudaEvent_t* evs[5] = {&h->stage_start, &h->stage_in[0], &h->stage_in[1], &h->stage_done[0], &h->stage_done[1]};
+    for (cudaEvent_t* ev : evs)
+        if (*ev) cudaEventDestroy(*ev), *ev = nullptr;
+    h->stage_x = nullptr;
+    h->stage_am = nullptr;
+    h->stage_mv = nullptr;
+    h->stage_copy = nullptr;
+    h->stage_rows = 0;
+}
+
 void free_basis(gs_basis* h) {
     if (!h) return;
     cudaFree(h->Q);
@@ -53,6 +68,7 @@ void free_basis(gs_basis* h) {
     cudaFree(h->Q16);
     cudaFree(h->Q16t);
     cudaFree(h->scratch);
+    release_staging(h);
     cudaFree(h->tc_Rh);
     cudaFree(h->tc_Rl);
     cudaFree(h->tc_Rth);
@@ -295,6 +311,80 @@ gs_status gs_project_similarity(const gs_basis* h, const float* X, long long N, 
                                       argmax ? argmax + c0 : nullptr, maxval ? maxval + c0 : nullptr, s);
             if (e != cudaSuccess) return from_cuda(e);
         }
+    }
+    return GS_OK;
+}
+
+gs_status gs_basis_reserve_staging(gs_basis* h, long long rows) {
+    if (!h) return GS_ERR_INVALID_ARG;
+    if (rows < 0) return GS_ERR_SHAPE;
+    DeviceGuard g(h->device);
+    if (!g.ok) return GS_ERR_CUDA;
+    release_staging(h);
+    if (rows == 0) return GS_OK;
+    const int ld = (h->D + 3) / 4 * 4;  // 16-byte rows, as the tensor-core path needs
+    bool ok = cudaMalloc(&h->stage_x, sizeof(float) * 2 * (size_t)rows * ld) == cudaSuccess &&
+              cudaMalloc(&h->stage_am, sizeof(int) * 2 * (size_t)rows) == cudaSuccess &&
+              cudaMalloc(&h->stage_mv, sizeof(float) * 2 * (size_t)rows) == cudaSuccess;
+    if (!ok) {
+        release_staging(h);
+        return GS_ERR_NOMEM;
+    }
+    ok = cudaStreamCreateWithFlags(&h->stage_copy, cudaStreamNonBlocking) == cudaSuccess &&
+         cudaEventCreateWithFlags(&h->stage_start, cudaEventDisableTiming) == cudaSuccess;
+    for (int b = 0; b < 2 && ok; ++b)
+        ok = cudaEventCreateWithFlags(&h->stage_in[b], cudaEventDisableTiming) == cudaSuccess &&
+             cudaEventCreateWithFlags(&h->stage_done[b], cudaEventDisableTiming) == cudaSuccess;
+    if (!ok) {
+        release_staging(h);
+        return GS_ERR_CUDA;
+    }
+    h->stage_rows = rows;
+    h->stage_ld = ld;
+    return GS_OK;
+}
+
+gs_status gs_project_similarity_host(const gs_basis* h, const float* X, long long N, int ldx, int mode,
+                                     float scale, unsigned flags, int* argmax, float* maxval, void* stream) {
+    if (!h || !valid_path(flags)) return GS_ERR_INVALID_ARG;
+    if (mode < GS_SCORE_RAW || mode > GS_SCORE_SOFTMAX || !isfinite(scale)) return GS_ERR_INVALID_ARG;
+    if (N < 0 || ldx < h->D) return GS_ERR_SHAPE;
+    if (N == 0) return GS_OK;
+    if (!X || (!argmax && !maxval)) return GS_ERR_INVALID_ARG;
+    if (h->stage_rows < 1) return GS_ERR_INVALID_ARG;  // gs_basis_reserve_staging first
+    DeviceGuard g(h->device);
+    if (!g.ok) return GS_ERR_CUDA;
+    cudaStream_t s = (cudaStream_t)stream;
+    const long long R = h->stage_rows;
+    // The copy stream starts after the work already on s (which may still read the slots).
+    // Chunk i goes through slot i & 1: its copy in (copy stream) waits until chunk i - 2 has
+    // finished with the slot; the kernel and the copies out (on s) wait for the copy in.
+    // s waits for every copy-stream event, so work enqueued on s later follows all of it.
+    cudaError_t e = cudaEventRecord(h->stage_start, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(h->stage_copy, h->stage_start, 0);
+    if (e != cudaSuccess) return from_cuda(e);
+    long long i = 0;
+    for (long long c0 = 0; c0 < N; c0 += R, ++i) {
+        const int b = (int)(i & 1);
+        const long long nc = std::min(R, N - c0);
+        float* sx = h->stage_x + (size_t)b * R * h->stage_ld;
+        int* sam = h->stage_am + (size_t)b * R;
+        float* smv = h->stage_mv + (size_t)b * R;
+        if (i >= 2) e = cudaStreamWaitEvent(h->stage_copy, h->stage_done[b], 0);
+        if (e == cudaSuccess)
+            e = cudaMemcpy2DAsync(sx, sizeof(float) * h->stage_ld, X + c0 * ldx, sizeof(float) * ldx,
+                                  sizeof(float) * h->D, nc, cudaMemcpyHostToDevice, h->stage_copy);
+        if (e == cudaSuccess) e = cudaEventRecord(h->stage_in[b], h->stage_copy);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(s, h->stage_in[b], 0);
+        if (e != cudaSuccess) return from_cuda(e);
+        gs_status st = gs_project_similarity(h, sx, nc, h->stage_ld, mode, scale, flags, nullptr, 0, nullptr, 0,
+                                             argmax ? sam : nullptr, maxval ? smv : nullptr, stream);
+        if (st != GS_OK) return st;
+        if (argmax) e = cudaMemcpyAsync(argmax + c0, sam, sizeof(int) * nc, cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess && maxval)
+            e = cudaMemcpyAsync(maxval + c0, smv, sizeof(float) * nc, cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaEventRecord(h->stage_done[b], s);
+        if (e != cudaSuccess) return from_cuda(e);
     }
     return GS_OK;
 }

@@ -47,6 +47,16 @@ struct gs_basis {
     void* tc_Qh = nullptr;
     void* tc_Ql = nullptr;
     bool has_split = false;         // tc_Rh / tc_Rl / tc_Rth / tc_Rtl exist
+    // device staging of gs_project_similarity_host (gs_basis_reserve_staging): two slots,
+    // each of stage_rows queries (row pitch stage_ld floats) and their argmax / maxval, a
+    // stream for the host-to-device copies and the events that order the two streams
+    float* stage_x = nullptr;   // 2 x stage_rows x stage_ld
+    int* stage_am = nullptr;    // 2 x stage_rows
+    float* stage_mv = nullptr;  // 2 x stage_rows
+    long long stage_rows = 0;
+    int stage_ld = 0;
+    cudaStream_t stage_copy = nullptr;
+    cudaEvent_t stage_start = nullptr, stage_in[2] = {nullptr, nullptr}, stage_done[2] = {nullptr, nullptr};
     // scratch for the multi-kernel paths (rows processed in chunks)
     float* scratch = nullptr;
     long long scratch_floats = 0;

@@ -30,7 +30,8 @@ GS_BUILD_NORMALIZE_ROWS = 1
 EXPORTS = ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_similarity",
            "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores", "gs_stream_status",
            "gs_status_string", "gs_version", "gs_project_similarity_static", "gs_similarity_coeffs",
-           "gs_selftest_wait_timeout", "gs_basis_import")
+           "gs_selftest_wait_timeout", "gs_basis_import", "gs_basis_reserve_staging",
+           "gs_project_similarity_host")
 
 
 class GramSpaceError(RuntimeError):
@@ -55,6 +56,8 @@ def load_library(path=LIB_PATH):
     L.gs_basis_info.argtypes = [vp, ctypes.POINTER(ip), ctypes.POINTER(ip), ctypes.POINTER(ip),
                                 ctypes.POINTER(vp), ctypes.POINTER(vp), ctypes.POINTER(vp)]
     L.gs_basis_destroy.argtypes = [vp]
+    L.gs_basis_reserve_staging.argtypes = [vp, i64]
+    L.gs_project_similarity_host.argtypes = [vp, vp, i64, ip, ip, f32, u32, vp, vp, vp]
     L.gs_basis_import.argtypes = [vp, ip, ip, ip, vp, ip, ip, vp, vp, ctypes.POINTER(vp)]
     L.gs_project_similarity.argtypes = [vp, vp, i64, ip, ip, f32, u32, vp, ip, vp, ip, vp, vp, vp]
     L.gs_similarity_coeffs.argtypes = [vp, vp, i64, ip, ip, f32, u32, vp, ip, vp, vp, vp]
@@ -70,7 +73,8 @@ def load_library(path=LIB_PATH):
     L.gs_version.restype = ctypes.c_int
     for name in ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_similarity",
                  "gs_similarity_coeffs", "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores",
-                 "gs_stream_status", "gs_selftest_wait_timeout", "gs_basis_import"):
+                 "gs_stream_status", "gs_selftest_wait_timeout", "gs_basis_import",
+                 "gs_basis_reserve_staging", "gs_project_similarity_host"):
         getattr(L, name).restype = ctypes.c_int
     _lib = L
     return L
@@ -195,6 +199,39 @@ def import_basis(Q, R, cnorm=None, stream=None):
                                _ld(R) if r else 1, _ptr(cnorm), _stream(stream), ctypes.byref(h))
     _check(st, "gs_basis_import")
     return Basis(h, R.device)
+
+
+def reserve_staging(basis, rows):
+    """Device staging for project_similarity_host (rows queries); see gs_basis_reserve_staging."""
+    L = load_library()
+    with torch.cuda.device(basis.device):
+        _check(L.gs_basis_reserve_staging(basis.handle, int(rows)), "gs_basis_reserve_staging")
+
+
+def project_similarity_host(basis, X, mode="raw", scale=1.0, path="auto", want_argmax=True, want_maxval=True,
+                            out=None, stream=None):
+    """Project + similarity of host queries X (N x D float32 CPU tensor, ideally pinned) into host
+    outputs; see gs_project_similarity_host.  Asynchronous on `stream`: synchronise before reading
+    the outputs, and keep X referenced (and unchanged) until then -- a pinned tensor freed earlier
+    returns its block to torch's host allocator, which can reuse it while the copy is queued."""
+    if X.is_cuda or X.dtype != torch.float32:
+        raise TypeError("X must be a float32 CPU tensor")
+    if X.dim() != 2 or X.shape[1] != basis.D:
+        raise ValueError(f"X must be N x {basis.D}")
+    N = X.shape[0]
+    out = dict(out or {})
+    pin = X.is_pinned()
+    if want_argmax and "argmax" not in out:
+        out["argmax"] = torch.empty(N, dtype=torch.int32, pin_memory=pin)
+    if want_maxval and "maxval" not in out:
+        out["maxval"] = torch.empty(N, dtype=torch.float32, pin_memory=pin)
+    L = load_library()
+    with torch.cuda.device(basis.device):
+        st = L.gs_project_similarity_host(basis.handle, _ptr(X), N, _ld(X), MODES[mode], float(scale),
+                                          PATHS[path], _ptr(out.get("argmax")), _ptr(out.get("maxval")),
+                                          _stream(stream))
+    _check(st, "gs_project_similarity_host")
+    return out
 
 
 def project_similarity(basis, X, mode="raw", scale=1.0, path="auto", want_Y=False, want_S=False,
