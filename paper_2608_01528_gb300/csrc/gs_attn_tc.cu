@@ -344,10 +344,258 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
+// ================================================================= one pass, key units spread over a cluster
+// With the row softmax and Lk <= 4 x 256, the G = ceil(Lk / 256) CTAs of a thread-block
+// cluster share each work item: CTA g computes the logits of keys [256 g, 256 g + 256)
+// for the item's 128 queries, once.  Each epilogue thread holds 128 logits of one
+// query row in registers (one TMEM read, after which the accumulator is released to
+// the MMA), takes their max m and p_j = exp(scale s_j - m) and sum l, and posts (m, l)
+// to every CTA of the cluster through distributed shared memory.  With all 2 G partial
+// results of its row a thread has the row's max M and sum L and writes
+// p_j exp(m - M) / L: one exponential per output.  The probabilities go out through a
+// swizzled shared-memory tile and TMA tensor stores (a 3-D map over B x Lq x Lk, so
+// rows past Lq and keys past Lk are clipped).  Compared with the two-pass kernel above
+// this halves the MMA work and the exponentials; the TMEM accumulator is
+// double-buffered over items, so an item's exchange and writes overlap the next
+// item's MMAs.
+//
+// Warp roles (320 threads): 0-7 epilogue (warp w: TMEM lanes 32 (w % 4) = query rows,
+// keys [128 (w / 4), +128) of the CTA's unit), 8 TMA producer (query and key K-blocks
+// into one stage), 9 TMEM allocator + MMA issuer.
+
+constexpr int kClMaxG = 4;
+constexpr int kClStageBytes = kQBlockBytes + kKStageBytes;  // 48 KB: query block, then key block
+constexpr int kClStages = 3;
+constexpr int kClThreads = 10 * 32;
+constexpr int kClStgBytes = 32 * 32 * 4;  // one output box: 32 query rows x 32 keys fp32 (128-byte rows)
+
+struct ClCtl {
+    uint64_t full[kClStages], empty[kClStages];
+    uint64_t d_full[2], d_empty[2];
+    uint64_t x_full[2];           // statistics of an item from every CTA's every key half (by item parity)
+    uint64_t mma_done;
+    float2 xch[2][2 * kClMaxG][kBM];  // [item parity][2 rank + key half][query row] = (max, sum)
+    uint32_t tmem_base;
+    int abort_flag;
+};
+
+__global__ void __launch_bounds__(kClThreads, 1)
+    k_attn_cl(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
+              const __grid_constant__ CUtensorMap tmap_a, const AttnParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+    uint8_t* St = base;                                          // kClStages x 48 KB
+    uint8_t* Stg = St + (size_t)kClStages * kClStageBytes;       // 8 warps x 2 x 4 KB output boxes
+    ClCtl& c = *reinterpret_cast<ClCtl*>(Stg + (size_t)kEpiWarps * 2 * kClStgBytes);
+    volatile int* abort_flag = &c.abort_flag;
+    unsigned* err = &g_err_attn;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    const int G = p.ntiles;  // CTAs per cluster = key units per row
+    const long long cid = cluster_id_x(), ncl = cluster_count_x();
+    const long long items = (long long)p.B * p.qtiles;
+    const int nitems = items > cid ? (int)((items - 1 - cid) / ncl + 1) : 0;
+    const int nkb = p.nkb;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kClStages; ++s) {
+            mbar_init(&c.full[s], 1);
+            mbar_init(&c.empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&c.d_full[b], 1);
+            mbar_init(&c.d_empty[b], kEpiWarps);
+            mbar_init(&c.x_full[b], 1);
+        }
+        mbar_init(&c.mma_done, 1);
+        c.abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 9) {
+        tmem_alloc(&c.tmem_base, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync_all();  // every CTA's barriers exist before any CTA arrives on them
+    tc_fence_after();
+    const uint32_t tmem = c.tmem_base;
+
+    auto item_bq = [&](int li, int& b, int& qt) {
+        const long long ig = cid + (long long)li * ncl;
+        b = (int)(ig / p.qtiles);
+        qt = (int)(ig % p.qtiles);
+    };
+
+    if (warp == 8) {
+        // ------------------------------------------------------------- query + key K-blocks via TMA
+        if (lane == 0) {
+            const uint64_t pol = l2_policy_evict_last();
+            RingPos st;
+            int it = 0;
+            bool ok = true;
+            for (int li = 0; li < nitems && ok; ++li) {
+                int b, qt;
+                item_bq(li, b, qt);
+                for (int kb = 0; kb < nkb; ++kb, ++it, st.next(kClStages)) {
+                    if (!mbar_wait_1t(&c.empty[st.idx], st.phase ^ 1u, abort_flag, err)) {
+                        ok = false;
+                        break;
+                    }
+                    uint8_t* dst = St + (size_t)st.idx * kClStageBytes;
+                    mbar_arrive_expect_tx(&c.full[st.idx], kClStageBytes);
+                    tma_load_2d(dst, &tmap_q, &c.full[st.idx], kb * kBK, b * p.Lq + qt * kBM, pol);
+                    tma_load_2d(dst + kQBlockBytes, &tmap_k, &c.full[st.idx], kb * kBK,
+                                b * p.Lk + (int)rank * kBN, pol);
+                }
+            }
+            for (int j = std::max(0, it - kClStages); j < it; ++j)
+                mbar_drain(&c.full[j % kClStages], (uint32_t)(j / kClStages) & 1u, err);
+        }
+    } else if (warp == 9) {
+        // ------------------------------------------------------------- MMA issue
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(kBN);
+            RingPos st;
+            bool ok = true;
+            for (int li = 0; li < nitems && ok; ++li) {
+                const int buf = li & 1;
+                if (!mbar_wait_1t(&c.d_empty[buf], ((uint32_t)(li >> 1) & 1u) ^ 1u, abort_flag, err)) break;
+                tc_fence_after();
+                const uint32_t d_tmem = tmem + (uint32_t)(buf * kBN);
+                for (int kb = 0; kb < nkb; ++kb, st.next(kClStages)) {
+                    if (!mbar_wait_1t(&c.full[st.idx], st.phase, abort_flag, err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(St + (size_t)st.idx * kClStageBytes);
+                    const uint64_t ad = sdesc_sw128(sa);
+                    const uint64_t bd = sdesc_sw128(sa + kQBlockBytes);
+#pragma unroll
+                    for (int k = 0; k < kBK / 16; ++k)
+                        mma_f16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
+                                   (kb | k) != 0 ? 1u : 0u);
+                    mma_commit(&c.empty[st.idx]);
+                }
+                if (ok) mma_commit(&c.d_full[buf]);
+            }
+            mma_commit(&c.mma_done);
+            mbar_drain(&c.mma_done, 0, err);
+        }
+    } else {
+        // ------------------------------------------------------------- epilogue
+        const int quad = warp & 3, kh = warp >> 2;
+        const int i = quad * 32 + lane;                   // query row within the item
+        const int key0 = (int)rank * kBN + kh * (kBN / 2);  // first of this warp's 128 keys
+        const int nvalid = min(kBN / 2, max(0, p.Lk - key0));
+        uint8_t* stg = Stg + (size_t)warp * 2 * kClStgBytes;
+        const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+        const uint32_t xbar = smem_u32(&c.x_full[0]);
+        for (int li = 0; li < nitems; ++li) {
+            int b, qt;
+            item_bq(li, b, qt);
+            const int buf = li & 1, par = li & 1;
+            const uint32_t ph = (uint32_t)(li >> 1) & 1u;
+            if (!mbar_wait_warp(&c.d_full[buf], ph, abort_flag, err)) break;
+            tc_fence_after();
+            float v[kBN / 2];
+            tmem_ld128(tmem + lane_base + (uint32_t)(buf * kBN + kh * (kBN / 2)), v);
+            // the logits are in registers: the accumulator goes back to the MMA
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&c.d_empty[buf]);
+            // this thread's part of its row: max m, p_j = exp(scale s_j - m), sum l
+            float mx8[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) mx8[k] = -INFINITY;
+#pragma unroll
+            for (int j = 0; j < kBN / 2; ++j) {
+                v[j] = j < nvalid ? p.scale * v[j] : -INFINITY;
+                mx8[j & 7] = fmaxf(mx8[j & 7], v[j]);
+            }
+            const float m = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                                  fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+            const float mref = m == -INFINITY ? 0.f : m;
+            float l8[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) l8[k] = 0.f;
+#pragma unroll
+            for (int j = 0; j < kBN / 2; ++j) {
+                v[j] = __expf(v[j] - mref);
+                l8[j & 7] += v[j];
+            }
+            const float l = ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
+            // post (m, l) to every CTA of the cluster, then merge the 2 G partial results of the row
+            {
+                const uint32_t slot = smem_u32(&c.xch[par][2 * rank + kh][i]);
+                const uint32_t bar = xbar + (uint32_t)(par * sizeof(uint64_t));
+                // the barrier's one arrival per phase carries the byte count of every CTA's
+                // posts; the posts are asynchronous stores that complete those bytes (a
+                // release-arrive after plain remote stores cost microseconds per item)
+                if (threadIdx.x == 0) mbar_arrive_expect_tx(&c.x_full[par], (uint32_t)(G * kEpiWarps * 32 * 8));
+                for (int g = 0; g < G; ++g)
+                    st_async_f32x2(mapa_shared(slot, (uint32_t)g), m, l, mapa_shared(bar, (uint32_t)g));
+            }
+            const bool got = mbar_wait_cluster(&c.x_full[par], ph, abort_flag, err);
+            if (!__all_sync(0xffffffffu, got)) break;
+            float f;
+            {
+                float M = -INFINITY;
+                for (int j = 0; j < 2 * G; ++j) M = fmaxf(M, c.xch[par][j][i].x);
+                float L = 0.f;
+                for (int j = 0; j < 2 * G; ++j) {
+                    const float2 e = c.xch[par][j][i];
+                    if (e.y > 0.f) L += e.y * __expf(e.x - M);
+                }
+                f = l > 0.f ? __expf(mref - M) / L : 0.f;
+            }
+            // four boxes of 32 keys: swizzled shared-memory tile (16-byte chunk k of row
+            // `lane` at chunk k ^ (lane % 8), the TMA's 128-byte swizzle), then a tensor store
+            const int x0 = key0, y = qt * kBM + quad * 32;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                uint8_t* sb = stg + (size_t)(q & 1) * kClStgBytes;
+                if (lane == 0) bulk_wait_read_1();  // the store that last read this buffer is done with it
+                __syncwarp();
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    const float4 o = make_float4(v[32 * q + 4 * k] * f, v[32 * q + 4 * k + 1] * f,
+                                                 v[32 * q + 4 * k + 2] * f, v[32 * q + 4 * k + 3] * f);
+                    *reinterpret_cast<float4*>(sb + lane * 128 + ((k ^ (lane & 7)) << 4)) = o;
+                }
+                fence_proxy_async();
+                __syncwarp();
+                if (lane == 0) {
+                    if (x0 + 32 * q < p.Lk && y < p.Lq) tma_store_3d(&tmap_a, sb, x0 + 32 * q, y, b);
+                    bulk_commit();
+                }
+            }
+        }
+        if (lane == 0) bulk_wait_all();
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync_all();  // no CTA leaves while a peer may still post into its shared memory
+    if (warp == 9) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+constexpr size_t kClSmemBytes =
+    1024 + (size_t)kClStages * kClStageBytes + (size_t)kEpiWarps * 2 * kClStgBytes + sizeof(ClCtl);
+static_assert(kClSmemBytes <= 227 * 1024, "cluster attention kernel shared memory exceeds the per-CTA limit");
+
 constexpr size_t kSmemBytes = 1024 + (size_t)kMaxKB * kQBlockBytes + (size_t)kKStages * kKStageBytes + sizeof(Ctl);
 static_assert(kSmemBytes <= 227 * 1024, "attention kernel shared memory exceeds the per-CTA limit");
 
 bool g_attr_set[64];
+bool g_cl_attr_set[64];
+int g_cl_max[64][kClMaxG + 1];  // active clusters of k_attn_cl per device and cluster size
 
 }  // namespace
 
@@ -382,6 +630,46 @@ cudaError_t launch_attn_tc(const void* Yq, const void* Yk, int B, int Lq, int Lk
         !make_tmap_2d(&tk, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, Yk, (long long)B * Lk, r, ldy, kBK, kBN,
                       CU_TENSOR_MAP_SWIZZLE_128B))
         return cudaErrorInvalidValue;
+    const long long items = (long long)B * p.qtiles;
+    CUtensorMap ta;
+    if (softmax && p.ntiles <= kClMaxG && Lk % 4 == 0 && (uintptr_t)A % 16 == 0 &&
+        make_tmap_3d(&ta, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, A, Lk, Lq, B, Lk, (long long)Lq * Lk, 32, 32,
+                     CU_TENSOR_MAP_SWIZZLE_128B)) {
+        // one pass: the key units of a row spread over a cluster of ntiles CTAs
+        const int G = p.ntiles;
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = (unsigned)G;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.blockDim = dim3(kClThreads);
+        cfg.dynamicSmemBytes = kClSmemBytes;
+        cfg.stream = s;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if (device < 0 || device >= 64) return cudaErrorInvalidDevice;
+        if (!g_cl_attr_set[device]) {
+            cudaError_t e =
+                cudaFuncSetAttribute(k_attn_cl, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kClSmemBytes);
+            if (e != cudaSuccess) return e;
+            g_cl_attr_set[device] = true;
+        }
+        int& ncl_max = g_cl_max[device][G];
+        if (ncl_max <= 0) {
+            int sms = 0;
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+            cfg.gridDim = dim3((unsigned)(std::max(sms, G) / G * G));
+            cudaError_t e = cudaOccupancyMaxActiveClusters(&ncl_max, k_attn_cl, &cfg);
+            if (e != cudaSuccess) return e;
+            if (ncl_max <= 0) return cudaErrorInvalidConfiguration;
+        }
+        const long long ncl = std::min<long long>(ncl_max, items);
+        cfg.gridDim = dim3((unsigned)(ncl * G));
+        cudaError_t e = cudaLaunchKernelEx(&cfg, k_attn_cl, tq, tk, ta, p);
+        if (e != cudaSuccess) return e;
+        return cudaGetLastError();
+    }
     if (device >= 0 && device < 64 && !g_attr_set[device]) {
         cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
         if (e != cudaSuccess) return e;
@@ -389,7 +677,6 @@ cudaError_t launch_attn_tc(const void* Yq, const void* Yk, int B, int Lq, int Lk
     }
     int sms = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
-    const long long items = (long long)B * p.qtiles;
     const int grid = (int)std::min<long long>(sms > 0 ? sms : 1, items);
     k_attn_tc<<<grid, kThreads, kSmemBytes, s>>>(tq, tk, p);
     return cudaGetLastError();
