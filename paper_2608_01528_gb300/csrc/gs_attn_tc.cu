@@ -53,6 +53,7 @@ struct AttnParams {
     int B, Lq, Lk, r, nkb;
     int qtiles, ntiles;      // query tiles per sequence, key tiles per sequence
     int passes;              // 2 with the row softmax, 1 for plain scaled logits
+    int qslice;              // cluster kernel: rows of the query tile each CTA loads for all (0: whole tile, own CTA only)
     float scale;
     float* A;                // B x Lq x Lk
     int a_vec;               // rows aligned for two-element stores (Lk even, A 8-byte aligned)
@@ -379,9 +380,32 @@ struct ClCtl {
     int abort_flag;
 };
 
+// 2^x on the special-function unit (ex2.approx.ftz: 2^-inf = 0).
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// max (MIN: min) of v[0, n), eight independent chains; MASK: n may be below the length
+template <bool MIN, bool MASK>
+__device__ __forceinline__ float row_extreme(const float* v, int n) {
+    float e8[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) e8[k] = MIN ? INFINITY : -INFINITY;
+#pragma unroll
+    for (int j = 0; j < kBN / 2; ++j)
+        if (!MASK || j < n) e8[j & 7] = MIN ? fminf(e8[j & 7], v[j]) : fmaxf(e8[j & 7], v[j]);
+    if (MIN)
+        return fminf(fminf(fminf(e8[0], e8[1]), fminf(e8[2], e8[3])), fminf(fminf(e8[4], e8[5]), fminf(e8[6], e8[7])));
+    return fmaxf(fmaxf(fmaxf(e8[0], e8[1]), fmaxf(e8[2], e8[3])), fmaxf(fmaxf(e8[4], e8[5]), fmaxf(e8[6], e8[7])));
+}
+
 __global__ void __launch_bounds__(kClThreads, 1)
     k_attn_cl(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
               const __grid_constant__ CUtensorMap tmap_a, const AttnParams p) {
+    // tmap_q boxes are p.qslice rows when the query tile is multicast (each CTA loads its
+    // slice for the whole cluster), else the whole 128-row tile
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
@@ -398,11 +422,14 @@ __global__ void __launch_bounds__(kClThreads, 1)
     const long long items = (long long)p.B * p.qtiles;
     const int nitems = items > cid ? (int)((items - 1 - cid) / ncl + 1) : 0;
     const int nkb = p.nkb;
+    const bool qmc = p.qslice > 0;
+    const uint16_t cmask = (uint16_t)((1u << G) - 1u);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kClStages; ++s) {
             mbar_init(&c.full[s], 1);
-            mbar_init(&c.empty[s], 1);
+            // with the multicast query tile a stage is free once every CTA's MMAs are done with it
+            mbar_init(&c.empty[s], qmc ? (uint32_t)G : 1u);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&c.d_full[b], 1);
@@ -446,7 +473,11 @@ __global__ void __launch_bounds__(kClThreads, 1)
                     }
                     uint8_t* dst = St + (size_t)st.idx * kClStageBytes;
                     mbar_arrive_expect_tx(&c.full[st.idx], kClStageBytes);
-                    tma_load_2d(dst, &tmap_q, &c.full[st.idx], kb * kBK, b * p.Lq + qt * kBM, pol);
+                    if (qmc)
+                        tma_load_2d_mc(dst + (size_t)rank * p.qslice * (kBK * 2), &tmap_q, &c.full[st.idx], kb * kBK,
+                                       b * p.Lq + qt * kBM + (int)rank * p.qslice, cmask, pol);
+                    else
+                        tma_load_2d(dst, &tmap_q, &c.full[st.idx], kb * kBK, b * p.Lq + qt * kBM, pol);
                     tma_load_2d(dst + kQBlockBytes, &tmap_k, &c.full[st.idx], kb * kBK,
                                 b * p.Lk + (int)rank * kBN, pol);
                 }
@@ -478,7 +509,10 @@ __global__ void __launch_bounds__(kClThreads, 1)
                     for (int k = 0; k < kBK / 16; ++k)
                         mma_f16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
                                    (kb | k) != 0 ? 1u : 0u);
-                    mma_commit(&c.empty[st.idx]);
+                    if (qmc)
+                        mma_commit_mc(&c.empty[st.idx], cmask);
+                    else
+                        mma_commit(&c.empty[st.idx]);
                 }
                 if (ok) mma_commit(&c.d_full[buf]);
             }
@@ -507,24 +541,24 @@ __global__ void __launch_bounds__(kClThreads, 1)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&c.d_empty[buf]);
-            // this thread's part of its row: max m, p_j = exp(scale s_j - m), sum l
-            float mx8[8];
-#pragma unroll
-            for (int k = 0; k < 8; ++k) mx8[k] = -INFINITY;
-#pragma unroll
-            for (int j = 0; j < kBN / 2; ++j) {
-                v[j] = j < nvalid ? p.scale * v[j] : -INFINITY;
-                mx8[j & 7] = fmaxf(mx8[j & 7], v[j]);
-            }
-            const float m = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                                  fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-            const float mref = m == -INFINITY ? 0.f : m;
+            // this thread's part of its row, in base-2 units (c2 = scale log2 e): the max m
+            // of c2 s_j, p_j = 2^(c2 s_j - m) and their sum l.  The max of c2 s_j is c2 times
+            // the max (or, for c2 < 0, the min) of the raw s_j; each p_j is then one fma and
+            // one ex2.  Keys past Lk (only in a row's last unit) are left out.
+            const float c2 = p.scale * 1.4426950408889634f;
+            float ext;
+            if (nvalid == kBN / 2)
+                ext = c2 >= 0.f ? row_extreme<false, false>(v, kBN / 2) : row_extreme<true, false>(v, kBN / 2);
+            else
+                ext = c2 >= 0.f ? row_extreme<false, true>(v, nvalid) : row_extreme<true, true>(v, nvalid);
+            const float m = nvalid > 0 ? c2 * ext : -INFINITY;
+            const float mref = nvalid > 0 ? m : 0.f;
             float l8[8];
 #pragma unroll
             for (int k = 0; k < 8; ++k) l8[k] = 0.f;
 #pragma unroll
             for (int j = 0; j < kBN / 2; ++j) {
-                v[j] = __expf(v[j] - mref);
+                v[j] = (nvalid == kBN / 2 || j < nvalid) ? ex2_approx(fmaf(v[j], c2, -mref)) : 0.f;
                 l8[j & 7] += v[j];
             }
             const float l = ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
@@ -541,16 +575,20 @@ __global__ void __launch_bounds__(kClThreads, 1)
             }
             const bool got = mbar_wait_cluster(&c.x_full[par], ph, abort_flag, err);
             if (!__all_sync(0xffffffffu, got)) break;
-            float f;
+            float f;  // p_j f = exp(scale s_j - row max) / row sum
             {
+                float2 e[2 * kClMaxG];
+#pragma unroll
+                for (int j = 0; j < 2 * kClMaxG; ++j)
+                    e[j] = j < 2 * G ? c.xch[par][j][i] : make_float2(-INFINITY, 0.f);
                 float M = -INFINITY;
-                for (int j = 0; j < 2 * G; ++j) M = fmaxf(M, c.xch[par][j][i].x);
+#pragma unroll
+                for (int j = 0; j < 2 * kClMaxG; ++j) M = fmaxf(M, e[j].x);
                 float L = 0.f;
-                for (int j = 0; j < 2 * G; ++j) {
-                    const float2 e = c.xch[par][j][i];
-                    if (e.y > 0.f) L += e.y * __expf(e.x - M);
-                }
-                f = l > 0.f ? __expf(mref - M) / L : 0.f;
+#pragma unroll
+                for (int j = 0; j < 2 * kClMaxG; ++j)
+                    if (e[j].y > 0.f) L += e[j].y * ex2_approx(e[j].x - M);
+                f = l > 0.f ? __fdividef(ex2_approx(mref - M), L) : 0.f;
             }
             // four boxes of 32 keys: swizzled shared-memory tile (16-byte chunk k of row
             // `lane` at chunk k ^ (lane % 8), the TMA's 128-byte swizzle), then a tensor store
@@ -621,6 +659,7 @@ cudaError_t launch_attn_tc(const void* Yq, const void* Yk, int B, int Lq, int Lk
     p.qtiles = (Lq + kBM - 1) / kBM;
     p.ntiles = (Lk + kBN - 1) / kBN;
     p.passes = softmax ? 2 : 1;
+    p.qslice = 0;
     p.scale = scale;
     p.A = A;
     p.a_vec = ((uintptr_t)A % 8 == 0) && (Lk % 2 == 0);
@@ -637,6 +676,13 @@ cudaError_t launch_attn_tc(const void* Yq, const void* Yk, int B, int Lq, int Lk
                      CU_TENSOR_MAP_SWIZZLE_128B)) {
         // one pass: the key units of a row spread over a cluster of ntiles CTAs
         const int G = p.ntiles;
+        // G = 2 or 4: each CTA loads 128 / G rows of the query tile for the whole cluster
+        CUtensorMap tqc = tq;
+        p.qslice = 0;
+        if ((G == 2 || G == 4) &&
+            make_tmap_2d(&tqc, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, Yq, (long long)B * Lq, r, ldy, kBK, kBM / G,
+                         CU_TENSOR_MAP_SWIZZLE_128B))
+            p.qslice = kBM / G;
         cudaLaunchConfig_t cfg = {};
         cudaLaunchAttribute attr[1];
         attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -666,7 +712,7 @@ cudaError_t launch_attn_tc(const void* Yq, const void* Yk, int B, int Lq, int Lk
         }
         const long long ncl = std::min<long long>(ncl_max, items);
         cfg.gridDim = dim3((unsigned)(ncl * G));
-        cudaError_t e = cudaLaunchKernelEx(&cfg, k_attn_cl, tq, tk, ta, p);
+        cudaError_t e = cudaLaunchKernelEx(&cfg, k_attn_cl, tqc, tk, ta, p);
         if (e != cudaSuccess) return e;
         return cudaGetLastError();
     }

@@ -233,12 +233,14 @@ def _attn_inputs(orc, R, B, Lq, Lk, seed=5):
 
 @pytest.mark.parametrize("B,Lq,Lk,r", [(3, 40, 40, 512), (2, 300, 700, 512), (1, 128, 256, 512),
                                         (2, 1024, 1024, 512), (2, 130, 520, 512), (1, 200, 1500, 512),
-                                        (2, 257, 900, 200), (1, 64, 2100, 72), (2, 50, 301, 512)])
+                                        (2, 257, 900, 200), (1, 64, 2100, 72), (2, 50, 301, 512),
+                                        (3, 300, 512, 136)])
 def test_tc_attention(gs, orc, attn_R, B, Lq, Lk, r):
     """bf16 compressed vectors, fp32 accumulation, row softmax over all keys; against
     the oracle run on the same bf16 inputs.  Lk <= 1024 (a multiple of 4) runs one pass
     with the key units of a row spread over a cluster of ceil(Lk / 256) CTAs (520: the
-    last unit has an empty key half); longer rows and Lk = 301 run the two-pass kernel.
+    last unit has an empty key half; with 2 or 4 CTAs each loads a slice of the query
+    tile for the whole cluster); longer rows and Lk = 301 run the two-pass kernel.
     r < 512 (the first r coordinates) leaves the last K-block partly beyond r."""
     tq, tk = _attn_inputs(orc, attn_R, B, Lq, Lk)
     if r < tq.shape[2]:
