@@ -348,34 +348,41 @@ __global__ void __launch_bounds__(kThreads, 1)
 // ================================================================= one pass, key units spread over a cluster
 // With the row softmax and Lk <= 4 x 256, the G = ceil(Lk / 256) CTAs of a thread-block
 // cluster share each work item: CTA g computes the logits of keys [256 g, 256 g + 256)
-// for the item's 128 queries, once.  Each epilogue thread holds 128 logits of one
-// query row in registers (one TMEM read, after which the accumulator is released to
-// the MMA), takes their max m and p_j = exp(scale s_j - m) and sum l, and posts (m, l)
-// to every CTA of the cluster through distributed shared memory.  With all 2 G partial
-// results of its row a thread has the row's max M and sum L and writes
-// p_j exp(m - M) / L: one exponential per output.  The probabilities go out through a
-// swizzled shared-memory tile and TMA tensor stores (a 3-D map over B x Lq x Lk, so
-// rows past Lq and keys past Lk are clipped).  Compared with the two-pass kernel above
-// this halves the MMA work and the exponentials; the TMEM accumulator is
-// double-buffered over items, so an item's exchange and writes overlap the next
-// item's MMAs.
+// for the item's 128 queries, once.  Each epilogue thread holds 64 logits of one query
+// row in registers (one TMEM read, after which the accumulator goes back to the MMA),
+// takes, in base-2 units, their max m, p_j = 2^(c s_j - m) (c = scale log2 e) and sum
+// l.  The four column quarters of each row are merged in shared memory, each CTA posts
+// its row results to every CTA of the cluster with asynchronous remote stores, and with
+// all G results a thread has the row's max M and sum L and writes p_j 2^(m - M) / L: one
+// exponential per output.  The probabilities go out through a swizzled shared-memory
+// tile and TMA tensor stores (a 3-D map over B x Lq x Lk, so rows past Lq and keys past
+// Lk are clipped).  Compared with the two-pass kernel above this halves the MMA work and
+// the exponentials; the TMEM accumulator is double-buffered over items, so an item's
+// exchange and writes overlap the next item's MMAs.  With G = 2 or 4 each CTA loads
+// 128 / G rows of the query tile and multicasts them to the whole cluster.
 //
-// Warp roles (320 threads): 0-7 epilogue (warp w: TMEM lanes 32 (w % 4) = query rows,
-// keys [128 (w / 4), +128) of the CTA's unit), 8 TMA producer (query and key K-blocks
-// into one stage), 9 TMEM allocator + MMA issuer.
+// Warp roles (576 threads): 0-15 epilogue (warp w: TMEM lanes 32 (w % 4) = query rows,
+// keys [64 (w / 4), +64) of the CTA's unit; warps 0-3 also merge and post the CTA's
+// row results), 16 TMA producer (query and key K-blocks into one stage), 17 TMEM
+// allocator + MMA issuer.
 
 constexpr int kClMaxG = 4;
 constexpr int kClStageBytes = kQBlockBytes + kKStageBytes;  // 48 KB: query block, then key block
 constexpr int kClStages = 3;
-constexpr int kClThreads = 10 * 32;
-constexpr int kClStgBytes = 32 * 32 * 4;  // one output box: 32 query rows x 32 keys fp32 (128-byte rows)
+constexpr int kClEpiWarps = 16;
+constexpr int kClCols = kBN / 4;            // keys per epilogue thread
+constexpr int kClProdWarp = 16, kClMmaWarp = 17;
+constexpr int kClThreads = 18 * 32;
+constexpr int kClStgBytes = 32 * 32 * 4;    // one output box: 32 query rows x 32 keys fp32 (128-byte rows)
 
 struct ClCtl {
     uint64_t full[kClStages], empty[kClStages];
     uint64_t d_full[2], d_empty[2];
-    uint64_t x_full[2];           // statistics of an item from every CTA's every key half (by item parity)
+    uint64_t p_full[2];           // the 16 warps' partial row results of an item (by item parity)
+    uint64_t x_full[2];           // every CTA's row results of an item (by item parity)
     uint64_t mma_done;
-    float2 xch[2][2 * kClMaxG][kBM];  // [item parity][2 rank + key half][query row] = (max, sum)
+    float2 part[2][4][kBM];       // [item parity][column quarter][query row] = (max, sum)
+    float2 xch[2][kClMaxG][kBM];  // [item parity][rank][query row] = (max, sum)
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -394,11 +401,24 @@ __device__ __forceinline__ float row_extreme(const float* v, int n) {
 #pragma unroll
     for (int k = 0; k < 8; ++k) e8[k] = MIN ? INFINITY : -INFINITY;
 #pragma unroll
-    for (int j = 0; j < kBN / 2; ++j)
+    for (int j = 0; j < kClCols; ++j)
         if (!MASK || j < n) e8[j & 7] = MIN ? fminf(e8[j & 7], v[j]) : fmaxf(e8[j & 7], v[j]);
     if (MIN)
         return fminf(fminf(fminf(e8[0], e8[1]), fminf(e8[2], e8[3])), fminf(fminf(e8[4], e8[5]), fminf(e8[6], e8[7])));
     return fmaxf(fmaxf(fmaxf(e8[0], e8[1]), fmaxf(e8[2], e8[3])), fmaxf(fmaxf(e8[4], e8[5]), fmaxf(e8[6], e8[7])));
+}
+
+// merge of partial (max, sum) pairs taken in base 2 (empty parts are (-inf, 0))
+__device__ __forceinline__ float2 merge_stats(const float2* e, int n) {
+    float M = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < kClMaxG; ++j)
+        if (j < n) M = fmaxf(M, e[j].x);
+    float L = 0.f;
+#pragma unroll
+    for (int j = 0; j < kClMaxG; ++j)
+        if (j < n && e[j].y > 0.f) L += e[j].y * ex2_approx(e[j].x - M);
+    return make_float2(M, L);
 }
 
 __global__ void __launch_bounds__(kClThreads, 1)
@@ -410,8 +430,8 @@ __global__ void __launch_bounds__(kClThreads, 1)
     const uint32_t raw = smem_u32(smem_raw);
     uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
     uint8_t* St = base;                                          // kClStages x 48 KB
-    uint8_t* Stg = St + (size_t)kClStages * kClStageBytes;       // 8 warps x 2 x 4 KB output boxes
-    ClCtl& c = *reinterpret_cast<ClCtl*>(Stg + (size_t)kEpiWarps * 2 * kClStgBytes);
+    uint8_t* Stg = St + (size_t)kClStages * kClStageBytes;       // 16 warps x 4 KB output box
+    ClCtl& c = *reinterpret_cast<ClCtl*>(Stg + (size_t)kClEpiWarps * kClStgBytes);
     volatile int* abort_flag = &c.abort_flag;
     unsigned* err = &g_err_attn;
 
@@ -433,14 +453,15 @@ __global__ void __launch_bounds__(kClThreads, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&c.d_full[b], 1);
-            mbar_init(&c.d_empty[b], kEpiWarps);
+            mbar_init(&c.d_empty[b], kClEpiWarps);
+            mbar_init(&c.p_full[b], kClEpiWarps);
             mbar_init(&c.x_full[b], 1);
         }
         mbar_init(&c.mma_done, 1);
         c.abort_flag = 0;
         fence_barrier_init();
     }
-    if (warp == 9) {
+    if (warp == kClMmaWarp) {
         tmem_alloc(&c.tmem_base, kTmemCols);
         tmem_relinquish();
     }
@@ -456,7 +477,7 @@ __global__ void __launch_bounds__(kClThreads, 1)
         qt = (int)(ig % p.qtiles);
     };
 
-    if (warp == 8) {
+    if (warp == kClProdWarp) {
         // ------------------------------------------------------------- query + key K-blocks via TMA
         if (lane == 0) {
             const uint64_t pol = l2_policy_evict_last();
@@ -485,7 +506,7 @@ __global__ void __launch_bounds__(kClThreads, 1)
             for (int j = std::max(0, it - kClStages); j < it; ++j)
                 mbar_drain(&c.full[j % kClStages], (uint32_t)(j / kClStages) & 1u, err);
         }
-    } else if (warp == 9) {
+    } else if (warp == kClMmaWarp) {
         // ------------------------------------------------------------- MMA issue
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16_f32(kBN);
@@ -521,11 +542,12 @@ __global__ void __launch_bounds__(kClThreads, 1)
         }
     } else {
         // ------------------------------------------------------------- epilogue
-        const int quad = warp & 3, kh = warp >> 2;
-        const int i = quad * 32 + lane;                   // query row within the item
-        const int key0 = (int)rank * kBN + kh * (kBN / 2);  // first of this warp's 128 keys
-        const int nvalid = min(kBN / 2, max(0, p.Lk - key0));
-        uint8_t* stg = Stg + (size_t)warp * 2 * kClStgBytes;
+        const int quad = warp & 3, cq = warp >> 2;
+        const int i = quad * 32 + lane;                       // query row within the item
+        const int key0 = (int)rank * kBN + cq * kClCols;      // first of this warp's 64 keys
+        const int nvalid = min(kClCols, max(0, p.Lk - key0));
+        const float c2 = p.scale * 1.4426950408889634f;
+        uint8_t* sb = Stg + (size_t)warp * kClStgBytes;
         const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
         const uint32_t xbar = smem_u32(&c.x_full[0]);
         for (int li = 0; li < nitems; ++li) {
@@ -535,20 +557,27 @@ __global__ void __launch_bounds__(kClThreads, 1)
             const uint32_t ph = (uint32_t)(li >> 1) & 1u;
             if (!mbar_wait_warp(&c.d_full[buf], ph, abort_flag, err)) break;
             tc_fence_after();
-            float v[kBN / 2];
-            tmem_ld128(tmem + lane_base + (uint32_t)(buf * kBN + kh * (kBN / 2)), v);
+            float v[kClCols];
+            {
+                uint32_t r[kClCols];
+                const uint32_t ta = tmem + lane_base + (uint32_t)(buf * kBN + cq * kClCols);
+                tmem_ld32_issue(ta, r);
+                tmem_ld32_issue(ta + 32u, r + 32);
+                tmem_wait_ld32(r);
+                tmem_wait_ld32(r + 32);
+#pragma unroll
+                for (int j = 0; j < kClCols; ++j) v[j] = __uint_as_float(r[j]);
+            }
             // the logits are in registers: the accumulator goes back to the MMA
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&c.d_empty[buf]);
-            // this thread's part of its row, in base-2 units (c2 = scale log2 e): the max m
-            // of c2 s_j, p_j = 2^(c2 s_j - m) and their sum l.  The max of c2 s_j is c2 times
-            // the max (or, for c2 < 0, the min) of the raw s_j; each p_j is then one fma and
-            // one ex2.  Keys past Lk (only in a row's last unit) are left out.
-            const float c2 = p.scale * 1.4426950408889634f;
+            // this thread's part of its row in base-2 units: max m of c s_j (c times the max,
+            // or for c < 0 the min, of the raw s_j), p_j = 2^(c s_j - m) by one fma and one
+            // ex2, and their sum l; keys past Lk (only in a row's last unit) are left out
             float ext;
-            if (nvalid == kBN / 2)
-                ext = c2 >= 0.f ? row_extreme<false, false>(v, kBN / 2) : row_extreme<true, false>(v, kBN / 2);
+            if (nvalid == kClCols)
+                ext = c2 >= 0.f ? row_extreme<false, false>(v, kClCols) : row_extreme<true, false>(v, kClCols);
             else
                 ext = c2 >= 0.f ? row_extreme<false, true>(v, nvalid) : row_extreme<true, true>(v, nvalid);
             const float m = nvalid > 0 ? c2 * ext : -INFINITY;
@@ -557,46 +586,47 @@ __global__ void __launch_bounds__(kClThreads, 1)
 #pragma unroll
             for (int k = 0; k < 8; ++k) l8[k] = 0.f;
 #pragma unroll
-            for (int j = 0; j < kBN / 2; ++j) {
-                v[j] = (nvalid == kBN / 2 || j < nvalid) ? ex2_approx(fmaf(v[j], c2, -mref)) : 0.f;
+            for (int j = 0; j < kClCols; ++j) {
+                v[j] = (nvalid == kClCols || j < nvalid) ? ex2_approx(fmaf(v[j], c2, -mref)) : 0.f;
                 l8[j & 7] += v[j];
             }
             const float l = ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
-            // post (m, l) to every CTA of the cluster, then merge the 2 G partial results of the row
-            {
-                const uint32_t slot = smem_u32(&c.xch[par][2 * rank + kh][i]);
+            // the four column quarters of each row meet in shared memory; warps 0-3 merge
+            // them and post the CTA's row result to every CTA of the cluster
+            c.part[par][cq][i] = make_float2(m, l);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&c.p_full[par]);
+            if (cq == 0) {
+                if (!mbar_wait_warp(&c.p_full[par], ph, abort_flag, err)) break;
+                float2 e[kClMaxG];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) e[k] = c.part[par][k][i];
+                const float2 rc = merge_stats(e, 4);
+                const uint32_t slot = smem_u32(&c.xch[par][rank][i]);
                 const uint32_t bar = xbar + (uint32_t)(par * sizeof(uint64_t));
                 // the barrier's one arrival per phase carries the byte count of every CTA's
                 // posts; the posts are asynchronous stores that complete those bytes (a
                 // release-arrive after plain remote stores cost microseconds per item)
-                if (threadIdx.x == 0) mbar_arrive_expect_tx(&c.x_full[par], (uint32_t)(G * kEpiWarps * 32 * 8));
+                if (threadIdx.x == 0) mbar_arrive_expect_tx(&c.x_full[par], (uint32_t)(G * kBM * 8));
                 for (int g = 0; g < G; ++g)
-                    st_async_f32x2(mapa_shared(slot, (uint32_t)g), m, l, mapa_shared(bar, (uint32_t)g));
+                    st_async_f32x2(mapa_shared(slot, (uint32_t)g), rc.x, rc.y, mapa_shared(bar, (uint32_t)g));
             }
             const bool got = mbar_wait_cluster(&c.x_full[par], ph, abort_flag, err);
             if (!__all_sync(0xffffffffu, got)) break;
             float f;  // p_j f = exp(scale s_j - row max) / row sum
             {
-                float2 e[2 * kClMaxG];
+                float2 e[kClMaxG];
 #pragma unroll
-                for (int j = 0; j < 2 * kClMaxG; ++j)
-                    e[j] = j < 2 * G ? c.xch[par][j][i] : make_float2(-INFINITY, 0.f);
-                float M = -INFINITY;
-#pragma unroll
-                for (int j = 0; j < 2 * kClMaxG; ++j) M = fmaxf(M, e[j].x);
-                float L = 0.f;
-#pragma unroll
-                for (int j = 0; j < 2 * kClMaxG; ++j)
-                    if (e[j].y > 0.f) L += e[j].y * ex2_approx(e[j].x - M);
-                f = l > 0.f ? __fdividef(ex2_approx(mref - M), L) : 0.f;
+                for (int k = 0; k < kClMaxG; ++k) e[k] = k < G ? c.xch[par][k][i] : make_float2(-INFINITY, 0.f);
+                const float2 rw = merge_stats(e, G);
+                f = l > 0.f ? __fdividef(ex2_approx(mref - rw.x), rw.y) : 0.f;
             }
-            // four boxes of 32 keys: swizzled shared-memory tile (16-byte chunk k of row
+            // two boxes of 32 keys: swizzled shared-memory tile (16-byte chunk k of row
             // `lane` at chunk k ^ (lane % 8), the TMA's 128-byte swizzle), then a tensor store
-            const int x0 = key0, y = qt * kBM + quad * 32;
+            const int y = qt * kBM + quad * 32;
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                uint8_t* sb = stg + (size_t)(q & 1) * kClStgBytes;
-                if (lane == 0) bulk_wait_read_1();  // the store that last read this buffer is done with it
+            for (int q = 0; q < kClCols / 32; ++q) {
+                if (lane == 0) bulk_wait_read_0();  // the previous store has read the tile
                 __syncwarp();
 #pragma unroll
                 for (int k = 0; k < 8; ++k) {
@@ -607,7 +637,7 @@ __global__ void __launch_bounds__(kClThreads, 1)
                 fence_proxy_async();
                 __syncwarp();
                 if (lane == 0) {
-                    if (x0 + 32 * q < p.Lk && y < p.Lq) tma_store_3d(&tmap_a, sb, x0 + 32 * q, y, b);
+                    if (key0 + 32 * q < p.Lk && y < p.Lq) tma_store_3d(&tmap_a, sb, key0 + 32 * q, y, b);
                     bulk_commit();
                 }
             }
@@ -618,14 +648,14 @@ __global__ void __launch_bounds__(kClThreads, 1)
     tc_fence_before();
     __syncthreads();
     cluster_sync_all();  // no CTA leaves while a peer may still post into its shared memory
-    if (warp == 9) {
+    if (warp == kClMmaWarp) {
         tc_fence_after();
         tmem_dealloc(tmem, kTmemCols);
     }
 }
 
 constexpr size_t kClSmemBytes =
-    1024 + (size_t)kClStages * kClStageBytes + (size_t)kEpiWarps * 2 * kClStgBytes + sizeof(ClCtl);
+    1024 + (size_t)kClStages * kClStageBytes + (size_t)kClEpiWarps * kClStgBytes + sizeof(ClCtl);
 static_assert(kClSmemBytes <= 227 * 1024, "cluster attention kernel shared memory exceeds the per-CTA limit");
 
 constexpr size_t kSmemBytes = 1024 + (size_t)kMaxKB * kQBlockBytes + (size_t)kKStages * kKStageBytes + sizeof(Ctl);
