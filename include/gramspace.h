@@ -25,8 +25,8 @@
  *  - Errors that only the device can see (a bounded wait that ran out, an
  *    input outside a fast path's numeric range) set a per-device error word;
  *    gs_stream_status() synchronises the stream and returns and clears it.
- *  - Only gs_build_basis, gs_basis_import and gs_basis_reserve_staging
- *    allocate device memory; the other calls allocate nothing.  N = 0 is a
+ *  - Only gs_build_basis, gs_build_basis_grouped, gs_basis_import and
+ *    gs_basis_reserve_staging allocate device memory; the other calls allocate nothing.  N = 0 is a
  *    valid no-op.
  *  - All functions are callable from any host thread; a gs_basis must not be
  *    destroyed while work that uses it is in flight.  Some paths keep
@@ -109,6 +109,53 @@ GS_API gs_status gs_build_basis(const float* C, int M, int D, int ldc, float ran
                          unsigned flags, void* stream, gs_basis** out);
 
 /*
+ * Grouped basis (Sec. 3.1: when D < M the codebook is rank-deficient, so its
+ * entries are partitioned into subsets of at most D, each subset gets its own
+ * orthonormal basis, and the reconstructions are concatenated into the full
+ * codebook layout).  The same construction holds several attribute codebooks
+ * (e.g. one per RAVEN attribute) in one handle, so one launch scores a query
+ * against all of them.
+ *
+ * Rows [group_offsets[g], group_offsets[g+1]) of C form group g; group_offsets
+ * is a HOST array of G + 1 increasing ints from 0 to M (1 <= G <= 256, every
+ * group non-empty).  Each group is orthonormalised alone exactly as
+ * gs_build_basis does (same rank_tol and flags), giving Q_g (r_g x D) and R_g.
+ * The handle holds the stacked Q = [Q_0; Q_1; ...] (r = r_0 + ... + r_(G-1)
+ * rows; rows of one group are orthonormal, rows of different groups need not
+ * be, and r may exceed D) and the block-diagonal R (M x r): row i of group g
+ * carries R_g's row in columns [s_g, s_g + r_g), s_g = r_0 + ... + r_(g-1), and
+ * zeros elsewhere.  C = R Q holds row by row, so every other call works on the
+ * handle unchanged: scores cover all M entries in the original layout, Gram-loc
+ * rows and prob-vectorized rows use the stacked coordinates, and reconstruction
+ * returns the concatenated codebook layout.  gs_basis_groups reports the group
+ * and coordinate offsets; gs_group_argmax picks the best entry per group.
+ * Synchronises `stream` once per group.  Errors as gs_build_basis; invalid
+ * offsets give GS_ERR_INVALID_ARG.
+ */
+GS_API gs_status gs_build_basis_grouped(const float* C, int M, int D, int ldc, const int* group_offsets, int G,
+                                        float rank_tol, unsigned flags, void* stream, gs_basis** out);
+
+/*
+ * Group layout of a handle: *G groups; row_offsets and coeff_offsets (HOST
+ * arrays of *G + 1 ints, either may be NULL; call once with both NULL to learn
+ * *G) receive the codebook-row and Gram-loc-coordinate ranges of each group.
+ * A handle from gs_build_basis or gs_basis_import is one group: {0, M}, {0, r}.
+ */
+GS_API gs_status gs_basis_groups(const gs_basis* h, int* G, int* row_offsets, int* coeff_offsets);
+
+/*
+ * Best entry of each group for each score row (hard selection per attribute,
+ * Sec. 2.2, on the scores of a grouped codebook): S is N x M fp32 (ld = lds >=
+ * group_offsets[G]); group g is columns [group_offsets[g], group_offsets[g+1])
+ * (HOST array of G + 1 increasing ints from 0, 1 <= G <= 256).  argmax (N x G
+ * int32, ld G) receives the index WITHIN the group of the first column holding
+ * the group's maximum, maxval (N x G fp32, ld G) that maximum; either may be
+ * NULL, not both.  N = 0 is a no-op.
+ */
+GS_API gs_status gs_group_argmax(const float* S, long long N, int lds, const int* group_offsets, int G,
+                                 int* argmax, float* maxval, void* stream);
+
+/*
  * Read-only view of a basis: sizes and device pointers to Q (r x D, ld = D),
  * R (M x r, ld = r) and cnorm (M, fp32 ||c_i||).  Any output pointer may be
  * NULL.  The pointers stay valid until gs_basis_destroy.
@@ -129,7 +176,10 @@ GS_API gs_status gs_basis_info(const gs_basis* h, int* M, int* D, int* r, const 
  *          because C = R Q with orthonormal Q)
  * Device pointers owned by the caller; the handle keeps its own copies.  The
  * rows of Q are taken as orthonormal and R as lower echelon (as a build leaves
- * them); neither is re-checked.  Synchronises `stream` before returning.
+ * them; for a grouped basis, orthonormal within each group and block diagonal,
+ * with r <= M); neither is re-checked.  A restored grouped basis reports one
+ * group (pass the offsets to gs_group_argmax explicitly).  Synchronises
+ * `stream` before returning.
  */
 GS_API gs_status gs_basis_import(const float* Q, int r, int D, int ldq, const float* R, int M, int ldr,
                                  const float* cnorm, void* stream, gs_basis** out);

@@ -93,6 +93,42 @@ def build_basis(C, tau=1e-6, normalize_rows=False, passes=2):
     return Q[:r].copy(), np.ascontiguousarray(R[:, :r]), cn
 
 
+def build_grouped(C, offsets, tau=1e-6, normalize_rows=False):
+    """Sec. 3.1, D < M: the entries are partitioned into subsets (rows [offsets[g],
+    offsets[g+1]) of C), each subset gets its own orthonormal basis, and the
+    reconstructions are concatenated.  Returns (Q, R, cnorm, coeff_offsets): Q stacks the
+    subsets' bases (r = sum of their ranks rows), R is block diagonal (subset g's
+    coefficients in columns [coeff_offsets[g], coeff_offsets[g+1])), so C = R Q."""
+    C = _f64(C)
+    M, D = C.shape
+    parts = [build_basis(C[offsets[g]:offsets[g + 1]], tau, normalize_rows) for g in range(len(offsets) - 1)]
+    coeff = [0]
+    for Qg, _, _ in parts:
+        coeff.append(coeff[-1] + Qg.shape[0])
+    Q = np.zeros((coeff[-1], D))
+    R = np.zeros((M, coeff[-1]))
+    cn = np.zeros(M)
+    for g, (Qg, Rg, cng) in enumerate(parts):
+        Q[coeff[g]:coeff[g + 1]] = Qg
+        R[offsets[g]:offsets[g + 1], coeff[g]:coeff[g + 1]] = Rg
+        cn[offsets[g]:offsets[g + 1]] = cng
+    return Q, R, cn, coeff
+
+
+def group_argmax(S, offsets):
+    """Best entry of each group (columns [offsets[g], offsets[g+1])) for each row of S:
+    (argmax within the group, first index of the maximum; maximum), each N x G."""
+    S = _f64(S)
+    G = len(offsets) - 1
+    am = np.zeros((S.shape[0], G), dtype=np.int32)
+    mv = np.zeros((S.shape[0], G))
+    for g in range(G):
+        block = S[:, offsets[g]:offsets[g + 1]]
+        am[:, g] = np.argmax(block, axis=1)
+        mv[:, g] = block.max(axis=1)
+    return am, mv
+
+
 def project(X, Q):
     """Y = X Q^T (Gram-loc of each query, Sec. 3.1) and the full-D norms ||x||."""
     X = _f64(X)

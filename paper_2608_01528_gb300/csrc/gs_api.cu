@@ -193,11 +193,66 @@ gs_status gs_build_basis(const float* C, int M, int D, int ldc, float rank_tol, 
     return GS_OK;
 }
 
+// increasing offsets 0 = off[0] < off[1] < ... < off[G] = M (M < 0: any last offset)
+static bool valid_offsets(const int* off, int G, int M) {
+    if (!off || G < 1 || G > gs::kMaxGroups || off[0] != 0) return false;
+    for (int g = 0; g < G; ++g)
+        if (off[g + 1] <= off[g]) return false;
+    return M < 0 || off[G] == M;
+}
+
+gs_status gs_build_basis_grouped(const float* C, int M, int D, int ldc, const int* group_offsets, int G,
+                                 float rank_tol, unsigned flags, void* stream, gs_basis** out) {
+    if (!out) return GS_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (!C || M < 1 || D < 1 || ldc < D) return M < 1 || D < 1 || ldc < D ? GS_ERR_SHAPE : GS_ERR_INVALID_ARG;
+    if (!valid_offsets(group_offsets, G, M)) return GS_ERR_INVALID_ARG;
+    if (!(rank_tol > 0.f) || !isfinite(rank_tol)) return GS_ERR_INVALID_ARG;
+    if (flags & ~GS_BUILD_NORMALIZE_ROWS) return GS_ERR_INVALID_ARG;
+    if ((uintptr_t)C % sizeof(float)) return GS_ERR_ALIGNMENT;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return GS_ERR_CUDA;
+    if (!device_supported(dev)) return GS_ERR_UNSUPPORTED;
+    gs_basis* h = new gs_basis();
+    h->device = dev;
+    gs_status st = gs::build_basis_grouped(C, M, D, ldc, group_offsets, G, (double)rank_tol,
+                                           (flags & GS_BUILD_NORMALIZE_ROWS) != 0, (cudaStream_t)stream, h);
+    if (st == GS_OK && gs::tc_available(dev)) st = gs::tc_prepare(h);
+    if (st != GS_OK) {
+        free_basis(h);
+        return st;
+    }
+    *out = h;
+    return GS_OK;
+}
+
+gs_status gs_basis_groups(const gs_basis* h, int* G, int* row_offsets, int* coeff_offsets) {
+    if (!h || !G) return GS_ERR_INVALID_ARG;
+    const bool grouped = !h->grp_rows.empty();
+    const int g = grouped ? (int)h->grp_rows.size() - 1 : 1;
+    *G = g;
+    for (int k = 0; k <= g; ++k) {
+        if (row_offsets) row_offsets[k] = grouped ? h->grp_rows[k] : (k ? h->M : 0);
+        if (coeff_offsets) coeff_offsets[k] = grouped ? h->grp_coeffs[k] : (k ? h->r : 0);
+    }
+    return GS_OK;
+}
+
+gs_status gs_group_argmax(const float* S, long long N, int lds, const int* group_offsets, int G, int* argmax,
+                          float* maxval, void* stream) {
+    if (N < 0) return GS_ERR_SHAPE;
+    if (!valid_offsets(group_offsets, G, -1)) return GS_ERR_INVALID_ARG;
+    if (lds < group_offsets[G]) return GS_ERR_SHAPE;
+    if (N == 0) return GS_OK;
+    if (!S || (!argmax && !maxval)) return GS_ERR_INVALID_ARG;
+    return from_cuda(gs::launch_group_argmax(S, N, lds, group_offsets, G, argmax, maxval, (cudaStream_t)stream));
+}
+
 gs_status gs_basis_import(const float* Q, int r, int D, int ldq, const float* R, int M, int ldr,
                           const float* cnorm, void* stream, gs_basis** out) {
     if (!out) return GS_ERR_INVALID_ARG;
     *out = nullptr;
-    if (M < 1 || D < 1 || r < 0 || r > std::min(M, D)) return GS_ERR_SHAPE;
+    if (M < 1 || D < 1 || r < 0 || r > M) return GS_ERR_SHAPE;  // r > D only for a grouped basis
     if (r > 0 && (ldq < D || ldr < r)) return GS_ERR_SHAPE;
     if (r > 0 && (!Q || !R)) return GS_ERR_INVALID_ARG;
     if (((uintptr_t)Q | (uintptr_t)R | (uintptr_t)cnorm) % sizeof(float)) return GS_ERR_ALIGNMENT;

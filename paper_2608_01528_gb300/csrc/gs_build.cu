@@ -22,6 +22,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <memory>
 #include <vector>
 
 #include "gs_internal.h"
@@ -319,28 +320,45 @@ unsigned take_device_error_build() {
 gs_status finalize_basis(const double* Qw, const double* R64, int ldr, const double* cn, int M, int D, int r,
                          cudaStream_t s, gs_basis* h);
 
-gs_status build_basis(const float* C, int M, int D, int ldc, double tau, bool normalize,
-                      cudaStream_t s, gs_basis* h) {
+// The fp64 factorisation C = R Q of M rows of C (Q: r x D orthonormal rows, R: M x r lower
+// echelon, ldr = min(M, D); cn: the rows' norms), kept on the device.
+struct Factor {
+    double* Qw = nullptr;
+    double* R64 = nullptr;
+    double* cn = nullptr;
+    int r = 0, ldr = 1;
+    Factor() = default;
+    Factor(const Factor&) = delete;
+    Factor& operator=(const Factor&) = delete;
+    ~Factor() {
+        cudaFree(Qw);
+        cudaFree(R64);
+        cudaFree(cn);
+    }
+};
+
+gs_status factor_rows(const float* C, int M, int D, int ldc, double tau, bool normalize, cudaStream_t s,
+                      Factor& f) {
     const int rmax = std::min(M, D);
     const int ldr = rmax;                       // R64 leading dimension
     const int ldh = std::max(1, ((M + 15) / 16) * 16);  // >= any r0
     const int dslice = std::max(kDotCols, ((D + 7) / 8 + kDotCols - 1) / kDotCols * kDotCols);
     const int nslices = (D + dslice - 1) / dslice;
 
-    DevBuf bV, bQw, bR64, bH, bHp, bcn, br;
+    DevBuf bV, bH, bHp, br;
     GS_CK(cudaMalloc(&bV.p, sizeof(double) * (size_t)kPanel * D));
-    GS_CK(cudaMalloc(&bQw.p, sizeof(double) * (size_t)rmax * D));
-    GS_CK(cudaMalloc(&bR64.p, sizeof(double) * (size_t)M * ldr));
+    GS_CK(cudaMalloc(&f.Qw, sizeof(double) * (size_t)rmax * D));
+    GS_CK(cudaMalloc(&f.R64, sizeof(double) * (size_t)M * ldr));
     GS_CK(cudaMalloc(&bH.p, sizeof(double) * (size_t)kPanel * ldh));
     GS_CK(cudaMalloc(&bHp.p, sizeof(double) * (size_t)nslices * kPanel * ldh));
-    GS_CK(cudaMalloc(&bcn.p, sizeof(double) * (size_t)M));
+    GS_CK(cudaMalloc(&f.cn, sizeof(double) * (size_t)M));
     GS_CK(cudaMalloc(&br.p, sizeof(int)));
     double* V = (double*)bV.p;
-    double* Qw = (double*)bQw.p;
-    double* R64 = (double*)bR64.p;
+    double* Qw = f.Qw;
+    double* R64 = f.R64;
     double* H = (double*)bH.p;
     double* Hp = (double*)bHp.p;
-    double* cn = (double*)bcn.p;
+    double* cn = f.cn;
     int* r_dev = (int*)br.p;
     GS_CK(cudaMemsetAsync(R64, 0, sizeof(double) * (size_t)M * ldr, s));
     GS_CK(cudaMemsetAsync(r_dev, 0, sizeof(int), s));
@@ -363,7 +381,63 @@ gs_status build_basis(const float* C, int M, int D, int ldc, double tau, bool no
     int r = 0;
     GS_CK(cudaMemcpyAsync(&r, r_dev, sizeof(int), cudaMemcpyDeviceToHost, s));
     GS_CK(cudaStreamSynchronize(s));
-    return finalize_basis(Qw, R64, ldr, cn, M, D, r, s, h);
+    f.r = r;
+    f.ldr = ldr;
+    return GS_OK;
+}
+
+gs_status build_basis(const float* C, int M, int D, int ldc, double tau, bool normalize,
+                      cudaStream_t s, gs_basis* h) {
+    Factor f;
+    gs_status st = factor_rows(C, M, D, ldc, tau, normalize, s, f);
+    if (st != GS_OK) return st;
+    return finalize_basis(f.Qw, f.R64, f.ldr, f.cn, M, D, f.r, s, h);
+}
+
+// Sec. 3.1, D < M: the entries are split into subsets, each gets its own orthonormal basis,
+// and the reconstructions are concatenated.  Group g (rows [off[g], off[g+1]) of C) is
+// factored alone; the handle holds the stacked Q = [Q_0; Q_1; ...] (r = sum of r_g rows) and
+// the block-diagonal R whose row i of group g holds R_g's row in columns [s_g, s_g + r_g),
+// s_g = r_0 + ... + r_(g-1).  C = R Q holds row by row, so every call on the handle works
+// unchanged (Q's rows are orthonormal within a group, not across groups).
+gs_status build_basis_grouped(const float* C, int M, int D, int ldc, const int* off, int G, double tau,
+                              bool normalize, cudaStream_t s, gs_basis* h) {
+    std::vector<std::unique_ptr<Factor>> fs;
+    int rt = 0;
+    for (int g = 0; g < G; ++g) {
+        fs.emplace_back(new Factor());
+        gs_status st = factor_rows(C + (size_t)off[g] * ldc, off[g + 1] - off[g], D, ldc, tau, normalize, s,
+                                   *fs.back());
+        if (st != GS_OK) return st;
+        rt += fs.back()->r;
+    }
+    const int ldr = std::max(rt, 1);
+    DevBuf bQ, bR, bcn;
+    GS_CK(cudaMalloc(&bQ.p, sizeof(double) * (size_t)ldr * D));
+    GS_CK(cudaMalloc(&bR.p, sizeof(double) * (size_t)M * ldr));
+    GS_CK(cudaMalloc(&bcn.p, sizeof(double) * (size_t)M));
+    double* Q = (double*)bQ.p;
+    double* R = (double*)bR.p;
+    double* cn = (double*)bcn.p;
+    GS_CK(cudaMemsetAsync(R, 0, sizeof(double) * (size_t)M * ldr, s));
+    h->grp_rows.assign(off, off + G + 1);
+    h->grp_coeffs.assign(1, 0);
+    int sg = 0;
+    for (int g = 0; g < G; ++g) {
+        const Factor& f = *fs[g];
+        const int mg = off[g + 1] - off[g];
+        if (f.r > 0) {
+            GS_CK(cudaMemcpyAsync(Q + (size_t)sg * D, f.Qw, sizeof(double) * (size_t)f.r * D,
+                                  cudaMemcpyDeviceToDevice, s));
+            GS_CK(cudaMemcpy2DAsync(R + (size_t)off[g] * ldr + sg, sizeof(double) * ldr, f.R64,
+                                    sizeof(double) * f.ldr, sizeof(double) * f.r, mg, cudaMemcpyDeviceToDevice,
+                                    s));
+        }
+        GS_CK(cudaMemcpyAsync(cn + off[g], f.cn, sizeof(double) * mg, cudaMemcpyDeviceToDevice, s));
+        sg += f.r;
+        h->grp_coeffs.push_back(sg);
+    }
+    return finalize_basis(Q, R, ldr, cn, M, D, rt, s, h);
 }
 
 // Everything a handle holds besides the fp64 factorisation: fp32 Q, R and norms for the

@@ -10,6 +10,8 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include <vector>
+
 #include "../../include/gramspace.h"
 
 struct gs_basis {
@@ -57,6 +59,9 @@ struct gs_basis {
     int stage_ld = 0;
     cudaStream_t stage_copy = nullptr;
     cudaEvent_t stage_start = nullptr, stage_in[2] = {nullptr, nullptr}, stage_done[2] = {nullptr, nullptr};
+    // grouped bases (gs_build_basis_grouped): rows [grp_rows[g], grp_rows[g+1]) of the codebook
+    // and coefficients [grp_coeffs[g], grp_coeffs[g+1]) belong to group g; empty otherwise
+    std::vector<int> grp_rows, grp_coeffs;
     // scratch for the multi-kernel paths (rows processed in chunks)
     float* scratch = nullptr;
     long long scratch_floats = 0;
@@ -76,6 +81,10 @@ constexpr int kMinF16Depth = 1024;
 // tensor maps.  Synchronises `s` once.
 gs_status build_basis(const float* C, int M, int D, int ldc, double tau, bool normalize,
                       cudaStream_t s, gs_basis* h);
+// one basis per group of rows (off: host, G + 1 increasing offsets from 0 to M), stacked into
+// one handle: Q = [Q_0; Q_1; ...], R block diagonal
+gs_status build_basis_grouped(const float* C, int M, int D, int ldc, const int* off, int G, double tau,
+                              bool normalize, cudaStream_t s, gs_basis* h);
 // a handle from a saved basis (fp32 Q r x D, R M x r, optional norms), same finalisation as a build
 gs_status import_basis(const float* Q, int ldq, const float* R, int ldr_in, const float* cnorm, int M, int D,
                        int r, cudaStream_t s, gs_basis* h);
@@ -111,6 +120,12 @@ cudaError_t launch_gemm_simt(const GemmArgs& g, cudaStream_t s);
 
 // per-row ||x||
 cudaError_t launch_rownorm(const float* X, long long N, int ldx, int D, float* out, cudaStream_t s);
+
+// per-row, per-group argmax (index within the group) and max over S (N x M, lds); groups are
+// column ranges [off[g], off[g+1]), G <= kMaxGroups; outputs N x G
+constexpr int kMaxGroups = 256;
+cudaError_t launch_group_argmax(const float* S, long long N, int lds, const int* off, int G, int* argmax,
+                                float* maxval, cudaStream_t s);
 
 // per-row argmax / maxval over S (N x M); SOFTMAX mode rewrites the row in place.
 cudaError_t launch_row_finish(float* S, long long N, int M, int lds, bool softmax, int* argmax,

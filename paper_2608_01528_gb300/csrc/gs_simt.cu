@@ -13,6 +13,7 @@
 //  k_row_finish   argmax / maxval / softmax over each score row
 //  k_row_softmax  softmax over each attention row
 //  k_rownorm      full-D query norms for cosine scores
+//  k_group_argmax argmax / max of each score row within each group of a grouped codebook
 
 #include <float.h>
 
@@ -291,6 +292,40 @@ __global__ void __launch_bounds__(256) k_rownorm(const float* __restrict__ X, lo
     if (lane == 0) out[n] = sqrtf(s);
 }
 
+// Column ranges of the groups of a grouped codebook, passed by value.
+struct GroupOffsets {
+    int G;
+    int off[kMaxGroups + 1];
+};
+
+// one warp per score row: for each group, the max over its columns and the index (within
+// the group) of its first occurrence
+__global__ void __launch_bounds__(256) k_group_argmax(const float* __restrict__ S, long long N, int lds,
+                                                       const GroupOffsets go, int* __restrict__ argmax,
+                                                       float* __restrict__ maxval) {
+    const int lane = threadIdx.x & 31;
+    const long long n = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (n >= N) return;
+    const float* s = S + (size_t)n * lds;
+    for (int g = 0; g < go.G; ++g) {
+        const int c0 = go.off[g], c1 = go.off[g + 1];
+        float bv = -INFINITY;
+        int bi = c1;
+        for (int j = c0 + lane; j < c1; j += 32) {
+            const float v = s[j];
+            if (v > bv) {  // columns rise with j: the first of equal values stays
+                bv = v;
+                bi = j;
+            }
+        }
+        warp_argmax(bv, bi);
+        if (lane == 0) {
+            if (argmax) argmax[(size_t)n * go.G + g] = bi - c0;
+            if (maxval) maxval[(size_t)n * go.G + g] = bv;
+        }
+    }
+}
+
 inline unsigned rows_grid(long long n) { return (unsigned)((n + 7) / 8); }
 
 }  // namespace
@@ -339,6 +374,17 @@ cudaError_t launch_row_finish(float* S, long long N, int M, int lds, bool softma
                               float* maxval, cudaStream_t s) {
     if (N <= 0) return cudaSuccess;
     k_row_finish<<<rows_grid(N), 256, 0, s>>>(S, N, M, lds, softmax ? 1 : 0, argmax, maxval);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_group_argmax(const float* S, long long N, int lds, const int* off, int G, int* argmax,
+                                float* maxval, cudaStream_t s) {
+    if (N <= 0) return cudaSuccess;
+    if (G < 1 || G > kMaxGroups) return cudaErrorInvalidValue;
+    GroupOffsets go;
+    go.G = G;
+    for (int g = 0; g <= G; ++g) go.off[g] = off[g];
+    k_group_argmax<<<rows_grid(N), 256, 0, s>>>(S, N, lds, go, argmax, maxval);
     return cudaGetLastError();
 }
 

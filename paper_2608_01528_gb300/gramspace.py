@@ -31,7 +31,7 @@ EXPORTS = ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_si
            "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores", "gs_stream_status",
            "gs_status_string", "gs_version", "gs_project_similarity_static", "gs_similarity_coeffs",
            "gs_selftest_wait_timeout", "gs_basis_import", "gs_basis_reserve_staging",
-           "gs_project_similarity_host")
+           "gs_project_similarity_host", "gs_build_basis_grouped", "gs_basis_groups", "gs_group_argmax")
 
 
 class GramSpaceError(RuntimeError):
@@ -59,6 +59,9 @@ def load_library(path=LIB_PATH):
     L.gs_basis_reserve_staging.argtypes = [vp, i64]
     L.gs_project_similarity_host.argtypes = [vp, vp, i64, ip, ip, f32, u32, vp, vp, vp]
     L.gs_basis_import.argtypes = [vp, ip, ip, ip, vp, ip, ip, vp, vp, ctypes.POINTER(vp)]
+    L.gs_build_basis_grouped.argtypes = [vp, ip, ip, ip, vp, ip, f32, u32, vp, ctypes.POINTER(vp)]
+    L.gs_basis_groups.argtypes = [vp, ctypes.POINTER(ip), vp, vp]
+    L.gs_group_argmax.argtypes = [vp, i64, ip, vp, ip, vp, vp, vp]
     L.gs_project_similarity.argtypes = [vp, vp, i64, ip, ip, f32, u32, vp, ip, vp, ip, vp, vp, vp]
     L.gs_similarity_coeffs.argtypes = [vp, vp, i64, ip, ip, f32, u32, vp, ip, vp, vp, vp]
     L.gs_prob_vectorize.argtypes = [vp, vp, i64, ip, vp, ip, ip, u32, vp]
@@ -74,7 +77,8 @@ def load_library(path=LIB_PATH):
     for name in ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_similarity",
                  "gs_similarity_coeffs", "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores",
                  "gs_stream_status", "gs_selftest_wait_timeout", "gs_basis_import",
-                 "gs_basis_reserve_staging", "gs_project_similarity_host"):
+                 "gs_basis_reserve_staging", "gs_project_similarity_host", "gs_build_basis_grouped",
+                 "gs_basis_groups", "gs_group_argmax"):
         getattr(L, name).restype = ctypes.c_int
     _lib = L
     return L
@@ -182,6 +186,58 @@ def build_basis(C, rank_tol=1e-6, normalize_rows=False, stream=None):
                               ctypes.byref(h))
     _check(st, "gs_build_basis")
     return Basis(h, C.device)
+
+
+def _offsets(group_offsets):
+    off = [int(o) for o in group_offsets]
+    return (ctypes.c_int * len(off))(*off), len(off) - 1
+
+
+def build_basis_grouped(C, group_offsets, rank_tol=1e-6, normalize_rows=False, stream=None):
+    """One Gram-Schmidt basis per group of rows of C (rows [off[g], off[g+1])), stacked in one
+    handle; see gs_build_basis_grouped."""
+    if not C.is_cuda or C.dtype != torch.float32:
+        raise TypeError("C must be a float32 CUDA tensor")
+    off, G = _offsets(group_offsets)
+    L = load_library()
+    h = ctypes.c_void_p()
+    with torch.cuda.device(C.device):
+        st = L.gs_build_basis_grouped(_ptr(C), C.shape[0], C.shape[1], _ld(C), off, G, float(rank_tol),
+                                      GS_BUILD_NORMALIZE_ROWS if normalize_rows else 0, _stream(stream),
+                                      ctypes.byref(h))
+    _check(st, "gs_build_basis_grouped")
+    return Basis(h, C.device)
+
+
+def basis_groups(basis):
+    """(row_offsets, coeff_offsets) of the basis' groups; see gs_basis_groups."""
+    L = load_library()
+    G = ctypes.c_int()
+    _check(L.gs_basis_groups(basis.handle, ctypes.byref(G), None, None), "gs_basis_groups")
+    rows = (ctypes.c_int * (G.value + 1))()
+    coeffs = (ctypes.c_int * (G.value + 1))()
+    _check(L.gs_basis_groups(basis.handle, ctypes.byref(G), rows, coeffs), "gs_basis_groups")
+    return list(rows), list(coeffs)
+
+
+def group_argmax(S, group_offsets, want_maxval=True, out=None, stream=None):
+    """Per-row, per-group argmax (index within the group) and max of scores S (N x M fp32, CUDA);
+    see gs_group_argmax.  Returns {"argmax": N x G int32, "maxval": N x G fp32}."""
+    if not S.is_cuda or S.dtype != torch.float32:
+        raise TypeError("S must be a float32 CUDA tensor")
+    off, G = _offsets(group_offsets)
+    N = S.shape[0]
+    out = dict(out or {})
+    if "argmax" not in out:
+        out["argmax"] = torch.empty((N, G), dtype=torch.int32, device=S.device)
+    if want_maxval and "maxval" not in out:
+        out["maxval"] = torch.empty((N, G), dtype=torch.float32, device=S.device)
+    L = load_library()
+    with torch.cuda.device(S.device):
+        st = L.gs_group_argmax(_ptr(S), N, _ld(S) if N else S.shape[1], off, G, _ptr(out.get("argmax")),
+                               _ptr(out.get("maxval")), _stream(stream))
+    _check(st, "gs_group_argmax")
+    return out
 
 
 def import_basis(Q, R, cnorm=None, stream=None):

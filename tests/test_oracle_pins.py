@@ -346,3 +346,74 @@ def test_golden_table3_arithmetic():
         assert abs(int(n) * float(per) - float(dec)) < 0.006
         assert abs(float(pipe) + float(dec) - float(total)) < 0.006
         assert abs(float(orig) / float(total) - float(speed)) < 0.006
+
+
+# ----------------------------------------------------------------- grouped bases (Sec. 3.1, D < M)
+def test_grouped_partition_closed_forms(orc):
+    """D < M: each subset of at most D entries gets its own orthonormal basis (its rank
+    from an independent routine), R is block diagonal, R Q = C exactly in fp64, and scores
+    through the stacked basis equal X C^T."""
+    rng = np.random.default_rng(20260101)
+    M, D = 40, 16
+    off = [0, 16, 32, 40]
+    C = (rng.integers(0, 2, size=(M, D)) * 2 - 1).astype(np.float64)
+    Q, R, cn, coeff = orc.build_grouped(C, off)
+    assert Q.shape[0] > D  # the stacked basis is wider than the space: only the partition fits it
+    for g in range(3):
+        Qg = Q[coeff[g]:coeff[g + 1]]
+        assert Qg.shape[0] == np.linalg.matrix_rank(C[off[g]:off[g + 1]])
+        assert np.abs(Qg @ Qg.T - np.eye(Qg.shape[0])).max() <= 1e-12
+        outside = np.ones(R.shape, dtype=bool)
+        outside[off[g]:off[g + 1], coeff[g]:coeff[g + 1]] = False
+        assert np.all(R[off[g]:off[g + 1]][outside[off[g]:off[g + 1]]] == 0.0)
+    assert np.abs(R @ Q - C).max() <= 1e-12
+    assert np.allclose(cn, np.linalg.norm(C, axis=1), rtol=1e-14)
+    X = rng.normal(size=(9, D))
+    ref = orc.project_similarity(X, Q, R, cn)
+    assert np.abs(ref["S"] - X @ C.T).max() <= 1e-10
+    assert np.abs(orc.reconstruct(R, Q) - C).max() <= 1e-12
+
+
+def test_grouped_single_group_is_plain_build(orc, tiny_case):
+    C = tiny_case[0]["C"]
+    Q, R, cn, coeff = orc.build_grouped(C, [0, C.shape[0]])
+    Q1, R1, cn1 = orc.build_basis(C)
+    assert coeff == [0, Q1.shape[0]]
+    assert np.array_equal(Q, Q1) and np.array_equal(R, R1) and np.array_equal(cn, cn1)
+
+
+def test_group_argmax_brute_force(orc):
+    """Per-group argmax (first index of the maximum within the group) against plain loops,
+    with ties planted inside groups."""
+    rng = np.random.default_rng(5)
+    S = rng.integers(-3, 4, size=(7, 12)).astype(np.float64)
+    S[0, 4:9] = 3.0
+    S[1, 0:3] = -1.0
+    off = [0, 3, 4, 9, 12]
+    am, mv = orc.group_argmax(S, off)
+    for n in range(S.shape[0]):
+        for g in range(len(off) - 1):
+            best = off[g]
+            for j in range(off[g] + 1, off[g + 1]):
+                if S[n, j] > S[n, best]:
+                    best = j
+            assert am[n, g] == best - off[g]
+            assert mv[n, g] == S[n, best]
+
+
+def test_grouped_attribute_codebooks(orc):
+    """The four attribute codebooks in one grouped basis: the scores of each attribute's
+    columns are that attribute's own X C_a^T, and the per-group argmax is the argmax against
+    each codebook alone."""
+    cases = synth.multiattr()
+    C = np.concatenate([a["C"] for a in cases]).astype(np.float64)
+    off = np.cumsum([0] + [a["C"].shape[0] for a in cases]).tolist()
+    Q, R, cn, coeff = orc.build_grouped(C, off)
+    assert coeff == off  # every attribute codebook has full rank
+    X = cases[2]["X"][:64].astype(np.float64)
+    S = orc.project_similarity(X, Q, R, cn)["S"]
+    am, _ = orc.group_argmax(S, off)
+    for g, a in enumerate(cases):
+        Sg = X @ a["C"].astype(np.float64).T
+        assert np.abs(S[:, off[g]:off[g + 1]] - Sg).max() <= 1e-9
+        assert np.array_equal(am[:, g], np.argmax(Sg, axis=1))
