@@ -442,7 +442,61 @@ def side_rows(gs, dev):
     out["attention"] = roof(ms, 2 * V3.numel() * 2 + A.numel() * 4, 2 * 64 * 1024 * 1024 * b5.r, "hbm")
     del b4, b5
     out["lookup_sweep"] = lookup_sweep(gs, dev)
+    out["grouped_attributes"] = grouped_attributes(gs, dev)
     return out
+
+
+def call_latency(fn, reps=50):
+    """Single-call latency in us: events around one call issued to an idle stream, median of
+    `reps` calls (host issue time included, as in a lookup)."""
+    import torch
+    for _ in range(5):
+        fn()
+    torch.cuda.synchronize()
+    s = torch.cuda.current_stream()
+    ts = []
+    for _ in range(reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(s)
+        fn()
+        b.record(s)
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b) * 1e3)
+    return round(statistics.median(ts), 1)
+
+
+def grouped_attributes(gs, dev):
+    """The four attribute codebooks (M = 5, 6, 10, 9, D = 1024; 512 queries each): one grouped
+    handle scoring all 2,048 queries against all 30 entries plus the per-group argmax (two
+    launches), against four handles called one after another.  Launch-bound sizes: latency
+    only, no roofline."""
+    import numpy as np
+    import torch
+    import synth
+    cases = synth.multiattr()
+    C = torch.from_numpy(np.concatenate([a["C"] for a in cases])).to(dev)
+    off = np.cumsum([0] + [a["C"].shape[0] for a in cases]).tolist()
+    X = torch.from_numpy(np.concatenate([a["X"] for a in cases])).to(dev)
+    bg = gs.build_basis_grouped(C, off)
+    S = torch.empty(X.shape[0], C.shape[0], device=dev)
+    gam = torch.empty(X.shape[0], len(cases), dtype=torch.int32, device=dev)
+    t_grouped = call_latency(lambda: (gs.project_similarity(bg, X, want_S=True, want_argmax=False,
+                                                            want_maxval=False, out={"S": S}),
+                                      gs.group_argmax(S, off, want_maxval=False, out={"argmax": gam})))
+    bs = [gs.build_basis(C[off[g]:off[g + 1]].contiguous()) for g in range(len(cases))]
+    Xs = [X[off_n:off_n + a["X"].shape[0]] for off_n, a in zip(np.cumsum([0] + [a["X"].shape[0] for a in cases]),
+                                                                  cases)]
+    ams = [torch.empty(x.shape[0], dtype=torch.int32, device=dev) for x in Xs]
+
+    def separate():
+        for b, x, am in zip(bs, Xs, ams):
+            gs.project_similarity(b, x, want_maxval=False, out={"argmax": am})
+
+    t_sep = call_latency(separate)
+    agree = all(torch.equal(ams[g], gam[n0:n0 + Xs[g].shape[0], g])
+                for g, n0 in enumerate(np.cumsum([0] + [x.shape[0] for x in Xs])[:-1]))
+    return {"queries": int(X.shape[0]), "groups": len(cases), "unit": "us per batch",
+            "grouped_one_handle": t_grouped, "four_handles": t_sep, "argmax_agree": bool(agree)}
 
 
 def lookup_sweep(gs, dev, reps=50):
@@ -456,19 +510,7 @@ def lookup_sweep(gs, dev, reps=50):
     import synth
 
     def latency(fn):
-        for _ in range(5):
-            fn()
-        torch.cuda.synchronize()
-        s = torch.cuda.current_stream()
-        ts = []
-        for _ in range(reps):
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a.record(s)
-            fn()
-            b.record(s)
-            torch.cuda.synchronize()
-            ts.append(a.elapsed_time(b) * 1e3)
-        return round(statistics.median(ts), 1)
+        return call_latency(fn, reps)
 
     res = {"M": 40, "lookups_per_batch": 1024, "unit": "us per batch", "D": [], "original_xct": [],
            "compressed_coeffs": [], "project_then_compressed": [], "argmax_agree": True}
