@@ -56,6 +56,8 @@ def lib():
         L.orc_attention.argtypes = [dp, dp, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                     ctypes.c_double, ctypes.c_int, dp]
         L.orc_memory_ratios.argtypes = [ctypes.c_long, ctypes.c_long, ctypes.c_long, dp]
+        L.orc_bind.argtypes = [dp, ctypes.c_long, ctypes.c_int, ctypes.c_int, dp, ctypes.c_long, ctypes.c_int,
+                               ctypes.c_int, dp]
         L.orc_num_threads.restype = ctypes.c_int
         L.orc_set_num_threads.argtypes = [ctypes.c_int]
         _lib = L
@@ -199,6 +201,29 @@ def attention(Yq, Yk, B, Lq, Lk, scale, apply_softmax=True):
     A = np.zeros((B, Lq, Lk))
     lib().orc_attention(_p(Yq), _p(Yk), B, Lq, Lk, r, float(scale), int(bool(apply_softmax)), _p(A))
     return A
+
+
+BIND, UNBIND = 0, 1
+
+
+def bind(X, Y, L, op=BIND):
+    """Block circular convolution (bind) or correlation (unbind) of the rows of X with the rows
+    of Y (or with Y's single row for every row of X), blocks of L components (Sec. 2.2, 3.3)."""
+    X = _f64(X)
+    Y = _f64(Y)
+    N, D = X.shape
+    if D % L:
+        raise ValueError("L must divide D")
+    ldy = 0 if Y.shape[0] == 1 and N != 1 else D
+    Z = np.zeros((N, D))
+    lib().orc_bind(_p(X), N, D, D, _p(Y), ldy, int(L), int(op), _p(Z))
+    return Z
+
+
+def reconstruct_bind(T, Q, Y, L, op=BIND):
+    """Bind (or unbind) reconstructed rows x = t Q with Y: the reconstruction at the transition
+    into component-wise operators, then the operator (Sec. 3.3)."""
+    return bind(reconstruct(T, Q), Y, L, op)
 
 
 def memory_ratios(M, D, k):

@@ -417,3 +417,62 @@ def test_grouped_attribute_codebooks(orc):
         Sg = X @ a["C"].astype(np.float64).T
         assert np.abs(S[:, off[g]:off[g + 1]] - Sg).max() <= 1e-9
         assert np.array_equal(am[:, g], np.argmax(Sg, axis=1))
+
+
+# ----------------------------------------------------------------- binding / unbinding (Sec. 2.2, 3.3)
+def _block_fft_conv(X, Y, L, correlate):
+    Z = np.zeros_like(X)
+    for b0 in range(0, X.shape[1], L):
+        fx = np.fft.fft(X[:, b0:b0 + L], axis=1)
+        fy = np.fft.fft(Y[:, b0:b0 + L], axis=1)
+        Z[:, b0:b0 + L] = np.real(np.fft.ifft(fx * (np.conj(fy) if correlate else fy), axis=1))
+    return Z
+
+
+@pytest.mark.parametrize("L", [48, 16, 12, 1])
+def test_bind_convolution_theorem(orc, L):
+    """Block circular convolution / correlation against the DFT's convolution theorem."""
+    rng = np.random.default_rng(L)
+    X = rng.normal(size=(5, 48))
+    Y = rng.normal(size=(5, 48))
+    assert np.abs(orc.bind(X, Y, L, orc.BIND) - _block_fft_conv(X, Y, L, False)).max() <= 1e-12
+    assert np.abs(orc.bind(X, Y, L, orc.UNBIND) - _block_fft_conv(X, Y, L, True)).max() <= 1e-12
+
+
+def test_bind_algebra(orc):
+    """Identity element, commutativity, and one partner broadcast over every row."""
+    rng = np.random.default_rng(2)
+    L, D = 16, 64
+    X = rng.normal(size=(6, D))
+    Y = rng.normal(size=(6, D))
+    delta = np.zeros((1, D))
+    delta[0, ::L] = 1.0
+    assert np.array_equal(orc.bind(X, delta, L), X)
+    assert np.array_equal(orc.bind(X, delta, L, orc.UNBIND), X)
+    assert np.abs(orc.bind(X, Y, L) - orc.bind(Y, X, L)).max() <= 1e-12
+    y1 = Y[:1]
+    assert np.array_equal(orc.bind(X, y1, L), orc.bind(X, np.repeat(y1, 6, axis=0), L))
+
+
+def test_unbind_inverts_unitary_binding(orc):
+    """Partners whose block spectra have unit modulus: unbinding recovers the bound vector."""
+    rng = np.random.default_rng(3)
+    L, D = 32, 128
+    Y = np.zeros((4, D))
+    for b0 in range(0, D, L):
+        ph = rng.uniform(-np.pi, np.pi, size=(4, L))
+        spec = np.exp(1j * ph)
+        spec[:, 0] = 1.0
+        spec[:, L // 2] = 1.0
+        spec[:, L // 2 + 1:] = np.conj(spec[:, 1:L // 2][:, ::-1])  # Hermitian: real blocks
+        Y[:, b0:b0 + L] = np.real(np.fft.ifft(spec, axis=1))
+    X = rng.normal(size=(4, D))
+    assert np.abs(orc.bind(orc.bind(X, Y, L), Y, L, orc.UNBIND) - X).max() <= 1e-12
+
+
+def test_reconstruct_bind_of_codebook(orc, tiny_case):
+    """Reconstructing R gives the codebook, so binding the reconstruction is binding C."""
+    t, (Q, R, _) = tiny_case
+    Y = np.random.default_rng(4).normal(size=(1, Q.shape[1]))
+    Z = orc.reconstruct_bind(R, Q, Y, 256)
+    assert np.abs(Z - orc.bind(t["C"], Y, 256)).max() <= 1e-9
