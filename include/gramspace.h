@@ -282,6 +282,43 @@ GS_API gs_status gs_prob_vectorize(const gs_basis* h, const float* P, long long 
 GS_API gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt,
                          float* Xhat, int ldxh, unsigned flags, void* stream);
 
+/* binding operators of gs_bind / gs_reconstruct_bind */
+#define GS_BIND 0   /* block circular convolution  */
+#define GS_UNBIND 1 /* block circular correlation  */
+
+/*
+ * Binding and unbinding, the component-wise operators of rule execution
+ * (Sec. 2.2: binding / unbinding with a modulo-style index computation;
+ * Sec. 3.3: the operators after reconstruction are based on circular
+ * convolution).  Rows are cut into blocks of L consecutive components (L
+ * divides D; L = D is one circular convolution over the whole vector) and,
+ * within block b of row n,
+ *   GS_BIND:   Z[n][bL+k] = sum_j X[n][bL+j] * Y[n][bL + ((k - j) mod L)]
+ *   GS_UNBIND: Z[n][bL+k] = sum_j X[n][bL+j] * Y[n][bL + ((j - k) mod L)]
+ * (unbinding with y undoes binding with y when y's block spectra have unit
+ * modulus, and approximately for random y).  X, Z: N x D fp32 (ld = ldx,
+ * ldz >= D); Y: N x D fp32 with ld = ldy >= D, or ldy = 0: Y's single row
+ * binds every row.  fp32 CUDA-core arithmetic, one sum per output in j order.
+ * Errors: GS_ERR_SHAPE (L does not divide D, ld too small), GS_ERR_INVALID_ARG.
+ */
+GS_API gs_status gs_bind(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L, int op,
+                         float* Z, int ldz, void* stream);
+
+/*
+ * Reconstruction followed by binding at the transition into component-wise
+ * operators (Sec. 3.3: reconstruction is placed immediately before binding and
+ * unbinding): Z = op(T Q, Y) with gs_reconstruct's T (N x r, t_dtype, ldt) and
+ * gs_bind's Y, L, op and Z.  The rows are processed in chunks whose
+ * reconstruction (at most 32 MiB) lives in the handle's scratch between the two
+ * kernels, so the reconstructed vectors stay in L2 rather than making a round
+ * trip through HBM.  flags picks the reconstruction path as in gs_reconstruct.
+ * Shares the handle's scratch with the other multi-kernel calls: order calls
+ * on one handle.
+ */
+GS_API gs_status gs_reconstruct_bind(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt,
+                                     const float* Y, long long ldy, int L, int op, float* Z, int ldz, unsigned flags,
+                                     void* stream);
+
 /*
  * Attention scores between compressed vectors (Sec. 2.2 attention score;
  * Sec. 3.2: attention computed by matrix multiplication is preserved on

@@ -538,16 +538,9 @@ gs_status gs_prob_vectorize(const gs_basis* h, const float* P, long long N, int 
     return GS_OK;
 }
 
-gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt, float* Xhat,
-                         int ldxh, unsigned flags, void* stream) {
-    if (!h || !valid_path(flags)) return GS_ERR_INVALID_ARG;
-    if (t_dtype != GS_F32 && t_dtype != GS_BF16) return GS_ERR_INVALID_ARG;
-    if (N < 0 || ldt < h->r || ldxh < h->D) return GS_ERR_SHAPE;
-    if (N == 0) return GS_OK;
-    if (!T || !Xhat) return GS_ERR_INVALID_ARG;
-    DeviceGuard g(h->device);
-    if (!g.ok) return GS_ERR_CUDA;
-    cudaStream_t s = (cudaStream_t)stream;
+// Xhat = T Q with the fp16 copy of T (tensor-core path) in `work` (work_floats floats).
+static gs_status reconstruct_rows(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt, float* Xhat,
+                                  int ldxh, unsigned flags, cudaStream_t s, float* work, long long work_floats) {
     const bool tc_ok = h->has_split && h->r >= 1 && t_dtype == GS_F32 && (uintptr_t)T % 16 == 0 && ldt % 4 == 0;
     if (flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && tc_ok && big_gemm(N, h->D, h->r))) {
         if (!tc_ok) return t_dtype != GS_F32 || !h->has_split ? GS_ERR_UNSUPPORTED : GS_ERR_ALIGNMENT;
@@ -555,15 +548,15 @@ gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, long lon
         // Xhat re-reads it), the basis' dithered fp16 Q^T, fp32 accumulation; rows in chunks
         // that fit the scratch
         const int ld16 = (h->r + 7) / 8 * 8;  // 16-byte rows for TMA
-        const long long chunk = std::min(h->scratch_floats * 2 / ld16, kMaxGemmRows) / 128 * 128;
+        const long long chunk = std::min(work_floats * 2 / ld16, kMaxGemmRows) / 128 * 128;
         if (chunk < 128) return GS_ERR_SHAPE;
         for (long long c0 = 0; c0 < N; c0 += chunk) {
             const long long nc = std::min(chunk, N - c0);
             const float* Tc = (const float*)T + (size_t)c0 * ldt;
-            gs_status st = from_cuda(gs::launch_round_f16(Tc, ldt, nc, h->r, h->scratch, ld16, s));
+            gs_status st = from_cuda(gs::launch_round_f16(Tc, ldt, nc, h->r, work, ld16, s));
             if (st != GS_OK) return st;
             gs::GemmTcArgs a{};
-            a.A = h->scratch; a.lda = ld16; a.m = nc; a.K = h->r; a.split = false; a.a_half = true;
+            a.A = work; a.lda = ld16; a.m = nc; a.K = h->r; a.split = false; a.a_half = true;
             a.B0 = h->Q16t; a.ldb = h->ldr16; a.n = h->D;
             a.C = Xhat + (size_t)c0 * ldxh; a.ldc = ldxh; a.c_bf16 = false; a.alpha = 1.f;
             st = from_cuda(gs::launch_gemm_tc(a, h->device, s));
@@ -581,6 +574,72 @@ gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, long lon
         a.m = nc; a.n = h->D; a.k = h->r; a.batch = 1; a.alpha = 1.f;
         cudaError_t e = gs::launch_gemm_simt(a, s);
         if (e != cudaSuccess) return from_cuda(e);
+    }
+    return GS_OK;
+}
+
+gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt, float* Xhat,
+                         int ldxh, unsigned flags, void* stream) {
+    if (!h || !valid_path(flags)) return GS_ERR_INVALID_ARG;
+    if (t_dtype != GS_F32 && t_dtype != GS_BF16) return GS_ERR_INVALID_ARG;
+    if (N < 0 || ldt < h->r || ldxh < h->D) return GS_ERR_SHAPE;
+    if (N == 0) return GS_OK;
+    if (!T || !Xhat) return GS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    if (!g.ok) return GS_ERR_CUDA;
+    return reconstruct_rows(h, T, t_dtype, N, ldt, Xhat, ldxh, flags, (cudaStream_t)stream, h->scratch,
+                            h->scratch_floats);
+}
+
+static gs_status check_bind_args(long long N, int D, int ldx, long long ldy, int L, int op, int ldz) {
+    if (op != GS_BIND && op != GS_UNBIND) return GS_ERR_INVALID_ARG;
+    if (N < 0 || D < 1 || L < 1 || D % L || ldx < D || ldz < D || (ldy != 0 && ldy < D)) return GS_ERR_SHAPE;
+    return GS_OK;
+}
+
+gs_status gs_bind(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L, int op, float* Z,
+                  int ldz, void* stream) {
+    gs_status st = check_bind_args(N, D, ldx, ldy, L, op, ldz);
+    if (st != GS_OK) return st;
+    if (N == 0) return GS_OK;
+    if (!X || !Y || !Z) return GS_ERR_INVALID_ARG;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return GS_ERR_CUDA;
+    if (!device_supported(dev)) return GS_ERR_UNSUPPORTED;
+    return from_cuda(gs::launch_bind(X, N, D, ldx, Y, ldy, L, op == GS_UNBIND, Z, ldz, (cudaStream_t)stream));
+}
+
+gs_status gs_reconstruct_bind(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt, const float* Y,
+                              long long ldy, int L, int op, float* Z, int ldz, unsigned flags, void* stream) {
+    if (!h || !valid_path(flags)) return GS_ERR_INVALID_ARG;
+    if (t_dtype != GS_F32 && t_dtype != GS_BF16) return GS_ERR_INVALID_ARG;
+    if (N < 0 || ldt < h->r) return GS_ERR_SHAPE;
+    gs_status st = check_bind_args(N, h->D, h->D, ldy, L, op, ldz);
+    if (st != GS_OK) return st;
+    if (N == 0) return GS_OK;
+    if (!T || !Y || !Z) return GS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    if (!g.ok) return GS_ERR_CUDA;
+    cudaStream_t s = (cudaStream_t)stream;
+    // rows in chunks: the reconstructed chunk (at most 32 MiB, so it stays in L2 between the two
+    // kernels) and the fp16 copy of its T rows share the handle's scratch
+    const int Dp = (h->D + 3) / 4 * 4, ld16 = (h->r + 7) / 8 * 8;
+    long long cr = std::min(h->scratch_floats / (Dp + ld16 / 2 + 1), (32LL << 20) / (4LL * Dp));
+    cr = std::min(cr, kMaxGemmRows);
+    if (cr >= 128) cr = cr / 128 * 128;
+    if (cr < 1) return GS_ERR_SHAPE;
+    float* xhat = h->scratch;
+    float* work = h->scratch + cr * Dp;
+    const long long work_floats = h->scratch_floats - cr * Dp;
+    const size_t tsize = t_dtype == GS_F32 ? 4 : 2;
+    for (long long c0 = 0; c0 < N; c0 += cr) {
+        const long long nc = std::min(cr, N - c0);
+        st = reconstruct_rows(h, (const char*)T + (size_t)c0 * ldt * tsize, t_dtype, nc, ldt, xhat, Dp, flags, s,
+                              work, work_floats);
+        if (st != GS_OK) return st;
+        st = from_cuda(gs::launch_bind(xhat, nc, h->D, Dp, Y + (size_t)c0 * ldy, ldy, L, op == GS_UNBIND,
+                                       Z + (size_t)c0 * ldz, ldz, s));
+        if (st != GS_OK) return st;
     }
     return GS_OK;
 }

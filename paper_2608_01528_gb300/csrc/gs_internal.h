@@ -127,6 +127,12 @@ constexpr int kMaxGroups = 256;
 cudaError_t launch_group_argmax(const float* S, long long N, int lds, const int* off, int G, int* argmax,
                                 float* maxval, cudaStream_t s);
 
+// block circular convolution (unbind: correlation) of rows of X with rows of Y (ldy = 0: Y's
+// row 0 for every row), blocks of L (L divides D); k_bind8 for L % 8 == 0 up to kMaxBindFastL
+constexpr int kMaxBindFastL = 4096;
+cudaError_t launch_bind(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L, bool unbind,
+                        float* Z, int ldz, cudaStream_t s);
+
 // per-row argmax / maxval over S (N x M); SOFTMAX mode rewrites the row in place.
 cudaError_t launch_row_finish(float* S, long long N, int M, int lds, bool softmax, int* argmax,
                               float* maxval, cudaStream_t s);

@@ -14,8 +14,12 @@
 //  k_row_softmax  softmax over each attention row
 //  k_rownorm      full-D query norms for cosine scores
 //  k_group_argmax argmax / max of each score row within each group of a grouped codebook
+//  k_bind8        block circular convolution / correlation (binding / unbinding), L % 8 == 0
+//  k_bind1        the same for any block length, one output per thread
 
 #include <float.h>
+
+#include <algorithm>
 
 #include "gs_internal.h"
 
@@ -326,6 +330,88 @@ __global__ void __launch_bounds__(256) k_group_argmax(const float* __restrict__ 
     }
 }
 
+// Binding (UNB = false: Z_k = sum_j X_j Y_(k-j mod L)) or unbinding (UNB = true:
+// Z_k = sum_j X_j Y_(j-k mod L)) within blocks of L components.  A CTA takes one block of
+// 256 / tpr rows (tpr = min(L / 8, 256) threads per row) and stages the rows' X and Y
+// blocks in shared memory, Y index-reversed for unbinding (Y'_m = Y_(-m mod L) turns the
+// correlation into a convolution).  A thread computes eight consecutive outputs
+// k0..k0+7: per eight-wide step of j it reads X_j..X_(j+7) (the same words for the whole
+// row: broadcast) and the sixteen Y' values (k0 - j - 8 .. k0 - j + 7) mod L -- two aligned
+// chunks, since L, k0 and j are multiples of 8 -- and does 64 fma.  ldy = 0: one partner row.
+template <bool UNB>
+__global__ void __launch_bounds__(256) k_bind8(const float* __restrict__ X, long long N, int ldx,
+                                                const float* __restrict__ Y, long long ldy, int L,
+                                                float* __restrict__ Z, int ldz, int zvec) {
+    extern __shared__ float4 bind_sm[];
+    const int tpr = min(L >> 3, 256);
+    const int rpc = 256 / tpr;
+    const int tr = threadIdx.x / tpr, tk = threadIdx.x - tr * tpr;
+    const long long n = (long long)blockIdx.x * rpc + tr;
+    const int b0 = blockIdx.y * L;
+    float* xs = reinterpret_cast<float*>(bind_sm) + (size_t)tr * 2 * L;
+    float* ys = xs + L;
+    if (tr < rpc && n < N) {
+        const float* x = X + (size_t)n * ldx + b0;
+        const float* y = Y + (size_t)n * ldy + b0;
+        for (int j = tk; j < L; j += tpr) {
+            xs[j] = x[j];
+            ys[j] = y[UNB ? (j == 0 ? 0 : L - j) : j];
+        }
+    }
+    __syncthreads();
+    if (tr >= rpc || n >= N) return;
+    for (int k0 = 8 * tk; k0 < L; k0 += 8 * tpr) {
+        float z[8];
+#pragma unroll
+        for (int t = 0; t < 8; ++t) z[t] = 0.f;
+        for (int j = 0; j < L; j += 8) {
+            int a = k0 - j - 8;
+            if (a < 0) a += L;
+            const int c = a + 8 == L ? 0 : a + 8;
+            float xv[8], w[16];
+            *reinterpret_cast<float4*>(xv) = *reinterpret_cast<const float4*>(xs + j);
+            *reinterpret_cast<float4*>(xv + 4) = *reinterpret_cast<const float4*>(xs + j + 4);
+            *reinterpret_cast<float4*>(w) = *reinterpret_cast<const float4*>(ys + a);
+            *reinterpret_cast<float4*>(w + 4) = *reinterpret_cast<const float4*>(ys + a + 4);
+            *reinterpret_cast<float4*>(w + 8) = *reinterpret_cast<const float4*>(ys + c);
+            *reinterpret_cast<float4*>(w + 12) = *reinterpret_cast<const float4*>(ys + c + 4);
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+#pragma unroll
+                for (int t = 0; t < 8; ++t) z[t] = fmaf(xv[u], w[8 + t - u], z[t]);
+        }
+        float* zo = Z + (size_t)n * ldz + b0 + k0;
+        if (zvec) {
+            reinterpret_cast<float4*>(zo)[0] = make_float4(z[0], z[1], z[2], z[3]);
+            reinterpret_cast<float4*>(zo)[1] = make_float4(z[4], z[5], z[6], z[7]);
+        } else {
+#pragma unroll
+            for (int t = 0; t < 8; ++t) zo[t] = z[t];
+        }
+    }
+}
+
+// Any block length: one thread per output, operands read through the cache.
+template <bool UNB>
+__global__ void __launch_bounds__(256) k_bind1(const float* __restrict__ X, long long N, int D, int ldx,
+                                                const float* __restrict__ Y, long long ldy, int L,
+                                                float* __restrict__ Z, int ldz) {
+    const long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= N * D) return;
+    const long long n = e / D;
+    const int d = (int)(e - n * D);
+    const int b0 = d - d % L, k = d - b0;
+    const float* x = X + (size_t)n * ldx + b0;
+    const float* y = Y + (size_t)n * ldy + b0;
+    float acc = 0.f;
+    for (int j = 0; j < L; ++j) {
+        int m = UNB ? j - k : k - j;
+        if (m < 0) m += L;
+        acc = fmaf(x[j], y[m], acc);
+    }
+    Z[(size_t)n * ldz + d] = acc;
+}
+
 inline unsigned rows_grid(long long n) { return (unsigned)((n + 7) / 8); }
 
 }  // namespace
@@ -385,6 +471,30 @@ cudaError_t launch_group_argmax(const float* S, long long N, int lds, const int*
     go.G = G;
     for (int g = 0; g <= G; ++g) go.off[g] = off[g];
     k_group_argmax<<<rows_grid(N), 256, 0, s>>>(S, N, lds, go, argmax, maxval);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_bind(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L, bool unbind,
+                        float* Z, int ldz, cudaStream_t s) {
+    if (N <= 0) return cudaSuccess;
+    if (L % 8 == 0 && L <= kMaxBindFastL && D / L <= 65535) {
+        const int tpr = std::min(L / 8, 256);
+        const int rpc = 256 / tpr;
+        const size_t smem = (size_t)rpc * 2 * L * sizeof(float);
+        const dim3 grid((unsigned)((N + rpc - 1) / rpc), (unsigned)(D / L));
+        const int zvec = ((uintptr_t)Z % 16 == 0 && ldz % 4 == 0) ? 1 : 0;
+        if (unbind)
+            k_bind8<true><<<grid, 256, smem, s>>>(X, N, ldx, Y, ldy, L, Z, ldz, zvec);
+        else
+            k_bind8<false><<<grid, 256, smem, s>>>(X, N, ldx, Y, ldy, L, Z, ldz, zvec);
+        return cudaGetLastError();
+    }
+    const long long total = N * D;
+    const unsigned blocks = (unsigned)((total + 255) / 256);
+    if (unbind)
+        k_bind1<true><<<blocks, 256, 0, s>>>(X, N, D, ldx, Y, ldy, L, Z, ldz);
+    else
+        k_bind1<false><<<blocks, 256, 0, s>>>(X, N, D, ldx, Y, ldy, L, Z, ldz);
     return cudaGetLastError();
 }
 

@@ -31,7 +31,8 @@ EXPORTS = ("gs_build_basis", "gs_basis_info", "gs_basis_destroy", "gs_project_si
            "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores", "gs_stream_status",
            "gs_status_string", "gs_version", "gs_project_similarity_static", "gs_similarity_coeffs",
            "gs_selftest_wait_timeout", "gs_basis_import", "gs_basis_reserve_staging",
-           "gs_project_similarity_host", "gs_build_basis_grouped", "gs_basis_groups", "gs_group_argmax")
+           "gs_project_similarity_host", "gs_build_basis_grouped", "gs_basis_groups", "gs_group_argmax",
+           "gs_bind", "gs_reconstruct_bind")
 
 
 class GramSpaceError(RuntimeError):
@@ -62,6 +63,8 @@ def load_library(path=LIB_PATH):
     L.gs_build_basis_grouped.argtypes = [vp, ip, ip, ip, vp, ip, f32, u32, vp, ctypes.POINTER(vp)]
     L.gs_basis_groups.argtypes = [vp, ctypes.POINTER(ip), vp, vp]
     L.gs_group_argmax.argtypes = [vp, i64, ip, vp, ip, vp, vp, vp]
+    L.gs_bind.argtypes = [vp, i64, ip, ip, vp, i64, ip, ip, vp, ip, vp]
+    L.gs_reconstruct_bind.argtypes = [vp, vp, ip, i64, ip, vp, i64, ip, ip, vp, ip, u32, vp]
     L.gs_project_similarity.argtypes = [vp, vp, i64, ip, ip, f32, u32, vp, ip, vp, ip, vp, vp, vp]
     L.gs_similarity_coeffs.argtypes = [vp, vp, i64, ip, ip, f32, u32, vp, ip, vp, vp, vp]
     L.gs_prob_vectorize.argtypes = [vp, vp, i64, ip, vp, ip, ip, u32, vp]
@@ -78,7 +81,7 @@ def load_library(path=LIB_PATH):
                  "gs_similarity_coeffs", "gs_prob_vectorize", "gs_reconstruct", "gs_attention_scores",
                  "gs_stream_status", "gs_selftest_wait_timeout", "gs_basis_import",
                  "gs_basis_reserve_staging", "gs_project_similarity_host", "gs_build_basis_grouped",
-                 "gs_basis_groups", "gs_group_argmax"):
+                 "gs_basis_groups", "gs_group_argmax", "gs_bind", "gs_reconstruct_bind"):
         getattr(L, name).restype = ctypes.c_int
     _lib = L
     return L
@@ -365,6 +368,47 @@ def reconstruct(basis, T, path="auto", out=None, stream=None):
                               _ptr(X), _ld(X), PATHS[path], _stream(stream))
     _check(st, "gs_reconstruct")
     return X
+
+
+BIND_OPS = {"bind": 0, "unbind": 1}
+
+
+def _partner(Y, N, D):
+    if not Y.is_cuda or Y.dtype != torch.float32 or Y.dim() != 2 or Y.shape[1] != D:
+        raise ValueError(f"Y must be a float32 CUDA tensor with {D} columns")
+    if Y.shape[0] == 1 and N != 1:
+        return 0  # one partner for every row
+    if Y.shape[0] != N:
+        raise ValueError("Y must have one row or one row per input row")
+    return _ld(Y)
+
+
+def bind(X, Y, L, op="bind", out=None, stream=None):
+    """Block circular convolution (op="bind") or correlation ("unbind") of the rows of X with
+    those of Y (or with Y's single row), blocks of L; see gs_bind."""
+    N, D = X.shape
+    ldy = _partner(Y, N, D)
+    Z = out if out is not None else torch.empty((N, D), dtype=torch.float32, device=X.device)
+    L_ = load_library()
+    with torch.cuda.device(X.device):
+        st = L_.gs_bind(_ptr(X), N, D, _ld(X) if N else D, _ptr(Y), ldy, int(L), BIND_OPS[op], _ptr(Z),
+                        _ld(Z) if N else D, _stream(stream))
+    _check(st, "gs_bind")
+    return Z
+
+
+def reconstruct_bind(basis, T, Y, L, op="bind", path="auto", out=None, stream=None):
+    """op(T Q, Y): reconstruction then binding, chunk by chunk through L2; see gs_reconstruct_bind."""
+    N = T.shape[0]
+    ldy = _partner(Y, N, basis.D)
+    Z = out if out is not None else torch.empty((N, basis.D), dtype=torch.float32, device=T.device)
+    L_ = load_library()
+    with torch.cuda.device(basis.device):
+        st = L_.gs_reconstruct_bind(basis.handle, _ptr(T), _dtype_code(T), N, _ld(T) if N else basis.r, _ptr(Y),
+                                    ldy, int(L), BIND_OPS[op], _ptr(Z), _ld(Z) if N else basis.D, PATHS[path],
+                                    _stream(stream))
+    _check(st, "gs_reconstruct_bind")
+    return Z
 
 
 def attention_scores(Yq, Yk, scale, apply_softmax=True, path="auto", out=None, stream=None):
