@@ -32,6 +32,9 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "project+similarity queries/s"
+# fp32 FMA peak of the binding kernel (bound "alu"): 152 SMs x 128 fp32 lanes x 2 flop at the
+# 2,070 MHz maximum SM clock
+FP32_PEAK_TFLOPS = round(152 * 128 * 2 * 2.07e9 / 1e12, 1)
 # rows per staging slot of the end-to-end leg (8192 x 8192 fp32 = 256 MiB a slot)
 E2E_CHUNK = 8192
 WORKLOAD = "large-batch fused project+similarity+argmax, bipolar M=256, D=8192, 65536 queries (sigma=1)"
@@ -440,7 +443,23 @@ def side_rows(gs, dev):
     A = torch.empty(64, 1024, 1024, device=dev)
     ms = timeit(lambda: gs.attention_scores(V3, V3, 1 / 64.0, out=A))
     out["attention"] = roof(ms, 2 * V3.numel() * 2 + A.numel() * 4, 2 * 64 * 1024 * 1024 * b5.r, "hbm")
-    del b4, b5
+    # reconstruct + bind at the transition into component-wise operators: 8,192 coefficient rows
+    # of the attention basis (r = 512, D = 4096), per-row partners, blocks of 256
+    Nb, Lb = 8192, 256
+    Tb = torch.from_numpy(synth.attention_probs(12, 1, Nb, b5.M, 1)).to(dev) @ b5.R
+    Yb = torch.randn(Nb, b5.D, device=dev)
+    Zb = torch.empty(Nb, b5.D, device=dev)
+    Xb = torch.empty(Nb, b5.D, device=dev)
+    ms_fused = timeit(lambda: gs.reconstruct_bind(b5, Tb, Yb, Lb, out=Zb))
+    ms_rec = timeit(lambda: gs.reconstruct(b5, Tb, out=Xb))
+    ms_bind = timeit(lambda: gs.bind(Xb, Yb, Lb, out=Zb))
+    bind_flops = 2 * Nb * b5.D * Lb
+    out["reconstruct_bind"] = {"ms": round(ms_fused, 4), "rows": Nb, "D": b5.D, "r": b5.r, "L": Lb,
+                               "reconstruct_ms": round(ms_rec, 4), "bind_ms": round(ms_bind, 4),
+                               "bind_tflops": round(bind_flops / (ms_bind / 1e3) / 1e12, 1),
+                               "bound": "alu", "alu_peak_tflops": FP32_PEAK_TFLOPS,
+                               "frac": round(bind_flops / (ms_bind / 1e3) / 1e12 / FP32_PEAK_TFLOPS, 4)}
+    del b4, b5, Xb, Yb, Zb
     out["lookup_sweep"] = lookup_sweep(gs, dev)
     out["grouped_attributes"] = grouped_attributes(gs, dev)
     return out

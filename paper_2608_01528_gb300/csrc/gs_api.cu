@@ -621,10 +621,10 @@ gs_status gs_reconstruct_bind(const gs_basis* h, const void* T, int t_dtype, lon
     DeviceGuard g(h->device);
     if (!g.ok) return GS_ERR_CUDA;
     cudaStream_t s = (cudaStream_t)stream;
-    // rows in chunks: the reconstructed chunk (at most 32 MiB, so it stays in L2 between the two
+    // rows in chunks: the reconstructed chunk (at most 64 MiB, so it stays in L2 between the two
     // kernels) and the fp16 copy of its T rows share the handle's scratch
     const int Dp = (h->D + 3) / 4 * 4, ld16 = (h->r + 7) / 8 * 8;
-    long long cr = std::min(h->scratch_floats / (Dp + ld16 / 2 + 1), (32LL << 20) / (4LL * Dp));
+    long long cr = std::min(h->scratch_floats / (Dp + ld16 / 2 + 1), (64LL << 20) / (4LL * Dp));
     cr = std::min(cr, kMaxGemmRows);
     if (cr >= 128) cr = cr / 128 * 128;
     if (cr < 1) return GS_ERR_SHAPE;

@@ -14,7 +14,8 @@
 //  k_row_softmax  softmax over each attention row
 //  k_rownorm      full-D query norms for cosine scores
 //  k_group_argmax argmax / max of each score row within each group of a grouped codebook
-//  k_bind8        block circular convolution / correlation (binding / unbinding), L % 8 == 0
+//  k_bind16       block circular convolution / correlation (binding / unbinding), L % 16 == 0
+//  k_bind8        the same for L % 8 == 0
 //  k_bind1        the same for any block length, one output per thread
 
 #include <float.h>
@@ -391,6 +392,68 @@ __global__ void __launch_bounds__(256) k_bind8(const float* __restrict__ X, long
     }
 }
 
+// The same with 16 x 16 register tiles (L % 16 == 0): a thread computes 16 consecutive
+// outputs; per 16-wide step of j it reads X_j..X_(j+15) (broadcast within the row) and the
+// 32 Y' values (k0 - j - 16 .. k0 - j + 15) mod L as two aligned 16-value segments, and does
+// 256 fma.  Y' is stored with 4 words of padding after every 16 (segment i at word 20 i), so
+// the segments of consecutive threads, 64 bytes apart unpadded, fall in disjoint banks.
+template <bool UNB>
+__global__ void __launch_bounds__(256) k_bind16(const float* __restrict__ X, long long N, int ldx,
+                                                 const float* __restrict__ Y, long long ldy, int L,
+                                                 float* __restrict__ Z, int ldz, int zvec) {
+    extern __shared__ float4 bind_sm16[];
+    const int tpr = min(L >> 4, 256);
+    const int rpc = 256 / tpr;
+    const int tr = threadIdx.x / tpr, tk = threadIdx.x - tr * tpr;
+    const long long n = (long long)blockIdx.x * rpc + tr;
+    const int b0 = blockIdx.y * L;
+    const int Lp = L + (L >> 2);  // padded length of Y'
+    float* xs = reinterpret_cast<float*>(bind_sm16) + (size_t)tr * (L + Lp);
+    float* ys = xs + L;
+    if (tr < rpc && n < N) {
+        const float* x = X + (size_t)n * ldx + b0;
+        const float* y = Y + (size_t)n * ldy + b0;
+        for (int j = tk; j < L; j += tpr) {
+            xs[j] = x[j];
+            ys[j + (j >> 4) * 4] = y[UNB ? (j == 0 ? 0 : L - j) : j];
+        }
+    }
+    __syncthreads();
+    if (tr >= rpc || n >= N) return;
+    for (int k0 = 16 * tk; k0 < L; k0 += 16 * tpr) {
+        float z[16];
+#pragma unroll
+        for (int t = 0; t < 16; ++t) z[t] = 0.f;
+        for (int j = 0; j < L; j += 16) {
+            int a = k0 - j - 16;
+            if (a < 0) a += L;
+            const int c = a + 16 == L ? 0 : a + 16;
+            float xv[16], w[32];
+            const float* sa = ys + a + (a >> 2);
+            const float* sc = ys + c + (c >> 2);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                *reinterpret_cast<float4*>(xv + 4 * q) = *reinterpret_cast<const float4*>(xs + j + 4 * q);
+                *reinterpret_cast<float4*>(w + 4 * q) = *reinterpret_cast<const float4*>(sa + 4 * q);
+                *reinterpret_cast<float4*>(w + 16 + 4 * q) = *reinterpret_cast<const float4*>(sc + 4 * q);
+            }
+#pragma unroll
+            for (int u = 0; u < 16; ++u)
+#pragma unroll
+                for (int t = 0; t < 16; ++t) z[t] = fmaf(xv[u], w[16 + t - u], z[t]);
+        }
+        float* zo = Z + (size_t)n * ldz + b0 + k0;
+        if (zvec) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                reinterpret_cast<float4*>(zo)[q] = make_float4(z[4 * q], z[4 * q + 1], z[4 * q + 2], z[4 * q + 3]);
+        } else {
+#pragma unroll
+            for (int t = 0; t < 16; ++t) zo[t] = z[t];
+        }
+    }
+}
+
 // Any block length: one thread per output, operands read through the cache.
 template <bool UNB>
 __global__ void __launch_bounds__(256) k_bind1(const float* __restrict__ X, long long N, int D, int ldx,
@@ -477,12 +540,23 @@ cudaError_t launch_group_argmax(const float* S, long long N, int lds, const int*
 cudaError_t launch_bind(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L, bool unbind,
                         float* Z, int ldz, cudaStream_t s) {
     if (N <= 0) return cudaSuccess;
+    const int zvec = ((uintptr_t)Z % 16 == 0 && ldz % 4 == 0) ? 1 : 0;
+    if (L % 16 == 0 && L <= kMaxBindFastL && D / L <= 65535) {
+        const int tpr = std::min(L / 16, 256);
+        const int rpc = 256 / tpr;
+        const size_t smem = (size_t)rpc * (2 * L + L / 4) * sizeof(float);
+        const dim3 grid((unsigned)((N + rpc - 1) / rpc), (unsigned)(D / L));
+        if (unbind)
+            k_bind16<true><<<grid, 256, smem, s>>>(X, N, ldx, Y, ldy, L, Z, ldz, zvec);
+        else
+            k_bind16<false><<<grid, 256, smem, s>>>(X, N, ldx, Y, ldy, L, Z, ldz, zvec);
+        return cudaGetLastError();
+    }
     if (L % 8 == 0 && L <= kMaxBindFastL && D / L <= 65535) {
         const int tpr = std::min(L / 8, 256);
         const int rpc = 256 / tpr;
         const size_t smem = (size_t)rpc * 2 * L * sizeof(float);
         const dim3 grid((unsigned)((N + rpc - 1) / rpc), (unsigned)(D / L));
-        const int zvec = ((uintptr_t)Z % 16 == 0 && ldz % 4 == 0) ? 1 : 0;
         if (unbind)
             k_bind8<true><<<grid, 256, smem, s>>>(X, N, ldx, Y, ldy, L, Z, ldz, zvec);
         else
