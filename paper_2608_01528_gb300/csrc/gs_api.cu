@@ -121,6 +121,7 @@ gs_status ps_two_gemm(const gs_basis* h, const float* X, long long N, int ldx, i
         gs::GemmTcArgs g2{};
         g2.A = Ybuf; g2.lda = r4; g2.m = nc; g2.K = r; g2.split = true;
         g2.B0 = h->tc_Rh; g2.B1 = h->tc_Rl; g2.ldb = h->tc_npad; g2.n = M;
+        g2.b_klo = h->kzero_host.data(); g2.b_khi = h->rlen_host.data();
         g2.C = Sbuf; g2.ldc = ldsb; g2.c_bf16 = false; g2.alpha = scale;
         if (mode == GS_SCORE_COSINE) { g2.rownorm = xn; g2.colnorm = h->cnorm; }
         e = gs::launch_gemm_tc(g2, h->device, s);
@@ -482,6 +483,7 @@ gs_status gs_similarity_coeffs(const gs_basis* h, const float* Y, long long N, i
             gs::GemmTcArgs a{};
             a.A = Yc; a.lda = ldy; a.m = nc; a.K = r; a.split = true;
             a.B0 = h->tc_Rh; a.B1 = h->tc_Rl; a.ldb = h->tc_npad; a.n = M;
+            a.b_klo = h->kzero_host.data(); a.b_khi = h->rlen_host.data();
             a.C = Sbuf; a.ldc = ldsb; a.c_bf16 = false; a.alpha = scale;
             if (xn) { a.rownorm = xn; a.colnorm = h->cnorm; }
             e = gs::launch_gemm_tc(a, h->device, s);
@@ -521,6 +523,7 @@ gs_status gs_prob_vectorize(const gs_basis* h, const float* P, long long N, int 
         gs::GemmTcArgs a{};
         a.A = P; a.lda = ldp; a.m = N; a.K = h->M; a.split = true;
         a.B0 = h->tc_Rth; a.B1 = h->tc_Rtl; a.ldb = h->tc_mpad; a.n = h->r;
+        a.b_klo = h->pivot_host.data(); a.b_khi = h->kM_host.data();
         a.C = V; a.ldc = ldv; a.c_bf16 = v_dtype == GS_BF16; a.alpha = 1.f;
         return from_cuda(gs::launch_gemm_tc(a, h->device, s));
     }

@@ -68,6 +68,7 @@ constexpr int kAPartBytes = kBM * kBK * 2;             // 16 KB
 constexpr int kBStageBytes = 256 * kBK * 2;            // 32 KB
 constexpr int kMaxSX = 4, kMaxSA = 4, kMaxSB = 4;
 constexpr int kTmemCols = 512;
+constexpr int kMaxTilesN = 64;  // column tiles whose K-block range can be trimmed
 
 // A operand modes: fp32 rounded to fp16 by the converters; fp32 split into bf16 hi / lo by
 // the converters (three products with B hi / lo); fp16 already, loaded by TMA straight into
@@ -86,6 +87,10 @@ struct GemmParams {
     float alpha;
     const float* rownorm;
     const float* colnorm;
+    // K-blocks [kb_lo[tn], kb_hi[tn]) of column tile tn (krange = 1); outside them B's rows of the
+    // tile are zero (R's echelon structure), so skipping them changes no sum
+    int krange;
+    int kb_lo[kMaxTilesN], kb_hi[kMaxTilesN];
 };
 
 struct Ctl {
@@ -100,7 +105,7 @@ struct Ctl {
 
 __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see kThreads)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b0,
-              const __grid_constant__ CUtensorMap tmap_b1, const GemmParams p) {
+              const __grid_constant__ CUtensorMap tmap_b1, const __grid_constant__ GemmParams p) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
@@ -114,7 +119,16 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // this CTA's tiles: blockIdx.x, blockIdx.x + gridDim.x, ...
     const int ntiles = p.tiles > blockIdx.x ? (int)((p.tiles - 1 - blockIdx.x) / gridDim.x + 1) : 0;
-    const int total_it = ntiles * p.nkb;
+    auto krange = [&](int tn, int& lo, int& hi) {
+        lo = p.krange ? p.kb_lo[tn] : 0;
+        hi = p.krange ? p.kb_hi[tn] : p.nkb;
+    };
+    int total_it = 0;  // K-blocks over this CTA's tiles
+    for (int lt = 0; lt < ntiles; ++lt) {
+        int lo, hi;
+        krange((int)((blockIdx.x + (long long)lt * gridDim.x) % p.tiles_n), lo, hi);
+        total_it += hi - lo;
+    }
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < p.sx; ++s) {
@@ -159,17 +173,21 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
             const uint64_t pol = l2_policy_evict_last();  // each row block is read once per N tile
             int it = 0;
             RingPos as;
-            long long tm = 0;
-            int tn = 0;
-            for (int kb = 0, lt = 0; it < total_it; ++it, as.next(p.sa)) {
-                const int s = as.idx;
-                if (!mbar_wait_1t(&c.a_empty[s], as.phase ^ 1u, abort_flag, err)) break;
-                if (kb == 0) tile_mn(lt, tm, tn);
-                mbar_arrive_expect_tx(&c.a_full[s], kAPartBytes);
-                tma_load_2d(As + (size_t)s * kAPartBytes, &tmap_a, &c.a_full[s], kb * kBK, (int)(tm * kBM), pol);
-                if (++kb == p.nkb) {
-                    kb = 0;
-                    ++lt;
+            bool ok = true;
+            for (int lt = 0; lt < ntiles && ok; ++lt) {
+                long long tm;
+                int tn, lo, hi;
+                tile_mn(lt, tm, tn);
+                krange(tn, lo, hi);
+                for (int kb = lo; kb < hi; ++kb, ++it, as.next(p.sa)) {
+                    const int s = as.idx;
+                    if (!mbar_wait_1t(&c.a_empty[s], as.phase ^ 1u, abort_flag, err)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&c.a_full[s], kAPartBytes);
+                    tma_load_2d(As + (size_t)s * kAPartBytes, &tmap_a, &c.a_full[s], kb * kBK, (int)(tm * kBM),
+                                pol);
                 }
             }
             for (int j = std::max(0, it - p.sa); j < it; ++j) mbar_drain(&c.a_full[j % p.sa], (uint32_t)(j / p.sa) & 1u, err);
@@ -180,17 +198,21 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
             const uint64_t pol = l2_policy_evict_first();
             int it = 0;
             RingPos xs;
-            long long tm = 0;
-            int tn = 0;
-            for (int kb = 0, lt = 0; it < total_it; ++it, xs.next(p.sx)) {
-                const int s = xs.idx;
-                if (!mbar_wait_1t(&c.x_empty[s], xs.phase ^ 1u, abort_flag, err)) break;
-                if (kb == 0) tile_mn(lt, tm, tn);
-                mbar_arrive_expect_tx(&c.x_full[s], kXStageBytes);
-                tma_load_2d(Xs + (size_t)s * kXStageBytes, &tmap_a, &c.x_full[s], kb * kBK, (int)(tm * kBM), pol);
-                if (++kb == p.nkb) {
-                    kb = 0;
-                    ++lt;
+            bool ok = true;
+            for (int lt = 0; lt < ntiles && ok; ++lt) {
+                long long tm;
+                int tn, lo, hi;
+                tile_mn(lt, tm, tn);
+                krange(tn, lo, hi);
+                for (int kb = lo; kb < hi; ++kb, ++it, xs.next(p.sx)) {
+                    const int s = xs.idx;
+                    if (!mbar_wait_1t(&c.x_empty[s], xs.phase ^ 1u, abort_flag, err)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&c.x_full[s], kXStageBytes);
+                    tma_load_2d(Xs + (size_t)s * kXStageBytes, &tmap_a, &c.x_full[s], kb * kBK, (int)(tm * kBM),
+                                pol);
                 }
             }
             for (int j = std::max(0, it - p.sx); j < it; ++j) mbar_drain(&c.x_full[j % p.sx], (uint32_t)(j / p.sx) & 1u, err);
@@ -200,25 +222,25 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
         if (lane == 0) {
             const uint64_t pol = l2_policy_evict_last();
             const uint32_t bytes = (uint32_t)p.nt * kBK * 2;
-            const int total = total_it * p.nb;
             int ib = 0;
             RingPos bs;
-            long long tm = 0;
-            int tn = 0;
-            for (int which = 0, kb = 0, lt = 0; ib < total; ++ib, bs.next(p.sb)) {
-                const int s = bs.idx;
-                if (!mbar_wait_1t(&c.b_empty[s], bs.phase ^ 1u, abort_flag, err)) break;
-                if (kb == 0 && which == 0) tile_mn(lt, tm, tn);
-                mbar_arrive_expect_tx(&c.b_full[s], bytes);
-                tma_load_2d(Bs + (size_t)s * kBStageBytes, which ? &tmap_b1 : &tmap_b0, &c.b_full[s], kb * kBK,
-                            tn * p.nt, pol);
-                if (++which == p.nb) {
-                    which = 0;
-                    if (++kb == p.nkb) {
-                        kb = 0;
-                        ++lt;
+            bool ok = true;
+            for (int lt = 0; lt < ntiles && ok; ++lt) {
+                long long tm;
+                int tn, lo, hi;
+                tile_mn(lt, tm, tn);
+                krange(tn, lo, hi);
+                for (int kb = lo; kb < hi && ok; ++kb)
+                    for (int which = 0; which < p.nb; ++which, ++ib, bs.next(p.sb)) {
+                        const int s = bs.idx;
+                        if (!mbar_wait_1t(&c.b_empty[s], bs.phase ^ 1u, abort_flag, err)) {
+                            ok = false;
+                            break;
+                        }
+                        mbar_arrive_expect_tx(&c.b_full[s], bytes);
+                        tma_load_2d(Bs + (size_t)s * kBStageBytes, which ? &tmap_b1 : &tmap_b0, &c.b_full[s],
+                                    kb * kBK, tn * p.nt, pol);
                     }
-                }
             }
             for (int j = std::max(0, ib - p.sb); j < ib; ++j) mbar_drain(&c.b_full[j % p.sb], (uint32_t)(j / p.sb) & 1u, err);
         }
@@ -233,7 +255,11 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                 if (!mbar_wait_1t(&c.d_empty[buf], ((uint32_t)(lt >> 1) & 1u) ^ 1u, abort_flag, err)) break;
                 tc_fence_after();
                 const uint32_t d_tmem = tmem + (uint32_t)(buf * 256);
-                for (int kb = 0; kb < p.nkb; ++kb, ra.next(p.sa)) {
+                long long tm;
+                int tn, lo, hi;
+                tile_mn(lt, tm, tn);
+                krange(tn, lo, hi);
+                for (int kb = lo; kb < hi; ++kb, ra.next(p.sa)) {
                     const int sa = ra.idx;
                     if (!mbar_wait_1t(&c.a_full[sa], ra.phase, abort_flag, err)) {
                         ok = false;
@@ -257,14 +283,14 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
 #pragma unroll
                         for (int k = 0; k < kBK / 16; ++k)
                             mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
-                                       (kb | k) != 0 ? 1u : 0u);
+                                       (kb != lo || k != 0) ? 1u : 0u);
                     } else {
                         const uint64_t al = sdesc_sw128(smem_u32(At + kAPartBytes));
                         const uint64_t b1 = sdesc_sw128(smem_u32(Bs + (size_t)sb1 * kBStageBytes));
 #pragma unroll
                         for (int k = 0; k < kBK / 16; ++k) {
                             mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
-                                       (kb | k) != 0 ? 1u : 0u);
+                                       (kb != lo || k != 0) ? 1u : 0u);
                             mma_f16_ss(d_tmem, al + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc, 1u);
                             mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b1 + (uint64_t)(2 * k), idesc, 1u);
                         }
@@ -496,6 +522,21 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     p.alpha = a.alpha;
     p.rownorm = a.rownorm;
     p.colnorm = a.colnorm;
+    p.krange = 0;
+    if (a.b_klo && a.b_khi && p.tiles_n <= kMaxTilesN) {
+        // per column tile: the K-blocks holding the tile's nonzero B entries
+        p.krange = 1;
+        for (int tn = 0; tn < p.tiles_n; ++tn) {
+            int lo = a.K, hi = 0;
+            for (int j = tn * p.nt; j < std::min(a.n, (tn + 1) * p.nt); ++j) {
+                lo = std::min(lo, a.b_klo[j]);
+                hi = std::max(hi, a.b_khi[j]);
+            }
+            const int kl = std::min(std::max(lo, 0), a.K) / kBK;
+            p.kb_lo[tn] = std::min(kl, p.nkb - 1);
+            p.kb_hi[tn] = std::min(p.nkb, std::max(p.kb_lo[tn] + 1, (hi + kBK - 1) / kBK));
+        }
+    }
     CUtensorMap ta, tb0, tb1;
     const CUtensorMapDataType bt = a.split ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
     const bool ta_ok = a.a_half ? make_tmap_2d(&ta, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, a.A, a.m, a.K, a.lda, kBK,

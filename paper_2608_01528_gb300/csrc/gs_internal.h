@@ -62,6 +62,10 @@ struct gs_basis {
     // grouped bases (gs_build_basis_grouped): rows [grp_rows[g], grp_rows[g+1]) of the codebook
     // and coefficients [grp_coeffs[g], grp_coeffs[g+1]) belong to group g; empty otherwise
     std::vector<int> grp_rows, grp_coeffs;
+    // host copies for the tensor-core GEMMs' K trimming (tc_prepare): R row i is zero from
+    // column rlen_host[i] on (B = R: K range [kzero_host[i] = 0, rlen_host[i])), and R column j
+    // is zero above row pivot_host[j] (B = R^T: K range [pivot_host[j], kM_host[j] = M))
+    std::vector<int> rlen_host, pivot_host, kzero_host, kM_host;
     // scratch for the multi-kernel paths (rows processed in chunks)
     float* scratch = nullptr;
     long long scratch_floats = 0;
@@ -161,6 +165,9 @@ struct GemmTcArgs {
     const void* B0; const void* B1; long long ldb; int n;
     void* C; long long ldc; bool c_bf16; float alpha;
     const float* rownorm; const float* colnorm;
+    // optional HOST arrays (n each): B row j is zero outside K columns [b_klo[j], b_khi[j]);
+    // K-blocks outside a column tile's union are skipped (exact: only zero products dropped)
+    const int* b_klo; const int* b_khi;
 };
 cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s);
 // fp32 rows -> fp16 (RN), for the fp16-A GEMM; values beyond the fp16 range set GS_DEV_ERR_RANGE

@@ -637,6 +637,17 @@ gs_status tc_prepare(gs_basis* h) {
     h->tc_npad = npad;
     h->tc_mpad = mpad;
     h->has_split = true;
+    // R's echelon structure on the host, for the GEMMs' K trimming
+    h->rlen_host.assign((size_t)h->M, 0);
+    if (cudaMemcpy(h->rlen_host.data(), h->rlen, sizeof(int) * (size_t)h->M, cudaMemcpyDeviceToHost) != cudaSuccess)
+        return GS_ERR_CUDA;
+    h->kzero_host.assign((size_t)h->M, 0);
+    h->kM_host.assign((size_t)h->r, h->M);
+    h->pivot_host.assign((size_t)h->r, h->M);
+    for (int j = 0, i = 0; j < h->r; ++j) {  // first row reaching column j (nondecreasing in j)
+        while (i < h->M && h->rlen_host[(size_t)i] <= j) ++i;
+        h->pivot_host[(size_t)j] = i;
+    }
     // the fused kernel keeps Y (r <= 256 columns) and S (M <= 256 columns) in TMEM
     if (h->r > 256 || h->M > 256) return GS_OK;
     // GEMM2 halves: up to 128 codewords each; K-blocks per half from the last nonzero of R
