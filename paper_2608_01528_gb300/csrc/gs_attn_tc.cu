@@ -348,23 +348,23 @@ __global__ void __launch_bounds__(kThreads, 1)
 // ================================================================= one pass, key units spread over a cluster
 // With the row softmax and Lk <= 4 x 256, the G = ceil(Lk / 256) CTAs of a thread-block
 // cluster share each work item: CTA g computes the logits of keys [256 g, 256 g + 256)
-// for the item's 128 queries, once.  Each epilogue thread holds 64 logits of one query
-// row in registers (one TMEM read, after which the accumulator goes back to the MMA),
-// takes, in base-2 units, their max m, p_j = 2^(c s_j - m) (c = scale log2 e) and sum
-// l.  The four column quarters of each row are merged in shared memory, each CTA posts
-// its row results to every CTA of the cluster with asynchronous remote stores, and with
-// all G results a thread has the row's max M and sum L and writes p_j 2^(m - M) / L: one
-// exponential per output.  The probabilities go out through a swizzled shared-memory
-// tile and TMA tensor stores (a 3-D map over B x Lq x Lk, so rows past Lq and keys past
-// Lk are clipped).  Compared with the two-pass kernel above this halves the MMA work and
-// the exponentials; the TMEM accumulator is double-buffered over items, so an item's
-// exchange and writes overlap the next item's MMAs.  With G = 2 or 4 each CTA loads
-// 128 / G rows of the query tile and multicasts them to the whole cluster.
+// for the item's 128 queries, once.  The epilogue warps form two teams that take the
+// items in turn (team t: items t, t + 2, ...; TMEM accumulator t), so one team's exchange
+// and writes overlap the other team's statistics.  A team thread owns one query row and
+// 128 of the unit's keys, read from TMEM in two 64-key passes: the statistics pass takes,
+// in base-2 units, the max m of c s_j (c = scale log2 e) and l = sum 2^(c s_j - m); the two
+// key halves of each row meet in shared memory, the team posts each row's CTA result to
+// every CTA of the cluster with asynchronous remote stores, and with all G results the
+// row's max M and sum L are known; the writing pass reads the logits again and writes
+// 2^(c s_j - M) / L.  The logits never leave the chip.  Outputs go through a 64-byte-
+// swizzled 32 x 16 fp32 tile per warp and TMA tensor stores over a 3-D map (B x Lq x Lk),
+// which clips rows past Lq and keys past Lk.  With G = 2 or 4 each CTA loads 128 / G rows
+// of the query tile and multicasts them to the whole cluster.
 //
-// Warp roles (576 threads): 0-15 epilogue (warp w: TMEM lanes 32 (w % 4) = query rows,
-// keys [64 (w / 4), +64) of the CTA's unit; warps 0-3 also merge and post the CTA's
-// row results), 16 TMA producer (query and key K-blocks into one stage), 17 TMEM
-// allocator + MMA issuer.
+// Warp roles (576 threads): 0-7 team 0 and 8-15 team 1 (warp w: TMEM lanes 32 (w % 4) =
+// query rows, keys [128 ((w / 4) % 2), +128) of the CTA's unit; warps with (w / 4) even also
+// merge and post their rows), 16 TMA producer (query and key K-blocks into one stage), 17
+// TMEM allocator + MMA issuer.
 
 constexpr int kClMaxG = 4;
 constexpr int kClStageBytes = kQBlockBytes + kKStageBytes;  // 48 KB: query block, then key block
@@ -373,16 +373,17 @@ constexpr int kClEpiWarps = 16;
 constexpr int kClCols = kBN / 4;            // keys per epilogue thread
 constexpr int kClProdWarp = 16, kClMmaWarp = 17;
 constexpr int kClThreads = 18 * 32;
-constexpr int kClStgBytes = 32 * 32 * 4;    // one output box: 32 query rows x 32 keys fp32 (128-byte rows)
+constexpr int kClStgCols = 16;             // one output box: 32 query rows x 16 keys fp32 (64-byte rows)
+constexpr int kClStgBytes = 32 * kClStgCols * 4;
 
 struct ClCtl {
     uint64_t full[kClStages], empty[kClStages];
-    uint64_t d_full[2], d_empty[2];
-    uint64_t p_full[2];           // the 16 warps' partial row results of an item (by item parity)
-    uint64_t x_full[2];           // every CTA's row results of an item (by item parity)
+    uint64_t d_full[2], d_empty[2];  // TMEM accumulator t, used by team t
+    uint64_t p_full[2];              // team t's two key halves of an item's rows are in part[t]
+    uint64_t x_full[2][2];           // team t, slot s: every CTA's row results of an item
     uint64_t mma_done;
-    float2 part[2][4][kBM];       // [item parity][column quarter][query row] = (max, sum)
-    float2 xch[2][kClMaxG][kBM];  // [item parity][rank][query row] = (max, sum)
+    float2 part[2][2][kBM];             // [team][key half][query row] = (max, sum)
+    float2 xch[2][2][kClMaxG][kBM];     // [team][slot][rank][query row] = (max, sum)
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -430,7 +431,7 @@ __global__ void __launch_bounds__(kClThreads, 1)
     const uint32_t raw = smem_u32(smem_raw);
     uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
     uint8_t* St = base;                                          // kClStages x 48 KB
-    uint8_t* Stg = St + (size_t)kClStages * kClStageBytes;       // 16 warps x 4 KB output box
+    uint8_t* Stg = St + (size_t)kClStages * kClStageBytes;       // 16 warps x 2 KB output box
     ClCtl& c = *reinterpret_cast<ClCtl*>(Stg + (size_t)kClEpiWarps * kClStgBytes);
     volatile int* abort_flag = &c.abort_flag;
     unsigned* err = &g_err_attn;
@@ -453,9 +454,10 @@ __global__ void __launch_bounds__(kClThreads, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&c.d_full[b], 1);
-            mbar_init(&c.d_empty[b], kClEpiWarps);
-            mbar_init(&c.p_full[b], kClEpiWarps);
-            mbar_init(&c.x_full[b], 1);
+            mbar_init(&c.d_empty[b], kClEpiWarps / 2);
+            mbar_init(&c.p_full[b], kClEpiWarps / 2);
+            mbar_init(&c.x_full[b][0], 1);
+            mbar_init(&c.x_full[b][1], 1);
         }
         mbar_init(&c.mma_done, 1);
         c.abort_flag = 0;
@@ -541,104 +543,127 @@ __global__ void __launch_bounds__(kClThreads, 1)
             mbar_drain(&c.mma_done, 0, err);
         }
     } else {
-        // ------------------------------------------------------------- epilogue
-        const int quad = warp & 3, cq = warp >> 2;
-        const int i = quad * 32 + lane;                       // query row within the item
-        const int key0 = (int)rank * kBN + cq * kClCols;      // first of this warp's 64 keys
-        const int nvalid = min(kClCols, max(0, p.Lk - key0));
+        // ------------------------------------------------------------- epilogue (two teams)
+        const int team = warp >> 3, quad = warp & 3, kh = (warp >> 2) & 1;
+        const int i = quad * 32 + lane;                          // query row within the item
+        const int keyh = (int)rank * kBN + kh * (kBN / 2);       // first of this warp's 128 keys
         const float c2 = p.scale * 1.4426950408889634f;
         uint8_t* sb = Stg + (size_t)warp * kClStgBytes;
         const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
-        const uint32_t xbar = smem_u32(&c.x_full[0]);
-        for (int li = 0; li < nitems; ++li) {
+        const uint32_t tcol = (uint32_t)(team * kBN + kh * (kBN / 2));
+        for (int li = team; li < nitems; li += 2) {
             int b, qt;
             item_bq(li, b, qt);
-            const int buf = li & 1, par = li & 1;
-            const uint32_t ph = (uint32_t)(li >> 1) & 1u;
-            if (!mbar_wait_warp(&c.d_full[buf], ph, abort_flag, err)) break;
+            const int k = li >> 1;                   // this team's k-th item
+            const uint32_t ph = (uint32_t)k & 1u;    // phase of d_full[team] / p_full[team]
+            const int xs = k & 1;                    // exchange slot (two per team)
+            const uint32_t xph = (uint32_t)(k >> 1) & 1u;
+            if (!mbar_wait_warp(&c.d_full[team], ph, abort_flag, err)) break;
             tc_fence_after();
-            float v[kClCols];
-            {
-                uint32_t r[kClCols];
-                const uint32_t ta = tmem + lane_base + (uint32_t)(buf * kBN + cq * kClCols);
-                tmem_ld32_issue(ta, r);
-                tmem_ld32_issue(ta + 32u, r + 32);
-                tmem_wait_ld32(r);
-                tmem_wait_ld32(r + 32);
+            // statistics pass over the two 64-key chunks: max m and sum l in base 2
+            float m = -INFINITY, l = 0.f;
+            for (int cc = 0; cc < 2; ++cc) {
+                const int nvalid = min(kClCols, max(0, p.Lk - (keyh + cc * kClCols)));
+                float v[kClCols];
+                {
+                    uint32_t r[kClCols];
+                    const uint32_t ta = tmem + lane_base + tcol + (uint32_t)(cc * kClCols);
+                    tmem_ld32_issue(ta, r);
+                    tmem_ld32_issue(ta + 32u, r + 32);
+                    tmem_wait_ld32(r);
+                    tmem_wait_ld32(r + 32);
 #pragma unroll
-                for (int j = 0; j < kClCols; ++j) v[j] = __uint_as_float(r[j]);
+                    for (int j = 0; j < kClCols; ++j) v[j] = __uint_as_float(r[j]);
+                }
+                if (nvalid == 0) continue;
+                float ext;
+                if (nvalid == kClCols)
+                    ext = c2 >= 0.f ? row_extreme<false, false>(v, kClCols) : row_extreme<true, false>(v, kClCols);
+                else
+                    ext = c2 >= 0.f ? row_extreme<false, true>(v, nvalid) : row_extreme<true, true>(v, nvalid);
+                const float mc = c2 * ext;
+                float l8[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) l8[q] = 0.f;
+#pragma unroll
+                for (int j = 0; j < kClCols; ++j)
+                    if (nvalid == kClCols || j < nvalid) l8[j & 7] += ex2_approx(fmaf(v[j], c2, -mc));
+                const float lc = ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
+                const float mn = fmaxf(m, mc);
+                l = (l > 0.f ? l * ex2_approx(m - mn) : 0.f) + lc * ex2_approx(mc - mn);
+                m = mn;
             }
-            // the logits are in registers: the accumulator goes back to the MMA
-            tc_fence_before();
+            // the row's two key halves meet in shared memory; the even-half warps merge them
+            // and post the CTA's result to every CTA of the cluster
+            c.part[team][kh][i] = make_float2(m, l);
             __syncwarp();
-            if (lane == 0) mbar_arrive(&c.d_empty[buf]);
-            // this thread's part of its row in base-2 units: max m of c s_j (c times the max,
-            // or for c < 0 the min, of the raw s_j), p_j = 2^(c s_j - m) by one fma and one
-            // ex2, and their sum l; keys past Lk (only in a row's last unit) are left out
-            float ext;
-            if (nvalid == kClCols)
-                ext = c2 >= 0.f ? row_extreme<false, false>(v, kClCols) : row_extreme<true, false>(v, kClCols);
-            else
-                ext = c2 >= 0.f ? row_extreme<false, true>(v, nvalid) : row_extreme<true, true>(v, nvalid);
-            const float m = nvalid > 0 ? c2 * ext : -INFINITY;
-            const float mref = nvalid > 0 ? m : 0.f;
-            float l8[8];
-#pragma unroll
-            for (int k = 0; k < 8; ++k) l8[k] = 0.f;
-#pragma unroll
-            for (int j = 0; j < kClCols; ++j) {
-                v[j] = (nvalid == kClCols || j < nvalid) ? ex2_approx(fmaf(v[j], c2, -mref)) : 0.f;
-                l8[j & 7] += v[j];
-            }
-            const float l = ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
-            // the four column quarters of each row meet in shared memory; warps 0-3 merge
-            // them and post the CTA's row result to every CTA of the cluster
-            c.part[par][cq][i] = make_float2(m, l);
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&c.p_full[par]);
-            if (cq == 0) {
-                if (!mbar_wait_warp(&c.p_full[par], ph, abort_flag, err)) break;
+            if (lane == 0) mbar_arrive(&c.p_full[team]);
+            if (kh == 0) {
+                if (!mbar_wait_warp(&c.p_full[team], ph, abort_flag, err)) break;
                 float2 e[kClMaxG];
-#pragma unroll
-                for (int k = 0; k < 4; ++k) e[k] = c.part[par][k][i];
-                const float2 rc = merge_stats(e, 4);
-                const uint32_t slot = smem_u32(&c.xch[par][rank][i]);
-                const uint32_t bar = xbar + (uint32_t)(par * sizeof(uint64_t));
+                e[0] = c.part[team][0][i];
+                e[1] = c.part[team][1][i];
+                const float2 rc = merge_stats(e, 2);
+                const uint32_t slot = smem_u32(&c.xch[team][xs][rank][i]);
+                const uint32_t bar = smem_u32(&c.x_full[team][xs]);
                 // the barrier's one arrival per phase carries the byte count of every CTA's
                 // posts; the posts are asynchronous stores that complete those bytes (a
                 // release-arrive after plain remote stores cost microseconds per item)
-                if (threadIdx.x == 0) mbar_arrive_expect_tx(&c.x_full[par], (uint32_t)(G * kBM * 8));
+                if (quad == 0 && lane == 0) mbar_arrive_expect_tx(&c.x_full[team][xs], (uint32_t)(G * kBM * 8));
                 for (int g = 0; g < G; ++g)
                     st_async_f32x2(mapa_shared(slot, (uint32_t)g), rc.x, rc.y, mapa_shared(bar, (uint32_t)g));
             }
-            const bool got = mbar_wait_cluster(&c.x_full[par], ph, abort_flag, err);
+            const bool got = mbar_wait_cluster(&c.x_full[team][xs], xph, abort_flag, err);
             if (!__all_sync(0xffffffffu, got)) break;
-            float f;  // p_j f = exp(scale s_j - row max) / row sum
+            float M, invL;
             {
                 float2 e[kClMaxG];
 #pragma unroll
-                for (int k = 0; k < kClMaxG; ++k) e[k] = k < G ? c.xch[par][k][i] : make_float2(-INFINITY, 0.f);
+                for (int q = 0; q < kClMaxG; ++q) e[q] = q < G ? c.xch[team][xs][q][i] : make_float2(-INFINITY, 0.f);
                 const float2 rw = merge_stats(e, G);
-                f = l > 0.f ? __fdividef(ex2_approx(mref - rw.x), rw.y) : 0.f;
+                M = rw.x;
+                invL = rw.y > 0.f ? __fdividef(1.f, rw.y) : 0.f;
             }
-            // two boxes of 32 keys: swizzled shared-memory tile (16-byte chunk k of row
-            // `lane` at chunk k ^ (lane % 8), the TMA's 128-byte swizzle), then a tensor store
+            // writing pass: 2^(c s_j - M) / L through 32 x 16 tiles (16-byte chunk q of row
+            // `lane` at chunk q ^ ((lane / 2) % 4), the TMA's 64-byte swizzle) and tensor stores
             const int y = qt * kBM + quad * 32;
+            for (int cc = 0; cc < 2; ++cc) {
+                float v[kClCols];
+                {
+                    uint32_t r[kClCols];
+                    const uint32_t ta = tmem + lane_base + tcol + (uint32_t)(cc * kClCols);
+                    tmem_ld32_issue(ta, r);
+                    tmem_ld32_issue(ta + 32u, r + 32);
+                    tmem_wait_ld32(r);
+                    tmem_wait_ld32(r + 32);
 #pragma unroll
-            for (int q = 0; q < kClCols / 32; ++q) {
-                if (lane == 0) bulk_wait_read_0();  // the previous store has read the tile
-                __syncwarp();
-#pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    const float4 o = make_float4(v[32 * q + 4 * k] * f, v[32 * q + 4 * k + 1] * f,
-                                                 v[32 * q + 4 * k + 2] * f, v[32 * q + 4 * k + 3] * f);
-                    *reinterpret_cast<float4*>(sb + lane * 128 + ((k ^ (lane & 7)) << 4)) = o;
+                    for (int j = 0; j < kClCols; ++j) v[j] = __uint_as_float(r[j]);
                 }
-                fence_proxy_async();
-                __syncwarp();
-                if (lane == 0) {
-                    if (key0 + 32 * q < p.Lk && y < p.Lq) tma_store_3d(&tmap_a, sb, key0 + 32 * q, y, b);
-                    bulk_commit();
+                if (cc == 1) {  // the accumulator has been read twice: back to the MMA
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&c.d_empty[team]);
+                }
+#pragma unroll
+                for (int q = 0; q < kClCols / kClStgCols; ++q) {
+                    const int x = keyh + cc * kClCols + q * kClStgCols;
+                    if (lane == 0) bulk_wait_read_0();  // the previous store has read the tile
+                    __syncwarp();
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const float* vv = v + q * kClStgCols + 4 * u;
+                        const float4 o = make_float4(ex2_approx(fmaf(vv[0], c2, -M)) * invL,
+                                                     ex2_approx(fmaf(vv[1], c2, -M)) * invL,
+                                                     ex2_approx(fmaf(vv[2], c2, -M)) * invL,
+                                                     ex2_approx(fmaf(vv[3], c2, -M)) * invL);
+                        *reinterpret_cast<float4*>(sb + lane * 64 + ((u ^ ((lane >> 1) & 3)) << 4)) = o;
+                    }
+                    fence_proxy_async();
+                    __syncwarp();
+                    if (lane == 0) {
+                        if (x < p.Lk && y < p.Lq) tma_store_3d(&tmap_a, sb, x, y, b);
+                        bulk_commit();
+                    }
                 }
             }
         }
@@ -702,8 +727,8 @@ cudaError_t launch_attn_tc(const void* Yq, const void* Yk, int B, int Lq, int Lk
     const long long items = (long long)B * p.qtiles;
     CUtensorMap ta;
     if (softmax && p.ntiles <= kClMaxG && Lk % 4 == 0 && (uintptr_t)A % 16 == 0 &&
-        make_tmap_3d(&ta, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, A, Lk, Lq, B, Lk, (long long)Lq * Lk, 32, 32,
-                     CU_TENSOR_MAP_SWIZZLE_128B)) {
+        make_tmap_3d(&ta, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, A, Lk, Lq, B, Lk, (long long)Lq * Lk, kClStgCols, 32,
+                     CU_TENSOR_MAP_SWIZZLE_64B)) {
         // one pass: the key units of a row spread over a cluster of ntiles CTAs
         const int G = p.ntiles;
         // G = 2 or 4: each CTA loads 128 / G rows of the query tile for the whole cluster
