@@ -53,7 +53,6 @@ struct AttnParams {
     int B, Lq, Lk, r, nkb;
     int qtiles, ntiles;      // query tiles per sequence, key tiles per sequence
     int passes;              // 2 with the row softmax, 1 for plain scaled logits
-    int qslice;              // cluster kernel: rows of the query tile each CTA loads for all (0: whole tile, own CTA only)
     float scale;
     float* A;                // B x Lq x Lk
     int a_vec;               // rows aligned for two-element stores (Lk even, A 8-byte aligned)
@@ -358,8 +357,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 // row's max M and sum L are known; the writing pass reads the logits again and writes
 // 2^(c s_j - M) / L.  The logits never leave the chip.  Outputs go through a 64-byte-
 // swizzled 32 x 16 fp32 tile per warp and TMA tensor stores over a 3-D map (B x Lq x Lk),
-// which clips rows past Lq and keys past Lk.  With G = 2 or 4 each CTA loads 128 / G rows
-// of the query tile and multicasts them to the whole cluster.
+// which clips rows past Lq and keys past Lk.  (Multicasting the query tile across the cluster
+// halved its L2 reads but tied every CTA's stage release to the slowest CTA: 2 % slower.)
 //
 // Warp roles (576 threads): 0-7 team 0 and 8-15 team 1 (warp w: TMEM lanes 32 (w % 4) =
 // query rows, keys [128 ((w / 4) % 2), +128) of the CTA's unit; warps with (w / 4) even also
@@ -425,8 +424,6 @@ __device__ __forceinline__ float2 merge_stats(const float2* e, int n) {
 __global__ void __launch_bounds__(kClThreads, 1)
     k_attn_cl(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
               const __grid_constant__ CUtensorMap tmap_a, const AttnParams p) {
-    // tmap_q boxes are p.qslice rows when the query tile is multicast (each CTA loads its
-    // slice for the whole cluster), else the whole 128-row tile
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
@@ -443,14 +440,11 @@ __global__ void __launch_bounds__(kClThreads, 1)
     const long long items = (long long)p.B * p.qtiles;
     const int nitems = items > cid ? (int)((items - 1 - cid) / ncl + 1) : 0;
     const int nkb = p.nkb;
-    const bool qmc = p.qslice > 0;
-    const uint16_t cmask = (uint16_t)((1u << G) - 1u);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kClStages; ++s) {
             mbar_init(&c.full[s], 1);
-            // with the multicast query tile a stage is free once every CTA's MMAs are done with it
-            mbar_init(&c.empty[s], qmc ? (uint32_t)G : 1u);
+            mbar_init(&c.empty[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&c.d_full[b], 1);
@@ -496,11 +490,7 @@ __global__ void __launch_bounds__(kClThreads, 1)
                     }
                     uint8_t* dst = St + (size_t)st.idx * kClStageBytes;
                     mbar_arrive_expect_tx(&c.full[st.idx], kClStageBytes);
-                    if (qmc)
-                        tma_load_2d_mc(dst + (size_t)rank * p.qslice * (kBK * 2), &tmap_q, &c.full[st.idx], kb * kBK,
-                                       b * p.Lq + qt * kBM + (int)rank * p.qslice, cmask, pol);
-                    else
-                        tma_load_2d(dst, &tmap_q, &c.full[st.idx], kb * kBK, b * p.Lq + qt * kBM, pol);
+                    tma_load_2d(dst, &tmap_q, &c.full[st.idx], kb * kBK, b * p.Lq + qt * kBM, pol);
                     tma_load_2d(dst + kQBlockBytes, &tmap_k, &c.full[st.idx], kb * kBK,
                                 b * p.Lk + (int)rank * kBN, pol);
                 }
@@ -532,10 +522,7 @@ __global__ void __launch_bounds__(kClThreads, 1)
                     for (int k = 0; k < kBK / 16; ++k)
                         mma_f16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
                                    (kb | k) != 0 ? 1u : 0u);
-                    if (qmc)
-                        mma_commit_mc(&c.empty[st.idx], cmask);
-                    else
-                        mma_commit(&c.empty[st.idx]);
+                    mma_commit(&c.empty[st.idx]);
                 }
                 if (ok) mma_commit(&c.d_full[buf]);
             }
@@ -714,7 +701,6 @@ cudaError_t launch_attn_tc(const void* Yq, const void* Yk, int B, int Lq, int Lk
     p.qtiles = (Lq + kBM - 1) / kBM;
     p.ntiles = (Lk + kBN - 1) / kBN;
     p.passes = softmax ? 2 : 1;
-    p.qslice = 0;
     p.scale = scale;
     p.A = A;
     p.a_vec = ((uintptr_t)A % 8 == 0) && (Lk % 2 == 0);
@@ -731,13 +717,6 @@ cudaError_t launch_attn_tc(const void* Yq, const void* Yk, int B, int Lq, int Lk
                      CU_TENSOR_MAP_SWIZZLE_64B)) {
         // one pass: the key units of a row spread over a cluster of ntiles CTAs
         const int G = p.ntiles;
-        // G = 2 or 4: each CTA loads 128 / G rows of the query tile for the whole cluster
-        CUtensorMap tqc = tq;
-        p.qslice = 0;
-        if ((G == 2 || G == 4) &&
-            make_tmap_2d(&tqc, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, Yq, (long long)B * Lq, r, ldy, kBK, kBM / G,
-                         CU_TENSOR_MAP_SWIZZLE_128B))
-            p.qslice = kBM / G;
         cudaLaunchConfig_t cfg = {};
         cudaLaunchAttribute attr[1];
         attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -767,7 +746,7 @@ cudaError_t launch_attn_tc(const void* Yq, const void* Yk, int B, int Lq, int Lk
         }
         const long long ncl = std::min<long long>(ncl_max, items);
         cfg.gridDim = dim3((unsigned)(ncl * G));
-        cudaError_t e = cudaLaunchKernelEx(&cfg, k_attn_cl, tqc, tk, ta, p);
+        cudaError_t e = cudaLaunchKernelEx(&cfg, k_attn_cl, tq, tk, ta, p);
         if (e != cudaSuccess) return e;
         return cudaGetLastError();
     }

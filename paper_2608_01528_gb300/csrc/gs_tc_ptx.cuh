@@ -231,17 +231,6 @@ static __device__ __forceinline__ void bulk_wait_read_0() {
 static __device__ __forceinline__ void bulk_wait_all() {
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
-// The same load multicast to every CTA of the cluster in `mask`: the box lands at the
-// same shared-memory offset in each and completes bytes on the mbarrier at the same
-// offset in each.
-static __device__ __forceinline__ void tma_load_2d_mc(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
-                                               uint16_t mask, uint64_t policy) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
-        ".L2::cache_hint [%0], [%1, {%3, %4}], [%2], %5, %6;" ::"r"(smem_u32(dst)),
-        "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(mask), "l"(policy)
-        : "memory");
-}
 static __device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst)),
                  "r"(ncols)
@@ -278,15 +267,6 @@ static __device__ __forceinline__ void mma_commit(uint64_t* bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                      smem_u32(bar))
                  : "memory");
-}
-// Arrives once on the mbarrier at `bar`'s offset in every CTA of the cluster in `mask`
-// when every previously issued MMA of this thread has completed.
-static __device__ __forceinline__ void mma_commit_mc(uint64_t* bar, uint16_t mask) {
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
-            smem_u32(bar)),
-        "h"(mask)
-        : "memory");
 }
 // 16 consecutive fp32 columns of this thread's TMEM lane.
 static __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {

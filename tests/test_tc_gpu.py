@@ -239,8 +239,8 @@ def test_tc_attention(gs, orc, attn_R, B, Lq, Lk, r):
     """bf16 compressed vectors, fp32 accumulation, row softmax over all keys; against
     the oracle run on the same bf16 inputs.  Lk <= 1024 (a multiple of 4) runs one pass
     with the key units of a row spread over a cluster of ceil(Lk / 256) CTAs (520: the
-    last unit has an empty key half; with 2 or 4 CTAs each loads a slice of the query
-    tile for the whole cluster); longer rows and Lk = 301 run the two-pass kernel.
+    last unit has an empty key half; 512: a cluster of two); longer rows and Lk = 301 run
+    the two-pass kernel.
     r < 512 (the first r coordinates) leaves the last K-block partly beyond r."""
     tq, tk = _attn_inputs(orc, attn_R, B, Lq, Lk)
     if r < tq.shape[2]:
