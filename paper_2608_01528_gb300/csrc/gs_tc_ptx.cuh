@@ -125,9 +125,6 @@ static __device__ __forceinline__ uint32_t mapa_shared(uint32_t saddr, uint32_t 
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
     return r;
 }
-static __device__ __forceinline__ void st_cluster_f32x2(uint32_t caddr, float a, float b) {
-    asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(caddr), "f"(a), "f"(b) : "memory");
-}
 // Asynchronous store of two floats into the shared memory of a CTA of the cluster
 // that completes 8 bytes of transactions on that CTA's mbarrier `cbar` (both
 // addresses shared::cluster, in the same CTA): the waiter sees the data once the
@@ -136,11 +133,6 @@ static __device__ __forceinline__ void st_async_f32x2(uint32_t caddr, float a, f
     asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];" ::"r"(caddr),
                  "f"(a), "f"(b), "r"(cbar)
                  : "memory");
-}
-// Arrive on an mbarrier of any CTA of the cluster; orders this thread's earlier
-// memory operations (e.g. its stores into that CTA's shared memory) before it.
-static __device__ __forceinline__ void mbar_arrive_cluster(uint32_t caddr) {
-    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(caddr) : "memory");
 }
 // Non-blocking test (test_wait, not try_wait): a thread suspended in try_wait on a
 // barrier that only other SMs arrive on was observed to wake late, by microseconds.
@@ -218,10 +210,6 @@ static __device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, cons
 }
 static __device__ __forceinline__ void bulk_commit() {
     asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-}
-// Until at most one of this thread's bulk groups is still reading shared memory.
-static __device__ __forceinline__ void bulk_wait_read_1() {
-    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
 }
 // Until none of this thread's bulk groups is still reading shared memory.
 static __device__ __forceinline__ void bulk_wait_read_0() {
@@ -317,9 +305,9 @@ static __device__ __forceinline__ void tmem_ld16x256b_x4(uint32_t taddr, float* 
 #pragma unroll
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
-// 128 consecutive fp32 columns of this thread's TMEM lane: four loads in flight, then
-// one wait.  Each wait names its registers as operands, so no use of them can be
-// scheduled before it.
+// 32 consecutive fp32 columns of this thread's TMEM lane, issued without waiting, so that
+// several loads are in flight; tmem_wait_ld32 then waits and names the registers as its
+// operands, so no use of them can be scheduled before the wait.
 static __device__ __forceinline__ void tmem_ld32_issue(uint32_t taddr, uint32_t* r) {
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
@@ -342,16 +330,6 @@ static __device__ __forceinline__ void tmem_wait_ld32(uint32_t* r) {
                  :
                  : "memory");
 }
-static __device__ __forceinline__ void tmem_ld128(uint32_t taddr, float* v) {
-    uint32_t r[128];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) tmem_ld32_issue(taddr + (uint32_t)(32 * q), r + 32 * q);
-#pragma unroll
-    for (int q = 0; q < 4; ++q) tmem_wait_ld32(r + 32 * q);
-#pragma unroll
-    for (int i = 0; i < 128; ++i) v[i] = __uint_as_float(r[i]);
-}
-
 // Stores 16 consecutive 32-bit columns of this thread's TMEM lane.
 static __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* v) {
     asm volatile(
@@ -360,12 +338,6 @@ static __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t*
         "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
         "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
         : "memory");
-}
-// Stores 8 consecutive 32-bit columns of this thread's TMEM lane.
-static __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t* v) {
-    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(v[0]),
-                 "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
-                 : "memory");
 }
 static __device__ __forceinline__ void tmem_wait_st() {
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
