@@ -24,8 +24,10 @@
 // vectorization V = P R (split, B0 / B1 = bf16 hi / lo of R^T).
 //
 // Tiles are 128 x nt (nt <= 256) with the fp32 accumulator double-buffered in
-// TMEM (2 x 256 columns); one persistent CTA per SM walks the tiles with the n
-// index fastest, so CTAs running at the same time share A rows in L2.
+// TMEM (2 x 256 columns), or, for a long K with A rounded to fp16 and n > 256, 128 x 512
+// (two 256-column accumulators filling TMEM, single-buffered: each converted A K-block
+// feeds both); one persistent CTA per SM walks the tiles with the n index fastest, so
+// CTAs running at the same time share A rows in L2.
 // Warp roles (608 threads): 0-3 and 15-18 epilogue (warp w reads TMEM lanes
 // 32 (w % 4)..+31; the two warps of a lane quadrant take alternate 32-column chunks,
 // so output-heavy products like reconstruct are not held up by the stores),
@@ -80,6 +82,7 @@ struct GemmParams {
     int n, K, nkb, nt, tiles_n;
     long long tiles;
     int amode, nb, parts;   // nb: B matrices per K-block; parts: A operand tiles per K-block
+    int halves;             // 256-column halves per tile: 2 = a 512-column tile, one accumulator
     int sx, sa, sb;
     void* C;
     long long ldc;
@@ -231,16 +234,17 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                 tile_mn(lt, tm, tn);
                 krange(tn, lo, hi);
                 for (int kb = lo; kb < hi && ok; ++kb)
-                    for (int which = 0; which < p.nb; ++which, ++ib, bs.next(p.sb)) {
-                        const int s = bs.idx;
-                        if (!mbar_wait_1t(&c.b_empty[s], bs.phase ^ 1u, abort_flag, err)) {
-                            ok = false;
-                            break;
+                    for (int hf = 0; hf < p.halves && ok; ++hf)
+                        for (int which = 0; which < p.nb; ++which, ++ib, bs.next(p.sb)) {
+                            const int s = bs.idx;
+                            if (!mbar_wait_1t(&c.b_empty[s], bs.phase ^ 1u, abort_flag, err)) {
+                                ok = false;
+                                break;
+                            }
+                            mbar_arrive_expect_tx(&c.b_full[s], bytes);
+                            tma_load_2d(Bs + (size_t)s * kBStageBytes, which ? &tmap_b1 : &tmap_b0, &c.b_full[s],
+                                        kb * kBK, (tn * p.halves + hf) * p.nt, pol);
                         }
-                        mbar_arrive_expect_tx(&c.b_full[s], bytes);
-                        tma_load_2d(Bs + (size_t)s * kBStageBytes, which ? &tmap_b1 : &tmap_b0, &c.b_full[s],
-                                    kb * kBK, tn * p.nt, pol);
-                    }
             }
             for (int j = std::max(0, ib - p.sb); j < ib; ++j) mbar_drain(&c.b_full[j % p.sb], (uint32_t)(j / p.sb) & 1u, err);
         }
@@ -250,9 +254,10 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
             const uint32_t idesc = p.amode == kABF16X2 ? idesc_bf16_f32(p.nt) : idesc_f16_f32(p.nt);
             RingPos ra, rb;
             bool ok = true;
+            const int nbuf = p.halves == 2 ? 1 : 2;  // a 512-column tile fills TMEM
             for (int lt = 0; lt < ntiles && ok; ++lt) {
-                const int buf = lt & 1;
-                if (!mbar_wait_1t(&c.d_empty[buf], ((uint32_t)(lt >> 1) & 1u) ^ 1u, abort_flag, err)) break;
+                const int buf = lt % nbuf;
+                if (!mbar_wait_1t(&c.d_empty[buf], ((uint32_t)(lt / nbuf) & 1u) ^ 1u, abort_flag, err)) break;
                 tc_fence_after();
                 const uint32_t d_tmem = tmem + (uint32_t)(buf * 256);
                 long long tm;
@@ -265,39 +270,61 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                         ok = false;
                         break;
                     }
-                    const int sb0 = rb.idx;
-                    if (!mbar_wait_1t(&c.b_full[sb0], rb.phase, abort_flag, err)) ok = false;
-                    rb.next(p.sb);
-                    int sb1 = sb0;
-                    if (p.nb == 2) {
-                        sb1 = rb.idx;
-                        if (ok && !mbar_wait_1t(&c.b_full[sb1], rb.phase, abort_flag, err)) ok = false;
-                        rb.next(p.sb);
-                    }
-                    if (!ok) break;
-                    tc_fence_after();
                     const uint8_t* At = As + (size_t)sa * p.parts * kAPartBytes;
                     const uint64_t ah = sdesc_sw128(smem_u32(At));
-                    const uint64_t b0 = sdesc_sw128(smem_u32(Bs + (size_t)sb0 * kBStageBytes));
-                    if (p.amode != kABF16X2) {
+                    if (p.halves == 1) {
+                        const int sb0 = rb.idx;
+                        if (!mbar_wait_1t(&c.b_full[sb0], rb.phase, abort_flag, err)) ok = false;
+                        rb.next(p.sb);
+                        int sb1 = sb0;
+                        if (p.nb == 2) {
+                            sb1 = rb.idx;
+                            if (ok && !mbar_wait_1t(&c.b_full[sb1], rb.phase, abort_flag, err)) ok = false;
+                            rb.next(p.sb);
+                        }
+                        if (!ok) break;
+                        tc_fence_after();
+                        const uint64_t b0 = sdesc_sw128(smem_u32(Bs + (size_t)sb0 * kBStageBytes));
+                        if (p.amode != kABF16X2) {
+#pragma unroll
+                            for (int k = 0; k < kBK / 16; ++k)
+                                mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
+                                           (kb != lo || k != 0) ? 1u : 0u);
+                        } else {
+                            const uint64_t al = sdesc_sw128(smem_u32(At + kAPartBytes));
+                            const uint64_t b1 = sdesc_sw128(smem_u32(Bs + (size_t)sb1 * kBStageBytes));
+#pragma unroll
+                            for (int k = 0; k < kBK / 16; ++k) {
+                                mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
+                                           (kb != lo || k != 0) ? 1u : 0u);
+                                mma_f16_ss(d_tmem, al + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc, 1u);
+                                mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b1 + (uint64_t)(2 * k), idesc, 1u);
+                            }
+                        }
+                        mma_commit(&c.a_empty[sa]);
+                        mma_commit(&c.b_empty[sb0]);
+                        if (p.nb == 2) mma_commit(&c.b_empty[sb1]);
+                        continue;
+                    }
+                    // 512-column tile (fp16 A, one B per half): the A K-block feeds both halves
+                    for (int hf = 0; hf < 2 && ok; ++hf) {
+                        const int sb0 = rb.idx;
+                        if (!mbar_wait_1t(&c.b_full[sb0], rb.phase, abort_flag, err)) {
+                            ok = false;
+                            break;
+                        }
+                        rb.next(p.sb);
+                        tc_fence_after();
+                        const uint32_t dh = d_tmem + (uint32_t)(hf * 256);
+                        const uint64_t b0 = sdesc_sw128(smem_u32(Bs + (size_t)sb0 * kBStageBytes));
 #pragma unroll
                         for (int k = 0; k < kBK / 16; ++k)
-                            mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
+                            mma_f16_ss(dh, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
                                        (kb != lo || k != 0) ? 1u : 0u);
-                    } else {
-                        const uint64_t al = sdesc_sw128(smem_u32(At + kAPartBytes));
-                        const uint64_t b1 = sdesc_sw128(smem_u32(Bs + (size_t)sb1 * kBStageBytes));
-#pragma unroll
-                        for (int k = 0; k < kBK / 16; ++k) {
-                            mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
-                                       (kb != lo || k != 0) ? 1u : 0u);
-                            mma_f16_ss(d_tmem, al + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc, 1u);
-                            mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b1 + (uint64_t)(2 * k), idesc, 1u);
-                        }
+                        mma_commit(&c.b_empty[sb0]);
                     }
+                    if (!ok) break;
                     mma_commit(&c.a_empty[sa]);
-                    mma_commit(&c.b_empty[sb0]);
-                    if (p.nb == 2) mma_commit(&c.b_empty[sb1]);
                 }
                 if (ok) mma_commit(&c.d_full[buf]);
             }
@@ -363,9 +390,11 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
         // TMEM is read in the 16x256b pattern so that each store writes whole sectors:
         // thread t holds rows (t/4) and (t/4 + 8) of a 16-lane half, 8 columns per quad.
         const int quad = warp & 3, kh = warp >= kEpi2 ? 1 : 0;  // lane quadrant, column chunks
+        const int nbuf = p.halves == 2 ? 1 : 2;
+        const int tw = p.nt * p.halves;  // tile width
         for (int lt = 0; lt < ntiles; ++lt) {
-            const int buf = lt & 1;
-            if (!mbar_wait_warp(&c.d_full[buf], (uint32_t)(lt >> 1) & 1u, abort_flag, err)) break;
+            const int buf = lt % nbuf;
+            if (!mbar_wait_warp(&c.d_full[buf], (uint32_t)(lt / nbuf) & 1u, abort_flag, err)) break;
             tc_fence_after();
             long long tm;
             int tn;
@@ -377,12 +406,12 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                 float rn[2];
 #pragma unroll
                 for (int h = 0; h < 2; ++h) rn[h] = (p.rownorm && row[h] < p.m) ? p.rownorm[row[h]] : 1.f;
-                for (int jc = 32 * kh; jc < p.nt; jc += 64) {
+                for (int jc = 32 * kh; jc < tw; jc += 64) {
                     float v[16];
                     tmem_ld16x256b_x4(tb + (uint32_t)jc, v);
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
-                        const int col = tn * p.nt + jc + 8 * j + 2 * (lane & 3);
+                        const int col = tn * tw + jc + 8 * j + 2 * (lane & 3);
 #pragma unroll
                         for (int h = 0; h < 2; ++h) {
                             if (row[h] >= p.m || col >= p.n) continue;
@@ -484,7 +513,11 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     p.K = a.K;
     p.nkb = (a.K + kBK - 1) / kBK;
     p.nt = a.n >= 256 ? 256 : (a.n + 31) / 32 * 32;
-    p.tiles_n = (a.n + p.nt - 1) / p.nt;
+    // a long K with fp32 A rounded to fp16 and more than 256 columns: 512-column tiles, so each
+    // converted A K-block feeds two 256-column MMAs (half the A loads and conversions per
+    // output; the single TMEM accumulator costs one epilogue per tile, small against the K loop)
+    p.halves = (!a.a_half && !a.split && a.n > 256 && p.nkb >= 32) ? 2 : 1;
+    p.tiles_n = (a.n + p.nt * p.halves - 1) / (p.nt * p.halves);
     p.tiles = ((a.m + kBM - 1) / kBM) * (long long)p.tiles_n;
     p.amode = a.a_half ? kAF16T : a.split ? kABF16X2 : kAF16;
     p.nb = a.split ? 2 : 1;
@@ -514,6 +547,10 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
         p.sa = kMaxSA;
         p.sb = kMaxSB;
     }
+    if (p.halves == 2) {  // two B boxes per K-block: B stages for two K-blocks
+        p.sx = 2;
+        p.sb = kMaxSB;
+    }
     if (gemm_smem_bytes(p.sx, p.sa, p.parts, p.sb) > cap) return cudaErrorInvalidConfiguration;
     p.C = a.C;
     p.ldc = a.ldc;
@@ -528,7 +565,7 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
         p.krange = 1;
         for (int tn = 0; tn < p.tiles_n; ++tn) {
             int lo = a.K, hi = 0;
-            for (int j = tn * p.nt; j < std::min(a.n, (tn + 1) * p.nt); ++j) {
+            for (int j = tn * p.nt * p.halves; j < std::min(a.n, (tn + 1) * p.nt * p.halves); ++j) {
                 lo = std::min(lo, a.b_klo[j]);
                 hi = std::max(hi, a.b_khi[j]);
             }
