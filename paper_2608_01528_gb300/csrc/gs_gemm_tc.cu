@@ -82,7 +82,6 @@ struct GemmParams {
     int n, K, nkb, nt, tiles_n;
     long long tiles;
     int amode, nb, parts;   // nb: B matrices per K-block; parts: A operand tiles per K-block
-    int halves;             // 256-column halves per tile: 2 = a 512-column tile, one accumulator
     int sx, sa, sb;
     void* C;
     long long ldc;
@@ -106,6 +105,9 @@ struct Ctl {
     int abort_flag;
 };
 
+// HALVES = 2: 128 x 512 tiles (two accumulators, fp16 A, one B); a template parameter so that the
+// ordinary kernel carries none of its control flow
+template <int HALVES>
 __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see kThreads)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b0,
               const __grid_constant__ CUtensorMap tmap_b1, const __grid_constant__ GemmParams p) {
@@ -234,7 +236,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                 tile_mn(lt, tm, tn);
                 krange(tn, lo, hi);
                 for (int kb = lo; kb < hi && ok; ++kb)
-                    for (int hf = 0; hf < p.halves && ok; ++hf)
+                    for (int hf = 0; hf < HALVES && ok; ++hf)
                         for (int which = 0; which < p.nb; ++which, ++ib, bs.next(p.sb)) {
                             const int s = bs.idx;
                             if (!mbar_wait_1t(&c.b_empty[s], bs.phase ^ 1u, abort_flag, err)) {
@@ -243,7 +245,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                             }
                             mbar_arrive_expect_tx(&c.b_full[s], bytes);
                             tma_load_2d(Bs + (size_t)s * kBStageBytes, which ? &tmap_b1 : &tmap_b0, &c.b_full[s],
-                                        kb * kBK, (tn * p.halves + hf) * p.nt, pol);
+                                        kb * kBK, (tn * HALVES + hf) * p.nt, pol);
                         }
             }
             for (int j = std::max(0, ib - p.sb); j < ib; ++j) mbar_drain(&c.b_full[j % p.sb], (uint32_t)(j / p.sb) & 1u, err);
@@ -254,7 +256,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
             const uint32_t idesc = p.amode == kABF16X2 ? idesc_bf16_f32(p.nt) : idesc_f16_f32(p.nt);
             RingPos ra, rb;
             bool ok = true;
-            const int nbuf = p.halves == 2 ? 1 : 2;  // a 512-column tile fills TMEM
+            const int nbuf = HALVES == 2 ? 1 : 2;  // a 512-column tile fills TMEM
             for (int lt = 0; lt < ntiles && ok; ++lt) {
                 const int buf = lt % nbuf;
                 if (!mbar_wait_1t(&c.d_empty[buf], ((uint32_t)(lt / nbuf) & 1u) ^ 1u, abort_flag, err)) break;
@@ -272,7 +274,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                     }
                     const uint8_t* At = As + (size_t)sa * p.parts * kAPartBytes;
                     const uint64_t ah = sdesc_sw128(smem_u32(At));
-                    if (p.halves == 1) {
+                    if (HALVES == 1) {
                         const int sb0 = rb.idx;
                         if (!mbar_wait_1t(&c.b_full[sb0], rb.phase, abort_flag, err)) ok = false;
                         rb.next(p.sb);
@@ -390,8 +392,8 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
         // TMEM is read in the 16x256b pattern so that each store writes whole sectors:
         // thread t holds rows (t/4) and (t/4 + 8) of a 16-lane half, 8 columns per quad.
         const int quad = warp & 3, kh = warp >= kEpi2 ? 1 : 0;  // lane quadrant, column chunks
-        const int nbuf = p.halves == 2 ? 1 : 2;
-        const int tw = p.nt * p.halves;  // tile width
+        const int nbuf = HALVES == 2 ? 1 : 2;
+        const int tw = p.nt * HALVES;  // tile width
         for (int lt = 0; lt < ntiles; ++lt) {
             const int buf = lt % nbuf;
             if (!mbar_wait_warp(&c.d_full[buf], (uint32_t)(lt / nbuf) & 1u, abort_flag, err)) break;
@@ -516,8 +518,8 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     // a long K with fp32 A rounded to fp16 and more than 256 columns: 512-column tiles, so each
     // converted A K-block feeds two 256-column MMAs (half the A loads and conversions per
     // output; the single TMEM accumulator costs one epilogue per tile, small against the K loop)
-    p.halves = (!a.a_half && !a.split && a.n > 256 && p.nkb >= 32) ? 2 : 1;
-    p.tiles_n = (a.n + p.nt * p.halves - 1) / (p.nt * p.halves);
+    const int halves = (!a.a_half && !a.split && a.n > 256 && p.nkb >= 32) ? 2 : 1;
+    p.tiles_n = (a.n + p.nt * halves - 1) / (p.nt * halves);
     p.tiles = ((a.m + kBM - 1) / kBM) * (long long)p.tiles_n;
     p.amode = a.a_half ? kAF16T : a.split ? kABF16X2 : kAF16;
     p.nb = a.split ? 2 : 1;
@@ -547,7 +549,7 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
         p.sa = kMaxSA;
         p.sb = kMaxSB;
     }
-    if (p.halves == 2) {  // two B boxes per K-block: B stages for two K-blocks
+    if (halves == 2) {  // two B boxes per K-block: B stages for two K-blocks
         p.sx = 2;
         p.sb = kMaxSB;
     }
@@ -565,7 +567,7 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
         p.krange = 1;
         for (int tn = 0; tn < p.tiles_n; ++tn) {
             int lo = a.K, hi = 0;
-            for (int j = tn * p.nt * p.halves; j < std::min(a.n, (tn + 1) * p.nt * p.halves); ++j) {
+            for (int j = tn * p.nt * halves; j < std::min(a.n, (tn + 1) * p.nt * halves); ++j) {
                 lo = std::min(lo, a.b_klo[j]);
                 hi = std::max(hi, a.b_khi[j]);
             }
@@ -586,14 +588,19 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
         return cudaErrorInvalidValue;
     const size_t smem = gemm_smem_bytes(p.sx, p.sa, p.parts, p.sb);
     if (device >= 0 && device < 64 && !g_attr_set[device]) {
-        cudaError_t e = cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cap);
+        cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cap);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(k_gemm_tc<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cap);
         if (e != cudaSuccess) return e;
         g_attr_set[device] = true;
     }
     int sms = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
     const int grid = (int)std::min<long long>(sms > 0 ? sms : 1, p.tiles);
-    k_gemm_tc<<<grid, kThreads, smem, s>>>(ta, tb0, tb1, p);
+    if (halves == 2)
+        k_gemm_tc<2><<<grid, kThreads, smem, s>>>(ta, tb0, tb1, p);
+    else
+        k_gemm_tc<1><<<grid, kThreads, smem, s>>>(ta, tb0, tb1, p);
     return cudaGetLastError();
 }
 
