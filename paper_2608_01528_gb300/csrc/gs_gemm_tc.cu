@@ -105,9 +105,9 @@ struct Ctl {
     int abort_flag;
 };
 
-// HALVES = 2: 128 x 512 tiles (two accumulators, fp16 A, one B); a template parameter so that the
-// ordinary kernel carries none of its control flow
-template <int HALVES>
+// AMODE: kAF16, kABF16X2 or kAF16T; HALVES = 2: 128 x 512 tiles (two accumulators, fp16 A, one
+// B).  Template parameters, so that each kernel carries only its own mode's control flow.
+template <int AMODE, int HALVES>
 __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see kThreads)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b0,
               const __grid_constant__ CUtensorMap tmap_b1, const __grid_constant__ GemmParams p) {
@@ -141,7 +141,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
             mbar_init(&c.x_empty[s], kCvtGroupWarps);
         }
         for (int s = 0; s < p.sa; ++s) {
-            mbar_init(&c.a_full[s], p.amode == kAF16T ? 1 : kCvtGroupWarps);
+            mbar_init(&c.a_full[s], AMODE == kAF16T ? 1 : kCvtGroupWarps);
             mbar_init(&c.a_empty[s], 1);
         }
         for (int s = 0; s < p.sb; ++s) {
@@ -171,7 +171,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
         tn = (int)(tg % p.tiles_n);
     };
 
-    if (warp == kAWarp && p.amode == kAF16T) {
+    if (warp == kAWarp && AMODE == kAF16T) {
         // ------------------------------------------------------------- A tiles (fp16) via TMA
         // straight into the swizzled A stages the MMA reads
         if (lane == 0) {
@@ -253,7 +253,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------- MMA issue
         if (lane == 0) {
-            const uint32_t idesc = p.amode == kABF16X2 ? idesc_bf16_f32(p.nt) : idesc_f16_f32(p.nt);
+            const uint32_t idesc = AMODE == kABF16X2 ? idesc_bf16_f32(p.nt) : idesc_f16_f32(p.nt);
             RingPos ra, rb;
             bool ok = true;
             const int nbuf = HALVES == 2 ? 1 : 2;  // a 512-column tile fills TMEM
@@ -287,7 +287,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                         if (!ok) break;
                         tc_fence_after();
                         const uint64_t b0 = sdesc_sw128(smem_u32(Bs + (size_t)sb0 * kBStageBytes));
-                        if (p.amode != kABF16X2) {
+                        if (AMODE != kABF16X2) {
 #pragma unroll
                             for (int k = 0; k < kBK / 16; ++k)
                                 mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
@@ -345,7 +345,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
             rx.next(p.sx);
             ra.next(p.sa);
         }
-        for (int it = g; p.amode != kAF16T && it < total_it; it += kCvtGroups) {
+        for (int it = g; AMODE != kAF16T && it < total_it; it += kCvtGroups) {
             const int sx = rx.idx, sa = ra.idx;
             if (!mbar_wait_warp(&c.x_full[sx], rx.phase, abort_flag, err) ||
                 !mbar_wait_warp(&c.a_empty[sa], ra.phase ^ 1u, abort_flag, err))
@@ -362,7 +362,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                 const float4 x = *reinterpret_cast<const float4*>(Xt + row * (kBK * 4) + c4 * 16);
                 const int off = row * 128 + (((c4 >> 1) ^ (row & 7)) * 16) + (c4 & 1) * 8;
                 uint2 hi;
-                if (p.amode == kAF16) {
+                if (AMODE == kAF16) {
                     amax = fmaxf(amax, fmaxf(fmaxf(fabsf(x.x), fabsf(x.y)), fmaxf(fabsf(x.z), fabsf(x.w))));
                     const __half2 h0 = __floats2half2_rn(x.x, x.y), h1 = __floats2half2_rn(x.z, x.w);
                     hi.x = *reinterpret_cast<const uint32_t*>(&h0);
@@ -588,19 +588,23 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
         return cudaErrorInvalidValue;
     const size_t smem = gemm_smem_bytes(p.sx, p.sa, p.parts, p.sb);
     if (device >= 0 && device < 64 && !g_attr_set[device]) {
-        cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cap);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(k_gemm_tc<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cap);
-        if (e != cudaSuccess) return e;
+        for (auto fn : {k_gemm_tc<kAF16, 1>, k_gemm_tc<kAF16, 2>, k_gemm_tc<kABF16X2, 1>, k_gemm_tc<kAF16T, 1>}) {
+            cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cap);
+            if (e != cudaSuccess) return e;
+        }
         g_attr_set[device] = true;
     }
     int sms = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
     const int grid = (int)std::min<long long>(sms > 0 ? sms : 1, p.tiles);
     if (halves == 2)
-        k_gemm_tc<2><<<grid, kThreads, smem, s>>>(ta, tb0, tb1, p);
+        k_gemm_tc<kAF16, 2><<<grid, kThreads, smem, s>>>(ta, tb0, tb1, p);
+    else if (p.amode == kAF16)
+        k_gemm_tc<kAF16, 1><<<grid, kThreads, smem, s>>>(ta, tb0, tb1, p);
+    else if (p.amode == kABF16X2)
+        k_gemm_tc<kABF16X2, 1><<<grid, kThreads, smem, s>>>(ta, tb0, tb1, p);
     else
-        k_gemm_tc<1><<<grid, kThreads, smem, s>>>(ta, tb0, tb1, p);
+        k_gemm_tc<kAF16T, 1><<<grid, kThreads, smem, s>>>(ta, tb0, tb1, p);
     return cudaGetLastError();
 }
 
