@@ -147,6 +147,9 @@ struct Ctl {
     int abort_flag;
 };
 
+// FULL = false: raw scores with only argmax / maxval out (the large-batch lookup); true: every
+// mode and output.  A template parameter, so the lookup kernel carries none of the other paths.
+template <bool FULL>
 __global__ void __launch_bounds__(kThreads, 1)
     k_ps_tc(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_q,
             const __grid_constant__ CUtensorMap tmap_rh, const __grid_constant__ CUtensorMap tmap_rl,
@@ -333,7 +336,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int l = threadIdx.x - (kCvt0 + g * kCvtGroupWarps) * 32;  // 0..127 within the group
         const int c4 = l & 15;                   // float4 column of the 64-wide K-block
         const int rbase = l >> 4;                // rows rbase + 8u, u < 16
-        const bool want_norm = p.mode == GS_SCORE_COSINE;
+        const bool want_norm = FULL && p.mode == GS_SCORE_COSINE;
         float nrm[kCvtRows];
 #pragma unroll
         for (int u = 0; u < kCvtRows; ++u) nrm[u] = 0.f;
@@ -422,7 +425,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tmem_ld32(ty + (uint32_t)jc, y);
                 else
                     tmem_ld16(ty + (uint32_t)jc, y);
-                if (p.Y && valid) {
+                if (FULL && p.Y && valid) {
                     float* dst = p.Y + (size_t)row * p.ldy + jc;
 #pragma unroll
                     for (int j = 0; j < 32; ++j)
@@ -470,7 +473,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int ci = ic + j;
                     if (ci >= p.M) break;
                     float g = p.scale * sv[j];
-                    if (p.mode == GS_SCORE_COSINE) {
+                    if (FULL && p.mode == GS_SCORE_COSINE) {
                         const float den = xnorm * p.cnorm[ci];
                         g = den > 0.f ? g / den : 0.f;
                     }
@@ -478,12 +481,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                         best = g;
                         besti = ci;
                     }
-                    if (p.mode == GS_SCORE_SOFTMAX) {
+                    if (FULL && p.mode == GS_SCORE_SOFTMAX) {
                         const float nm = fmaxf(run_max, g);
                         run_sum = run_sum * __expf(run_max - nm) + __expf(g - nm);
                         run_max = nm;
                     }
-                    if (p.S && valid) p.S[(size_t)row * p.lds + ci] = g;
+                    if (FULL && p.S && valid) p.S[(size_t)row * p.lds + ci] = g;
                 }
             }
             tc_fence_before();
@@ -491,7 +494,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (lane == 0) mbar_arrive(&c.s_empty);
             if (!valid) continue;
             float outmax = best;
-            if (p.mode == GS_SCORE_SOFTMAX) {
+            if (FULL && p.mode == GS_SCORE_SOFTMAX) {
                 const float inv = 1.f / run_sum;
                 outmax = __expf(best - run_max) * inv;
                 if (p.S) {
@@ -671,14 +674,18 @@ gs_status tc_prepare(gs_basis* h) {
         !make_tmap_2d(&h->tmap_rl, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, h->tc_Rl, mpad, npad, npad, kBK,
                       h->tc_half_rows, CU_TENSOR_MAP_SWIZZLE_128B))
         return GS_ERR_CUDA;
-    if (cudaFuncSetAttribute(k_ps_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemCap) !=
-        cudaSuccess)
+    if (cudaFuncSetAttribute(k_ps_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemCap) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(k_ps_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemCap) !=
+            cudaSuccess)
         return GS_ERR_CUDA;
     // the fused kernel needs all of its threads resident in one CTA; otherwise the
     // basis simply has no fused tensor-core similarity path
-    cudaFuncAttributes fa;
-    if (cudaFuncGetAttributes(&fa, k_ps_tc) != cudaSuccess) return GS_ERR_CUDA;
-    h->has_tmap_q16 = fa.maxThreadsPerBlock >= kThreads;
+    cudaFuncAttributes fa, fb;
+    if (cudaFuncGetAttributes(&fa, k_ps_tc<false>) != cudaSuccess ||
+        cudaFuncGetAttributes(&fb, k_ps_tc<true>) != cudaSuccess)
+        return GS_ERR_CUDA;
+    h->has_tmap_q16 = fa.maxThreadsPerBlock >= kThreads && fb.maxThreadsPerBlock >= kThreads;
     return GS_OK;
 }
 
@@ -722,7 +729,10 @@ cudaError_t launch_ps_tc(const gs_basis* h, const float* X, long long N, int ldx
     p.lds = lds;
     p.argmax = argmax;
     p.maxval = maxval;
-    k_ps_tc<<<grid, kThreads, ps_smem_bytes(g, p.xstage), s>>>(tmx, h->tmap_q16, h->tmap_rh, h->tmap_rl, p);
+    if (mode == GS_SCORE_RAW && !Y && !S)
+        k_ps_tc<false><<<grid, kThreads, ps_smem_bytes(g, p.xstage), s>>>(tmx, h->tmap_q16, h->tmap_rh, h->tmap_rl, p);
+    else
+        k_ps_tc<true><<<grid, kThreads, ps_smem_bytes(g, p.xstage), s>>>(tmx, h->tmap_q16, h->tmap_rh, h->tmap_rl, p);
     return cudaGetLastError();
 }
 
