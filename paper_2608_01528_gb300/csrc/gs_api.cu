@@ -460,6 +460,9 @@ gs_status gs_similarity_coeffs(const gs_basis* h, const float* Y, long long N, i
     const bool tc_ok = h->has_split && r >= 1 && (uintptr_t)Y % 16 == 0 && ldy % 4 == 0;
     const bool tensor = flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && tc_ok && big_gemm(N, M, r));
     if (tensor && !tc_ok) return h->has_split && r >= 1 ? GS_ERR_ALIGNMENT : GS_ERR_UNSUPPORTED;
+    if (!tensor && r >= 1 && r <= gs::kMaxCoeffsWarpR)  // small r: one fused launch, no scratch
+        return from_cuda(gs::launch_coeffs_warp(Y, N, ldy, r, h->R, h->ldr, M, h->cnorm, mode, scale, S, lds, argmax,
+                                                maxval, s));
     // scratch per row: ||y|| (cosine) and the score row when S is not an output
     const long long per_row = (mode == GS_SCORE_COSINE ? 1 : 0) + (S ? 0 : M);
     const long long chunk = std::min(per_row ? h->scratch_floats / per_row : N, kMaxGemmRows);

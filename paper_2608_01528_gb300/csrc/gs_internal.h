@@ -102,6 +102,12 @@ cudaError_t launch_ps_warp(const float* X, long long N, int ldx, int D, const fl
                            float* Y, int ldy, float* S, int lds, int* argmax, float* maxval,
                            cudaStream_t s);
 
+// similarity of Gram-loc queries Y (N x r, r <= 64), one warp per query; every mode, S optional
+constexpr int kMaxCoeffsWarpR = 64;
+cudaError_t launch_coeffs_warp(const float* Y, long long N, int ldy, int r, const float* R, int ldr, int M,
+                               const float* cnorm, int mode, float scale, float* S, int lds, int* argmax,
+                               float* maxval, cudaStream_t s);
+
 // C = alpha * A * op(B), batched over `batch` with element strides.
 //   A: m x k (lda), B: trans ? n x k : k x n (ldb); types MAT_F32 / MAT_BF16.
 //   rownorm/colnorm (optional): C[i][j] /= rownorm[i]*colnorm[j] (0 if product is 0)

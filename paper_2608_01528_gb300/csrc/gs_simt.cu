@@ -7,6 +7,7 @@
 //
 //  k_ps_warp      fused project + similarity, one warp per query, r <= 32
 //                 (Sec. 3.1 t = U^T x; Sec. 2.2 similarity; Eq. 2-3)
+//  k_coeffs_warp  similarity of Gram-loc queries, one warp per query, r <= 64 (Sec. 3.2, Eq. 2)
 //  k_gemm         tiled fp32 GEMM with scale / cosine / bf16 epilogues; used for
 //                 Y = X Q^T, S = Y R^T, V = P R (Sec. 2.2 / 3.3), Xhat = T Q
 //                 (Sec. 3.1 / 3.3) and batched attention logits (Sec. 2.2)
@@ -95,6 +96,69 @@ __global__ void __launch_bounds__(256) k_ps_warp(const float* __restrict__ X, lo
         g *= scale;
         if (mode == GS_SCORE_COSINE) {
             const float den = xnorm * cnorm[i];
+            g = den > 0.f ? g / den : 0.f;
+        }
+        return g;
+    };
+    float bv = -FLT_MAX;
+    int bi = 0x7fffffff;
+    for (int i = lane; i < M; i += 32) {
+        const float g = score(i);
+        if (g > bv) {
+            bv = g;
+            bi = i;
+        }
+        if (S && mode != GS_SCORE_SOFTMAX) S[(size_t)n * lds + i] = g;
+    }
+    warp_argmax(bv, bi);
+    if (bi == 0x7fffffff) bi = 0;
+    float outmax = bv;
+    if (mode == GS_SCORE_SOFTMAX) {
+        float z = 0.f;
+        for (int i = lane; i < M; i += 32) z += __expf(score(i) - bv);
+        z = warp_sum(z);
+        const float inv = 1.f / z;
+        if (S)
+            for (int i = lane; i < M; i += 32) S[(size_t)n * lds + i] = __expf(score(i) - bv) * inv;
+        outmax = inv;
+    }
+    if (lane == 0) {
+        if (argmax) argmax[n] = M > 0 ? bi : 0;
+        if (maxval) maxval[n] = M > 0 ? outmax : 0.f;
+    }
+}
+
+// Scores of queries given by their Gram-loc rows y (r <= 64): every lane holds the whole row
+// (broadcast loads), lane l scores codewords l, l + 32, ...; ||y|| stands for ||x|| in the
+// cosine mode (Eq. 3: equal for x in span(C)).  One launch for a small-batch lookup.
+constexpr int kCoefR = 64;
+
+__global__ void __launch_bounds__(256) k_coeffs_warp(const float* __restrict__ Yg, long long N, int ldy, int r,
+                                                      const float* __restrict__ R, int ldr, int M,
+                                                      const float* __restrict__ cnorm, int mode, float scale,
+                                                      float* __restrict__ S, int lds, int* __restrict__ argmax,
+                                                      float* __restrict__ maxval) {
+    const int lane = threadIdx.x & 31;
+    const long long n = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (n >= N) return;
+    const float* yr = Yg + (size_t)n * ldy;
+    float y[kCoefR];
+    float yy = 0.f;
+#pragma unroll
+    for (int j = 0; j < kCoefR; ++j) {
+        y[j] = j < r ? __ldg(yr + j) : 0.f;
+        yy = fmaf(y[j], y[j], yy);
+    }
+    const float ynorm = sqrtf(yy);
+    auto score = [&](int i) {
+        const float* Ri = R + (size_t)i * ldr;
+        float g = 0.f;
+#pragma unroll
+        for (int j = 0; j < kCoefR; ++j)
+            if (j < r) g = fmaf(y[j], __ldg(Ri + j), g);
+        g *= scale;
+        if (mode == GS_SCORE_COSINE) {
+            const float den = ynorm * cnorm[i];
             g = den > 0.f ? g / den : 0.f;
         }
         return g;
@@ -485,6 +549,16 @@ cudaError_t launch_ps_warp(const float* X, long long N, int ldx, int D, const fl
                            cudaStream_t s) {
     k_ps_warp<<<rows_grid(N), 256, 0, s>>>(X, N, ldx, D, Q, r, R, ldr, M, cnorm, mode, scale, Y, ldy,
                                            S, lds, argmax, maxval);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_coeffs_warp(const float* Y, long long N, int ldy, int r, const float* R, int ldr, int M,
+                               const float* cnorm, int mode, float scale, float* S, int lds, int* argmax,
+                               float* maxval, cudaStream_t s) {
+    if (N <= 0) return cudaSuccess;
+    if (r > kCoefR) return cudaErrorInvalidValue;
+    k_coeffs_warp<<<rows_grid(N), 256, 0, s>>>(Y, N, ldy, r, R, ldr, M, cnorm, mode, scale, S, lds, argmax,
+                                               maxval);
     return cudaGetLastError();
 }
 

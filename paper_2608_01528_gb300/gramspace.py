@@ -100,8 +100,8 @@ def _ptr(t):
     return ctypes.c_void_p(t.data_ptr()) if t is not None else None
 
 
-def _stream(stream):
-    s = stream if stream is not None else torch.cuda.current_stream()
+def _stream(stream, device=None):
+    s = stream if stream is not None else torch.cuda.current_stream(device)
     return ctypes.c_void_p(s.cuda_stream)
 
 
@@ -313,11 +313,11 @@ def project_similarity(basis, X, mode="raw", scale=1.0, path="auto", want_Y=Fals
         out["maxval"] = torch.empty(N, dtype=torch.float32, device=dev)
     Y, S = out.get("Y"), out.get("S")
     L = load_library()
-    with torch.cuda.device(dev):
-        st = L.gs_project_similarity(basis.handle, _ptr(X), N, _ld(X), MODES[mode], float(scale), PATHS[path],
-                                     _ptr(Y), _ld(Y) if Y is not None and Y.numel() else max(basis.r, 1),
-                                     _ptr(S), _ld(S) if S is not None and S.numel() else max(basis.M, 1),
-                                     _ptr(out.get("argmax")), _ptr(out.get("maxval")), _stream(stream))
+    # the handle's calls switch to the basis' device themselves: only the stream is looked up here
+    st = L.gs_project_similarity(basis.handle, _ptr(X), N, _ld(X), MODES[mode], float(scale), PATHS[path],
+                                 _ptr(Y), _ld(Y) if Y is not None and Y.numel() else max(basis.r, 1),
+                                 _ptr(S), _ld(S) if S is not None and S.numel() else max(basis.M, 1),
+                                 _ptr(out.get("argmax")), _ptr(out.get("maxval")), _stream(stream, dev))
     _check(st, "gs_project_similarity")
     return out
 
@@ -337,11 +337,10 @@ def similarity_coeffs(basis, Y, mode="raw", scale=1.0, path="auto", want_S=False
         out["maxval"] = torch.empty(N, dtype=torch.float32, device=dev)
     S = out.get("S")
     L = load_library()
-    with torch.cuda.device(dev):
-        st = L.gs_similarity_coeffs(basis.handle, _ptr(Y) if Y.numel() else None, N,
-                                    _ld(Y) if Y.numel() else max(basis.r, 1), MODES[mode], float(scale),
-                                    PATHS[path], _ptr(S), _ld(S) if S is not None and S.numel() else max(basis.M, 1),
-                                    _ptr(out.get("argmax")), _ptr(out.get("maxval")), _stream(stream))
+    st = L.gs_similarity_coeffs(basis.handle, _ptr(Y) if Y.numel() else None, N,
+                                _ld(Y) if Y.numel() else max(basis.r, 1), MODES[mode], float(scale),
+                                PATHS[path], _ptr(S), _ld(S) if S is not None and S.numel() else max(basis.M, 1),
+                                _ptr(out.get("argmax")), _ptr(out.get("maxval")), _stream(stream, dev))
     _check(st, "gs_similarity_coeffs")
     return out
 
