@@ -1,0 +1,73 @@
+"""GPU parity of the bench's side rows at their full sizes, in the launch configuration the bench
+times: every output computed, a seeded sample of rows checked against the oracle run with the
+GPU's own basis (so only the kernels' arithmetic differs), bounds as in the other parity tests:
+X̂ within 1e-4 ||t|| (fp16 tensor-core reconstruction), V within 1e-4 sum_i |p_i| ||c_i|| +
+2^-8 |V*| (bf16 output), binding within the fp32-sum bound plus the reconstruction error carried
+through the block (see test_bind_gpu).
+"""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from test_bind_gpu import check_bind
+from test_parity_gpu import cuda, host
+
+pytestmark = pytest.mark.gpu
+
+
+def sample_rows(n, k, seed):
+    return np.sort(np.random.default_rng(seed).choice(n, k, replace=False))
+
+
+def test_reconstruct_rankdef_full_size(gs, orc):
+    """16,384 x 922 coefficients -> 16,384 x 10,000 (the bench's reconstruct row)."""
+    C4, _ = synth.rankdef_codebook()
+    b = gs.build_basis(cuda(C4))
+    r4 = (b.r + 3) // 4 * 4
+    g = torch.Generator().manual_seed(17)
+    T = torch.randn(16384, r4, generator=g).to("cuda:0")[:, :b.r]
+    Xh = gs.reconstruct(b, T)
+    gs.stream_status()
+    rows = sample_rows(16384, 64, 1)
+    Tr = host(T[torch.from_numpy(rows).to(T.device)])
+    ref = orc.reconstruct(Tr, host(b.Q))
+    got = host(Xh[torch.from_numpy(rows).to(T.device)])
+    bound = 1e-4 * np.linalg.norm(Tr, axis=1)
+    assert np.all(np.abs(got - ref).max(axis=1) <= bound)
+
+
+def test_prob_vectorize_attention_full_size(gs, orc):
+    """65,536 x 512 probabilities -> bf16 Gram-loc rows (the bench's prob-vectorize row)."""
+    a = synth.attention()
+    b = gs.build_basis(cuda(a["C"]))
+    V = gs.prob_vectorize(b, cuda(a["Pq"]), dtype=torch.bfloat16)
+    gs.stream_status()
+    rows = sample_rows(a["Pq"].shape[0], 256, 2)
+    P = a["Pq"][rows].astype(np.float64)
+    R = host(b.R)
+    ref = P @ R
+    got = host(V[torch.from_numpy(rows).to(V.device)])
+    cn = np.linalg.norm(R, axis=1)
+    bound = 1e-4 * (np.abs(P) @ cn)[:, None] + 2.0 ** -8 * np.abs(ref)
+    assert np.all(np.abs(got - ref) <= bound)
+
+
+def test_reconstruct_bind_full_size(gs, orc):
+    """8,192 rows of the attention basis bound with per-row partners in blocks of 256 (the bench's
+    reconstruct + bind row)."""
+    a = synth.attention(B=1, L=1)
+    b = gs.build_basis(cuda(a["C"]))
+    N, L = 8192, 256
+    P = synth.attention_probs(12, 1, N, b.M, 1)
+    T = (torch.from_numpy(P).to("cuda:0") @ b.R).contiguous()
+    g = torch.Generator().manual_seed(19)
+    Y = torch.randn(N, b.D, generator=g).to("cuda:0")
+    Z = gs.reconstruct_bind(b, T, Y, L)
+    gs.stream_status()
+    rows = sample_rows(N, 32, 3)
+    idx = torch.from_numpy(rows).to(T.device)
+    Tr, Yr = host(T[idx]), host(Y[idx])
+    Xo = orc.reconstruct(Tr, host(b.Q))
+    Zo = orc.bind(Xo, Yr, L)
+    check_bind(Z[idx], Zo, Xo, Yr, L, e_rec=1e-4 * np.linalg.norm(Tr, axis=1))
