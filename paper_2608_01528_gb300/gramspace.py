@@ -6,8 +6,11 @@ PyTorch's plumbing), and every step of the computation runs in the library's
 CUDA kernels.  There is no CPU fallback: if the library is not built, or no
 sm_103 device is present, calls raise.
 
-Names follow the C ABI: build_basis, project_similarity, prob_vectorize,
-reconstruct, attention_scores, stream_status.
+Names follow the C ABI (gs_ prefix dropped): build_basis, build_basis_grouped,
+basis_groups, import_basis, project_similarity, project_similarity_host (with
+reserve_staging), project_similarity_static, similarity_coeffs, group_argmax,
+prob_vectorize, reconstruct, reconstruct_bind, bind, attention_scores,
+stream_status, selftest_wait_timeout.
 """
 from __future__ import annotations
 
