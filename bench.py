@@ -439,10 +439,12 @@ def side_rows(gs, dev):
     Vq = torch.empty(Pq.shape[0], b5.r, dtype=torch.bfloat16, device=dev)
     ms = timeit(lambda: gs.prob_vectorize(b5, Pq, out=Vq))
     out["probvec_attention"] = roof(ms, Pq.numel() * 4 + Vq.numel() * 2, 2 * Pq.shape[0] * b5.M * b5.r, "hbm")
-    V3 = Vq.reshape(64, 1024, -1)
+    # queries and keys from independent probabilities (64 MiB each), scores 256 MiB
+    Vk = gs.prob_vectorize(b5, torch.from_numpy(a["Pk"]).to(dev), dtype=torch.bfloat16)
+    Vq3, Vk3 = Vq.reshape(64, 1024, -1), Vk.reshape(64, 1024, -1)
     A = torch.empty(64, 1024, 1024, device=dev)
-    ms = timeit(lambda: gs.attention_scores(V3, V3, 1 / 64.0, out=A))
-    out["attention"] = roof(ms, 2 * V3.numel() * 2 + A.numel() * 4, 2 * 64 * 1024 * 1024 * b5.r, "hbm")
+    ms = timeit(lambda: gs.attention_scores(Vq3, Vk3, 1 / 64.0, out=A))
+    out["attention"] = roof(ms, (Vq3.numel() + Vk3.numel()) * 2 + A.numel() * 4, 2 * 64 * 1024 * 1024 * b5.r, "hbm")
     # reconstruct + bind at the transition into component-wise operators: 8,192 coefficient rows
     # of the attention basis (r = 512, D = 4096), per-row partners, blocks of 256
     Nb, Lb = 8192, 256
