@@ -454,13 +454,18 @@ def side_rows(gs, dev):
     Xb = torch.empty(Nb, b5.D, device=dev)
     ms_fused = timeit(lambda: gs.reconstruct_bind(b5, Tb, Yb, Lb, out=Zb))
     ms_rec = timeit(lambda: gs.reconstruct(b5, Tb, out=Xb))
+    # binding through block spectra (the default): X, Y read and Z written once, 12 D bytes a row
     ms_bind = timeit(lambda: gs.bind(Xb, Yb, Lb, out=Zb))
-    bind_flops = 2 * Nb * b5.D * Lb
+    bind_bytes = 3 * Nb * b5.D * 4
+    # the direct sum for comparison: 2 L flops per output on the fp32 lanes
+    ms_direct = timeit(lambda: gs.bind(Xb, Yb, Lb, method="direct", out=Zb))
+    direct_tflops = 2 * Nb * b5.D * Lb / (ms_direct / 1e3) / 1e12
     out["reconstruct_bind"] = {"ms": round(ms_fused, 4), "rows": Nb, "D": b5.D, "r": b5.r, "L": Lb,
                                "reconstruct_ms": round(ms_rec, 4), "bind_ms": round(ms_bind, 4),
-                               "bind_tflops": round(bind_flops / (ms_bind / 1e3) / 1e12, 1),
-                               "bound": "alu", "alu_peak_tflops": FP32_PEAK_TFLOPS,
-                               "frac": round(bind_flops / (ms_bind / 1e3) / 1e12 / FP32_PEAK_TFLOPS, 4)}
+                               "bind_gbs": round(bind_bytes / (ms_bind / 1e3) / 1e9, 1), "bound": "hbm",
+                               "frac": round(bind_bytes / (ms_bind / 1e3) / 1e9 / peaks["hbm_gbs"], 4),
+                               "bind_direct_ms": round(ms_direct, 4), "bind_direct_tflops": round(direct_tflops, 1),
+                               "bind_direct_alu_frac": round(direct_tflops / FP32_PEAK_TFLOPS, 4)}
     del b4, b5, Xb, Yb, Zb
     out["lookup_sweep"] = lookup_sweep(gs, dev)
     out["grouped_attributes"] = grouped_attributes(gs, dev)

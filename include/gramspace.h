@@ -282,9 +282,12 @@ GS_API gs_status gs_prob_vectorize(const gs_basis* h, const float* P, long long 
 GS_API gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt,
                          float* Xhat, int ldxh, unsigned flags, void* stream);
 
-/* binding operators of gs_bind / gs_reconstruct_bind */
+/* binding operators of gs_bind / gs_reconstruct_bind, optionally OR-ed with one method */
 #define GS_BIND 0   /* block circular convolution  */
 #define GS_UNBIND 1 /* block circular correlation  */
+#define GS_BIND_DIRECT 2   /* the direct sum: one fp32 sum of L products per output    */
+#define GS_BIND_SPECTRAL 4 /* through block spectra (convolution theorem): L a power
+                              of two in [64, 4096], rows 8-byte aligned               */
 
 /*
  * Binding and unbinding, the component-wise operators of rule execution
@@ -298,8 +301,22 @@ GS_API gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, l
  * (unbinding with y undoes binding with y when y's block spectra have unit
  * modulus, and approximately for random y).  X, Z: N x D fp32 (ld = ldx,
  * ldz >= D); Y: N x D fp32 with ld = ldy >= D, or ldy = 0: Y's single row
- * binds every row.  fp32 CUDA-core arithmetic, one sum per output in j order.
- * Errors: GS_ERR_SHAPE (L does not divide D, ld too small), GS_ERR_INVALID_ARG.
+ * binds every row.  Methods (op | method), both fp32 CUDA-core arithmetic:
+ *   GS_BIND_DIRECT: one sum per output in j order; |error| <= L 2^-22
+ *     ||x_b|| ||y_b|| per output of block b.
+ *   GS_BIND_SPECTRAL: z = IDFT(DFT(x) DFT(y)) per block (conj(DFT(y)) to
+ *     unbind) with fp32 radix-2^k transforms, ~5 L log2 L flops per block
+ *     instead of 2 L^2; |error| <= sqrt(2L) (3 e + 4u) ||x_b|| ||y_b||, where
+ *     u = 2^-24, e = K eta / (1 - K eta) + 10u, eta = 10u and K = log2(L) + 2
+ *     (log2(L) + 1 for L <= 512): the transform error bound of the radix-2
+ *     FFT (Higham, Accuracy and Stability of Numerical Algorithms, Thm 24.2)
+ *     carried through the product and the inverse; typical errors are far
+ *     smaller than the direct sum's.
+ *   neither: GS_BIND_SPECTRAL where it applies, else GS_BIND_DIRECT.
+ * Errors: GS_ERR_SHAPE (L does not divide D, ld too small), GS_ERR_INVALID_ARG
+ * (unknown op or both methods), GS_ERR_UNSUPPORTED (GS_BIND_SPECTRAL with an L
+ * it does not take), GS_ERR_ALIGNMENT (GS_BIND_SPECTRAL with a pointer or ld
+ * that leaves a row start off an 8-byte boundary).
  */
 GS_API gs_status gs_bind(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L, int op,
                          float* Z, int ldz, void* stream);
@@ -308,7 +325,7 @@ GS_API gs_status gs_bind(const float* X, long long N, int D, int ldx, const floa
  * Reconstruction followed by binding at the transition into component-wise
  * operators (Sec. 3.3: reconstruction is placed immediately before binding and
  * unbinding): Z = op(T Q, Y) with gs_reconstruct's T (N x r, t_dtype, ldt) and
- * gs_bind's Y, L, op and Z.  The rows are processed in chunks whose
+ * gs_bind's Y, L, op (with its method) and Z.  The rows are processed in chunks whose
  * reconstruction (at most 64 MiB) lives in the handle's scratch between the two
  * kernels, so the reconstructed vectors stay in L2 rather than making a round
  * trip through HBM.  flags picks the reconstruction path as in gs_reconstruct.

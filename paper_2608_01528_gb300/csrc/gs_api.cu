@@ -598,9 +598,26 @@ gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, long lon
 }
 
 static gs_status check_bind_args(long long N, int D, int ldx, long long ldy, int L, int op, int ldz) {
-    if (op != GS_BIND && op != GS_UNBIND) return GS_ERR_INVALID_ARG;
+    if (op < 0 || (op & ~(GS_UNBIND | GS_BIND_DIRECT | GS_BIND_SPECTRAL)) ||
+        ((op & GS_BIND_DIRECT) && (op & GS_BIND_SPECTRAL)))
+        return GS_ERR_INVALID_ARG;
     if (N < 0 || D < 1 || L < 1 || D % L || ldx < D || ldz < D || (ldy != 0 && ldy < D)) return GS_ERR_SHAPE;
     return GS_OK;
+}
+
+// one binding launch: the spectral kernel unless the direct sum is asked for or the spectral
+// kernel cannot take the shape; a forced spectral method that cannot run is an error
+static gs_status bind_rows(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L, int op,
+                           float* Z, int ldz, cudaStream_t s) {
+    const bool unbind = (op & GS_UNBIND) != 0;
+    const bool spec = gs::bind_spectral_supported(L, X, ldx, Y, ldy, Z, ldz);
+    if ((op & GS_BIND_SPECTRAL) && !spec) {
+        const bool l_ok = L >= gs::kMinBindSpectralL && L <= gs::kMaxBindSpectralL && !(L & (L - 1));
+        return l_ok ? GS_ERR_ALIGNMENT : GS_ERR_UNSUPPORTED;
+    }
+    if (spec && !(op & GS_BIND_DIRECT))
+        return from_cuda(gs::launch_bind_spectral(X, N, D, ldx, Y, ldy, L, unbind, Z, ldz, s));
+    return from_cuda(gs::launch_bind(X, N, D, ldx, Y, ldy, L, unbind, Z, ldz, s));
 }
 
 gs_status gs_bind(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L, int op, float* Z,
@@ -612,7 +629,7 @@ gs_status gs_bind(const float* X, long long N, int D, int ldx, const float* Y, l
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return GS_ERR_CUDA;
     if (!device_supported(dev)) return GS_ERR_UNSUPPORTED;
-    return from_cuda(gs::launch_bind(X, N, D, ldx, Y, ldy, L, op == GS_UNBIND, Z, ldz, (cudaStream_t)stream));
+    return bind_rows(X, N, D, ldx, Y, ldy, L, op, Z, ldz, (cudaStream_t)stream);
 }
 
 gs_status gs_reconstruct_bind(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt, const float* Y,
@@ -630,6 +647,8 @@ gs_status gs_reconstruct_bind(const gs_basis* h, const void* T, int t_dtype, lon
     // rows in chunks: the reconstructed chunk (at most 64 MiB, so it stays in L2 between the two
     // kernels) and the fp16 copy of its T rows share the handle's scratch
     const int Dp = (h->D + 3) / 4 * 4, ld16 = (h->r + 7) / 8 * 8;
+    if ((op & GS_BIND_SPECTRAL) && !gs::bind_spectral_supported(L, h->scratch, Dp, Y, ldy, Z, ldz))
+        return bind_rows(h->scratch, 0, h->D, Dp, Y, ldy, L, op, Z, ldz, s);  // the method's error, no launch
     long long cr = std::min(h->scratch_floats / (Dp + ld16 / 2 + 1), (64LL << 20) / (4LL * Dp));
     cr = std::min(cr, kMaxGemmRows);
     if (cr >= 128) cr = cr / 128 * 128;
@@ -643,8 +662,7 @@ gs_status gs_reconstruct_bind(const gs_basis* h, const void* T, int t_dtype, lon
         st = reconstruct_rows(h, (const char*)T + (size_t)c0 * ldt * tsize, t_dtype, nc, ldt, xhat, Dp, flags, s,
                               work, work_floats);
         if (st != GS_OK) return st;
-        st = from_cuda(gs::launch_bind(xhat, nc, h->D, Dp, Y + (size_t)c0 * ldy, ldy, L, op == GS_UNBIND,
-                                       Z + (size_t)c0 * ldz, ldz, s));
+        st = bind_rows(xhat, nc, h->D, Dp, Y + (size_t)c0 * ldy, ldy, L, op, Z + (size_t)c0 * ldz, ldz, s);
         if (st != GS_OK) return st;
     }
     return GS_OK;

@@ -142,6 +142,13 @@ cudaError_t launch_group_argmax(const float* S, long long N, int lds, const int*
 constexpr int kMaxBindFastL = 4096;
 cudaError_t launch_bind(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L, bool unbind,
                         float* Z, int ldz, cudaStream_t s);
+// the same through block spectra (gs_bind_spec.cu): L a power of two in [kMinBindSpectralL,
+// kMaxBindSpectralL], rows 8-byte aligned (bind_spectral_supported)
+constexpr int kMinBindSpectralL = 64;
+constexpr int kMaxBindSpectralL = 4096;
+bool bind_spectral_supported(int L, const float* X, int ldx, const float* Y, long long ldy, const float* Z, int ldz);
+cudaError_t launch_bind_spectral(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L,
+                                 bool unbind, float* Z, int ldz, cudaStream_t s);
 
 // per-row argmax / maxval over S (N x M); SOFTMAX mode rewrites the row in place.
 cudaError_t launch_row_finish(float* S, long long N, int M, int lds, bool softmax, int* argmax,

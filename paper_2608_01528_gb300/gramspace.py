@@ -373,6 +373,7 @@ def reconstruct(basis, T, path="auto", out=None, stream=None):
 
 
 BIND_OPS = {"bind": 0, "unbind": 1}
+BIND_METHODS = {"auto": 0, "direct": 2, "spectral": 4}
 
 
 def _partner(Y, N, D):
@@ -385,30 +386,32 @@ def _partner(Y, N, D):
     return _ld(Y)
 
 
-def bind(X, Y, L, op="bind", out=None, stream=None):
+def bind(X, Y, L, op="bind", method="auto", out=None, stream=None):
     """Block circular convolution (op="bind") or correlation ("unbind") of the rows of X with
-    those of Y (or with Y's single row), blocks of L; see gs_bind."""
+    those of Y (or with Y's single row), blocks of L; method "direct" (the sum per output),
+    "spectral" (block transforms) or "auto"; see gs_bind."""
     N, D = X.shape
     ldy = _partner(Y, N, D)
     Z = out if out is not None else torch.empty((N, D), dtype=torch.float32, device=X.device)
     L_ = load_library()
     with torch.cuda.device(X.device):
-        st = L_.gs_bind(_ptr(X), N, D, _ld(X) if N else D, _ptr(Y), ldy, int(L), BIND_OPS[op], _ptr(Z),
-                        _ld(Z) if N else D, _stream(stream))
+        st = L_.gs_bind(_ptr(X), N, D, _ld(X) if N else D, _ptr(Y), ldy, int(L), BIND_OPS[op] | BIND_METHODS[method],
+                        _ptr(Z), _ld(Z) if N else D, _stream(stream))
     _check(st, "gs_bind")
     return Z
 
 
-def reconstruct_bind(basis, T, Y, L, op="bind", path="auto", out=None, stream=None):
-    """op(T Q, Y): reconstruction then binding, chunk by chunk through L2; see gs_reconstruct_bind."""
+def reconstruct_bind(basis, T, Y, L, op="bind", path="auto", method="auto", out=None, stream=None):
+    """op(T Q, Y): reconstruction then binding, chunk by chunk through L2; see gs_reconstruct_bind
+    (path: the reconstruction's kernels, method: the binding's, as in bind)."""
     N = T.shape[0]
     ldy = _partner(Y, N, basis.D)
     Z = out if out is not None else torch.empty((N, basis.D), dtype=torch.float32, device=T.device)
     L_ = load_library()
     with torch.cuda.device(basis.device):
         st = L_.gs_reconstruct_bind(basis.handle, _ptr(T), _dtype_code(T), N, _ld(T) if N else basis.r, _ptr(Y),
-                                    ldy, int(L), BIND_OPS[op], _ptr(Z), _ld(Z) if N else basis.D, PATHS[path],
-                                    _stream(stream))
+                                    ldy, int(L), BIND_OPS[op] | BIND_METHODS[method], _ptr(Z),
+                                    _ld(Z) if N else basis.D, PATHS[path], _stream(stream))
     _check(st, "gs_reconstruct_bind")
     return Z
 

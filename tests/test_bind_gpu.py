@@ -1,10 +1,16 @@
 """GPU parity of binding / unbinding (gs_bind) and reconstruct-then-bind (gs_reconstruct_bind)
-against the float64 oracle.
+against the float64 oracle (the direct sums of the definition).
 
-Bound per output of block b (fp32 sums of L products in j order, and for the fused call the
-reconstruction error on top): |Z - Z*| <= L 2^-22 ||x_b|| ||y_b|| + e_rec sqrt(L) ||y_b||, with
-e_rec = 1e-4 ||t|| on the fp16 tensor-core reconstruction (the reconstruct bound) and 0 on the fp32
-path, where ||x_b||, ||y_b|| are the norms of the row's blocks.
+Bound per output of block b, with ||x_b||, ||y_b|| the norms of the row's blocks:
+  direct method (fp32 sums of L products in j order): |Z - Z*| <= L 2^-22 ||x_b|| ||y_b||;
+  spectral method (fp32 radix-2^k transforms of the blocks, the product, the inverse):
+  |Z - Z*| <= sqrt(2L) (3e + 4u) ||x_b|| ||y_b||, u = 2^-24, e = K eta / (1 - K eta) + 10u,
+  eta = 10u, K = log2(L) + 1 (two Stockham passes, L <= 512) or log2(L) + 2 (three): the
+  radix-2 FFT bound ||fl(F w) - F w|| <= K eta ||F w|| (Higham, Thm 24.2; one extra twiddle
+  multiply per pass) through the split, the product (max|Y_k| <= sqrt(L) ||y_b||) and the
+  inverse transform.
+For the fused call the reconstruction error adds e_rec sqrt(L) ||y_b||, e_rec = 1e-4 ||t|| on the
+fp16 tensor-core reconstruction (the reconstruct bound) and 0 on the fp32 path.
 """
 import numpy as np
 import pytest
@@ -15,17 +21,32 @@ from test_parity_gpu import cuda, host
 
 pytestmark = pytest.mark.gpu
 
+U32 = 2.0 ** -24
+
 
 def block_norms(A, L):
     N, D = A.shape
     return np.sqrt((A.astype(np.float64).reshape(N, D // L, L) ** 2).sum(axis=2))
 
 
-def check_bind(Z, Zo, X, Y, L, e_rec=None):
+def spectral_applies(L):
+    return 64 <= L <= 4096 and L & (L - 1) == 0
+
+
+def bind_error_factor(L, method):
+    if method == "direct":
+        return L * 2.0 ** -22
+    K = int(np.log2(L)) + (1 if L <= 512 else 2)
+    eta = 10 * U32
+    e = K * eta / (1 - K * eta) + 10 * U32
+    return np.sqrt(2 * L) * (3 * e + 4 * U32)
+
+
+def check_bind(Z, Zo, X, Y, L, e_rec=None, method="direct"):
     N, D = Zo.shape
     nx = block_norms(X, L)
     ny = block_norms(np.broadcast_to(Y, (N, D)), L)
-    bound = L * 2.0 ** -22 * nx * ny
+    bound = bind_error_factor(L, method) * nx * ny
     if e_rec is not None:
         bound = bound + e_rec[:, None] * np.sqrt(L) * ny
     err = np.abs(host(Z) - Zo).reshape(N, D // L, L).max(axis=2)
@@ -37,18 +58,44 @@ def check_bind(Z, Zo, X, Y, L, e_rec=None):
     (50, 960, 24, False, "unbind"), (33, 1000, 10, True, "bind"), (5, 4096, 4096, False, "bind"),
     (300, 3000, 1000, False, "unbind"), (1, 64, 64, True, "bind")])
 def test_bind_matches_oracle(gs, orc, N, D, L, bcast, op):
-    """Block lengths on both kernels (L % 8 == 0: the shared-memory kernel, up to L = 4096;
-    L = 10: one output per thread), one partner for all rows, padded leading dimensions."""
+    """The direct method on all its kernels (L % 16, L % 8 == 0: shared-memory tiles up to L =
+    4096; L = 10: one output per thread), one partner for all rows, padded leading dimensions."""
     rng = np.random.default_rng(N + D + L)
     X = rng.normal(size=(N, D)).astype(np.float32)
     Y = rng.normal(size=(1 if bcast else N, D)).astype(np.float32)
     Xp = torch.zeros((N, D + 8), device="cuda:0")
     Xp[:, :D] = cuda(X)
     Zp = torch.zeros((N, D + 3), device="cuda:0")  # odd row pitch: element stores
-    Z = gs.bind(Xp[:, :D], cuda(Y), L, op, out=Zp[:, :D])
+    Z = gs.bind(Xp[:, :D], cuda(Y), L, op, method="direct", out=Zp[:, :D])
     gs.stream_status()
     Zo = orc.bind(X, Y, L, orc.UNBIND if op == "unbind" else orc.BIND)
     check_bind(Z, Zo, X, Y, L)
+
+
+@pytest.mark.parametrize("N,D,L,bcast,op", [
+    (5, 192, 64, False, "bind"), (70, 64, 64, True, "unbind"), (3, 256, 128, False, "unbind"),
+    (37, 1024, 256, False, "bind"), (17, 256, 256, False, "unbind"), (9, 1536, 512, True, "bind"),
+    (37, 1024, 1024, False, "unbind"), (3, 4096, 2048, False, "bind"), (5, 4096, 4096, False, "unbind"),
+    (3000, 1024, 64, False, "bind")])
+def test_bind_spectral_matches_oracle(gs, orc, N, D, L, bcast, op):
+    """The spectral method at every block length it takes (L = 64 ... 4096: two and three
+    Stockham passes), partial last groups of blocks, one partner for all rows, padded even row
+    pitches, and 48,000 blocks (more groups than resident CTAs: the persistent loop)."""
+    rng = np.random.default_rng(N + D + L + 1)
+    X = rng.normal(size=(N, D)).astype(np.float32)
+    Y = rng.normal(size=(1 if bcast else N, D)).astype(np.float32)
+    Xp = torch.zeros((N, D + 6), device="cuda:0")
+    Xp[:, :D] = cuda(X)
+    Zp = torch.full((N, D + 2), 7.0, device="cuda:0")
+    Z = gs.bind(Xp[:, :D], cuda(Y), L, op, method="spectral", out=Zp[:, :D])
+    gs.stream_status()
+    Zo = orc.bind(X, Y, L, orc.UNBIND if op == "unbind" else orc.BIND)
+    check_bind(Z, Zo, X, Y, L, method="spectral")
+    assert torch.all(Zp[:, D:] == 7.0)  # nothing written past a row's D outputs
+    # the automatic choice is the spectral kernel here: identical results
+    Za = gs.bind(Xp[:, :D], cuda(Y), L, op)
+    gs.stream_status()
+    assert torch.equal(Za, Z)
 
 
 def test_unbind_recovers_unit_spectrum_binding(gs):
@@ -61,13 +108,15 @@ def test_unbind_recovers_unit_spectrum_binding(gs):
     Y = np.real(np.fft.ifft(spec, axis=2)).reshape(N, D).astype(np.float32)
     X = rng.normal(size=(N, D)).astype(np.float32)
     Xd, Yd = cuda(X), cuda(Y)
-    back = gs.bind(gs.bind(Xd, Yd, L), Yd, L, "unbind")
-    gs.stream_status()
-    assert np.abs(host(back) - X).max() <= 1e-4 * np.abs(X).max()
+    for method in ("direct", "spectral"):
+        back = gs.bind(gs.bind(Xd, Yd, L, method=method), Yd, L, "unbind", method=method)
+        gs.stream_status()
+        assert np.abs(host(back) - X).max() <= 1e-4 * np.abs(X).max()
 
 
-@pytest.mark.parametrize("path", ["simt", "tensor"])
-def test_reconstruct_bind_matches_oracle(gs, orc, path):
+@pytest.mark.parametrize("path,method", [("simt", "direct"), ("tensor", "direct"), ("simt", "spectral"),
+                                         ("tensor", "auto")])
+def test_reconstruct_bind_matches_oracle(gs, orc, path, method):
     """op(T Q, Y) on the attention codebook's basis (r = 512, D = 4096, blocks of 256); against
     the oracle run with the GPU's basis, so only the kernels' arithmetic differs."""
     a = synth.attention(B=1, L=1)
@@ -78,12 +127,12 @@ def test_reconstruct_bind_matches_oracle(gs, orc, path):
     T = T.astype(np.float32)
     Y = rng.normal(size=(N, b.D)).astype(np.float32)
     for op in ("bind", "unbind"):
-        Z = gs.reconstruct_bind(b, cuda(T), cuda(Y), 256, op, path=path)
+        Z = gs.reconstruct_bind(b, cuda(T), cuda(Y), 256, op, path=path, method=method)
         gs.stream_status()
         Zo = orc.reconstruct_bind(T, host(b.Q), Y, 256, orc.UNBIND if op == "unbind" else orc.BIND)
         Xo = orc.reconstruct(T, host(b.Q))
         e_rec = 1e-4 * np.linalg.norm(T.astype(np.float64), axis=1) if path == "tensor" else None
-        check_bind(Z, Zo, Xo, Y, 256, e_rec)
+        check_bind(Z, Zo, Xo, Y, 256, e_rec, method="direct" if method == "direct" else "spectral")
 
 
 def test_reconstruct_bind_codebook_and_broadcast(gs, orc):
@@ -93,10 +142,11 @@ def test_reconstruct_bind_codebook_and_broadcast(gs, orc):
     Y = np.random.default_rng(3).normal(size=(1, 1024)).astype(np.float32)
     Rp = torch.zeros((b.M, 8), device="cuda:0")
     Rp[:, :b.r] = b.R
-    Z = gs.reconstruct_bind(b, Rp[:, :b.r], cuda(Y), 128)
-    gs.stream_status()
-    Zo = orc.bind(t["C"], Y, 128)
-    check_bind(Z, Zo, t["C"], Y, 128, e_rec=np.full(b.M, 1e-5 * np.sqrt(1024)))
+    for method in ("direct", "spectral"):
+        Z = gs.reconstruct_bind(b, Rp[:, :b.r], cuda(Y), 128, method=method)
+        gs.stream_status()
+        Zo = orc.bind(t["C"], Y, 128)
+        check_bind(Z, Zo, t["C"], Y, 128, e_rec=np.full(b.M, 1e-5 * np.sqrt(1024)), method=method)
 
 
 def test_bind_argument_errors(gs):
@@ -107,3 +157,16 @@ def test_bind_argument_errors(gs):
     assert gs.bind(torch.zeros((0, 100), device="cuda:0"), X[:1], 50).shape == (0, 100)
     with pytest.raises(ValueError):
         gs.bind(X, X[:2], 50)
+    # the spectral method: block lengths it does not take, rows off an 8-byte boundary
+    with pytest.raises(gs.GramSpaceError) as ei:
+        gs.bind(X, X, 50, method="spectral")
+    assert ei.value.status == gs.GS_ERR_UNSUPPORTED
+    W = torch.zeros((4, 131), device="cuda:0")
+    with pytest.raises(gs.GramSpaceError) as ei:
+        gs.bind(W[:, :128], W[:, :128], 64, method="spectral")
+    assert ei.value.status == gs.GS_ERR_ALIGNMENT
+    # unknown op bits, or both methods at once
+    lib = gs.load_library()
+    p = X.data_ptr()
+    for op in (8, 2 | 4, -1):
+        assert lib.gs_bind(p, 4, 100, 100, p, 100, 50, op, p, 100, None) == gs.GS_ERR_INVALID_ARG

@@ -2,7 +2,7 @@
 times: every output computed, a seeded sample of rows checked against the oracle run with the
 GPU's own basis (so only the kernels' arithmetic differs), bounds as in the other parity tests:
 X̂ within 1e-4 ||t|| (fp16 tensor-core reconstruction), V within 1e-4 sum_i |p_i| ||c_i|| +
-2^-8 |V*| (bf16 output), binding within the fp32-sum bound plus the reconstruction error carried
+2^-8 |V*| (bf16 output), binding within the spectral method's bound plus the reconstruction error carried
 through the block (see test_bind_gpu).
 """
 import numpy as np
@@ -70,4 +70,4 @@ def test_reconstruct_bind_full_size(gs, orc):
     Tr, Yr = host(T[idx]), host(Y[idx])
     Xo = orc.reconstruct(Tr, host(b.Q))
     Zo = orc.bind(Xo, Yr, L)
-    check_bind(Z[idx], Zo, Xo, Yr, L, e_rec=1e-4 * np.linalg.norm(Tr, axis=1))
+    check_bind(Z[idx], Zo, Xo, Yr, L, e_rec=1e-4 * np.linalg.norm(Tr, axis=1), method="spectral")
