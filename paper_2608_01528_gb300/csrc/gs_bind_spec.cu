@@ -20,8 +20,11 @@
 // consecutive floats) and the last inverse pass writes the output rows, so the
 // intermediate spectra live only in shared memory.
 //
-//  k_bind_spec<H, UNB>   a CTA takes groups of U = 2048/H blocks (x and y: 4096
-//                        complex points), persistent over the grid
+//  k_bind_spec<H, UNB>   teams of T threads (a warp for L <= 512, L/16 threads above)
+//                        each take groups of U blocks (x and y: 16 T complex points in
+//                        the team's own shared buffer), persistent over the grid; a
+//                        team synchronises only itself, so teams in different phases
+//                        (loads in flight, transforms) overlap on an SM
 
 #include <stdint.h>
 
@@ -33,8 +36,11 @@ namespace gs {
 namespace {
 
 constexpr int kSpecThreads = 256;
-constexpr int kSpecPoints = 4096;                           // complex points of a forward group
-constexpr int kSpecBuf = kSpecPoints + kSpecPoints / 16;    // padded buffer length (float2)
+// threads of a team and complex points of its group (16 per thread: a radix-16 pass is one
+// butterfly per thread)
+constexpr int spec_team(int H) { return H <= 256 ? 32 : H / 8; }
+constexpr int spec_points(int H) { return 16 * spec_team(H); }
+constexpr int spec_buf(int H) { return spec_points(H) + spec_points(H) / 16; }  // padded length (float2)
 
 // one float2 of padding after every 16: the stride-R writes of a first pass and the
 // strided reads of the others then fall in distinct banks
@@ -55,12 +61,43 @@ constexpr int spec_passes(int H) { return H <= 256 ? 2 : 3; }
 // twiddle-table floats of pass p (p >= 1): (R - 1) rows of Ns entries
 constexpr int spec_ns(int H, int p) { return p == 0 ? 1 : spec_ns(H, p - 1) * spec_radix(H, p - 1); }
 constexpr int spec_tw_len(int H, int p) { return (spec_radix(H, p) - 1) * spec_ns(H, p); }
+// two padded buffers per team, then the tables
 constexpr size_t spec_smem_bytes(int H) {
-    return sizeof(float2) * ((size_t)2 * kSpecBuf + H + spec_tw_len(H, 1) + (spec_passes(H) > 2 ? spec_tw_len(H, 2) : 0));
+    return sizeof(float2) * ((size_t)(kSpecThreads / spec_team(H)) * 2 * spec_buf(H) + H + spec_tw_len(H, 1) +
+                             (spec_passes(H) > 2 ? spec_tw_len(H, 2) : 0));
 }
 
-__device__ __forceinline__ float2 c_add(float2 a, float2 b) { return make_float2(a.x + b.x, a.y + b.y); }
-__device__ __forceinline__ float2 c_sub(float2 a, float2 b) { return make_float2(a.x - b.x, a.y - b.y); }
+template <int T>
+__device__ __forceinline__ void team_sync(int team) {
+    if constexpr (T == 32) {
+        __syncwarp();
+    } else {
+        asm volatile("bar.sync %0, %1;\n" ::"r"(team + 1), "r"(T) : "memory");
+    }
+}
+
+// complex add / subtract as one paired fp32 instruction (sm_100+), lane by lane round to
+// nearest: the same results as two scalar operations
+__device__ __forceinline__ unsigned long long f2_pack(float2 a) {
+    unsigned long long r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a.x), "f"(a.y));
+    return r;
+}
+__device__ __forceinline__ float2 f2_unpack(unsigned long long v) {
+    float2 a;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(a.x), "=f"(a.y) : "l"(v));
+    return a;
+}
+__device__ __forceinline__ float2 c_add(float2 a, float2 b) {
+    unsigned long long r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(f2_pack(a)), "l"(f2_pack(b)));
+    return f2_unpack(r);
+}
+__device__ __forceinline__ float2 c_sub(float2 a, float2 b) {
+    unsigned long long r;
+    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(f2_pack(a)), "l"(f2_pack(b)));
+    return f2_unpack(r);
+}
 __device__ __forceinline__ float2 c_mul(float2 a, float2 b) {
     return make_float2(fmaf(a.x, b.x, -a.y * b.y), fmaf(a.x, b.y, a.y * b.x));
 }
@@ -129,43 +166,54 @@ struct SpecRows {
     int nb, L, ldx, ldz;
 };
 
-__device__ __forceinline__ long long unit_row(long long unit, int nb, int& b) {
-    const long long n = unit / nb;
-    b = (int)(unit - n * nb);
+// row n and block b of unit (n0, b0) + i, i < U: a few steps of b past the row's nb blocks
+__device__ __forceinline__ long long unit_row(long long n0, int b0, int i, int nb, int& b) {
+    long long n = n0;
+    b = b0 + i;
+    while (b >= nb) {
+        b -= nb;
+        ++n;
+    }
     return n;
 }
 
-// Stockham pass of radix R over sub-transforms of size NS, shared -> shared, nseq sequences
-template <int H, int R, int NS>
-__device__ __forceinline__ void spec_pass_ss(const float2* __restrict__ src, float2* __restrict__ dst, int nseq,
-                                             const float2* __restrict__ tw) {
+// Stockham pass of radix R over sub-transforms of size NS, src -> dst (a team's two buffers),
+// nseq sequences; the team synchronises at the end
+template <int H, int T, int R, int NS>
+__device__ __forceinline__ void spec_pass(const float2* __restrict__ src, float2* __restrict__ dst, int nseq,
+                                          const float2* __restrict__ tw, int t, int team) {
     constexpr int NB = H / R;
-    for (int bf = threadIdx.x; bf < nseq * NB; bf += kSpecThreads) {
+    for (int bf = t; bf < nseq * NB; bf += T) {
         const int s = bf / NB, j = bf % NB, k = j % NS;
         float2 v[R];
 #pragma unroll
         for (int r = 0; r < R; ++r) v[r] = src[pad16(s * H + j + r * NB)];
+        if constexpr (NS > 1) {
 #pragma unroll
-        for (int r = 1; r < R; ++r) v[r] = c_mul(v[r], tw[(r - 1) * NS + k]);
+            for (int r = 1; r < R; ++r) v[r] = c_mul(v[r], tw[(r - 1) * NS + k]);
+        }
         dft<R>(v);
         const int base = s * H + (j - k) * R + k;
 #pragma unroll
         for (int r = 0; r < R; ++r) dst[pad16(base + r * NS)] = v[r];
     }
+    team_sync<T>(team);
 }
 
-// first forward pass (Ns = 1, no twiddles): the 2U blocks of a group from global memory
-template <int H, int R>
-__device__ __forceinline__ void spec_pass_load(const SpecRows& p, long long u0, int U, float2* __restrict__ dst) {
-    constexpr int NB = H / R;
-    for (int bf = threadIdx.x; bf < 2 * U * NB; bf += kSpecThreads) {
+// first forward pass (Ns = 1, no twiddles) straight from the rows into dst: sequence s < U is
+// the x block of unit u0 + s, s >= U the y block of unit u0 + s - U
+template <int H, int T, int R>
+__device__ __forceinline__ void spec_pass_load(const SpecRows& p, long long u0, long long n0, int b0,
+                                               float2* __restrict__ dst, int t, int team) {
+    constexpr int U = spec_points(H) / 2 / H, NB = H / R;
+    for (int bf = t; bf < 2 * U * NB; bf += T) {
         const int s = bf / NB, j = bf % NB;
         const int i = s < U ? s : s - U;
         if (u0 + i >= p.units) continue;
         int b;
-        const long long n = unit_row(u0 + i, p.nb, b);
-        const float2* g = reinterpret_cast<const float2*>(
-            s < U ? p.X + (size_t)n * p.ldx + (size_t)b * p.L : p.Y + (size_t)n * p.ldy + (size_t)b * p.L);
+        const long long n = unit_row(n0, b0, i, p.nb, b);
+        const float* row = s < U ? p.X + (size_t)n * p.ldx : p.Y + (size_t)n * p.ldy;
+        const float2* g = reinterpret_cast<const float2*>(row + (size_t)b * p.L);
         float2 v[R];
 #pragma unroll
         for (int r = 0; r < R; ++r) v[r] = __ldcs(g + j + r * NB);
@@ -173,93 +221,102 @@ __device__ __forceinline__ void spec_pass_load(const SpecRows& p, long long u0, 
 #pragma unroll
         for (int r = 0; r < R; ++r) dst[pad16(s * H + j * R + r)] = v[r];
     }
+    team_sync<T>(team);
 }
 
 // last inverse pass: z_2n + i z_2n+1 = conj(F_n) / (8H) straight to the output rows
-template <int H, int R, int NS>
-__device__ __forceinline__ void spec_pass_store(const SpecRows& p, long long u0, int U,
-                                                const float2* __restrict__ src, const float2* __restrict__ tw) {
-    constexpr int NB = H / R;
+template <int H, int T, int R, int NS>
+__device__ __forceinline__ void spec_pass_store(const SpecRows& p, long long u0, long long n0, int b0,
+                                                const float2* __restrict__ buf, const float2* __restrict__ tw,
+                                                int t) {
+    constexpr int U = spec_points(H) / 2 / H, NB = H / R;
     static_assert(NB == NS, "the last pass completes the transform");
     constexpr float scale = 1.0f / (8.0f * H);
-    for (int bf = threadIdx.x; bf < U * NB; bf += kSpecThreads) {
+    for (int bf = t; bf < U * NB; bf += T) {
         const int s = bf / NB, j = bf % NB;
         if (u0 + s >= p.units) continue;
         float2 v[R];
 #pragma unroll
-        for (int r = 0; r < R; ++r) v[r] = src[pad16(s * H + j + r * NB)];
+        for (int r = 0; r < R; ++r) v[r] = buf[pad16(s * H + j + r * NB)];
 #pragma unroll
         for (int r = 1; r < R; ++r) v[r] = c_mul(v[r], tw[(r - 1) * NS + j]);
         dft<R>(v);
         int b;
-        const long long n = unit_row(u0 + s, p.nb, b);
+        const long long n = unit_row(n0, b0, s, p.nb, b);
         float2* g = reinterpret_cast<float2*>(p.Z + (size_t)n * p.ldz + (size_t)b * p.L);
 #pragma unroll
         for (int r = 0; r < R; ++r) __stcs(g + j + r * NS, make_float2(v[r].x * scale, -v[r].y * scale));
     }
 }
 
-// 2 X_k of a real block from W = DFT_H(packed pairs): (A + B) - i t_k (A - B),
-// A = W_k, B = conj(W_(H-k) mod H), t_k = e^{-2 pi i k / L}
-__device__ __forceinline__ float2 real_split(float2 a, float2 b_conj, float2 t) {
-    return c_add(c_add(a, b_conj), c_mul_negi(c_mul(t, c_sub(a, b_conj))));
+// 2 X_k and 2 X_H-k of a real block from W = DFT_H(packed pairs), t = e^{-2 pi i k / L}:
+// with A = W_k, B = conj(W_H-k), S = A + B and G = t (A - B),
+//   2 X_k = S - i G,   2 X_H-k = conj(S) - i conj(G)
+// (the second is the first's formula at H - k, where the roles of A and B swap and
+// t_H-k = -conj(t))
+__device__ __forceinline__ void real_split(float2 wk, float2 wm, float2 t, float2& xk, float2& xm) {
+    const float2 a = wk, b = c_conj(wm);
+    const float2 S = c_add(a, b), G = c_mul(t, c_sub(a, b));
+    xk = make_float2(S.x + G.y, S.y - G.x);
+    xm = make_float2(S.x - G.y, -S.y - G.x);
 }
 
-// point-wise pass: spectra of x (sequences 0..U-1) and y (U..2U-1) in src; writes, per block,
-// conj of the packed spectrum W''_k = (P_k + conj P_H-k) + i conj(t_k) (P_k - conj P_H-k) of the
-// product P = X Y (X conj Y to unbind), ready for the inverse transform by the forward passes
-template <int H, bool UNB>
-__device__ __forceinline__ void spec_pointwise(const float2* __restrict__ src, float2* __restrict__ dst, int U,
-                                               const float2* __restrict__ tws) {
-    constexpr int HH = H / 2;
-    for (int it = threadIdx.x; it < U * HH; it += kSpecThreads) {
+// point-wise pass, in place: from the spectra of x (sequences 0..U-1) and y (U..2U-1), writes
+// over x, per block, conj of the packed spectrum W''_k = (P_k + conj P_H-k) + i conj(t_k)
+// (P_k - conj P_H-k) of the product P = X Y (X conj Y to unbind), ready for the inverse
+// transform by forward passes.  With E = P_k + conj P_H-k and G = conj(t_k) (P_k - conj P_H-k):
+// W''_k = E + i G and W''_H-k = conj(E) + i conj(G).  A thread owns the pair (k, H - k) (and
+// k = 0 with H/2), so it alone reads and writes those positions.
+template <int H, int T, bool UNB>
+__device__ __forceinline__ void spec_pointwise(float2* __restrict__ buf, const float2* __restrict__ tws, int t,
+                                               int team) {
+    constexpr int U = spec_points(H) / 2 / H, HH = H / 2;
+    for (int it = t; it < U * HH; it += T) {
         const int i = it / HH, k = it % HH;
         // pad16(s H + k) = pad16(s H) + pad16(k): H is a multiple of 16
-        const float2* wx = src + pad16(i * H);
-        const float2* wy = src + pad16((U + i) * H);
-        float2* out = dst + pad16(i * H);
+        float2* wx = buf + pad16(i * H);
+        const float2* wy = buf + pad16((U + i) * H);
         if (k == 0) {
             // k = 0 and k = H (real: sums of the even and odd samples), k = H/2 (its own partner)
             const float2 ax = wx[pad16(0)], ay = wy[pad16(0)];
             const float p0 = 4.f * (ax.x + ax.y) * (ay.x + ay.y);
             const float ph = 4.f * (ax.x - ax.y) * (ay.x - ay.y);
-            out[pad16(0)] = make_float2(p0 + ph, ph - p0);
             const float2 bx = wx[pad16(HH)], by = wy[pad16(HH)];
             // 2 X_H/2 = 2 conj(W_H/2); W''_H/2 = 2 conj(P_H/2), stored conjugated: 2 P_H/2
             const float2 xq = make_float2(2.f * bx.x, -2.f * bx.y), yq = make_float2(2.f * by.x, -2.f * by.y);
             const float2 pq = UNB ? c_mulconj(xq, yq) : c_mul(xq, yq);
-            out[pad16(HH)] = make_float2(2.f * pq.x, 2.f * pq.y);
+            wx[pad16(0)] = make_float2(p0 + ph, ph - p0);
+            wx[pad16(HH)] = make_float2(2.f * pq.x, 2.f * pq.y);
             continue;
         }
         const int km = H - k;
-        const float2 t = tws[k];                              // e^{-2 pi i k / L}
-        const float2 tm = make_float2(-t.x, t.y);             // e^{-2 pi i (H - k) / L} = -conj(t)
-        const float2 axk = wx[pad16(k)], axm = wx[pad16(km)];
-        const float2 ayk = wy[pad16(k)], aym = wy[pad16(km)];
-        const float2 xk = real_split(axk, c_conj(axm), t), xm = real_split(axm, c_conj(axk), tm);
-        const float2 yk = real_split(ayk, c_conj(aym), t), ym = real_split(aym, c_conj(ayk), tm);
+        const float2 t1 = tws[k];  // e^{-2 pi i k / L}
+        float2 xk, xm, yk, ym;
+        real_split(wx[pad16(k)], wx[pad16(km)], t1, xk, xm);
+        real_split(wy[pad16(k)], wy[pad16(km)], t1, yk, ym);
         const float2 pk = UNB ? c_mulconj(xk, yk) : c_mul(xk, yk);
         const float2 pm = UNB ? c_mulconj(xm, ym) : c_mul(xm, ym);
-        // W''_k with conj(t_k); W''_H-k with conj(t_H-k) = -t_k
-        const float2 dk = c_sub(pk, c_conj(pm)), dm = c_sub(pm, c_conj(pk));
-        const float2 wk = c_add(c_add(pk, c_conj(pm)), c_mul_i(c_mul(c_conj(t), dk)));
-        const float2 wm = c_add(c_add(pm, c_conj(pk)), c_mul_i(c_mul(make_float2(-t.x, -t.y), dm)));
-        out[pad16(k)] = c_conj(wk);
-        out[pad16(km)] = c_conj(wm);
+        const float2 pmc = c_conj(pm);
+        const float2 E = c_add(pk, pmc), G = c_mul(c_conj(t1), c_sub(pk, pmc));
+        // stored conjugated: conj(E + iG) and conj(conj(E) + i conj(G))
+        wx[pad16(k)] = make_float2(E.x - G.y, -E.y - G.x);
+        wx[pad16(km)] = make_float2(E.x + G.y, E.y - G.x);
     }
+    team_sync<T>(team);
 }
 
 template <int H, bool UNB>
 __global__ void __launch_bounds__(kSpecThreads) k_bind_spec(SpecRows p, long long groups) {
-    constexpr int U = kSpecPoints / 2 / H;
+    constexpr int T = spec_team(H), U = spec_points(H) / 2 / H, TEAMS = kSpecThreads / T;
     constexpr int P = spec_passes(H);
     constexpr int R0 = spec_radix(H, 0), R1 = spec_radix(H, 1), R2 = spec_radix(H, 2);
     constexpr int NS1 = spec_ns(H, 1), NS2 = spec_ns(H, 2);
     extern __shared__ float2 spec_sm[];
-    float2* bufA = spec_sm;
-    float2* bufB = bufA + kSpecBuf;
-    float2* tws = bufB + kSpecBuf;  // e^{-2 pi i k / L}, k < H
-    float2* tw1 = tws + H;          // pass 1: e^{-2 pi i r k / (Ns R)}, row r - 1, column k
+    const int team = threadIdx.x / T, t = threadIdx.x % T;
+    float2* bufA = spec_sm + (size_t)team * 2 * spec_buf(H);
+    float2* bufB = bufA + spec_buf(H);
+    float2* tws = spec_sm + (size_t)TEAMS * 2 * spec_buf(H);  // e^{-2 pi i k / L}, k < H
+    float2* tw1 = tws + H;  // pass 1: e^{-2 pi i r k / (Ns R)}, row r - 1, column k
     float2* tw2 = tw1 + spec_tw_len(H, 1);
     for (int k = threadIdx.x; k < H; k += kSpecThreads) {
         float s, c;
@@ -281,56 +338,43 @@ __global__ void __launch_bounds__(kSpecThreads) k_bind_spec(SpecRows p, long lon
         }
     }
     __syncthreads();
-    for (long long g = blockIdx.x; g < groups; g += gridDim.x) {
+    const long long stride = (long long)gridDim.x * TEAMS;
+    const long long g0 = (long long)blockIdx.x * TEAMS + team;
+    // (row, block) of the group's first unit, stepped along with the group index
+    long long n0 = g0 * U / p.nb;
+    int b0 = (int)(g0 * U - n0 * p.nb);
+    const long long dn = stride * U / p.nb;
+    const int db = (int)(stride * U - dn * p.nb);
+    for (long long g = g0; g < groups; g += stride) {
         const long long u0 = g * U;
         // forward transforms of the group's x and y blocks
-        spec_pass_load<H, R0>(p, u0, U, bufA);
-        __syncthreads();
-        float2* fin;
-        float2* other;
+        spec_pass_load<H, T, R0>(p, u0, n0, b0, bufA, t, team);
+        spec_pass<H, T, R1, NS1>(bufA, bufB, 2 * U, tw1, t, team);
         if constexpr (P == 2) {
-            spec_pass_ss<H, R1, NS1>(bufA, bufB, 2 * U, tw1);
-            fin = bufB;
-            other = bufA;
+            spec_pointwise<H, T, UNB>(bufB, tws, t, team);
+            // inverse transforms of the products (forward passes on conjugated spectra)
+            spec_pass<H, T, R0, 1>(bufB, bufA, U, nullptr, t, team);
+            spec_pass_store<H, T, R1, NS1>(p, u0, n0, b0, bufA, tw1, t);
         } else {
-            spec_pass_ss<H, R1, NS1>(bufA, bufB, 2 * U, tw1);
-            __syncthreads();
-            spec_pass_ss<H, R2, NS2>(bufB, bufA, 2 * U, tw2);
-            fin = bufA;
-            other = bufB;
+            spec_pass<H, T, R2, NS2>(bufB, bufA, 2 * U, tw2, t, team);
+            spec_pointwise<H, T, UNB>(bufA, tws, t, team);
+            spec_pass<H, T, R0, 1>(bufA, bufB, U, nullptr, t, team);
+            spec_pass<H, T, R1, NS1>(bufB, bufA, U, tw1, t, team);
+            spec_pass_store<H, T, R2, NS2>(p, u0, n0, b0, bufA, tw2, t);
         }
-        __syncthreads();
-        spec_pointwise<H, UNB>(fin, other, U, tws);
-        __syncthreads();
-        // inverse transform of the products (forward passes on conjugated spectra)
-        {
-            constexpr int NB = H / R0;
-            for (int bf = threadIdx.x; bf < U * NB; bf += kSpecThreads) {
-                const int s = bf / NB, j = bf % NB;
-                float2 v[R0];
-#pragma unroll
-                for (int r = 0; r < R0; ++r) v[r] = other[pad16(s * H + j + r * NB)];
-                dft<R0>(v);
-#pragma unroll
-                for (int r = 0; r < R0; ++r) fin[pad16(s * H + j * R0 + r)] = v[r];
-            }
+        team_sync<T>(team);  // the last pass has read bufA before the next group's first pass writes it
+        n0 += dn;
+        b0 += db;
+        if (b0 >= p.nb) {
+            b0 -= p.nb;
+            ++n0;
         }
-        __syncthreads();
-        if constexpr (P == 2) {
-            spec_pass_store<H, R1, NS1>(p, u0, U, fin, tw1);
-        } else {
-            spec_pass_ss<H, R1, NS1>(fin, other, U, tw1);
-            __syncthreads();
-            spec_pass_store<H, R2, NS2>(p, u0, U, other, tw2);
-        }
-        // the next group's first pass writes bufA: every thread has passed the barrier after
-        // the last read of bufA above, and the pass that follows it reads only the other buffer
     }
 }
 
 template <int H>
 cudaError_t launch_h(const SpecRows& p, bool unbind, cudaStream_t s) {
-    constexpr int U = kSpecPoints / 2 / H;
+    constexpr int U = spec_points(H) / 2 / H, TEAMS = kSpecThreads / spec_team(H);
     constexpr size_t smem = spec_smem_bytes(H);
     static bool attr_set[2] = {false, false};
     auto kern = unbind ? k_bind_spec<H, true> : k_bind_spec<H, false>;
@@ -345,7 +389,8 @@ cudaError_t launch_h(const SpecRows& p, bool unbind, cudaStream_t s) {
     if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kSpecThreads, smem);
     if (e != cudaSuccess) return e;
     const long long groups = (p.units + U - 1) / U;
-    const long long grid = std::min<long long>(groups, (long long)std::max(sms, 1) * std::max(occ, 1));
+    const long long ctas = (groups + TEAMS - 1) / TEAMS;
+    const long long grid = std::min<long long>(ctas, (long long)std::max(sms, 1) * std::max(occ, 1));
     kern<<<(unsigned)grid, kSpecThreads, smem, s>>>(p, groups);
     return cudaGetLastError();
 }

@@ -76,11 +76,11 @@ def test_bind_matches_oracle(gs, orc, N, D, L, bcast, op):
     (5, 192, 64, False, "bind"), (70, 64, 64, True, "unbind"), (3, 256, 128, False, "unbind"),
     (37, 1024, 256, False, "bind"), (17, 256, 256, False, "unbind"), (9, 1536, 512, True, "bind"),
     (37, 1024, 1024, False, "unbind"), (3, 4096, 2048, False, "bind"), (5, 4096, 4096, False, "unbind"),
-    (3000, 1024, 64, False, "bind")])
+    (6000, 1024, 64, False, "bind")])
 def test_bind_spectral_matches_oracle(gs, orc, N, D, L, bcast, op):
     """The spectral method at every block length it takes (L = 64 ... 4096: two and three
     Stockham passes), partial last groups of blocks, one partner for all rows, padded even row
-    pitches, and 48,000 blocks (more groups than resident CTAs: the persistent loop)."""
+    pitches, and 96,000 blocks (more groups than resident teams: the persistent loop)."""
     rng = np.random.default_rng(N + D + L + 1)
     X = rng.normal(size=(N, D)).astype(np.float32)
     Y = rng.normal(size=(1 if bcast else N, D)).astype(np.float32)
