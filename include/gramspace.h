@@ -325,10 +325,10 @@ GS_API gs_status gs_bind(const float* X, long long N, int D, int ldx, const floa
  * Reconstruction followed by binding at the transition into component-wise
  * operators (Sec. 3.3: reconstruction is placed immediately before binding and
  * unbinding): Z = op(T Q, Y) with gs_reconstruct's T (N x r, t_dtype, ldt) and
- * gs_bind's Y, L, op (with its method) and Z.  The rows are processed in chunks whose
- * reconstruction (at most 64 MiB) lives in the handle's scratch between the two
- * kernels, so the reconstructed vectors stay in L2 rather than making a round
- * trip through HBM.  flags picks the reconstruction path as in gs_reconstruct.
+ * gs_bind's Y, L, op (with its method) and Z.  The rows are processed in chunks
+ * whose reconstruction lives in the handle's scratch between the two kernels
+ * (the caller needs no N x D buffer for the reconstructed vectors).  flags picks
+ * the reconstruction path as in gs_reconstruct.
  * Shares the handle's scratch with the other multi-kernel calls: order calls
  * on one handle.
  */

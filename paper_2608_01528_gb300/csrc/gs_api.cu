@@ -644,13 +644,13 @@ gs_status gs_reconstruct_bind(const gs_basis* h, const void* T, int t_dtype, lon
     DeviceGuard g(h->device);
     if (!g.ok) return GS_ERR_CUDA;
     cudaStream_t s = (cudaStream_t)stream;
-    // rows in chunks: the reconstructed chunk (at most 64 MiB, so it stays in L2 between the two
-    // kernels) and the fp16 copy of its T rows share the handle's scratch
+    // rows in chunks as large as the handle's scratch takes (the reconstructed rows and the fp16
+    // copy of their T rows): fewer, fuller reconstruction launches.  Chunks sized for L2 (64 MiB)
+    // measured slower: the GEMM's last wave per chunk cost more than the L2 hits saved.
     const int Dp = (h->D + 3) / 4 * 4, ld16 = (h->r + 7) / 8 * 8;
     if ((op & GS_BIND_SPECTRAL) && !gs::bind_spectral_supported(L, h->scratch, Dp, Y, ldy, Z, ldz))
         return bind_rows(h->scratch, 0, h->D, Dp, Y, ldy, L, op, Z, ldz, s);  // the method's error, no launch
-    long long cr = std::min(h->scratch_floats / (Dp + ld16 / 2 + 1), (64LL << 20) / (4LL * Dp));
-    cr = std::min(cr, kMaxGemmRows);
+    long long cr = std::min(h->scratch_floats / (Dp + ld16 / 2 + 1), kMaxGemmRows);
     if (cr >= 128) cr = cr / 128 * 128;
     if (cr < 1) return GS_ERR_SHAPE;
     float* xhat = h->scratch;

@@ -402,7 +402,7 @@ def bind(X, Y, L, op="bind", method="auto", out=None, stream=None):
 
 
 def reconstruct_bind(basis, T, Y, L, op="bind", path="auto", method="auto", out=None, stream=None):
-    """op(T Q, Y): reconstruction then binding, chunk by chunk through L2; see gs_reconstruct_bind
+    """op(T Q, Y): reconstruction then binding, chunk by chunk through the basis' scratch; see gs_reconstruct_bind
     (path: the reconstruction's kernels, method: the binding's, as in bind)."""
     N = T.shape[0]
     ldy = _partner(Y, N, basis.D)

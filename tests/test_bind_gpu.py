@@ -149,6 +149,27 @@ def test_reconstruct_bind_codebook_and_broadcast(gs, orc):
         check_bind(Z, Zo, t["C"], Y, 128, e_rec=np.full(b.M, 1e-5 * np.sqrt(1024)), method=method)
 
 
+def test_reconstruct_bind_several_chunks(gs, orc):
+    """3,000 rows on the tiny basis (M = 8, D = 1024), whose scratch holds 1,024 reconstructed
+    rows: three chunks, the last one partial, each reconstructed then bound before the next."""
+    t = synth.tiny()
+    b = gs.build_basis(cuda(t["C"]))
+    rng = np.random.default_rng(5)
+    N = 3000
+    P = rng.dirichlet(np.ones(b.M), size=N)
+    Tp = torch.zeros((N, 8), device="cuda:0")
+    Tp[:, :b.r] = torch.from_numpy(P).to("cuda:0", torch.float32) @ b.R
+    Y = rng.normal(size=(N, 1024)).astype(np.float32)
+    Tr = host(Tp[:, :b.r])
+    Xo = orc.reconstruct(Tr, host(b.Q))
+    for method in ("direct", "spectral"):
+        for op in ("bind", "unbind"):
+            Z = gs.reconstruct_bind(b, Tp[:, :b.r], cuda(Y), 128, op, method=method)
+            gs.stream_status()
+            Zo = orc.bind(Xo, Y, 128, orc.UNBIND if op == "unbind" else orc.BIND)
+            check_bind(Z, Zo, Xo, Y, 128, e_rec=1e-4 * np.linalg.norm(Tr, axis=1), method=method)
+
+
 def test_bind_argument_errors(gs):
     X = torch.zeros((4, 100), device="cuda:0")
     with pytest.raises(gs.GramSpaceError) as ei:
