@@ -179,9 +179,10 @@ __device__ __forceinline__ long long unit_row(long long n0, int b0, int i, int n
 
 // Stockham pass of radix R over sub-transforms of size NS, src -> dst (a team's two buffers),
 // nseq sequences; the team synchronises at the end
-template <int H, int T, int R, int NS>
+template <int H, int T, int R, int NS, bool TWR = false>
 __device__ __forceinline__ void spec_pass(const float2* __restrict__ src, float2* __restrict__ dst, int nseq,
-                                          const float2* __restrict__ tw, int t, int team) {
+                                          const float2* __restrict__ tw, int t, int team,
+                                          const float2* twr = nullptr) {
     constexpr int NB = H / R;
     for (int bf = t; bf < nseq * NB; bf += T) {
         const int s = bf / NB, j = bf % NB, k = j % NS;
@@ -190,7 +191,7 @@ __device__ __forceinline__ void spec_pass(const float2* __restrict__ src, float2
         for (int r = 0; r < R; ++r) v[r] = src[pad16(s * H + j + r * NB)];
         if constexpr (NS > 1) {
 #pragma unroll
-            for (int r = 1; r < R; ++r) v[r] = c_mul(v[r], tw[(r - 1) * NS + k]);
+            for (int r = 1; r < R; ++r) v[r] = c_mul(v[r], TWR ? twr[r - 1] : tw[(r - 1) * NS + k]);
         }
         dft<R>(v);
         const int base = s * H + (j - k) * R + k;
@@ -225,10 +226,10 @@ __device__ __forceinline__ void spec_pass_load(const SpecRows& p, long long u0, 
 }
 
 // last inverse pass: z_2n + i z_2n+1 = conj(F_n) / (8H) straight to the output rows
-template <int H, int T, int R, int NS>
+template <int H, int T, int R, int NS, bool TWR = false>
 __device__ __forceinline__ void spec_pass_store(const SpecRows& p, long long u0, long long n0, int b0,
                                                 const float2* __restrict__ buf, const float2* __restrict__ tw,
-                                                int t) {
+                                                int t, const float2* twr = nullptr) {
     constexpr int U = spec_points(H) / 2 / H, NB = H / R;
     static_assert(NB == NS, "the last pass completes the transform");
     constexpr float scale = 1.0f / (8.0f * H);
@@ -239,7 +240,7 @@ __device__ __forceinline__ void spec_pass_store(const SpecRows& p, long long u0,
 #pragma unroll
         for (int r = 0; r < R; ++r) v[r] = buf[pad16(s * H + j + r * NB)];
 #pragma unroll
-        for (int r = 1; r < R; ++r) v[r] = c_mul(v[r], tw[(r - 1) * NS + j]);
+        for (int r = 1; r < R; ++r) v[r] = c_mul(v[r], TWR ? twr[r - 1] : tw[(r - 1) * NS + j]);
         dft<R>(v);
         int b;
         const long long n = unit_row(n0, b0, s, p.nb, b);
@@ -306,7 +307,7 @@ __device__ __forceinline__ void spec_pointwise(float2* __restrict__ buf, const f
 }
 
 template <int H, bool UNB>
-__global__ void __launch_bounds__(kSpecThreads) k_bind_spec(SpecRows p, long long groups) {
+__global__ void __launch_bounds__(kSpecThreads, 3) k_bind_spec(SpecRows p, long long groups) {
     constexpr int T = spec_team(H), U = spec_points(H) / 2 / H, TEAMS = kSpecThreads / T;
     constexpr int P = spec_passes(H);
     constexpr int R0 = spec_radix(H, 0), R1 = spec_radix(H, 1), R2 = spec_radix(H, 2);
@@ -338,6 +339,14 @@ __global__ void __launch_bounds__(kSpecThreads) k_bind_spec(SpecRows p, long lon
         }
     }
     __syncthreads();
+    // two-pass warp teams: a thread's butterflies all sit at the same k = t mod NS1 in the second
+    // pass (and the last inverse pass), so it keeps those R1 - 1 twiddles in registers
+    constexpr bool TWR = P == 2 && T % NS1 == 0 && R1 <= 8;
+    float2 twr[R1 - 1];
+    if constexpr (TWR) {
+#pragma unroll
+        for (int r = 1; r < R1; ++r) twr[r - 1] = tw1[(r - 1) * NS1 + t % NS1];
+    }
     const long long stride = (long long)gridDim.x * TEAMS;
     const long long g0 = (long long)blockIdx.x * TEAMS + team;
     // (row, block) of the group's first unit, stepped along with the group index
@@ -349,12 +358,12 @@ __global__ void __launch_bounds__(kSpecThreads) k_bind_spec(SpecRows p, long lon
         const long long u0 = g * U;
         // forward transforms of the group's x and y blocks
         spec_pass_load<H, T, R0>(p, u0, n0, b0, bufA, t, team);
-        spec_pass<H, T, R1, NS1>(bufA, bufB, 2 * U, tw1, t, team);
+        spec_pass<H, T, R1, NS1, TWR>(bufA, bufB, 2 * U, tw1, t, team, twr);
         if constexpr (P == 2) {
             spec_pointwise<H, T, UNB>(bufB, tws, t, team);
             // inverse transforms of the products (forward passes on conjugated spectra)
             spec_pass<H, T, R0, 1>(bufB, bufA, U, nullptr, t, team);
-            spec_pass_store<H, T, R1, NS1>(p, u0, n0, b0, bufA, tw1, t);
+            spec_pass_store<H, T, R1, NS1, TWR>(p, u0, n0, b0, bufA, tw1, t, twr);
         } else {
             spec_pass<H, T, R2, NS2>(bufB, bufA, 2 * U, tw2, t, team);
             spec_pointwise<H, T, UNB>(bufA, tws, t, team);
