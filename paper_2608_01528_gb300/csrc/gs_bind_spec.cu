@@ -22,9 +22,9 @@
 //
 //  k_bind_spec<H, UNB>   teams of T threads (a warp for L <= 512, L/16 threads above)
 //                        each take groups of U blocks (x and y: 16 T complex points in
-//                        the team's own shared buffer), persistent over the grid; a
-//                        team synchronises only itself, so teams in different phases
-//                        (loads in flight, transforms) overlap on an SM
+//                        the team's own pair of shared buffers), persistent over the
+//                        grid; a team synchronises only itself, so teams in different
+//                        phases (loads in flight, transforms) overlap on an SM
 
 #include <stdint.h>
 
@@ -58,7 +58,7 @@ constexpr int spec_radix(int H, int p) {
                        : 1;
 }
 constexpr int spec_passes(int H) { return H <= 256 ? 2 : 3; }
-// twiddle-table floats of pass p (p >= 1): (R - 1) rows of Ns entries
+// twiddle-table entries of pass p (p >= 1): (R - 1) rows of Ns entries
 constexpr int spec_ns(int H, int p) { return p == 0 ? 1 : spec_ns(H, p - 1) * spec_radix(H, p - 1); }
 constexpr int spec_tw_len(int H, int p) { return (spec_radix(H, p) - 1) * spec_ns(H, p); }
 // two padded buffers per team, then the tables
@@ -105,7 +105,6 @@ __device__ __forceinline__ float2 c_mulconj(float2 a, float2 b) {  // a * conj(b
     return make_float2(fmaf(a.x, b.x, a.y * b.y), fmaf(a.y, b.x, -a.x * b.y));
 }
 __device__ __forceinline__ float2 c_conj(float2 a) { return make_float2(a.x, -a.y); }
-__device__ __forceinline__ float2 c_mul_i(float2 a) { return make_float2(-a.y, a.x); }     // i a
 __device__ __forceinline__ float2 c_mul_negi(float2 a) { return make_float2(a.y, -a.x); }  // -i a
 
 // z e^{-2 pi i t / 16}, t in [0, 8): the constant twiddles of butterflies up to radix 16
@@ -385,21 +384,25 @@ template <int H>
 cudaError_t launch_h(const SpecRows& p, bool unbind, cudaStream_t s) {
     constexpr int U = spec_points(H) / 2 / H, TEAMS = kSpecThreads / spec_team(H);
     constexpr size_t smem = spec_smem_bytes(H);
-    static bool attr_set[2] = {false, false};
+    // per device and operator: the shared-memory opt-in, done once, and the resident CTAs per SM
+    static int resident[64][2];
     auto kern = unbind ? k_bind_spec<H, true> : k_bind_spec<H, false>;
-    if (!attr_set[unbind]) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        attr_set[unbind] = true;
-    }
-    int dev = 0, sms = 0, occ = 0;
+    int dev = 0, sms = 0;
     cudaError_t e = cudaGetDevice(&dev);
-    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kSpecThreads, smem);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (resident[dev][unbind] == 0) {
+        int occ = 0;
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kSpecThreads, smem);
+        if (e != cudaSuccess) return e;
+        resident[dev][unbind] = std::max(occ, 1);
+    }
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
     const long long groups = (p.units + U - 1) / U;
     const long long ctas = (groups + TEAMS - 1) / TEAMS;
-    const long long grid = std::min<long long>(ctas, (long long)std::max(sms, 1) * std::max(occ, 1));
+    const long long grid = std::min<long long>(ctas, (long long)std::max(sms, 1) * resident[dev][unbind]);
     kern<<<(unsigned)grid, kSpecThreads, smem, s>>>(p, groups);
     return cudaGetLastError();
 }
