@@ -313,6 +313,7 @@ GS_API gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, l
  *     carried through the product and the inverse; typical errors are far
  *     smaller than the direct sum's.
  *   neither: GS_BIND_SPECTRAL where it applies, else GS_BIND_DIRECT.
+ * Z must not overlap X or Y.
  * Errors: GS_ERR_SHAPE (L does not divide D, ld too small), GS_ERR_INVALID_ARG
  * (unknown op or both methods), GS_ERR_UNSUPPORTED (GS_BIND_SPECTRAL with an L
  * it does not take), GS_ERR_ALIGNMENT (GS_BIND_SPECTRAL with a pointer or ld
