@@ -287,7 +287,7 @@ GS_API gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, l
 #define GS_UNBIND 1 /* block circular correlation  */
 #define GS_BIND_DIRECT 2   /* the direct sum: one fp32 sum of L products per output    */
 #define GS_BIND_SPECTRAL 4 /* through block spectra (convolution theorem): L a power
-                              of two in [64, 4096], rows 8-byte aligned               */
+                              of two in [64, 8192], rows 8-byte aligned               */
 
 /*
  * Binding and unbinding, the component-wise operators of rule execution

@@ -35,11 +35,13 @@
 namespace gs {
 namespace {
 
-constexpr int kSpecThreads = 256;
 // threads of a team and complex points of its group (16 per thread: a radix-16 pass is one
-// butterfly per thread)
+// butterfly per thread), threads of a CTA (256, or one team of 512 for H = 4096) and CTAs an
+// SM should hold (the register budget: 85 a thread at 3 CTAs of 256)
 constexpr int spec_team(int H) { return H <= 256 ? 32 : H / 8; }
 constexpr int spec_points(int H) { return 16 * spec_team(H); }
+constexpr int spec_cta(int H) { return spec_team(H) > 256 ? spec_team(H) : 256; }
+constexpr int spec_min_ctas(int H) { return spec_cta(H) > 256 ? 1 : 3; }
 constexpr int spec_buf(int H) { return spec_points(H) + spec_points(H) / 16; }  // padded length (float2)
 
 // one float2 of padding after every 16: the stride-R writes of a first pass and the
@@ -55,6 +57,7 @@ constexpr int spec_radix(int H, int p) {
            : H == 512  ? 8
            : H == 1024 ? (p == 0 ? 16 : 8)
            : H == 2048 ? (p < 2 ? 16 : 8)
+           : H == 4096 ? 16
                        : 1;
 }
 constexpr int spec_passes(int H) { return H <= 256 ? 2 : 3; }
@@ -63,7 +66,7 @@ constexpr int spec_ns(int H, int p) { return p == 0 ? 1 : spec_ns(H, p - 1) * sp
 constexpr int spec_tw_len(int H, int p) { return (spec_radix(H, p) - 1) * spec_ns(H, p); }
 // two padded buffers per team, then the tables
 constexpr size_t spec_smem_bytes(int H) {
-    return sizeof(float2) * ((size_t)(kSpecThreads / spec_team(H)) * 2 * spec_buf(H) + H + spec_tw_len(H, 1) +
+    return sizeof(float2) * ((size_t)(spec_cta(H) / spec_team(H)) * 2 * spec_buf(H) + H + spec_tw_len(H, 1) +
                              (spec_passes(H) > 2 ? spec_tw_len(H, 2) : 0));
 }
 
@@ -306,8 +309,8 @@ __device__ __forceinline__ void spec_pointwise(float2* __restrict__ buf, const f
 }
 
 template <int H, bool UNB>
-__global__ void __launch_bounds__(kSpecThreads, 3) k_bind_spec(SpecRows p, long long groups) {
-    constexpr int T = spec_team(H), U = spec_points(H) / 2 / H, TEAMS = kSpecThreads / T;
+__global__ void __launch_bounds__(spec_cta(H), spec_min_ctas(H)) k_bind_spec(SpecRows p, long long groups) {
+    constexpr int T = spec_team(H), U = spec_points(H) / 2 / H, NT = spec_cta(H), TEAMS = NT / T;
     constexpr int P = spec_passes(H);
     constexpr int R0 = spec_radix(H, 0), R1 = spec_radix(H, 1), R2 = spec_radix(H, 2);
     constexpr int NS1 = spec_ns(H, 1), NS2 = spec_ns(H, 2);
@@ -318,19 +321,19 @@ __global__ void __launch_bounds__(kSpecThreads, 3) k_bind_spec(SpecRows p, long 
     float2* tws = spec_sm + (size_t)TEAMS * 2 * spec_buf(H);  // e^{-2 pi i k / L}, k < H
     float2* tw1 = tws + H;  // pass 1: e^{-2 pi i r k / (Ns R)}, row r - 1, column k
     float2* tw2 = tw1 + spec_tw_len(H, 1);
-    for (int k = threadIdx.x; k < H; k += kSpecThreads) {
+    for (int k = threadIdx.x; k < H; k += NT) {
         float s, c;
         sincospif((float)k / (float)H, &s, &c);
         tws[k] = make_float2(c, -s);
     }
-    for (int e = threadIdx.x; e < spec_tw_len(H, 1); e += kSpecThreads) {
+    for (int e = threadIdx.x; e < spec_tw_len(H, 1); e += NT) {
         const int r = e / NS1 + 1, k = e % NS1;
         float s, c;
         sincospif(2.0f * (float)(r * k) / (float)(NS1 * R1), &s, &c);
         tw1[e] = make_float2(c, -s);
     }
     if constexpr (P > 2) {
-        for (int e = threadIdx.x; e < spec_tw_len(H, 2); e += kSpecThreads) {
+        for (int e = threadIdx.x; e < spec_tw_len(H, 2); e += NT) {
             const int r = e / NS2 + 1, k = e % NS2;
             float s, c;
             sincospif(2.0f * (float)(r * k) / (float)(NS2 * R2), &s, &c);
@@ -382,7 +385,7 @@ __global__ void __launch_bounds__(kSpecThreads, 3) k_bind_spec(SpecRows p, long 
 
 template <int H>
 cudaError_t launch_h(const SpecRows& p, bool unbind, cudaStream_t s) {
-    constexpr int U = spec_points(H) / 2 / H, TEAMS = kSpecThreads / spec_team(H);
+    constexpr int U = spec_points(H) / 2 / H, NT = spec_cta(H), TEAMS = NT / spec_team(H);
     constexpr size_t smem = spec_smem_bytes(H);
     // per device and operator: the shared-memory opt-in, done once, and the resident CTAs per SM
     static int resident[64][2];
@@ -394,7 +397,7 @@ cudaError_t launch_h(const SpecRows& p, bool unbind, cudaStream_t s) {
     if (resident[dev][unbind] == 0) {
         int occ = 0;
         e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kSpecThreads, smem);
+        if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, NT, smem);
         if (e != cudaSuccess) return e;
         resident[dev][unbind] = std::max(occ, 1);
     }
@@ -403,7 +406,7 @@ cudaError_t launch_h(const SpecRows& p, bool unbind, cudaStream_t s) {
     const long long groups = (p.units + U - 1) / U;
     const long long ctas = (groups + TEAMS - 1) / TEAMS;
     const long long grid = std::min<long long>(ctas, (long long)std::max(sms, 1) * resident[dev][unbind]);
-    kern<<<(unsigned)grid, kSpecThreads, smem, s>>>(p, groups);
+    kern<<<(unsigned)grid, NT, smem, s>>>(p, groups);
     return cudaGetLastError();
 }
 
@@ -437,6 +440,7 @@ cudaError_t launch_bind_spectral(const float* X, long long N, int D, int ldx, co
         case 1024: return launch_h<512>(p, unbind, s);
         case 2048: return launch_h<1024>(p, unbind, s);
         case 4096: return launch_h<2048>(p, unbind, s);
+        case 8192: return launch_h<4096>(p, unbind, s);
         default: return cudaErrorInvalidValue;
     }
 }

@@ -145,7 +145,7 @@ cudaError_t launch_bind(const float* X, long long N, int D, int ldx, const float
 // the same through block spectra (gs_bind_spec.cu): L a power of two in [kMinBindSpectralL,
 // kMaxBindSpectralL], rows 8-byte aligned (bind_spectral_supported)
 constexpr int kMinBindSpectralL = 64;
-constexpr int kMaxBindSpectralL = 4096;
+constexpr int kMaxBindSpectralL = 8192;
 bool bind_spectral_supported(int L, const float* X, int ldx, const float* Y, long long ldy, const float* Z, int ldz);
 cudaError_t launch_bind_spectral(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L,
                                  bool unbind, float* Z, int ldz, cudaStream_t s);

@@ -29,10 +29,6 @@ def block_norms(A, L):
     return np.sqrt((A.astype(np.float64).reshape(N, D // L, L) ** 2).sum(axis=2))
 
 
-def spectral_applies(L):
-    return 64 <= L <= 4096 and L & (L - 1) == 0
-
-
 def bind_error_factor(L, method):
     if method == "direct":
         return L * 2.0 ** -22
@@ -76,10 +72,11 @@ def test_bind_matches_oracle(gs, orc, N, D, L, bcast, op):
     (5, 192, 64, False, "bind"), (70, 64, 64, True, "unbind"), (3, 256, 128, False, "unbind"),
     (37, 1024, 256, False, "bind"), (17, 256, 256, False, "unbind"), (9, 1536, 512, True, "bind"),
     (37, 1024, 1024, False, "unbind"), (3, 4096, 2048, False, "bind"), (5, 4096, 4096, False, "unbind"),
-    (6000, 1024, 64, False, "bind")])
+    (2, 8192, 8192, False, "bind"), (3, 16384, 8192, True, "unbind"), (6000, 1024, 64, False, "bind")])
 def test_bind_spectral_matches_oracle(gs, orc, N, D, L, bcast, op):
-    """The spectral method at every block length it takes (L = 64 ... 4096: two and three
-    Stockham passes), partial last groups of blocks, one partner for all rows, padded even row
+    """The spectral method at every block length it takes (L = 64 ... 8192: two and three
+    Stockham passes; L = 8192 as whole-vector binding of D = 8192 rows, on 512-thread CTAs),
+    partial last groups of blocks, one partner for all rows, padded even row
     pitches, and 96,000 blocks (more groups than resident teams: the persistent loop)."""
     rng = np.random.default_rng(N + D + L + 1)
     X = rng.normal(size=(N, D)).astype(np.float32)
