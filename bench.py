@@ -457,6 +457,8 @@ def side_rows(gs, dev):
     # binding through block spectra (the default): X, Y read and Z written once, 12 D bytes a row
     ms_bind = timeit(lambda: gs.bind(Xb, Yb, Lb, out=Zb))
     bind_bytes = 3 * Nb * b5.D * 4
+    # one partner row for every row (its block spectra computed once per CTA): 8 D bytes a row
+    ms_bcast = timeit(lambda: gs.bind(Xb, Yb[:1], Lb, out=Zb))
     # the direct sum for comparison: 2 L flops per output on the fp32 lanes
     ms_direct = timeit(lambda: gs.bind(Xb, Yb, Lb, method="direct", out=Zb))
     direct_tflops = 2 * Nb * b5.D * Lb / (ms_direct / 1e3) / 1e12
@@ -464,6 +466,7 @@ def side_rows(gs, dev):
                                "reconstruct_ms": round(ms_rec, 4), "bind_ms": round(ms_bind, 4),
                                "bind_gbs": round(bind_bytes / (ms_bind / 1e3) / 1e9, 1), "bound": "hbm",
                                "frac": round(bind_bytes / (ms_bind / 1e3) / 1e9 / peaks["hbm_gbs"], 4),
+                               "bind_one_partner_ms": round(ms_bcast, 4),
                                "bind_direct_ms": round(ms_direct, 4), "bind_direct_tflops": round(direct_tflops, 1),
                                "bind_direct_alu_frac": round(direct_tflops / FP32_PEAK_TFLOPS, 4)}
     del b4, b5, Xb, Yb, Zb

@@ -158,7 +158,7 @@ __device__ __forceinline__ void dft(float2 (&v)[R]) {
     for (int i = 0; i < R; ++i) v[i] = t[i];
 }
 
-// Sequence s of a group (s < U: x of block u0 + s; s >= U: y of block u0 + s - U) in global memory.
+// The rows of one launch: X, Y (ldy = 0: Y's one row partners every row), Z; N rows of nb blocks.
 struct SpecRows {
     const float* X;
     const float* Y;
@@ -204,18 +204,20 @@ __device__ __forceinline__ void spec_pass(const float2* __restrict__ src, float2
 }
 
 // first forward pass (Ns = 1, no twiddles) straight from the rows into dst: sequence s < U is
-// the x block of unit u0 + s, s >= U the y block of unit u0 + s - U
-template <int H, int T, int R>
+// the x block of unit u0 + s, s >= U the y block of unit u0 + s - U (BC: all 2U sequences are x
+// blocks, units u0 .. u0 + 2U - 1)
+template <int H, int T, int R, bool BC>
 __device__ __forceinline__ void spec_pass_load(const SpecRows& p, long long u0, long long n0, int b0,
                                                float2* __restrict__ dst, int t, int team) {
     constexpr int U = spec_points(H) / 2 / H, NB = H / R;
     for (int bf = t; bf < 2 * U * NB; bf += T) {
         const int s = bf / NB, j = bf % NB;
-        const int i = s < U ? s : s - U;
+        const bool isx = BC || s < U;
+        const int i = isx ? s : s - U;
         if (u0 + i >= p.units) continue;
         int b;
         const long long n = unit_row(n0, b0, i, p.nb, b);
-        const float* row = s < U ? p.X + (size_t)n * p.ldx : p.Y + (size_t)n * p.ldy;
+        const float* row = isx ? p.X + (size_t)n * p.ldx : p.Y + (size_t)n * p.ldy;
         const float2* g = reinterpret_cast<const float2*>(row + (size_t)b * p.L);
         float2 v[R];
 #pragma unroll
@@ -228,14 +230,14 @@ __device__ __forceinline__ void spec_pass_load(const SpecRows& p, long long u0, 
 }
 
 // last inverse pass: z_2n + i z_2n+1 = conj(F_n) / (8H) straight to the output rows
-template <int H, int T, int R, int NS, bool TWR = false>
+template <int H, int T, int R, int NS, int UX, bool TWR = false>
 __device__ __forceinline__ void spec_pass_store(const SpecRows& p, long long u0, long long n0, int b0,
                                                 const float2* __restrict__ buf, const float2* __restrict__ tw,
                                                 int t, const float2* twr = nullptr) {
-    constexpr int U = spec_points(H) / 2 / H, NB = H / R;
+    constexpr int NB = H / R;
     static_assert(NB == NS, "the last pass completes the transform");
     constexpr float scale = 1.0f / (8.0f * H);
-    for (int bf = t; bf < U * NB; bf += T) {
+    for (int bf = t; bf < UX * NB; bf += T) {
         const int s = bf / NB, j = bf % NB;
         if (u0 + s >= p.units) continue;
         float2 v[R];
@@ -269,16 +271,24 @@ __device__ __forceinline__ void real_split(float2 wk, float2 wm, float2 t, float
 // (P_k - conj P_H-k) of the product P = X Y (X conj Y to unbind), ready for the inverse
 // transform by forward passes.  With E = P_k + conj P_H-k and G = conj(t_k) (P_k - conj P_H-k):
 // W''_k = E + i G and W''_H-k = conj(E) + i conj(G).  A thread owns the pair (k, H - k) (and
-// k = 0 with H/2), so it alone reads and writes those positions.
-template <int H, int T, bool UNB>
-__device__ __forceinline__ void spec_pointwise(float2* __restrict__ buf, const float2* __restrict__ tws, int t,
-                                               int team) {
-    constexpr int U = spec_points(H) / 2 / H, HH = H / 2;
-    for (int it = t; it < U * HH; it += T) {
+// k = 0 with H/2), so it alone reads and writes those positions.  BC: all 2U sequences are x
+// spectra and y's spectrum of block b is ytab + pad16(b H), shared by every row.
+template <int H, int T, bool UNB, bool BC>
+__device__ __forceinline__ void spec_pointwise(float2* __restrict__ buf, const float2* __restrict__ tws,
+                                               const float2* __restrict__ ytab, int b0, int nb, int t, int team) {
+    constexpr int U = spec_points(H) / 2 / H, HH = H / 2, UX = BC ? 2 * U : U;
+    for (int it = t; it < UX * HH; it += T) {
         const int i = it / HH, k = it % HH;
         // pad16(s H + k) = pad16(s H) + pad16(k): H is a multiple of 16
         float2* wx = buf + pad16(i * H);
-        const float2* wy = buf + pad16((U + i) * H);
+        const float2* wy;
+        if constexpr (BC) {
+            int b;
+            unit_row(0, b0, i, nb, b);
+            wy = ytab + pad16(b * H);
+        } else {
+            wy = buf + pad16((U + i) * H);
+        }
         if (k == 0) {
             // k = 0 and k = H (real: sums of the even and odd samples), k = H/2 (its own partner)
             const float2 ax = wx[pad16(0)], ay = wy[pad16(0)];
@@ -308,9 +318,10 @@ __device__ __forceinline__ void spec_pointwise(float2* __restrict__ buf, const f
     team_sync<T>(team);
 }
 
-template <int H, bool UNB>
+template <int H, bool UNB, bool BC>
 __global__ void __launch_bounds__(spec_cta(H), spec_min_ctas(H)) k_bind_spec(SpecRows p, long long groups) {
     constexpr int T = spec_team(H), U = spec_points(H) / 2 / H, NT = spec_cta(H), TEAMS = NT / T;
+    constexpr int UX = BC ? 2 * U : U;  // blocks of x a group transforms
     constexpr int P = spec_passes(H);
     constexpr int R0 = spec_radix(H, 0), R1 = spec_radix(H, 1), R2 = spec_radix(H, 2);
     constexpr int NS1 = spec_ns(H, 1), NS2 = spec_ns(H, 2);
@@ -321,6 +332,7 @@ __global__ void __launch_bounds__(spec_cta(H), spec_min_ctas(H)) k_bind_spec(Spe
     float2* tws = spec_sm + (size_t)TEAMS * 2 * spec_buf(H);  // e^{-2 pi i k / L}, k < H
     float2* tw1 = tws + H;  // pass 1: e^{-2 pi i r k / (Ns R)}, row r - 1, column k
     float2* tw2 = tw1 + spec_tw_len(H, 1);
+    float2* ytab = tw2 + (P > 2 ? spec_tw_len(H, 2) : 0);  // BC: y's spectrum of each block
     for (int k = threadIdx.x; k < H; k += NT) {
         float s, c;
         sincospif((float)k / (float)H, &s, &c);
@@ -349,29 +361,53 @@ __global__ void __launch_bounds__(spec_cta(H), spec_min_ctas(H)) k_bind_spec(Spe
 #pragma unroll
         for (int r = 1; r < R1; ++r) twr[r - 1] = tw1[(r - 1) * NS1 + t % NS1];
     }
+    if constexpr (BC) {
+        // the one partner row's block spectra, once per CTA: team by team, block by block
+        constexpr int NB0 = H / R0;
+        for (int b = team; b < p.nb; b += TEAMS) {
+            const float2* g = reinterpret_cast<const float2*>(p.Y + (size_t)b * p.L);
+            for (int j = t; j < NB0; j += T) {
+                float2 v[R0];
+#pragma unroll
+                for (int r = 0; r < R0; ++r) v[r] = __ldg(g + j + r * NB0);
+                dft<R0>(v);
+#pragma unroll
+                for (int r = 0; r < R0; ++r) bufA[pad16(j * R0 + r)] = v[r];
+            }
+            team_sync<T>(team);
+            float2* yb = ytab + pad16(b * H);
+            if constexpr (P == 2) {
+                spec_pass<H, T, R1, NS1, TWR>(bufA, yb, 1, tw1, t, team, twr);
+            } else {
+                spec_pass<H, T, R1, NS1>(bufA, bufB, 1, tw1, t, team);
+                spec_pass<H, T, R2, NS2>(bufB, yb, 1, tw2, t, team);
+            }
+        }
+        __syncthreads();
+    }
     const long long stride = (long long)gridDim.x * TEAMS;
     const long long g0 = (long long)blockIdx.x * TEAMS + team;
     // (row, block) of the group's first unit, stepped along with the group index
-    long long n0 = g0 * U / p.nb;
-    int b0 = (int)(g0 * U - n0 * p.nb);
-    const long long dn = stride * U / p.nb;
-    const int db = (int)(stride * U - dn * p.nb);
+    long long n0 = g0 * UX / p.nb;
+    int b0 = (int)(g0 * UX - n0 * p.nb);
+    const long long dn = stride * UX / p.nb;
+    const int db = (int)(stride * UX - dn * p.nb);
     for (long long g = g0; g < groups; g += stride) {
-        const long long u0 = g * U;
-        // forward transforms of the group's x and y blocks
-        spec_pass_load<H, T, R0>(p, u0, n0, b0, bufA, t, team);
+        const long long u0 = g * UX;
+        // forward transforms of the group's x (and y) blocks
+        spec_pass_load<H, T, R0, BC>(p, u0, n0, b0, bufA, t, team);
         spec_pass<H, T, R1, NS1, TWR>(bufA, bufB, 2 * U, tw1, t, team, twr);
         if constexpr (P == 2) {
-            spec_pointwise<H, T, UNB>(bufB, tws, t, team);
+            spec_pointwise<H, T, UNB, BC>(bufB, tws, ytab, b0, p.nb, t, team);
             // inverse transforms of the products (forward passes on conjugated spectra)
-            spec_pass<H, T, R0, 1>(bufB, bufA, U, nullptr, t, team);
-            spec_pass_store<H, T, R1, NS1, TWR>(p, u0, n0, b0, bufA, tw1, t, twr);
+            spec_pass<H, T, R0, 1>(bufB, bufA, UX, nullptr, t, team);
+            spec_pass_store<H, T, R1, NS1, UX, TWR>(p, u0, n0, b0, bufA, tw1, t, twr);
         } else {
             spec_pass<H, T, R2, NS2>(bufB, bufA, 2 * U, tw2, t, team);
-            spec_pointwise<H, T, UNB>(bufA, tws, t, team);
-            spec_pass<H, T, R0, 1>(bufA, bufB, U, nullptr, t, team);
-            spec_pass<H, T, R1, NS1>(bufB, bufA, U, tw1, t, team);
-            spec_pass_store<H, T, R2, NS2>(p, u0, n0, b0, bufA, tw2, t);
+            spec_pointwise<H, T, UNB, BC>(bufA, tws, ytab, b0, p.nb, t, team);
+            spec_pass<H, T, R0, 1>(bufA, bufB, UX, nullptr, t, team);
+            spec_pass<H, T, R1, NS1>(bufB, bufA, UX, tw1, t, team);
+            spec_pass_store<H, T, R2, NS2, UX>(p, u0, n0, b0, bufA, tw2, t);
         }
         team_sync<T>(team);  // the last pass has read bufA before the next group's first pass writes it
         n0 += dn;
@@ -383,29 +419,37 @@ __global__ void __launch_bounds__(spec_cta(H), spec_min_ctas(H)) k_bind_spec(Spe
     }
 }
 
+constexpr size_t kSpecSmemCap = 227 * 1024;
+
 template <int H>
 cudaError_t launch_h(const SpecRows& p, bool unbind, cudaStream_t s) {
     constexpr int U = spec_points(H) / 2 / H, NT = spec_cta(H), TEAMS = NT / spec_team(H);
-    constexpr size_t smem = spec_smem_bytes(H);
-    // per device and operator: the shared-memory opt-in, done once, and the resident CTAs per SM
-    static int resident[64][2];
-    auto kern = unbind ? k_bind_spec<H, true> : k_bind_spec<H, false>;
-    int dev = 0, sms = 0;
+    // one partner row: its block spectra are computed once per CTA and kept in shared memory
+    // (nb padded blocks after the tables) when they fit
+    const size_t ytab = sizeof(float2) * (size_t)p.nb * (H + H / 16);
+    const bool bc = p.ldy == 0 && spec_smem_bytes(H) + ytab <= kSpecSmemCap;
+    const size_t smem = spec_smem_bytes(H) + (bc ? ytab : 0);
+    // per device, operator and partner layout: the shared-memory opt-in (to the cap), done once;
+    // the resident CTAs per SM for this launch's shared memory
+    static bool opted[64][2][2];
+    auto kern = bc ? (unbind ? k_bind_spec<H, true, true> : k_bind_spec<H, false, true>)
+                   : (unbind ? k_bind_spec<H, true, false> : k_bind_spec<H, false, false>);
+    int dev = 0, sms = 0, occ = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-    if (resident[dev][unbind] == 0) {
-        int occ = 0;
-        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, NT, smem);
+    if (!opted[dev][unbind][bc]) {
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSpecSmemCap);
         if (e != cudaSuccess) return e;
-        resident[dev][unbind] = std::max(occ, 1);
+        opted[dev][unbind][bc] = true;
     }
-    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, NT, smem);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
-    const long long groups = (p.units + U - 1) / U;
+    const long long per_group = bc ? 2 * U : U;
+    const long long groups = (p.units + per_group - 1) / per_group;
     const long long ctas = (groups + TEAMS - 1) / TEAMS;
-    const long long grid = std::min<long long>(ctas, (long long)std::max(sms, 1) * resident[dev][unbind]);
+    const long long grid = std::min<long long>(ctas, (long long)std::max(sms, 1) * std::max(occ, 1));
     kern<<<(unsigned)grid, NT, smem, s>>>(p, groups);
     return cudaGetLastError();
 }

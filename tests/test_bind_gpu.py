@@ -72,11 +72,15 @@ def test_bind_matches_oracle(gs, orc, N, D, L, bcast, op):
     (5, 192, 64, False, "bind"), (70, 64, 64, True, "unbind"), (3, 256, 128, False, "unbind"),
     (37, 1024, 256, False, "bind"), (17, 256, 256, False, "unbind"), (9, 1536, 512, True, "bind"),
     (37, 1024, 1024, False, "unbind"), (3, 4096, 2048, False, "bind"), (5, 4096, 4096, False, "unbind"),
-    (2, 8192, 8192, False, "bind"), (3, 16384, 8192, True, "unbind"), (6000, 1024, 64, False, "bind")])
+    (2, 8192, 8192, False, "bind"), (3, 16384, 8192, True, "unbind"), (6000, 1024, 64, False, "bind"),
+    (7, 4096, 1024, True, "bind"), (5, 8192, 4096, True, "unbind"), (40, 2048, 128, True, "unbind"),
+    (6000, 1024, 64, True, "unbind")])
 def test_bind_spectral_matches_oracle(gs, orc, N, D, L, bcast, op):
     """The spectral method at every block length it takes (L = 64 ... 8192: two and three
     Stockham passes; L = 8192 as whole-vector binding of D = 8192 rows, on 512-thread CTAs),
-    partial last groups of blocks, one partner for all rows, padded even row
+    partial last groups of blocks, one partner for all rows (its block spectra cached in shared
+    memory, two- and three-pass plans; at L = 8192 they do not fit and every team transforms the
+    partner itself), padded even row
     pitches, and 96,000 blocks (more groups than resident teams: the persistent loop)."""
     rng = np.random.default_rng(N + D + L + 1)
     X = rng.normal(size=(N, D)).astype(np.float32)
