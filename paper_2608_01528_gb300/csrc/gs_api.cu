@@ -605,16 +605,19 @@ static gs_status check_bind_args(long long N, int D, int ldx, long long ldy, int
     return GS_OK;
 }
 
+// why a forced spectral method cannot run: a block length it does not take, else alignment
+static gs_status spectral_error(int L) {
+    const bool l_ok = L >= gs::kMinBindSpectralL && L <= gs::kMaxBindSpectralL && !(L & (L - 1));
+    return l_ok ? GS_ERR_ALIGNMENT : GS_ERR_UNSUPPORTED;
+}
+
 // one binding launch: the spectral kernel unless the direct sum is asked for or the spectral
 // kernel cannot take the shape; a forced spectral method that cannot run is an error
 static gs_status bind_rows(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L, int op,
                            float* Z, int ldz, cudaStream_t s) {
     const bool unbind = (op & GS_UNBIND) != 0;
     const bool spec = gs::bind_spectral_supported(L, X, ldx, Y, ldy, Z, ldz);
-    if ((op & GS_BIND_SPECTRAL) && !spec) {
-        const bool l_ok = L >= gs::kMinBindSpectralL && L <= gs::kMaxBindSpectralL && !(L & (L - 1));
-        return l_ok ? GS_ERR_ALIGNMENT : GS_ERR_UNSUPPORTED;
-    }
+    if ((op & GS_BIND_SPECTRAL) && !spec) return spectral_error(L);
     if (spec && !(op & GS_BIND_DIRECT))
         return from_cuda(gs::launch_bind_spectral(X, N, D, ldx, Y, ldy, L, unbind, Z, ldz, s));
     return from_cuda(gs::launch_bind(X, N, D, ldx, Y, ldy, L, unbind, Z, ldz, s));
@@ -649,7 +652,7 @@ gs_status gs_reconstruct_bind(const gs_basis* h, const void* T, int t_dtype, lon
     // measured slower: the GEMM's last wave per chunk cost more than the L2 hits saved.
     const int Dp = (h->D + 3) / 4 * 4, ld16 = (h->r + 7) / 8 * 8;
     if ((op & GS_BIND_SPECTRAL) && !gs::bind_spectral_supported(L, h->scratch, Dp, Y, ldy, Z, ldz))
-        return bind_rows(h->scratch, 0, h->D, Dp, Y, ldy, L, op, Z, ldz, s);  // the method's error, no launch
+        return spectral_error(L);
     long long cr = std::min(h->scratch_floats / (Dp + ld16 / 2 + 1), kMaxGemmRows);
     if (cr >= 128) cr = cr / 128 * 128;
     if (cr < 1) return GS_ERR_SHAPE;
