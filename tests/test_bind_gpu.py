@@ -187,6 +187,14 @@ def test_bind_argument_errors(gs):
     with pytest.raises(gs.GramSpaceError) as ei:
         gs.bind(W[:, :128], W[:, :128], 64, method="spectral")
     assert ei.value.status == gs.GS_ERR_ALIGNMENT
+    # the fused call checks the forced method before it reconstructs anything
+    t = synth.tiny()
+    b = gs.build_basis(cuda(t["C"]))
+    Zr = torch.full((4, 1024), 5.0, device="cuda:0")
+    with pytest.raises(gs.GramSpaceError) as ei:
+        gs.reconstruct_bind(b, b.R[:4], torch.zeros((4, 1024), device="cuda:0"), 32, method="spectral", out=Zr)
+    assert ei.value.status == gs.GS_ERR_UNSUPPORTED
+    assert torch.all(Zr == 5.0)
     # unknown op bits, or both methods at once
     lib = gs.load_library()
     p = X.data_ptr()
