@@ -56,3 +56,18 @@ def test_host_side_argument_checks_need_no_device(lib):
     assert lib.gs_attention_scores(None, None, 5, 1, 1, 1, 1, 1, 1.0, 1, None, 0, None) == g.GS_ERR_INVALID_ARG
     assert lib.gs_attention_scores(None, None, 0, 1, 1, 1, 4, 2, 1.0, 1, None, 0, None) == g.GS_ERR_SHAPE
     assert lib.gs_attention_scores(None, None, 0, 0, 4, 4, 4, 4, 1.0, 1, None, 0, None) == g.GS_OK
+
+
+def test_bind_argument_checks_need_no_device(lib):
+    """gs_bind rejects unknown operator bits, both methods at once and inconsistent shapes on
+    the host; N = 0 is a no-op."""
+    from paper_2608_01528_gb300 import gramspace as g
+    dummy = 16  # never dereferenced: every call below returns before touching memory
+    for op in (8, g.BIND_METHODS["direct"] | g.BIND_METHODS["spectral"], -1):
+        assert lib.gs_bind(dummy, 4, 100, 100, dummy, 100, 50, op, dummy, 100, None) == g.GS_ERR_INVALID_ARG
+    assert lib.gs_bind(dummy, 4, 100, 100, dummy, 100, 30, 0, dummy, 100, None) == g.GS_ERR_SHAPE  # L | D
+    assert lib.gs_bind(dummy, 4, 100, 99, dummy, 100, 50, 0, dummy, 100, None) == g.GS_ERR_SHAPE  # ldx < D
+    assert lib.gs_bind(dummy, 4, 100, 100, dummy, 60, 50, 0, dummy, 100, None) == g.GS_ERR_SHAPE  # 0 < ldy < D
+    assert lib.gs_bind(dummy, 0, 100, 100, dummy, 0, 50, g.BIND_METHODS["spectral"], dummy, 100,
+                       None) == g.GS_OK
+    assert lib.gs_bind(None, 4, 100, 100, None, 0, 50, 0, None, 100, None) == g.GS_ERR_INVALID_ARG
