@@ -97,6 +97,51 @@ def traffic_record(kernel_file, key):
         return None
 
 
+def _cpulist(text):
+    cpus = set()
+    for part in text.strip().split(","):
+        if not part:
+            continue
+        a, _, b = part.partition("-")
+        cpus.update(range(int(a), int(b or a) + 1))
+    return cpus
+
+
+class NearGpuHost:
+    """Runs the calling thread on the CPUs attached to the GPU while host buffers are pinned, so
+    the pinned pages land on the GPU's NUMA node (pages pinned on the far socket of a two-socket
+    node cross the socket link on every host <-> device copy); the affinity is restored after."""
+
+    def __init__(self, index):
+        self.index = index
+        self.saved = None
+        self.node = None
+        self.cpus = 0
+
+    def __enter__(self):
+        import torch
+        try:
+            p = torch.cuda.get_device_properties(self.index)
+            bus = "%04x:%02x:%02x.0" % (p.pci_domain_id, p.pci_bus_id, p.pci_device_id)
+            base = os.path.join("/sys/bus/pci/devices", bus)
+            with open(os.path.join(base, "numa_node")) as f:
+                self.node = int(f.read())
+            with open(os.path.join(base, "local_cpulist")) as f:
+                local = _cpulist(f.read())
+            self.saved = os.sched_getaffinity(0)
+            near = local & self.saved
+            if near:
+                os.sched_setaffinity(0, near)
+                self.cpus = len(near)
+        except (AttributeError, OSError, ValueError):
+            pass
+        return self
+
+    def __exit__(self, *a):
+        if self.saved:
+            os.sched_setaffinity(0, self.saved)
+
+
 class ClockSampler:
     """nvidia-smi clock / throttle samples while the timed region runs."""
 
@@ -261,7 +306,10 @@ def main():
     w = synth.large(rows=(0, args.rows)) if args.rows else synth.large()
     N, D = w["X"].shape
     M = w["C"].shape[0]
-    Xh = torch.from_numpy(w["X"]).pin_memory()
+    with NearGpuHost(local) as host:
+        Xh = torch.from_numpy(w["X"]).pin_memory()
+        amh = torch.empty(N, dtype=torch.int32).pin_memory()
+        mvh = torch.empty(N, dtype=torch.float32).pin_memory()
     X = Xh.to(dev)
     C = torch.from_numpy(w["C"]).to(dev)
     torch.cuda.synchronize()
@@ -316,8 +364,6 @@ def main():
     # end to end through the host-memory entry point: pinned host queries in, argmax /
     # maxval out, streamed through the basis' two staging slots (chunk i copied in while
     # chunk i - 1 is scored); the staging is reserved once, before the timed region
-    amh = torch.empty(N, dtype=torch.int32).pin_memory()
-    mvh = torch.empty(N, dtype=torch.float32).pin_memory()
     houts = {"argmax": amh, "maxval": mvh}
     gs.reserve_staging(basis, min(N, E2E_CHUNK))
 
@@ -337,7 +383,8 @@ def main():
     ms_e2e = max_over_ranks(f0.elapsed_time(f1), pg, dev)
     e2e = {"value": job_throughput(N, ws, ke, ms_e2e), "unit": "queries/s",
            "h2d_bytes_per_step": N * D * 4, "d2h_bytes_per_step": N * 8,
-           "call": "gs_project_similarity_host", "chunk_rows": min(N, E2E_CHUNK)}
+           "call": "gs_project_similarity_host", "chunk_rows": min(N, E2E_CHUNK),
+           "host_numa_node": host.node, "host_cpus_near_gpu": host.cpus}
     ok = ok and bool(np.array_equal(amh.numpy(), w["labels"]))
 
     # roofline of the dominant (only, on the tensor-core path) kernel of the step
