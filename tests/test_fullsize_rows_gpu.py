@@ -71,3 +71,18 @@ def test_reconstruct_bind_full_size(gs, orc):
     Xo = orc.reconstruct(Tr, host(b.Q))
     Zo = orc.bind(Xo, Yr, L)
     check_bind(Z[idx], Zo, Xo, Yr, L, e_rec=1e-4 * np.linalg.norm(Tr, axis=1), method="spectral")
+
+
+def test_bind_one_partner_full_size(gs, orc):
+    """8,192 x 4,096 rows bound with one partner row in blocks of 256 (the bench's one-partner
+    binding: the partner's block spectra cached per CTA), sampled rows against the oracle."""
+    g = torch.Generator().manual_seed(23)
+    X = torch.randn(8192, 4096, generator=g).to("cuda:0")
+    Y = torch.randn(1, 4096, generator=g).to("cuda:0")
+    Z = gs.bind(X, Y, 256)
+    gs.stream_status()
+    rows = sample_rows(8192, 32, 4)
+    Xr = host(X[torch.from_numpy(rows).to(X.device)])
+    Yh = host(Y)
+    Zo = orc.bind(Xr, Yh, 256)
+    check_bind(Z[torch.from_numpy(rows).to(X.device)], Zo, Xr, Yh, 256, method="spectral")
