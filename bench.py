@@ -35,6 +35,8 @@ METRIC = "project+similarity queries/s"
 # fp32 FMA peak of the binding kernel (bound "alu"): 152 SMs x 128 fp32 lanes x 2 flop at the
 # 2,070 MHz maximum SM clock
 FP32_PEAK_TFLOPS = round(152 * 128 * 2 * 2.07e9 / 1e12, 1)
+# GB300's nominal HBM3e bandwidth, reported beside the measured copy rate
+NOMINAL_HBM_GBS = 8000.0
 # rows per staging slot of the end-to-end leg (8192 x 8192 fp32 = 256 MiB a slot)
 E2E_CHUNK = 8192
 WORKLOAD = "large-batch fused project+similarity+argmax, bipolar M=256, D=8192, 65536 queries (sigma=1)"
@@ -396,7 +398,8 @@ def main():
     roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
             "frac": round(achieved / peaks["hbm_gbs"], 4), "peak_src": peaks["src"],
             "traffic": traffic_record("gs_tc.cu", "k_ps_tc/large") if tc else None, "kernel": kernel,
-            "algorithmic_bytes_per_launch": alg_bytes}
+            "algorithmic_bytes_per_launch": alg_bytes,
+            "frac_of_nominal": round(achieved / NOMINAL_HBM_GBS, 4), "nominal_peak": NOMINAL_HBM_GBS}
 
     rows = None
     if not args.no_rows and rank == 0:
