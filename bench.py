@@ -135,7 +135,7 @@ class NearGpuHost:
             if near:
                 os.sched_setaffinity(0, near)
                 self.cpus = len(near)
-        except (AttributeError, OSError, ValueError):
+        except Exception:  # best effort: no sysfs entry, no affinity API, no device properties
             pass
         return self
 

@@ -65,3 +65,19 @@ def test_reference_arm_is_silent_off_rank_zero(monkeypatch, capsys):
     monkeypatch.setattr(sys, "argv", ["bench.py", "--impl", "reference", "--gpus", "2", "--steps", "1"])
     bench.main()
     assert capsys.readouterr().out == ""
+
+
+def test_cpu_list_parsing():
+    assert bench._cpulist("0-3,8-11,16\n") == {0, 1, 2, 3, 8, 9, 10, 11, 16}
+    assert bench._cpulist("5") == {5}
+    assert bench._cpulist("") == set()
+
+
+def test_near_gpu_host_is_best_effort_and_restores_affinity():
+    """Without a device (or its sysfs entry) the NUMA pinning is skipped; the thread's CPU
+    affinity is the same after the block as before it."""
+    before = os.sched_getaffinity(0)
+    with bench.NearGpuHost(0) as host:
+        pass
+    assert os.sched_getaffinity(0) == before
+    assert host.cpus == 0 or host.node is not None
