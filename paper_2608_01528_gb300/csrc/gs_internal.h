@@ -138,8 +138,9 @@ cudaError_t launch_group_argmax(const float* S, long long N, int lds, const int*
                                 float* maxval, cudaStream_t s);
 
 // block circular convolution (unbind: correlation) of rows of X with rows of Y (ldy = 0: Y's
-// row 0 for every row), blocks of L (L divides D); k_bind8 for L % 8 == 0 up to kMaxBindFastL
-constexpr int kMaxBindFastL = 4096;
+// row 0 for every row), blocks of L (L divides D): k_bind_reg for L <= 32 with L % 4 == 0,
+// k_bind16 / k_bind8 for L % 16 / L % 8 == 0 up to kMaxBindFastL, k_bind1 otherwise
+constexpr int kMaxBindFastL = 16384;
 cudaError_t launch_bind(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L, bool unbind,
                         float* Z, int ldz, cudaStream_t s);
 // the same through block spectra (gs_bind_spec.cu): L a power of two in [kMinBindSpectralL,

@@ -17,6 +17,7 @@
 //  k_group_argmax argmax / max of each score row within each group of a grouped codebook
 //  k_bind16       block circular convolution / correlation (binding / unbinding), L % 16 == 0
 //  k_bind8        the same for L % 8 == 0
+//  k_bind_reg     the same for short blocks (L <= 32), one block per thread in registers
 //  k_bind1        the same for any block length, one output per thread
 
 #include <float.h>
@@ -518,6 +519,55 @@ __global__ void __launch_bounds__(256) k_bind16(const float* __restrict__ X, lon
     }
 }
 
+// Short blocks (L <= 32, L % 4 == 0): one thread per block, its X and Y blocks in registers
+// (float4 loads when every row start is 16-byte aligned), L sums of L products in j order;
+// consecutive threads take consecutive blocks of a row, so a warp's loads and stores are
+// contiguous.  The tiled kernels above would give each row's few outputs a thread group of
+// their own and read rows 4 L bytes at a time.
+template <int L, bool UNB>
+__global__ void __launch_bounds__(256) k_bind_reg(const float* __restrict__ X, long long N, int nb, int ldx,
+                                                   const float* __restrict__ Y, long long ldy,
+                                                   float* __restrict__ Z, int ldz, int vec) {
+    const long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= N * nb) return;
+    const long long n = e / nb;
+    const int b = (int)(e - n * nb);
+    const float* x = X + (size_t)n * ldx + (size_t)b * L;
+    const float* y = Y + (size_t)n * ldy + (size_t)b * L;
+    float* z = Z + (size_t)n * ldz + (size_t)b * L;
+    float xv[L], yv[L], zv[L];
+    if (vec) {
+#pragma unroll
+        for (int q = 0; q < L / 4; ++q) {
+            const float4 a = __ldcs(reinterpret_cast<const float4*>(x) + q);
+            const float4 c = __ldg(reinterpret_cast<const float4*>(y) + q);
+            xv[4 * q] = a.x, xv[4 * q + 1] = a.y, xv[4 * q + 2] = a.z, xv[4 * q + 3] = a.w;
+            yv[4 * q] = c.x, yv[4 * q + 1] = c.y, yv[4 * q + 2] = c.z, yv[4 * q + 3] = c.w;
+        }
+    } else {
+#pragma unroll
+        for (int j = 0; j < L; ++j) {
+            xv[j] = x[j];
+            yv[j] = y[j];
+        }
+    }
+#pragma unroll
+    for (int k = 0; k < L; ++k) {
+        float acc = 0.f;
+#pragma unroll
+        for (int j = 0; j < L; ++j) acc = fmaf(xv[j], yv[UNB ? (j - k + L) % L : (k - j + L) % L], acc);
+        zv[k] = acc;
+    }
+    if (vec) {
+#pragma unroll
+        for (int q = 0; q < L / 4; ++q)
+            __stcs(reinterpret_cast<float4*>(z) + q, make_float4(zv[4 * q], zv[4 * q + 1], zv[4 * q + 2], zv[4 * q + 3]));
+    } else {
+#pragma unroll
+        for (int k = 0; k < L; ++k) z[k] = zv[k];
+    }
+}
+
 // Any block length: one thread per output, operands read through the cache.
 template <bool UNB>
 __global__ void __launch_bounds__(256) k_bind1(const float* __restrict__ X, long long N, int D, int ldx,
@@ -611,9 +661,49 @@ cudaError_t launch_group_argmax(const float* S, long long N, int lds, const int*
     return cudaGetLastError();
 }
 
+template <int L>
+static cudaError_t launch_bind_reg(const float* X, long long N, int D, int ldx, const float* Y, long long ldy,
+                                   bool unbind, float* Z, int ldz, cudaStream_t s) {
+    const int nb = D / L;
+    const int vec = ((uintptr_t)X % 16 == 0 && (uintptr_t)Y % 16 == 0 && (uintptr_t)Z % 16 == 0 && ldx % 4 == 0 &&
+                     ldy % 4 == 0 && ldz % 4 == 0)
+                        ? 1
+                        : 0;
+    const unsigned blocks = (unsigned)((N * nb + 255) / 256);
+    if (unbind)
+        k_bind_reg<L, true><<<blocks, 256, 0, s>>>(X, N, nb, ldx, Y, ldy, Z, ldz, vec);
+    else
+        k_bind_reg<L, false><<<blocks, 256, 0, s>>>(X, N, nb, ldx, Y, ldy, Z, ldz, vec);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_bind(const float* X, long long N, int D, int ldx, const float* Y, long long ldy, int L, bool unbind,
                         float* Z, int ldz, cudaStream_t s) {
     if (N <= 0) return cudaSuccess;
+    switch (L) {
+        case 4: return launch_bind_reg<4>(X, N, D, ldx, Y, ldy, unbind, Z, ldz, s);
+        case 8: return launch_bind_reg<8>(X, N, D, ldx, Y, ldy, unbind, Z, ldz, s);
+        case 12: return launch_bind_reg<12>(X, N, D, ldx, Y, ldy, unbind, Z, ldz, s);
+        case 16: return launch_bind_reg<16>(X, N, D, ldx, Y, ldy, unbind, Z, ldz, s);
+        case 20: return launch_bind_reg<20>(X, N, D, ldx, Y, ldy, unbind, Z, ldz, s);
+        case 24: return launch_bind_reg<24>(X, N, D, ldx, Y, ldy, unbind, Z, ldz, s);
+        case 28: return launch_bind_reg<28>(X, N, D, ldx, Y, ldy, unbind, Z, ldz, s);
+        case 32: return launch_bind_reg<32>(X, N, D, ldx, Y, ldy, unbind, Z, ldz, s);
+        default: break;
+    }
+    // the staged kernels hold a row's X and Y blocks in shared memory: opt in past 48 KB once
+    static bool opted[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (!opted[dev]) {
+        for (auto fn : {k_bind16<true>, k_bind16<false>, k_bind8<true>, k_bind8<false>}) {
+            e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+            if (e != cudaSuccess) return e;
+        }
+        opted[dev] = true;
+    }
     const int zvec = ((uintptr_t)Z % 16 == 0 && ldz % 4 == 0) ? 1 : 0;
     if (L % 16 == 0 && L <= kMaxBindFastL && D / L <= 65535) {
         const int tpr = std::min(L / 16, 256);

@@ -54,8 +54,9 @@ def check_bind(Z, Zo, X, Y, L, e_rec=None, method="direct"):
     (50, 960, 24, False, "unbind"), (33, 1000, 10, True, "bind"), (5, 4096, 4096, False, "bind"),
     (300, 3000, 1000, False, "unbind"), (1, 64, 64, True, "bind")])
 def test_bind_matches_oracle(gs, orc, N, D, L, bcast, op):
-    """The direct method on all its kernels (L % 16, L % 8 == 0: shared-memory tiles up to L =
-    4096; L = 10: one output per thread), one partner for all rows, padded leading dimensions."""
+    """The direct method on all its kernels (L % 16, L % 8 == 0: shared-memory tiles; L <= 32:
+    registers, here with an odd output pitch (element stores); L = 10: one output per thread),
+    one partner for all rows, padded leading dimensions."""
     rng = np.random.default_rng(N + D + L)
     X = rng.normal(size=(N, D)).astype(np.float32)
     Y = rng.normal(size=(1 if bcast else N, D)).astype(np.float32)
@@ -63,6 +64,21 @@ def test_bind_matches_oracle(gs, orc, N, D, L, bcast, op):
     Xp[:, :D] = cuda(X)
     Zp = torch.zeros((N, D + 3), device="cuda:0")  # odd row pitch: element stores
     Z = gs.bind(Xp[:, :D], cuda(Y), L, op, method="direct", out=Zp[:, :D])
+    gs.stream_status()
+    Zo = orc.bind(X, Y, L, orc.UNBIND if op == "unbind" else orc.BIND)
+    check_bind(Z, Zo, X, Y, L)
+
+
+@pytest.mark.parametrize("N,D,L,bcast,op", [
+    (300, 1024, 4, False, "bind"), (97, 960, 12, True, "unbind"), (300, 1024, 16, False, "unbind"),
+    (33, 2048, 32, True, "bind"), (7, 640, 20, False, "bind"), (2, 8192, 8192, False, "unbind")])
+def test_bind_direct_short_and_long_blocks(gs, orc, N, D, L, bcast, op):
+    """The direct sum on short blocks (L <= 32: a block per thread in registers, float4 rows)
+    and on a block longer than 48 KB of staging (L = 8192: the shared-memory opt-in)."""
+    rng = np.random.default_rng(N + D + L + 2)
+    X = rng.normal(size=(N, D)).astype(np.float32)
+    Y = rng.normal(size=(1 if bcast else N, D)).astype(np.float32)
+    Z = gs.bind(cuda(X), cuda(Y), L, op, method="direct")
     gs.stream_status()
     Zo = orc.bind(X, Y, L, orc.UNBIND if op == "unbind" else orc.BIND)
     check_bind(Z, Zo, X, Y, L)
