@@ -32,7 +32,8 @@
 // 32 (w % 4)..+31; the two warps of a lane quadrant take alternate 32-column chunks,
 // so output-heavy products like reconstruct are not held up by the stores),
 // 4 TMA producer of A, 5 TMEM allocator + MMA issuer, 6 TMA producer of B,
-// 7-14 converters in two groups taking alternate K-blocks.  Every mbarrier wait
+// 7-14 converters in two groups taking alternate K-blocks (with A loaded by TMA they
+// join the epilogue: four warps per lane quadrant).  Every mbarrier wait
 // is bounded (see gs_tc_ptx.cuh); on expiry the CTA records GS_DEV_ERR_TIMEOUT,
 // unwinds, waits for its own copies and MMAs, frees TMEM and returns.
 
@@ -111,6 +112,8 @@ template <int AMODE, int HALVES>
 __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see kThreads)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b0,
               const __grid_constant__ CUtensorMap tmap_b1, const __grid_constant__ GemmParams p) {
+    // A loaded by TMA leaves the converter warps idle: they store output tiles instead
+    constexpr bool kCvtEpi = AMODE == kAF16T;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
@@ -150,7 +153,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&c.d_full[b], 1);
-            mbar_init(&c.d_empty[b], kEpiWarpsTotal);
+            mbar_init(&c.d_empty[b], kCvtEpi ? kEpiWarpsTotal + kCvtWarps : kEpiWarpsTotal);
         }
         mbar_init(&c.mma_done, 1);
         c.abort_flag = 0;
@@ -333,7 +336,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
             mma_commit(&c.mma_done);
             mbar_drain(&c.mma_done, 0, err);
         }
-    } else if (warp >= kCvt0 && warp < kEpi2) {
+    } else if (!kCvtEpi && warp >= kCvt0 && warp < kEpi2) {
         // ------------------------------------------------------------- converters
         const int g = (warp - kCvt0) / kCvtGroupWarps;
         const int l = threadIdx.x - (kCvt0 + g * kCvtGroupWarps) * 32;  // 0..127
@@ -388,10 +391,15 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
         }
         if (amax > 65504.f) atomicOr(err, GS_DEV_ERR_RANGE);
     } else {
-        // ------------------------------------------------------------- epilogue (warps 0-3, 15-18)
+        // ------------------------------------------------------------- epilogue (warps 0-3, 15-18,
+        // and with A loaded by TMA the idle converter warps 7-14 as well)
         // TMEM is read in the 16x256b pattern so that each store writes whole sectors:
         // thread t holds rows (t/4) and (t/4 + 8) of a 16-lane half, 8 columns per quad.
-        const int quad = warp & 3, kh = warp >= kEpi2 ? 1 : 0;  // lane quadrant, column chunks
+        // The warps of a lane quadrant take alternate 32-column chunks: two per quadrant, or
+        // four when the converter warps join.
+        const int quad = warp & 3;  // lane quadrant
+        const int chunk = warp < kCvt0 ? 0 : warp >= kEpi2 ? 1 : 2 + (warp - kCvt0) / kCvtGroupWarps;
+        constexpr int nchunks = kCvtEpi ? 4 : 2;
         const int nbuf = HALVES == 2 ? 1 : 2;
         const int tw = p.nt * HALVES;  // tile width
         for (int lt = 0; lt < ntiles; ++lt) {
@@ -408,7 +416,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                 float rn[2];
 #pragma unroll
                 for (int h = 0; h < 2; ++h) rn[h] = (p.rownorm && row[h] < p.m) ? p.rownorm[row[h]] : 1.f;
-                for (int jc = 32 * kh; jc < tw; jc += 64) {
+                for (int jc = 32 * chunk; jc < tw; jc += 32 * nchunks) {
                     float v[16];
                     tmem_ld16x256b_x4(tb + (uint32_t)jc, v);
 #pragma unroll
