@@ -71,3 +71,32 @@ def test_bind_argument_checks_need_no_device(lib):
     assert lib.gs_bind(dummy, 0, 100, 100, dummy, 0, 50, g.BIND_METHODS["spectral"], dummy, 100,
                        None) == g.GS_OK
     assert lib.gs_bind(None, 4, 100, 100, None, 0, 50, 0, None, 100, None) == g.GS_ERR_INVALID_ARG
+
+
+def test_plain_c_client(lib, tmp_path):
+    """The header is plain C (C99, -pedantic, no warnings) and a C program links against the
+    library and calls it: the boundary needs no C++ or torch on the caller's side."""
+    import shutil
+    import subprocess
+    from paper_2608_01528_gb300 import build
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "client.c"
+    src.write_text(
+        "#include <stdio.h>\n"
+        "#include \"gramspace.h\"\n"
+        "int main(void) {\n"
+        "    printf(\"%d %s\\n\", gs_version(), gs_status_string(GS_ERR_SHAPE));\n"
+        "    /* L = 30 does not divide D = 100: rejected on the host */\n"
+        "    return gs_bind(0, 4, 100, 100, 0, 0, 30, GS_BIND | GS_BIND_DIRECT, 0, 100, 0) == GS_ERR_SHAPE ? 0 : 1;\n"
+        "}\n")
+    exe = tmp_path / "client"
+    libdir = os.path.dirname(build.LIB)
+    p = subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-I",
+                        os.path.join(ROOT, "include"), str(src), "-L", libdir, "-lgramspace",
+                        f"-Wl,-rpath,{libdir}", "-o", str(exe)], capture_output=True, text=True)
+    assert p.returncode == 0, p.stderr
+    r = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert r.returncode == 0, r.stdout + r.stderr
+    assert r.stdout.split()[1] == "GS_ERR_SHAPE"
