@@ -1,41 +1,23 @@
 """GPU parity of binding / unbinding (gs_bind) and reconstruct-then-bind (gs_reconstruct_bind)
-against the float64 oracle (the direct sums of the definition).
-
-Bound per output of block b, with ||x_b||, ||y_b|| the norms of the row's blocks:
-  direct method (fp32 sums of L products in j order): |Z - Z*| <= L 2^-22 ||x_b|| ||y_b||;
-  spectral method (fp32 radix-2^k transforms of the blocks, the product, the inverse):
-  |Z - Z*| <= sqrt(2L) (3e + 4u) ||x_b|| ||y_b||, u = 2^-24, e = K eta / (1 - K eta) + 10u,
-  eta = 10u, K = log2(L) + 1 (two Stockham passes, L <= 512) or log2(L) + 2 (three): the
-  radix-2 FFT bound ||fl(F w) - F w|| <= K eta ||F w|| (Higham, Thm 24.2; one extra twiddle
-  multiply per pass) through the split, the product (max|Y_k| <= sqrt(L) ||y_b||) and the
-  inverse transform.
-For the fused call the reconstruction error adds e_rec sqrt(L) ||y_b||, e_rec = 1e-4 ||t|| on the
-fp16 tensor-core reconstruction (the reconstruct bound) and 0 on the fp32 path.
+against the float64 oracle (the direct sums of the definition), within the per-output bounds of
+tests/bounds.py (direct sum, or the transform bound of the spectral method).  For the fused call
+the reconstruction error adds e_rec sqrt(L) ||y_b||, e_rec = 1e-4 ||t|| on the fp16 tensor-core
+reconstruction (the reconstruct bound) and 0 on the fp32 path.
 """
 import numpy as np
 import pytest
 import torch
 
 import synth
+from bounds import bind_error_factor
 from test_parity_gpu import cuda, host
 
 pytestmark = pytest.mark.gpu
-
-U32 = 2.0 ** -24
 
 
 def block_norms(A, L):
     N, D = A.shape
     return np.sqrt((A.astype(np.float64).reshape(N, D // L, L) ** 2).sum(axis=2))
-
-
-def bind_error_factor(L, method):
-    if method == "direct":
-        return L * 2.0 ** -22
-    K = int(np.log2(L)) + (1 if L <= 512 else 2)
-    eta = 10 * U32
-    e = K * eta / (1 - K * eta) + 10 * U32
-    return np.sqrt(2 * L) * (3 * e + 4 * U32)
 
 
 def check_bind(Z, Zo, X, Y, L, e_rec=None, method="direct"):
