@@ -74,8 +74,8 @@ typedef enum gs_score_mode {
 } gs_score_mode;
 
 /* gs_build_basis flags */
-#define GS_BUILD_NORMALIZE_ROWS 0x1u /* build on c_i / ||c_i|| ("each atomic vector
-                                        undergoes normalization", Sec. 3.1)       */
+#define GS_BUILD_NORMALIZE_ROWS 0x1u /* build on c_i / ||c_i|| (the atoms scaled to
+                                        unit length first, Sec. 3.1)              */
 
 /* path-selection flags of the apply calls (at most one) */
 #define GS_PATH_AUTO 0x0u   /* pick by problem size                                 */
@@ -86,7 +86,7 @@ typedef enum gs_score_mode {
 typedef struct gs_basis gs_basis;
 
 /*
- * Basis construction (Sec. 3.1, Eq. 1; built once "during initialization" by
+ * Basis construction (Sec. 3.1, Eq. 1; built once, at initialisation, by
  * Gram-Schmidt, Sec. 3.3; rank k = algebraic rank, Sec. 3.2).
  *
  * Orthonormalises the rows of C (M x D, fp32, ld = ldc) in row order by
@@ -366,8 +366,12 @@ GS_API gs_status gs_attention_scores(const void* Yq, const void* Yk, int in_dtyp
  * every GPU that loads it until exit), processed in chunks of rows; a problem
  * with r + M + 1 > 4,194,304 is rejected with GS_ERR_SHAPE.  The first call on
  * a device looks up that array's device address (cudaGetSymbolAddress) with
- * the device current, so make that first call before any stream capture.  All
- * calls on a device share the array: calls that overlap on the GPU race.
+ * the device current, so make that first call before any stream capture; the
+ * address is kept per device context and looked up again after the context
+ * changes (cudaDeviceReset), so the first call after a reset must also come
+ * before any capture.  All calls on a device share the array: calls that
+ * overlap on the GPU race.  `stream` must belong to the current device
+ * (GS_ERR_INVALID_ARG otherwise).
  * Errors: GS_ERR_INVALID_ARG, GS_ERR_SHAPE, GS_ERR_CUDA, GS_ERR_UNSUPPORTED.
  */
 GS_API gs_status gs_project_similarity_static(const float* Q, int r, int D, const float* R, int M,
@@ -382,7 +386,6 @@ GS_API gs_status gs_project_similarity_static(const float* Q, int r, int D, cons
  */
 GS_API gs_status gs_stream_status(void* stream);
 
-/* Static, human-readable name of a status code. */
 /*
  * Self-test of the device-side failure detection (the paper has no counterpart:
  * this checks the library's own machinery).  Every wait of the tensor-core
@@ -395,6 +398,7 @@ GS_API gs_status gs_stream_status(void* stream);
  */
 GS_API gs_status gs_selftest_wait_timeout(void* stream);
 
+/* Static, human-readable name of a status code. */
 GS_API const char* gs_status_string(gs_status s);
 
 /* Library version, major*10000 + minor*100 + patch. */

@@ -72,12 +72,12 @@ static double dot(const double* a, const double* b, int n) {
 }
 
 /*
- * Basis construction (Sec. 3.1, Eq. 1; "During initialization ... generated by
- * Gram-Schmidt orthogonalization of the codebook", Sec. 3.3).
+ * Basis construction (Sec. 3.1, Eq. 1; Sec. 3.3 builds the basis once, at
+ * initialisation, by Gram-Schmidt orthogonalisation of the codebook).
  *
  * For each codeword row c_i in order:
- *   v = c_i (optionally c_i/||c_i||: "each atomic vector undergoes
- *   normalization", Sec. 3.1);
+ *   v = c_i (optionally c_i/||c_i||: Sec. 3.1 scales the atoms to unit
+ *   length);
  *   `passes` times: for j = 0 .. r-1 in order, h = <q_j, v> with the current
  *   v (modified GS), v -= h q_j, R[i][j] += h;
  *   if ||v|| > tau * ||c_i||: q_r = v / ||v||, R[i][r] = ||v||, r += 1.

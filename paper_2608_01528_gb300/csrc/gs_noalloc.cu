@@ -11,8 +11,12 @@
 // The array is a fixed 16 MiB per device (kStaticScratchFloats floats) and is
 // held by every GPU that loads this library until the process exits.  In host
 // code its name is only a host-side stand-in, so the entry point looks up the
-// device address with cudaGetSymbolAddress once per device (the first call on
-// a device, with that device current) and passes that address to the kernels.
+// device address with cudaGetSymbolAddress once per device context (the first
+// call on a device, with that device current) and passes that address to the
+// kernels.  The address is cached together with the context's unique id: after
+// cudaDeviceReset the device gets a new primary context (the module, and the
+// array with it, is loaded again), the ids differ, and the next call looks the
+// address up again instead of using one the old context owned.
 // Every call on a device shares the one array: calls that overlap on the GPU
 // (different streams, or several host threads) race on it.  Nothing in the
 // array needs to start at zero: each chunk writes every scratch element it
@@ -30,20 +34,60 @@ constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) float g_static_scratch[kStaticScratchFloats];
 
-float* g_scratch_dev[kMaxDevices];  // device address of g_static_scratch, per device
+float* g_scratch_dev[kMaxDevices];               // device address of g_static_scratch, per device
+unsigned long long g_scratch_ctx[kMaxDevices];   // id of the context that address belongs to
 std::mutex g_scratch_mu;
 
-// Device address of the static scratch on `dev` (looked up on first use).
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
+
+// Unique id of the current context (0 when it cannot be read: the address is then looked up
+// on every call, which is correct, only slower).
+unsigned long long current_ctx_id() {
+    static CtxGetCurrentFn get_current = nullptr;
+    static CtxGetIdFn get_id = nullptr;
+    static bool looked_up = false;
+    if (!looked_up) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_current = (CtxGetCurrentFn)p;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_id = (CtxGetIdFn)p;
+        looked_up = true;
+    }
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS)
+        return 0;
+    return id;
+}
+
+// Device address of the static scratch on `dev` (looked up on first use in each context).
 gs_status static_scratch(int dev, float** out) {
     if (dev < 0 || dev >= kMaxDevices) return GS_ERR_UNSUPPORTED;
     std::lock_guard<std::mutex> lock(g_scratch_mu);
-    if (!g_scratch_dev[dev]) {
+    const unsigned long long ctx = current_ctx_id();
+    if (!g_scratch_dev[dev] || ctx == 0 || ctx != g_scratch_ctx[dev]) {
         void* p = nullptr;
+        g_scratch_dev[dev] = nullptr;
         if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p) return GS_ERR_CUDA;
         g_scratch_dev[dev] = static_cast<float*>(p);
+        g_scratch_ctx[dev] = ctx;
     }
     *out = g_scratch_dev[dev];
     return GS_OK;
+}
+
+// A stream created on another device than the current one: its kernels would get this
+// device's scratch address.  The special handles (legacy and per-thread default streams)
+// always belong to the current device.
+bool stream_on_other_device(cudaStream_t s, int dev) {
+    if (s == nullptr || s == cudaStreamLegacy || s == cudaStreamPerThread) return false;
+    int sdev = -1;
+    return cudaStreamGetDevice(s, &sdev) != cudaSuccess || sdev != dev;
 }
 
 gs_status from_cuda(cudaError_t e) { return e == cudaSuccess ? GS_OK : GS_ERR_CUDA; }
@@ -66,10 +110,11 @@ extern "C" GS_API gs_status gs_project_similarity_static(const float* Q, int r, 
     cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
     cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
     if (major != 10 || minor != 3) return GS_ERR_UNSUPPORTED;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (stream_on_other_device(s, dev)) return GS_ERR_INVALID_ARG;
     float* scr = nullptr;
     gs_status st = static_scratch(dev, &scr);
     if (st != GS_OK) return st;
-    cudaStream_t s = (cudaStream_t)stream;
     long long chunk = kStaticScratchFloats / per_row;
     if (chunk > kMaxRowsPerGemm) chunk = kMaxRowsPerGemm;
     for (long long c0 = 0; c0 < N; c0 += chunk) {

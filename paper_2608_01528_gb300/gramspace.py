@@ -437,17 +437,37 @@ def project_similarity_static(Q, R, cnorm, X, mode="raw", scale=1.0, want_argmax
                               out=None, stream=None):
     """Project + similarity from a caller-held basis without any device allocation by the
     library; see gs_project_similarity_static.  Q: r x D, R: M x r, cnorm: M (fp32, CUDA)."""
+    # the C entry takes ld(Q) = D and ld(R) = r and reads cnorm[0..M): every shape is checked here,
+    # before any pointer reaches the library
+    if Q.dim() != 2 or R.dim() != 2 or X.dim() != 2 or cnorm.dim() != 1:
+        raise ValueError("Q, R, X must be 2-D and cnorm 1-D")
     N = X.shape[0]
     r, D = Q.shape
     M = R.shape[0]
+    if R.shape[1] != r:
+        raise ValueError(f"R must be M x r with r = {r} (Q's rows), got {tuple(R.shape)}")
+    if X.shape[1] != D:
+        raise ValueError(f"X must be N x {D} (Q's columns), got {tuple(X.shape)}")
+    if cnorm.shape[0] != M:
+        raise ValueError(f"cnorm must hold M = {M} entries, got {cnorm.shape[0]}")
+    for t in (Q, R):
+        if t.numel() and not t.is_contiguous():
+            raise ValueError("Q and R must be contiguous")
     out = dict(out or {})
+    for key, dt in (("argmax", torch.int32), ("maxval", torch.float32)):
+        t = out.get(key)
+        if t is not None and (t.dtype != dt or t.dim() != 1 or t.shape[0] != N or not t.is_contiguous()):
+            raise ValueError(f"out[{key!r}] must be a contiguous {dt} vector of N = {N} entries")
+    for name, t in (("Q", Q), ("R", R), ("cnorm", cnorm), ("X", X)):
+        if t.dtype != torch.float32:
+            raise TypeError(f"{name} must be float32, got {t.dtype}")
+    tensors = [Q, R, cnorm, X] + [t for t in out.values() if t is not None]
+    if any(not t.is_cuda for t in tensors) or len({t.device for t in tensors}) != 1:
+        raise TypeError("Q, R, cnorm, X and the outputs must be CUDA tensors on one device")
     if want_argmax and "argmax" not in out:
         out["argmax"] = torch.empty(N, dtype=torch.int32, device=X.device)
     if want_maxval and "maxval" not in out:
         out["maxval"] = torch.empty(N, dtype=torch.float32, device=X.device)
-    for t in (Q, R):
-        if t.numel() and not t.is_contiguous():
-            raise ValueError("Q and R must be contiguous")
     L = load_library()
     with torch.cuda.device(X.device):
         st = L.gs_project_similarity_static(_ptr(Q) if Q.numel() else None, r, D, _ptr(R) if R.numel() else None,

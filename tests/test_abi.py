@@ -100,3 +100,30 @@ def test_plain_c_client(lib, tmp_path):
     r = subprocess.run([str(exe)], capture_output=True, text=True)
     assert r.returncode == 0, r.stdout + r.stderr
     assert r.stdout.split()[1] == "GS_ERR_SHAPE"
+
+
+def test_static_entry_wrapper_rejects_mismatched_tensors():
+    """project_similarity_static checks shapes, dtypes and devices before any pointer reaches the
+    library: the C entry assumes ld(Q) = D, ld(R) = r and M norms, so a mismatch there would read
+    or write past a buffer on the device.  CPU tensors reach no CUDA call."""
+    import torch
+    from paper_2608_01528_gb300 import gramspace as g
+    r, D, M, N = 4, 16, 6, 3
+    Q, R, cn, X = torch.zeros(r, D), torch.zeros(M, r), torch.zeros(M), torch.zeros(N, D)
+    bad_shapes = [
+        (Q, torch.zeros(M, r + 1), cn, X),   # R wider than r
+        (Q, R, cn, torch.zeros(N, D - 1)),   # X narrower than D
+        (Q, R, torch.zeros(M - 1), X),       # too few norms
+        (Q.reshape(-1), R, cn, X),           # Q not 2-D
+    ]
+    for args in bad_shapes:
+        with pytest.raises(ValueError):
+            g.project_similarity_static(*args)
+    with pytest.raises(ValueError):
+        g.project_similarity_static(Q, R, cn, X, out={"argmax": torch.zeros(N - 1, dtype=torch.int32)})
+    with pytest.raises(ValueError):
+        g.project_similarity_static(Q, R, cn, X, out={"maxval": torch.zeros(N, dtype=torch.float64)})
+    with pytest.raises(TypeError):
+        g.project_similarity_static(Q, R, cn, X.to(torch.bfloat16))
+    with pytest.raises(TypeError):  # right shapes and dtypes, but host tensors
+        g.project_similarity_static(Q, R, cn, X)

@@ -307,3 +307,21 @@ def test_strided_inputs(gs, orc):
     out = gs.project_similarity(b, big[:, :1024], want_S=True)
     ref = orc.project_similarity(t["X"], Qo, Ro, cno)
     check_scores(out, ref, t["X"], cno)
+
+
+def test_reconstruct_multiattr(gs, orc):
+    """The multi-attribute workload's reconstruct step: each attribute's prob-vectorized rows
+    V = P R (512 per attribute) back to D = 1024, against the oracle's reconstruction with the
+    GPU's basis (1e-4 ||v||) and against the basis-free P C (1e-4 sum_i |p_i| ||c_i||)."""
+    for a in synth.multiattr():
+        b = gs.build_basis(cuda(a["C"]))
+        V = gs.prob_vectorize(b, cuda(a["P"]))
+        Xh = gs.reconstruct(b, V)
+        gs.stream_status()
+        Vh = host(V)
+        ref = orc.reconstruct(Vh, host(b.Q))
+        assert np.all(np.abs(host(Xh) - ref) <= 1e-4 * np.linalg.norm(Vh, axis=1)[:, None])
+        P = a["P"].astype(np.float64)
+        cn = np.linalg.norm(a["C"].astype(np.float64), axis=1)
+        PC = P @ a["C"].astype(np.float64)
+        assert np.all(np.abs(host(Xh) - PC) <= 1e-4 * (np.abs(P) @ cn)[:, None])
