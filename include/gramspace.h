@@ -59,9 +59,11 @@ typedef enum gs_status {
     GS_ERR_NOMEM = 4,        /* a device allocation failed                          */
     GS_ERR_CUDA = 5,         /* a CUDA runtime / driver call failed                 */
     GS_ERR_TIMEOUT = 6,      /* a bounded device-side wait gave up (device word)    */
-    GS_ERR_RANGE = 7,        /* an input exceeded the fp16 range of the tensor-core
-                                path (|x| > 65504); results of that call are invalid,
-                                rerun it with GS_PATH_SIMT (device word)            */
+    GS_ERR_RANGE = 7,        /* a query row of the fused tensor-core similarity has a
+                                squared norm that is not a finite fp32 number (an
+                                entry near 2^64 or beyond, or an infinity); results of
+                                that call are invalid, rerun it with GS_PATH_SIMT
+                                (device word)                                        */
     GS_ERR_UNSUPPORTED = 8   /* no sm_103 device, or a forced path cannot run      */
 } gs_status;
 
@@ -200,10 +202,17 @@ GS_API gs_status gs_basis_destroy(gs_basis* h);
  *   S      N x M fp32, ld = lds          maxval  N fp32 (S at argmax)
  * At least one output must be non-NULL.  When r = 0 every score is 0 (softmax:
  * 1/M) and argmax is 0.
- * Tensor-core path (GS_PATH_AUTO picks it for large N with r <= 256): X is
- * rounded to fp16 on the fly (|x| must stay below 65504, else GS_ERR_RANGE is
- * raised on the device word), Q is a fixed fp16 copy with unbiased dithered
- * rounding, fp32 accumulation; the scores S = Y R^T are taken in fp32.
+ * Tensor-core path (GS_PATH_AUTO picks it for large N): X is rounded to fp16
+ * on the fly (D >= 1024; shorter rows are split into bf16 hi / lo), Q is a
+ * fixed fp16 copy with unbiased dithered rounding, fp32 accumulation; the
+ * scores S = Y R^T are taken with Y and R split into bf16 hi / lo.  One fp16
+ * rounding of a row is accurate while 2^-8 sqrt(D) <= ||x|| <= 2^15; the kernels
+ * find every other nonzero row from its norm and compute it again within the
+ * same call -- the fused kernel (r <= 256, M <= 256) redoes the row's tile on
+ * x 2^s with an exact power of two s that brings ||x|| 2^s to [2^14, 2^15), the
+ * two-GEMM path (wider bases) recomputes the row's Y in fp32 -- so the results
+ * meet the same relative bound for queries of any magnitude.  Only a row whose
+ * squared norm is not a finite fp32 number raises GS_ERR_RANGE (fused kernel).
  * Requires X 16-byte aligned and ldx % 4 == 0 on the tensor-core path.
  */
 GS_API gs_status gs_project_similarity(const gs_basis* h, const float* X, long long N, int ldx,
@@ -278,6 +287,12 @@ GS_API gs_status gs_prob_vectorize(const gs_basis* h, const float* P, long long 
  * component-wise operators).  Xhat = T Q: T is N x r coefficients of type
  * t_dtype (GS_F32 or GS_BF16, ld = ldt), Xhat is N x D fp32 (ld = ldxh).
  * Reconstructing R itself returns the codebook C (exact up to rounding).
+ * Tensor-core path (GS_PATH_AUTO for large N with fp32 T, 16-byte aligned,
+ * ldt % 4 == 0): each row of T is multiplied by an exact power of two that
+ * brings its largest magnitude to [2^14, 2^15), rounded once to fp16 into the
+ * handle's scratch, multiplied by the dithered fp16 Q with fp32 accumulation,
+ * and the row's scale is undone in fp32, so the result is accurate for rows of
+ * any magnitude (down to a largest entry of 2^-112).  Otherwise fp32 CUDA cores.
  */
 GS_API gs_status gs_reconstruct(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt,
                          float* Xhat, int ldxh, unsigned flags, void* stream);

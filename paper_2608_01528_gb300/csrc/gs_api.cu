@@ -88,24 +88,40 @@ gs_status ps_two_gemm(const gs_basis* h, const float* X, long long N, int ldx, i
                       int ldy, float* S, int lds, int* argmax, float* maxval, cudaStream_t s) {
     const int r = h->r, M = h->M, D = h->D;
     const int r4 = (r + 3) / 4 * 4;  // padded ld of the Y scratch (16-byte rows for TMA)
-    const long long per_row = (long long)r4 + M + 1;
+    const long long per_row = (long long)r4 + M + 3;
     long long chunk = std::min(h->scratch_floats / per_row, kMaxGemmRows);
     if (chunk < 1) return GS_ERR_SHAPE;
     const bool need_s = S || argmax || maxval;
+    const bool f16 = D >= gs::kMinF16Depth;  // one fp16 rounding of X (else the bf16 hi / lo split)
     for (long long c0 = 0; c0 < N; c0 += chunk) {
         const long long nc = std::min(chunk, N - c0);
         float* Ybuf = h->scratch;
         float* xn = Ybuf + nc * r4;
-        float* Sscr = xn + nc;
+        float* xn2 = xn + nc;       // 2 x nc: the rows' ||x||^2 in two partial sums (fp16 GEMM1)
+        float* Sscr = xn2 + 2 * nc;
         gs::GemmTcArgs g1{};
         g1.A = X + c0 * ldx; g1.lda = ldx; g1.m = nc; g1.K = D;
-        g1.split = D < gs::kMinF16Depth;  // short rows: bf16 hi / lo split instead of one fp16 rounding
+        g1.split = !f16;
         g1.B0 = g1.split ? h->tc_Qh : (const void*)h->Q16;
         g1.B1 = g1.split ? h->tc_Ql : nullptr;
         g1.ldb = h->ldq16; g1.n = r;
         g1.C = Ybuf; g1.ldc = r4; g1.c_bf16 = false; g1.alpha = 1.f;
+        g1.xn2_out = f16 ? xn2 : nullptr;
         cudaError_t e = gs::launch_gemm_tc(g1, h->device, s);
         if (e != cudaSuccess) return from_cuda(e);
+        if (f16) {
+            // rows that one fp16 rounding cannot hold accurately (||x|| > 2^15, or ||x|| <
+            // 2^-8 sqrt(D) where fp16's subnormals start to matter): their Y rows are computed
+            // again in fp32; the 64-row blocks without such a row return at once
+            gs::GemmArgs f{};
+            f.A = X + c0 * ldx; f.a_type = gs::MAT_F32; f.lda = ldx;
+            f.B = h->Q; f.b_type = gs::MAT_F32; f.ldb = D; f.b_trans = true;
+            f.C = Ybuf; f.c_type = gs::MAT_F32; f.ldc = r4;
+            f.m = nc; f.n = r; f.k = D; f.batch = 1; f.alpha = 1.f;
+            f.gate_xn2 = xn2; f.gate_ld = nc; f.gate_lo = (float)D * 0x1p-16f; f.gate_hi = 0x1p30f;
+            e = gs::launch_gemm_simt(f, s);
+            if (e != cudaSuccess) return from_cuda(e);
+        }
         if (Y) {
             e = cudaMemcpy2DAsync(Y + c0 * ldy, sizeof(float) * ldy, Ybuf, sizeof(float) * r4, sizeof(float) * r, nc,
                                   cudaMemcpyDeviceToDevice, s);
@@ -551,20 +567,24 @@ static gs_status reconstruct_rows(const gs_basis* h, const void* T, int t_dtype,
     if (flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && tc_ok && big_gemm(N, h->D, h->r))) {
         if (!tc_ok) return t_dtype != GS_F32 || !h->has_split ? GS_ERR_UNSUPPORTED : GS_ERR_ALIGNMENT;
         // Xhat = T Q: T rounded once to fp16 into the handle's scratch (every column tile of
-        // Xhat re-reads it), the basis' dithered fp16 Q^T, fp32 accumulation; rows in chunks
-        // that fit the scratch
+        // Xhat re-reads it) after an exact power-of-two scale per row, the basis' dithered fp16
+        // Q^T, fp32 accumulation, the row scales undone in the epilogue; rows in chunks that
+        // fit the scratch (ld16 halves and one float per row)
         const int ld16 = (h->r + 7) / 8 * 8;  // 16-byte rows for TMA
-        const long long chunk = std::min(work_floats * 2 / ld16, kMaxGemmRows) / 128 * 128;
+        const long long chunk = std::min(work_floats / (ld16 / 2 + 1), kMaxGemmRows) / 128 * 128;
         if (chunk < 128) return GS_ERR_SHAPE;
         for (long long c0 = 0; c0 < N; c0 += chunk) {
             const long long nc = std::min(chunk, N - c0);
             const float* Tc = (const float*)T + (size_t)c0 * ldt;
-            gs_status st = from_cuda(gs::launch_round_f16(Tc, ldt, nc, h->r, work, ld16, s));
+            // T rows scaled by exact powers of two into fp16's range, the scales undone in fp32
+            float* rowmul = work + (size_t)chunk * ld16 / 2;
+            gs_status st = from_cuda(gs::launch_round_f16(Tc, ldt, nc, h->r, work, ld16, rowmul, s));
             if (st != GS_OK) return st;
             gs::GemmTcArgs a{};
             a.A = work; a.lda = ld16; a.m = nc; a.K = h->r; a.split = false; a.a_half = true;
             a.B0 = h->Q16t; a.ldb = h->ldr16; a.n = h->D;
             a.C = Xhat + (size_t)c0 * ldxh; a.ldc = ldxh; a.c_bf16 = false; a.alpha = 1.f;
+            a.rowmul = rowmul;
             st = from_cuda(gs::launch_gemm_tc(a, h->device, s));
             if (st != GS_OK) return st;
         }

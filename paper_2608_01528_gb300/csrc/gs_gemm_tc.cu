@@ -37,6 +37,8 @@
 // is bounded (see gs_tc_ptx.cuh); on expiry the CTA records GS_DEV_ERR_TIMEOUT,
 // unwinds, waits for its own copies and MMAs, frees TMEM and returns.
 
+#include <float.h>
+
 #include <algorithm>
 
 #include "gs_internal.h"
@@ -94,6 +96,8 @@ struct GemmParams {
     // tile are zero (R's echelon structure), so skipping them changes no sum
     int krange;
     int kb_lo[kMaxTilesN], kb_hi[kMaxTilesN];
+    float* xn2;             // kAF16 (optional): per converter group, the rows' partial ||a||^2 (2 x m)
+    const float* rowmul;    // optional: outputs of row i multiplied by rowmul[i]
 };
 
 struct Ctl {
@@ -342,6 +346,29 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
         const int l = threadIdx.x - (kCvt0 + g * kCvtGroupWarps) * 32;  // 0..127
         const int c4 = l & 15, rbase = l >> 4;
         float amax = 0.f;
+        // kAF16 with xn2: this group's part of each row's ||a||^2 over the current tile.  The 16
+        // lanes that share rows (one row phase, c4 = lane & 15) fold their 16 per-row K-block sums
+        // together in a butterfly after each K-block, so that lane c4 keeps the sum of row
+        // rbase + 8 c4 in one register; it is written out (for column tile 0, which every row
+        // block has) when the group moves to the next tile.
+        const bool want_xn2 = AMODE == kAF16 && p.xn2 != nullptr;
+        float nacc = 0.f;
+        int lt = 0, tile_end = 0;  // tile of the K-blocks being converted, and its end in `it`
+        if (ntiles > 0) {
+            long long tm;
+            int tn, lo, hi;
+            tile_mn(0, tm, tn);
+            krange(tn, lo, hi);
+            tile_end = hi - lo;
+        }
+        auto flush_xn2 = [&]() {
+            long long tm;
+            int tn;
+            tile_mn(lt, tm, tn);
+            const long long row = tm * kBM + rbase + kCvtRowStep * c4;
+            if (tn == 0 && row < p.m) p.xn2[(long long)g * p.m + row] = nacc;
+            nacc = 0.f;
+        };
         // ring positions of K-block g, then advanced by the two groups' K-blocks each step
         RingPos rx, ra;
         for (int j = 0; j < g; ++j) {
@@ -349,6 +376,17 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
             ra.next(p.sa);
         }
         for (int it = g; AMODE != kAF16T && it < total_it; it += kCvtGroups) {
+            if (want_xn2) {
+                while (it >= tile_end) {  // this group is done with tile lt
+                    flush_xn2();
+                    ++lt;
+                    long long tm;
+                    int tn, lo, hi;
+                    tile_mn(lt, tm, tn);
+                    krange(tn, lo, hi);
+                    tile_end += hi - lo;
+                }
+            }
             const int sx = rx.idx, sa = ra.idx;
             if (!mbar_wait_warp(&c.x_full[sx], rx.phase, abort_flag, err) ||
                 !mbar_wait_warp(&c.a_empty[sa], ra.phase ^ 1u, abort_flag, err))
@@ -359,7 +397,8 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
             }
             const uint8_t* Xt = Xs + (size_t)sx * kXStageBytes;
             uint8_t* At = As + (size_t)sa * p.parts * kAPartBytes;
-#pragma unroll 4
+            float nrm[kCvtRows];  // this K-block's part of ||a||^2 of each of the thread's rows
+#pragma unroll
             for (int u = 0; u < kCvtRows; ++u) {
                 const int row = rbase + kCvtRowStep * u;
                 const float4 x = *reinterpret_cast<const float4*>(Xt + row * (kBK * 4) + c4 * 16);
@@ -367,6 +406,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                 uint2 hi;
                 if (AMODE == kAF16) {
                     amax = fmaxf(amax, fmaxf(fmaxf(fabsf(x.x), fabsf(x.y)), fmaxf(fabsf(x.z), fabsf(x.w))));
+                    nrm[u] = fmaf(x.x, x.x, fmaf(x.y, x.y, fmaf(x.z, x.z, x.w * x.w)));
                     const __half2 h0 = __floats2half2_rn(x.x, x.y), h1 = __floats2half2_rn(x.z, x.w);
                     hi.x = *reinterpret_cast<const uint32_t*>(&h0);
                     hi.y = *reinterpret_cast<const uint32_t*>(&h1);
@@ -388,8 +428,30 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                 mbar_arrive(&c.a_full[sa]);
                 mbar_arrive(&c.x_empty[sx]);
             }
+            if (want_xn2) {
+                // butterfly over the 16 lanes of a row phase: after the step with lane bit b, a
+                // lane holds half as many rows, those whose index u has bit b equal to its own
+#pragma unroll
+                for (int w = kCvtRows / 2; w >= 1; w >>= 1) {
+                    const bool up = (lane & w) != 0;
+#pragma unroll
+                    for (int j = 0; j < w; ++j) {
+                        const float send = up ? nrm[j] : nrm[j + w];
+                        const float keep = up ? nrm[j + w] : nrm[j];
+                        nrm[j] = keep + __shfl_xor_sync(0xffffffffu, send, w);
+                    }
+                }
+                nacc += nrm[0];  // the K-block's sum for row rbase + 8 c4
+            }
         }
-        if (amax > 65504.f) atomicOr(err, GS_DEV_ERR_RANGE);
+        if (want_xn2) {
+            while (lt < ntiles) {  // the last tile (and any tile with no K-block of this group)
+                flush_xn2();
+                ++lt;
+            }
+        }
+        // with xn2 the caller recomputes the rows outside fp16's range; otherwise they are an error
+        if (!want_xn2 && amax > 65504.f) atomicOr(err, GS_DEV_ERR_RANGE);
     } else {
         // ------------------------------------------------------------- epilogue (warps 0-3, 15-18,
         // and with A loaded by TMA the idle converter warps 7-14 as well)
@@ -413,9 +475,12 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                 const int lrow = quad * 32 + half * 16;
                 const uint32_t tb = tmem + ((uint32_t)lrow << 16) + (uint32_t)(buf * 256);
                 const long long row[2] = {tm * kBM + lrow + (lane >> 2), tm * kBM + lrow + (lane >> 2) + 8};
-                float rn[2];
+                float rn[2], rm[2];
 #pragma unroll
-                for (int h = 0; h < 2; ++h) rn[h] = (p.rownorm && row[h] < p.m) ? p.rownorm[row[h]] : 1.f;
+                for (int h = 0; h < 2; ++h) {
+                    rn[h] = (p.rownorm && row[h] < p.m) ? p.rownorm[row[h]] : 1.f;
+                    rm[h] = (p.rowmul && row[h] < p.m) ? p.rowmul[row[h]] * p.alpha : p.alpha;
+                }
                 for (int jc = 32 * chunk; jc < tw; jc += 32 * nchunks) {
                     float v[16];
                     tmem_ld16x256b_x4(tb + (uint32_t)jc, v);
@@ -425,7 +490,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
 #pragma unroll
                         for (int h = 0; h < 2; ++h) {
                             if (row[h] >= p.m || col >= p.n) continue;
-                            float g0 = p.alpha * v[4 * j + 2 * h], g1 = p.alpha * v[4 * j + 2 * h + 1];
+                            float g0 = rm[h] * v[4 * j + 2 * h], g1 = rm[h] * v[4 * j + 2 * h + 1];
                             if (p.colnorm) {
                                 const float d0 = rn[h] * p.colnorm[col];
                                 const float d1 = col + 1 < p.n ? rn[h] * p.colnorm[col + 1] : 0.f;
@@ -475,35 +540,68 @@ size_t gemm_smem_bytes(int sx, int sa, int parts, int sb) {
 
 bool g_attr_set[64];
 
-// fp32 rows -> fp16 (RN), four columns per thread (X 16-byte aligned, ldx % 4 == 0;
-// out rows 8-byte aligned); values beyond the fp16 range are flagged
-__global__ void k_round_f16(const float* __restrict__ X, long long ldx, long long rows, int cols,
-                            __half* __restrict__ out, long long ldo) {
-    const int c4n = (cols + 3) / 4;
-    const long long total = rows * c4n;
-    float amax = 0.f;
-    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
-        const long long row = i / c4n;
-        const int c = (int)(i - row * c4n) * 4;
-        const float* src = X + row * ldx + c;
-        __half* dst = out + row * ldo + c;
-        if (c + 4 <= cols) {
-            const float4 v = *reinterpret_cast<const float4*>(src);
-            amax = fmaxf(amax, fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w))));
-            const __half2 h0 = __floats2half2_rn(v.x, v.y), h1 = __floats2half2_rn(v.z, v.w);
-            uint2 pk;
-            pk.x = *reinterpret_cast<const uint32_t*>(&h0);
-            pk.y = *reinterpret_cast<const uint32_t*>(&h1);
-            *reinterpret_cast<uint2*>(dst) = pk;
-        } else {
-            for (int j = 0; c + j < cols; ++j) {
-                amax = fmaxf(amax, fabsf(src[j]));
-                dst[j] = __float2half_rn(src[j]);
+// fp32 rows -> fp16 (RN), one warp per row: the row's largest magnitude a sets an exact scale 2^s
+// with 2^14 <= a 2^s < 2^15, so every scaled value is inside fp16's range and the row's mass far
+// above its subnormals; rowmul[row] = 2^-s undoes it in the GEMM's fp32 epilogue.  A zero row, or
+// one holding a non-finite value, keeps s = 0; rows whose largest magnitude is below 2^-112 take
+// the largest exact scale, 2^126.  Rows of up to 32 x 4 x kRoundRegs columns are read once into
+// registers; longer rows are read twice.  (X 16-byte aligned, ldx % 4 == 0; out rows 8-byte
+// aligned.)
+constexpr int kRoundRegs = 8;
+
+__device__ __forceinline__ float amax4(float a, float4 v) {
+    return fmaxf(a, fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w))));
+}
+
+__device__ __forceinline__ void store_h4(__half* dst, float4 v, float sc) {
+    const __half2 h0 = __floats2half2_rn(v.x * sc, v.y * sc), h1 = __floats2half2_rn(v.z * sc, v.w * sc);
+    uint2 pk;
+    pk.x = *reinterpret_cast<const uint32_t*>(&h0);
+    pk.y = *reinterpret_cast<const uint32_t*>(&h1);
+    *reinterpret_cast<uint2*>(dst) = pk;
+}
+
+__global__ void __launch_bounds__(256) k_round_f16(const float* __restrict__ X, long long ldx, long long rows,
+                                                   int cols, __half* __restrict__ out, long long ldo,
+                                                   float* __restrict__ rowmul) {
+    const int lane = threadIdx.x & 31;
+    const long long nw = (long long)gridDim.x * (blockDim.x >> 5);
+    const int c4n = cols / 4;
+    const bool in_regs = c4n <= 32 * kRoundRegs;
+    for (long long row = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); row < rows; row += nw) {
+        const float* src = X + row * ldx;
+        __half* dst = out + row * ldo;
+        float4 v[kRoundRegs];
+        float amax = 0.f;
+        if (in_regs) {
+#pragma unroll
+            for (int j = 0; j < kRoundRegs; ++j) {
+                const int c = lane + 32 * j;
+                v[j] = c < c4n ? *reinterpret_cast<const float4*>(src + 4 * c) : make_float4(0.f, 0.f, 0.f, 0.f);
+                amax = amax4(amax, v[j]);
             }
+        } else {
+            for (int c = lane; c < c4n; c += 32) amax = amax4(amax, *reinterpret_cast<const float4*>(src + 4 * c));
         }
+        const float tail = 4 * c4n + lane < cols ? src[4 * c4n + lane] : 0.f;  // cols % 4 elements
+        amax = fmaxf(amax, fabsf(tail));
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+        int e = 0;  // 2^14 <= amax 2^e < 2^15
+        if (amax > 0.f && amax <= FLT_MAX) e = min(14 - ilogbf(amax), 126);
+        const float sc = __int_as_float((127 + e) << 23);
+        if (in_regs) {
+#pragma unroll
+            for (int j = 0; j < kRoundRegs; ++j) {
+                const int c = lane + 32 * j;
+                if (c < c4n) store_h4(dst + 4 * c, v[j], sc);
+            }
+        } else {
+            for (int c = lane; c < c4n; c += 32) store_h4(dst + 4 * c, *reinterpret_cast<const float4*>(src + 4 * c), sc);
+        }
+        if (4 * c4n + lane < cols) dst[4 * c4n + lane] = __float2half_rn(tail * sc);
+        if (lane == 0) rowmul[row] = __int_as_float((127 - e) << 23);
     }
-    if (amax > 65504.f) atomicOr(&g_err_gemm, GS_DEV_ERR_RANGE);
 }
 
 }  // namespace
@@ -569,6 +667,8 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     p.alpha = a.alpha;
     p.rownorm = a.rownorm;
     p.colnorm = a.colnorm;
+    p.xn2 = p.amode == kAF16 ? a.xn2_out : nullptr;
+    p.rowmul = a.rowmul;
     p.krange = 0;
     if (a.b_klo && a.b_khi && p.tiles_n <= kMaxTilesN) {
         // per column tile: the K-blocks holding the tile's nonzero B entries
@@ -621,11 +721,10 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
 namespace gs {
 
 cudaError_t launch_round_f16(const float* X, long long ldx, long long rows, int cols, void* out, long long ldo,
-                             cudaStream_t s) {
+                             float* rowmul, cudaStream_t s) {
     if (rows <= 0 || cols <= 0) return cudaSuccess;
-    const long long work = rows * ((cols + 3) / 4);
-    const int grid = (int)std::min<long long>((work + 255) / 256, 152LL * 8);
-    k_round_f16<<<grid, 256, 0, s>>>(X, ldx, rows, cols, static_cast<__half*>(out), ldo);
+    const int grid = (int)std::min<long long>((rows + 7) / 8, 152LL * 8);  // 8 rows (warps) per block
+    k_round_f16<<<grid, 256, 0, s>>>(X, ldx, rows, cols, static_cast<__half*>(out), ldo, rowmul);
     return cudaGetLastError();
 }
 

@@ -120,6 +120,10 @@ struct GemmArgs {
     float alpha;
     const float* rownorm; const float* colnorm;
     const int* b_rowlen;  // optional (b_trans only): row j of B is zero beyond b_rowlen[j]
+    // optional gate (batch 1, no split): only 64-row tiles holding a row i whose squared norm
+    // gate_xn2[i] + gate_xn2[gate_ld + i] is nonzero and outside [gate_lo, gate_hi] are computed;
+    // the other blocks return at once (rewrites the rows that one fp16 rounding could not hold)
+    const float* gate_xn2; long long gate_ld; float gate_lo, gate_hi;
     int ksplit;           // > 1 (batch 1, fp32 C only): K is cut into ksplit chunks, one per
                           // grid z index; each chunk's m x n partial product goes to kpart
                           // (ksplit x m x n floats, caller's workspace) and a second kernel
@@ -182,11 +186,20 @@ struct GemmTcArgs {
     // optional HOST arrays (n each): B row j is zero outside K columns [b_klo[j], b_khi[j]);
     // K-blocks outside a column tile's union are skipped (exact: only zero products dropped)
     const int* b_klo; const int* b_khi;
+    // fp16-rounded fp32 A only (optional): the converters write each row's squared norm, as two
+    // partial sums xn2_out[row] + xn2_out[m + row] (2 x m floats), so the caller can find the rows
+    // that one fp16 rounding cannot represent accurately
+    float* xn2_out;
+    // optional (m floats): every output of row i is multiplied by rowmul[i] (the inverse of an
+    // exact power-of-two scale applied to A's row before its fp16 rounding)
+    const float* rowmul;
 };
 cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s);
-// fp32 rows -> fp16 (RN), for the fp16-A GEMM; values beyond the fp16 range set GS_DEV_ERR_RANGE
+// fp32 rows -> fp16 (RN) for the fp16-A GEMM, each row first multiplied by the exact power of two
+// 2^s that brings its largest magnitude to [2^14, 2^15) (inside fp16's range, far above its
+// subnormals); rowmul[row] receives 2^-s.  Rows that are zero or hold a non-finite value keep s = 0.
 cudaError_t launch_round_f16(const float* X, long long ldx, long long rows, int cols, void* out, long long ldo,
-                             cudaStream_t s);
+                             float* rowmul, cudaStream_t s);
 
 // ----------------------------------------------------------------- attention scores on tcgen05 (gs_attn_tc.cu)
 // bf16 Yq (B x Lq x r) and Yk (B x Lk x r), row stride ldy; fp32 A (B x Lq x Lk, dense).

@@ -201,16 +201,15 @@ __device__ __forceinline__ float ld_elem(const void* p, long long i) {
     return __bfloat162float(((const __nv_bfloat16*)p)[i]);
 }
 
+// One 64 x 64 output tile (rows m0.., columns n0..) of batch b, or of K chunk kz with ksplit;
+// called by every thread of the block.
 template <int TA, int TB, int TC, bool BT>
-__global__ void __launch_bounds__(256) k_gemm(GemmArgs g) {
-    __shared__ float As[kTK][kTM + 4];
-    __shared__ __align__(16) float Bs[kTK][kTN + 4];
+__device__ __forceinline__ void gemm_tile(const GemmArgs& g, long long m0, int n0, int kz,
+                                          float (&As)[kTK][kTM + 4], float (&Bs)[kTK][kTN + 4]) {
     const int tid = threadIdx.x;
     const int tx = tid % 16, ty = tid / 16;
-    const long long m0 = (long long)blockIdx.y * kTM;
-    const int n0 = blockIdx.x * kTN;
     const bool split = g.ksplit > 1;
-    const int b = split ? 0 : blockIdx.z;
+    const int b = split ? 0 : kz;
     const char* Ab = (const char*)g.A + (size_t)b * g.a_bstride * (TA == MAT_F32 ? 4 : 2);
     const char* Bb = (const char*)g.B + (size_t)b * g.b_bstride * (TB == MAT_F32 ? 4 : 2);
     int kend = g.k;
@@ -230,7 +229,7 @@ __global__ void __launch_bounds__(256) k_gemm(GemmArgs g) {
     int kbeg = 0;
     if (split) {  // this block's chunk of K (chunks are whole kTK steps)
         const int chunk = ((g.k + g.ksplit - 1) / g.ksplit + kTK - 1) / kTK * kTK;
-        kbeg = blockIdx.z * chunk;
+        kbeg = kz * chunk;
         kend = min(kend, kbeg + chunk);
     }
     float acc[4][4] = {};
@@ -281,12 +280,46 @@ __global__ void __launch_bounds__(256) k_gemm(GemmArgs g) {
                 v = den > 0.f ? v / den : 0.f;
             }
             if (TC == MAT_F32) {
-                if (split) g.kpart[((size_t)blockIdx.z * g.m + gm) * g.n + gn] = v;
+                if (split) g.kpart[((size_t)kz * g.m + gm) * g.n + gn] = v;
                 else ((float*)Cb)[gm * g.ldc + gn] = v;
             } else {
                 ((__nv_bfloat16*)Cb)[gm * g.ldc + gn] = __float2bfloat16_rn(v);
             }
         }
+    }
+}
+
+template <int TA, int TB, int TC, bool BT>
+__global__ void __launch_bounds__(256) k_gemm(GemmArgs g) {
+    __shared__ float As[kTK][kTM + 4];
+    __shared__ __align__(16) float Bs[kTK][kTN + 4];
+    gemm_tile<TA, TB, TC, BT>(g, (long long)blockIdx.y * kTM, blockIdx.x * kTN, blockIdx.z, As, Bs);
+}
+
+// The gated product (gate_xn2): persistent blocks walk the 64 x 64 tiles, n fastest, and compute
+// only those whose 64 rows hold a selected row; with no such row the launch is one pass over
+// the norms.
+template <int TA, int TB, int TC, bool BT>
+__global__ void __launch_bounds__(256) k_gemm_gated(GemmArgs g) {
+    __shared__ float As[kTK][kTM + 4];
+    __shared__ __align__(16) float Bs[kTK][kTN + 4];
+    const int tiles_n = (g.n + kTN - 1) / kTN;
+    const long long tiles = (g.m + kTM - 1) / kTM * tiles_n;
+    long long last_m0 = -1;
+    bool any = false;
+    for (long long t = blockIdx.x; t < tiles; t += gridDim.x) {
+        const long long m0 = t / tiles_n * kTM;
+        if (m0 != last_m0) {
+            bool mine = false;
+            if (threadIdx.x < kTM && m0 + threadIdx.x < g.m) {
+                const long long i = m0 + threadIdx.x;
+                const float xn2 = g.gate_xn2[i] + g.gate_xn2[g.gate_ld + i];
+                mine = xn2 > 0.f && !(xn2 >= g.gate_lo && xn2 <= g.gate_hi);
+            }
+            any = __syncthreads_or(mine) != 0;
+            last_m0 = m0;
+        }
+        if (any) gemm_tile<TA, TB, TC, BT>(g, m0, (int)(t % tiles_n) * kTN, 0, As, Bs);
     }
 }
 
@@ -615,6 +648,18 @@ cudaError_t launch_coeffs_warp(const float* Y, long long N, int ldy, int r, cons
 cudaError_t launch_gemm_simt(const GemmArgs& g, cudaStream_t s) {
     if (g.m <= 0 || g.n <= 0 || g.batch <= 0) return cudaSuccess;
     if (g.ksplit > 1 && (g.batch != 1 || g.c_type != MAT_F32 || !g.kpart)) return cudaErrorInvalidValue;
+    if (g.gate_xn2) {
+        if (g.batch != 1 || g.ksplit > 1 || g.a_type != MAT_F32 || g.b_type != MAT_F32 || g.c_type != MAT_F32 ||
+            !g.b_trans)
+            return cudaErrorInvalidValue;
+        int dev = 0, sms = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        const long long tiles = (g.m + kTM - 1) / kTM * ((g.n + kTN - 1) / kTN);
+        const int grid = (int)std::min<long long>(tiles, 4LL * std::max(sms, 1));
+        k_gemm_gated<MAT_F32, MAT_F32, MAT_F32, true><<<grid, 256, 0, s>>>(g);
+        return cudaGetLastError();
+    }
     dim3 grid((unsigned)((g.n + kTN - 1) / kTN), (unsigned)((g.m + kTM - 1) / kTM),
               (unsigned)(g.ksplit > 1 ? g.ksplit : g.batch));
     if (grid.y > 65535u) return cudaErrorInvalidConfiguration;

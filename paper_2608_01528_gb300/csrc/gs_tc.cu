@@ -123,6 +123,7 @@ struct PsParams {
     int sx, sa, sb;         // ring depths: fp32 X staging, fp16 A, B operand tiles
     int box_rows;           // rows of each X TMA box (>= every tile's rows)
     int xstage;             // bytes between X staging tiles (box_rows x 256, 1 KB aligned)
+    float xn2_lo, xn2_hi;   // rows with ||x||^2 outside [lo, hi] (and > 0) are redone scaled
     const float* cnorm;     // M
     int mode;
     float scale;
@@ -141,11 +142,49 @@ struct Ctl {
     uint64_t y_full, s_full, s_empty, gemm2_done;
     uint64_t ysplit[kMaxKR];  // Y columns [64 k, 64 k + 64) split in TMEM (GEMM2 K-block k may start)
     uint64_t xn_full[2], xn_empty[2];
+    uint64_t dec_full[2];     // redo decision of regular tile t published in slot t % 2
     uint64_t mma_done;
     float xn[2][kBM];  // ||x||^2 per row, both converter groups add into it
+    int8_t rsc[2][kBM];      // per-row exponent s of the redo's scale 2^s, for the tile in that slot
+    int redo[2][kEpiWarps];  // per epilogue warp: some row of its lane quadrant needs the redo
     uint32_t tmem_base;
     int abort_flag;
 };
+
+// Exact power of two 2^k (|k| <= 126).
+__device__ __forceinline__ float pow2f(int k) { return __int_as_float((127 + k) << 23); }
+
+// The exponent s that brings a row of squared norm xn2 to 2^14 <= ||x|| 2^s < 2^15: every
+// element then lies below 2^15 (inside fp16's range) and the row's mass far above fp16's
+// subnormals.  s lies in [-49, 89] for any finite positive fp32 xn2; rows whose squared norm is
+// not a finite positive number keep s = 0.
+__device__ __forceinline__ int row_scale_exp(float xn2) {
+    if (!(xn2 > 0.f) || !(xn2 <= FLT_MAX)) return 0;
+    return 14 - (ilogbf(xn2) >> 1);  // ilogbf(xn2) >> 1 = floor(log2 ||x||)
+}
+
+// Processing order of a CTA's tiles: regular tile t, and once tile t + 1 has been handed on, the
+// redo of tile t when its epilogue asked for one (the decision is published in slot t % 2, so it
+// is always known by then and nobody waits on it in the common case).  body(t, redo, q) runs one
+// tile; q counts processed tiles (the per-tile barrier phases and the norm buffers follow it).
+// wait(bar, parity) is the role's bounded wait.  Returns false when a wait or the body gave up.
+template <class Wait, class Body>
+__device__ __forceinline__ bool walk_tiles(const CtaRows& cr, Ctl& c, Wait wait, Body body) {
+    int q = 0;
+    for (int t = 0; t <= cr.ntiles; ++t) {
+        if (t < cr.ntiles && !body(t, false, q++)) return false;
+        if (t >= 1) {
+            const int d = t - 1, slot = d & 1;
+            if (!wait(&c.dec_full[slot], (uint32_t)(d >> 1) & 1u)) return false;
+            const volatile int* rd = c.redo[slot];
+            bool again = false;
+#pragma unroll
+            for (int w = 0; w < kEpiWarps; ++w) again |= rd[w] != 0;
+            if (again && !body(d, true, q++)) return false;
+        }
+    }
+    return true;
+}
 
 // FULL = false: raw scores with only argmax / maxval out (the large-batch lookup); true: every
 // mode and output.  A template parameter, so the lookup kernel carries none of the other paths.
@@ -188,6 +227,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int b = 0; b < 2; ++b) {
             mbar_init(&c.xn_full[b], kCvtWarps);
             mbar_init(&c.xn_empty[b], kEpiWarps);
+            mbar_init(&c.dec_full[b], kEpiWarps);
         }
         mbar_init(&c.mma_done, 1);
         c.abort_flag = 0;
@@ -202,6 +242,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = c.tmem_base;
+    auto wait_1t = [&](uint64_t* bar, uint32_t par) { return mbar_wait_1t(bar, par, abort_flag, &g_err_tc); };
+    auto wait_warp = [&](uint64_t* bar, uint32_t par) { return mbar_wait_warp(bar, par, abort_flag, &g_err_tc); };
 
     if (warp == kXWarp) {
         // ------------------------------------------------------------- X tiles via TMA
@@ -210,19 +252,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t bytes = (uint32_t)p.box_rows * kBK * 4;
             int it = 0;
             RingPos xs;
-            bool ok = true;
-            for (int t = 0; t < cr.ntiles && ok; ++t) {
+            walk_tiles(cr, c, wait_1t, [&](int t, bool, int) {
                 const TileRange tr = cr.tile(t);
                 for (int kb = 0; kb < p.nkb; ++kb, ++it, xs.next(p.sx)) {
-                    if (!mbar_wait_1t(&c.x_empty[xs.idx], xs.phase ^ 1u, abort_flag, &g_err_tc)) {
-                        ok = false;
-                        break;
-                    }
+                    if (!wait_1t(&c.x_empty[xs.idx], xs.phase ^ 1u)) return false;
                     mbar_arrive_expect_tx(&c.x_full[xs.idx], bytes);
                     tma_load_2d(Xs + (size_t)xs.idx * p.xstage, &tmap_x, &c.x_full[xs.idx], kb * kBK, (int)tr.row0,
                                 pol);
                 }
-            }
+                return true;
+            });
             // every copy this thread started lands before the CTA can exit
             for (int j = std::max(0, it - p.sx); j < it; ++j) mbar_drain(&c.x_full[j % p.sx], (uint32_t)(j / p.sx) & 1u, &g_err_tc);
         }
@@ -235,25 +274,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t qbytes = (uint32_t)p.npad * kBK * 2, rbytes = 2u * (uint32_t)p.half_rows * kBK * 2;
             const uint32_t rl_off = (uint32_t)p.half_rows * kBK * 2;  // Rl after Rh in the slot
             const int per_tile = p.nkb + p.nkr_h[0] + p.nkr_h[1];
-            const int total = cr.ntiles * per_tile;
             int it = 0;
             RingPos bs;
-            for (int k = 0; it < total; ++it, bs.next(p.sb), k = k + 1 == per_tile ? 0 : k + 1) {
-                const int s = bs.idx;
-                if (!mbar_wait_1t(&c.b_empty[s], bs.phase ^ 1u, abort_flag, &g_err_tc)) break;
-                uint8_t* dst = Bs + (size_t)s * kBStageBytes;
-                if (k < p.nkb) {
-                    mbar_arrive_expect_tx(&c.b_full[s], qbytes);
-                    tma_load_2d(dst, &tmap_q, &c.b_full[s], k * kBK, 0, pol);
-                } else {
-                    const int j = k - p.nkb;
-                    const int h = j < p.nkr_h[0] ? 0 : 1;
-                    const int kr = h ? j - p.nkr_h[0] : j;
-                    mbar_arrive_expect_tx(&c.b_full[s], rbytes);
-                    tma_load_2d(dst, &tmap_rh, &c.b_full[s], kr * kBK, h * p.half_rows, pol);
-                    tma_load_2d(dst + rl_off, &tmap_rl, &c.b_full[s], kr * kBK, h * p.half_rows, pol);
+            walk_tiles(cr, c, wait_1t, [&](int, bool, int) {
+                for (int k = 0; k < per_tile; ++k, ++it, bs.next(p.sb)) {
+                    const int s = bs.idx;
+                    if (!wait_1t(&c.b_empty[s], bs.phase ^ 1u)) return false;
+                    uint8_t* dst = Bs + (size_t)s * kBStageBytes;
+                    if (k < p.nkb) {
+                        mbar_arrive_expect_tx(&c.b_full[s], qbytes);
+                        tma_load_2d(dst, &tmap_q, &c.b_full[s], k * kBK, 0, pol);
+                    } else {
+                        const int j = k - p.nkb;
+                        const int h = j < p.nkr_h[0] ? 0 : 1;
+                        const int kr = h ? j - p.nkr_h[0] : j;
+                        mbar_arrive_expect_tx(&c.b_full[s], rbytes);
+                        tma_load_2d(dst, &tmap_rh, &c.b_full[s], kr * kBK, h * p.half_rows, pol);
+                        tma_load_2d(dst + rl_off, &tmap_rl, &c.b_full[s], kr * kBK, h * p.half_rows, pol);
+                    }
                 }
-            }
+                return true;
+            });
             for (int j = std::max(0, it - p.sb); j < it; ++j) mbar_drain(&c.b_full[j % p.sb], (uint32_t)(j / p.sb) & 1u, &g_err_tc);
         }
     } else if (warp == kMmaWarp) {
@@ -263,17 +304,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t idesc2 = idesc_bf16_f32(p.half_rows);
             const uint32_t y_tmem = tmem, s_tmem = tmem + kSCol;
             RingPos ra, rb;
-            bool ok = true;
-            for (int t = 0; t < cr.ntiles && ok; ++t) {
-                const uint32_t pt = (uint32_t)t & 1u;
+            walk_tiles(cr, c, wait_1t, [&](int, bool, int q) {
+                const uint32_t pt = (uint32_t)q & 1u;
                 // GEMM1: Y = X Q^T into columns [0, npad)
                 for (int kb = 0; kb < p.nkb; ++kb, ra.next(p.sa), rb.next(p.sb)) {
                     const int sa = ra.idx, sb = rb.idx;
-                    if (!mbar_wait_1t(&c.a_full[sa], ra.phase, abort_flag, &g_err_tc) ||
-                        !mbar_wait_1t(&c.b_full[sb], rb.phase, abort_flag, &g_err_tc)) {
-                        ok = false;
-                        break;
-                    }
+                    if (!wait_1t(&c.a_full[sa], ra.phase) || !wait_1t(&c.b_full[sb], rb.phase)) return false;
                     tc_fence_after();
                     const uint64_t ad = sdesc_sw128(smem_u32(As + (size_t)sa * kAStageBytes));
                     const uint64_t bd = sdesc_sw128(smem_u32(Bs + (size_t)sb * kBStageBytes));
@@ -284,22 +320,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mma_commit(&c.a_empty[sa]);
                     mma_commit(&c.b_empty[sb]);
                 }
-                if (!ok) break;
                 mma_commit(&c.y_full);
                 // GEMM2: S = Yh Rh + Yl Rh + Yh Rl into columns [256, 256 + mpad), once the
                 // epilogue has split Y in place and released the previous tile's S
-                if (!mbar_wait_1t(&c.s_empty, pt ^ 1u, abort_flag, &g_err_tc)) break;
+                if (!wait_1t(&c.s_empty, pt ^ 1u)) return false;
                 int nsplit = 0;  // K-blocks of Y known to be split; the epilogue signals each one
-                for (int h = 0; h < p.nh && ok; ++h) {
+                for (int h = 0; h < p.nh; ++h) {
                     const uint32_t s_half = s_tmem + (uint32_t)(h * p.half_rows);
                     for (int kr = 0; kr < p.nkr_h[h]; ++kr, rb.next(p.sb)) {
-                        for (; nsplit <= kr && ok; ++nsplit)
-                            ok = mbar_wait_1t(&c.ysplit[nsplit], pt, abort_flag, &g_err_tc);
+                        for (; nsplit <= kr; ++nsplit)
+                            if (!wait_1t(&c.ysplit[nsplit], pt)) return false;
                         const int sr = rb.idx;
-                        if (!ok || !mbar_wait_1t(&c.b_full[sr], rb.phase, abort_flag, &g_err_tc)) {
-                            ok = false;
-                            break;
-                        }
+                        if (!wait_1t(&c.b_full[sr], rb.phase)) return false;
                         tc_fence_after();
                         const uint32_t rs = smem_u32(Bs + (size_t)sr * kBStageBytes);
                         const uint64_t rh = sdesc_sw128(rs);
@@ -319,13 +351,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                         mma_commit(&c.b_empty[sr]);
                     }
                 }
-                if (!ok) break;
                 mma_commit(&c.s_full);
                 // the next tile's GEMM1 overwrites the columns GEMM2 reads: wait for it to finish
                 mma_commit(&c.gemm2_done);
-                if (!mbar_wait_1t(&c.gemm2_done, pt, abort_flag, &g_err_tc)) break;
+                if (!wait_1t(&c.gemm2_done, pt)) return false;
                 tc_fence_after();
-            }
+                return true;
+            });
             // all MMAs issued by this thread complete before TMEM is released
             mma_commit(&c.mma_done);
             mbar_drain(&c.mma_done, 0, &g_err_tc);
@@ -336,25 +368,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int l = threadIdx.x - (kCvt0 + g * kCvtGroupWarps) * 32;  // 0..127 within the group
         const int c4 = l & 15;                   // float4 column of the 64-wide K-block
         const int rbase = l >> 4;                // rows rbase + 8u, u < 16
-        const bool want_norm = FULL && p.mode == GS_SCORE_COSINE;
         float nrm[kCvtRows];
 #pragma unroll
         for (int u = 0; u < kCvtRows; ++u) nrm[u] = 0.f;
         float amax = 0.f;
         int it = 0;
         RingPos rx, ra;  // every K-block advances both rings; this group takes those with it % 2 == g
-        bool ok = true;
-        for (int t = 0; t < cr.ntiles && ok; ++t) {
+        walk_tiles(cr, c, wait_warp, [&](int t, bool redo, int q) {
             const TileRange tr = cr.tile(t);
-            const int b = t & 1;
+            const int b = q & 1;
+            const int8_t* rs = c.rsc[t & 1];  // the rows' scale exponents (redo only)
             for (int kb = 0; kb < p.nkb; ++kb, ++it, rx.next(p.sx), ra.next(p.sa)) {
                 if ((it & 1) != g) continue;
                 const int sx = rx.idx, sa = ra.idx;
-                if (!mbar_wait_warp(&c.x_full[sx], rx.phase, abort_flag, &g_err_tc) ||
-                    !mbar_wait_warp(&c.a_empty[sa], ra.phase ^ 1u, abort_flag, &g_err_tc)) {
-                    ok = false;
-                    break;
-                }
+                if (!wait_warp(&c.x_full[sx], rx.phase) || !wait_warp(&c.a_empty[sa], ra.phase ^ 1u)) return false;
                 const uint8_t* Xt = Xs + (size_t)sx * p.xstage;
                 uint8_t* At = As + (size_t)sa * kAStageBytes;
 #pragma unroll
@@ -362,8 +389,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int row = rbase + kCvtRowStep * u;
                     float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
                     if (row < tr.nrows) x = *reinterpret_cast<const float4*>(Xt + row * (kBK * 4) + c4 * 16);
-                    if (want_norm) nrm[u] = fmaf(x.x, x.x, fmaf(x.y, x.y, fmaf(x.z, x.z, fmaf(x.w, x.w, nrm[u]))));
-                    amax = fmaxf(amax, fmaxf(fmaxf(fabsf(x.x), fabsf(x.y)), fmaxf(fabsf(x.z), fabsf(x.w))));
+                    if (redo) {  // exact power-of-two scale: the fp16 rounding below loses nothing to range
+                        const float sc = pow2f(rs[row]);
+                        x.x *= sc;
+                        x.y *= sc;
+                        x.z *= sc;
+                        x.w *= sc;
+                        amax = fmaxf(amax, fmaxf(fmaxf(fabsf(x.x), fabsf(x.y)), fmaxf(fabsf(x.z), fabsf(x.w))));
+                    }
+                    nrm[u] = fmaf(x.x, x.x, fmaf(x.y, x.y, fmaf(x.z, x.z, fmaf(x.w, x.w, nrm[u]))));
                     const __half2 h0 = __floats2half2_rn(x.x, x.y);
                     const __half2 h1 = __floats2half2_rn(x.z, x.w);
                     uint2 pk;
@@ -379,7 +413,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mbar_arrive(&c.x_empty[sx]);
                 }
             }
-            if (!ok) break;
             // tile finished: this group's part of ||x||^2 of each row is added into shared memory
 #pragma unroll
             for (int u = 0; u < kCvtRows; ++u) {
@@ -390,8 +423,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 v += __shfl_xor_sync(0xffffffffu, v, 1);
                 nrm[u] = v;
             }
-            if (!mbar_wait_warp(&c.xn_empty[b], ((uint32_t)(t >> 1) & 1u) ^ 1u, abort_flag, &g_err_tc)) break;
-            if (want_norm && (lane & 15) == 0) {
+            if (!wait_warp(&c.xn_empty[b], ((uint32_t)(q >> 1) & 1u) ^ 1u)) return false;
+            if ((lane & 15) == 0) {
 #pragma unroll
                 for (int u = 0; u < kCvtRows; ++u) atomicAdd(&c.xn[b][rbase + kCvtRowStep * u], nrm[u]);
             }
@@ -399,21 +432,25 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (lane == 0) mbar_arrive(&c.xn_full[b]);
 #pragma unroll
             for (int u = 0; u < kCvtRows; ++u) nrm[u] = 0.f;
-        }
+            return true;
+        });
+        // only a redone row can still leave fp16's range (a norm that is not a finite fp32 number)
         if (amax > 65504.f) atomicOr(&g_err_tc, GS_DEV_ERR_RANGE);
     } else {
         // ------------------------------------------------------------- epilogue (warps 0-3)
         const int i = threadIdx.x;  // row within the tile = TMEM lane
         const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
         const uint32_t ty = tmem + lane_base, ts = tmem + lane_base + kSCol;
-        for (int t = 0; t < cr.ntiles; ++t) {
-            const uint32_t pt = (uint32_t)t & 1u;
-            const int b = t & 1;
-            if (!mbar_wait_warp(&c.y_full, pt, abort_flag, &g_err_tc)) break;
+        walk_tiles(cr, c, wait_warp, [&](int t, bool redo, int q) {
+            const uint32_t pt = (uint32_t)q & 1u;
+            const int b = q & 1;
+            if (!wait_warp(&c.y_full, pt)) return false;
             tc_fence_after();
             const TileRange tr = cr.tile(t);
             const bool valid = i < tr.nrows;
             const long long row = tr.row0 + i;
+            // a redone tile ran on x 2^s: Y and ||x|| come back multiplied by 2^s
+            const float unscale = redo ? pow2f(-c.rsc[t & 1][i]) : 1.f;
             // split Y in place: chunk of 16 fp32 columns -> 8 columns bf16(Y) + 8 columns
             // bf16(Y - bf16(Y)), read 32 columns per TMEM load wait.  Each finished K-block
             // of 64 columns is signalled on its own, so GEMM2 starts on it while the rest
@@ -425,6 +462,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tmem_ld32(ty + (uint32_t)jc, y);
                 else
                     tmem_ld16(ty + (uint32_t)jc, y);
+                if (redo) {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) y[j] *= unscale;
+                }
                 if (FULL && p.Y && valid) {
                     float* dst = p.Y + (size_t)row * p.ldy + jc;
 #pragma unroll
@@ -452,12 +493,27 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (lane == 0) mbar_arrive(&c.ysplit[jc >> 6]);
                 }
             }
-            if (!mbar_wait_warp(&c.xn_full[b], (uint32_t)(t >> 1) & 1u, abort_flag, &g_err_tc)) break;
-            const float xnorm = sqrtf(c.xn[b][i]);
+            if (!wait_warp(&c.xn_full[b], (uint32_t)(q >> 1) & 1u)) return false;
+            const float xn2 = c.xn[b][i];
             c.xn[b][i] = 0.f;  // ready for the tile after next (both groups add into it)
             __syncwarp();
             if (lane == 0) mbar_arrive(&c.xn_empty[b]);
-            if (!mbar_wait_warp(&c.s_full, pt, abort_flag, &g_err_tc)) break;
+            const float xnorm = sqrtf(xn2) * unscale;
+            if (!redo) {
+                // one fp16 rounding of x is accurate when every element is inside fp16's range
+                // (||x|| <= 2^15) and the row's mass is far above its subnormals (||x|| >= 2^-8
+                // sqrt(D): the subnormals' absolute errors, at most 2^-25 each, then add at most
+                // 2^-19 ||x|| to the error of <x, q_j>); any other nonzero row has its tile redone
+                // with an exact power-of-two scale (a norm that is not a number keeps scale 1)
+                const bool bad = xn2 > 0.f && !(xn2 >= p.xn2_lo && xn2 <= p.xn2_hi);
+                const int slot = t & 1;
+                c.rsc[slot][i] = (int8_t)row_scale_exp(xn2);
+                const unsigned any = __ballot_sync(0xffffffffu, bad);
+                if (lane == 0) c.redo[slot][warp] = any != 0u;
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&c.dec_full[slot]);
+            }
+            if (!wait_warp(&c.s_full, pt)) return false;
             tc_fence_after();
             float best = -FLT_MAX, run_max = -FLT_MAX, run_sum = 0.f;
             int besti = 0;
@@ -492,7 +548,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&c.s_empty);
-            if (!valid) continue;
+            if (!valid) return true;
             float outmax = best;
             if (FULL && p.mode == GS_SCORE_SOFTMAX) {
                 const float inv = 1.f / run_sum;
@@ -504,7 +560,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (p.argmax) p.argmax[row] = besti;
             if (p.maxval) p.maxval[row] = outmax;
-        }
+            return true;
+        });
     }
 
     tc_fence_before();
@@ -720,6 +777,9 @@ cudaError_t launch_ps_tc(const gs_basis* h, const float* X, long long N, int ldx
     p.sb = g.sb;
     p.box_rows = box_rows;
     p.xstage = ps_xstage(box_rows);
+    // one fp16 rounding of a row is accurate for 2^-8 sqrt(D) <= ||x|| <= 2^15; other rows are redone
+    p.xn2_lo = (float)h->D * 0x1p-16f;
+    p.xn2_hi = 0x1p30f;
     p.cnorm = h->cnorm;
     p.mode = mode;
     p.scale = scale;
