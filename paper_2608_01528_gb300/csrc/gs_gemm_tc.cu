@@ -26,7 +26,8 @@
 // Tiles are 128 x nt (nt <= 256) with the fp32 accumulator double-buffered in
 // TMEM (2 x 256 columns), or, for a long K with A rounded to fp16 and n > 256, 128 x 512
 // (two 256-column accumulators filling TMEM, single-buffered: each converted A K-block
-// feeds both); one persistent CTA per SM walks the tiles with the n index fastest, so
+// feeds both); one persistent CTA per SM walks the tiles with the n index fastest (rotated
+// each wave so that no CTA keeps one column tile), so
 // CTAs running at the same time share A rows in L2.
 // Warp roles (608 threads): 0-3 and 15-18 epilogue (warp w reads TMEM lanes
 // 32 (w % 4)..+31; the two warps of a lane quadrant take alternate 32-column chunks,
@@ -96,6 +97,7 @@ struct GemmParams {
     // tile are zero (R's echelon structure), so skipping them changes no sum
     int krange;
     int kb_lo[kMaxTilesN], kb_hi[kMaxTilesN];
+    int rotate;             // the grid is a multiple of tiles_n: column tiles rotate by one each wave
     float* xn2;             // kAF16 (optional): per converter group, the rows' partial ||a||^2 (2 x m)
     const float* rowmul;    // optional: outputs of row i multiplied by rowmul[i]
 };
@@ -135,10 +137,24 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
         lo = p.krange ? p.kb_lo[tn] : 0;
         hi = p.krange ? p.kb_hi[tn] : p.nkb;
     };
+    // Tile lt of this CTA is tile index tg = blockIdx.x + lt gridDim.x: row block tg / tiles_n and
+    // column tile tg mod tiles_n, rotated by one each wave (lt) when the grid is a multiple of
+    // tiles_n (p.rotate).  CTAs working at the same time share A row blocks in L2, and no CTA keeps
+    // one column tile: with trimmed K ranges (R's echelon structure) column tiles differ in length,
+    // and the CTAs fixed to the longest would set the kernel's time.  (A wave then covers whole row
+    // blocks, so the rotation permutes each block's column tiles; with any other grid the plain
+    // order already moves every CTA through the column tiles.)
+    auto tile_mn = [&](int lt, long long& tm, int& tn) {
+        const long long tg = blockIdx.x + (long long)lt * gridDim.x;
+        tm = tg / p.tiles_n;
+        tn = (int)((tg + (p.rotate ? lt : 0)) % p.tiles_n);
+    };
     int total_it = 0;  // K-blocks over this CTA's tiles
     for (int lt = 0; lt < ntiles; ++lt) {
-        int lo, hi;
-        krange((int)((blockIdx.x + (long long)lt * gridDim.x) % p.tiles_n), lo, hi);
+        long long tm;
+        int tn, lo, hi;
+        tile_mn(lt, tm, tn);
+        krange(tn, lo, hi);
         total_it += hi - lo;
     }
 
@@ -171,12 +187,6 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = c.tmem_base;
-
-    auto tile_mn = [&](int lt, long long& tm, int& tn) {
-        const long long tg = blockIdx.x + (long long)lt * gridDim.x;
-        tm = tg / p.tiles_n;
-        tn = (int)(tg % p.tiles_n);
-    };
 
     if (warp == kAWarp && AMODE == kAF16T) {
         // ------------------------------------------------------------- A tiles (fp16) via TMA
@@ -705,6 +715,7 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     int sms = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
     const int grid = (int)std::min<long long>(sms > 0 ? sms : 1, p.tiles);
+    p.rotate = grid % p.tiles_n == 0 ? 1 : 0;
     if (halves == 2)
         k_gemm_tc<kAF16, 2><<<grid, kThreads, smem, s>>>(ta, tb0, tb1, p);
     else if (p.amode == kAF16)
