@@ -503,6 +503,8 @@ def side_rows(gs, dev):
     Zb = torch.empty(Nb, b5.D, device=dev)
     Xb = torch.empty(Nb, b5.D, device=dev)
     ms_fused = timeit(lambda: gs.reconstruct_bind(b5, Tb, Yb, Lb, out=Zb))
+    # one partner row for every row: the basis rows are bound once, one reconstruction GEMM
+    ms_fused_one = timeit(lambda: gs.reconstruct_bind(b5, Tb, Yb[:1], Lb, out=Zb))
     ms_rec = timeit(lambda: gs.reconstruct(b5, Tb, out=Xb))
     # binding through block spectra (the default): X, Y read and Z written once, 12 D bytes a row
     ms_bind = timeit(lambda: gs.bind(Xb, Yb, Lb, out=Zb))
@@ -517,6 +519,8 @@ def side_rows(gs, dev):
                                "bind_gbs": round(bind_bytes / (ms_bind / 1e3) / 1e9, 1), "bound": "hbm",
                                "frac": round(bind_bytes / (ms_bind / 1e3) / 1e9 / peaks["hbm_gbs"], 4),
                                "bind_one_partner_ms": round(ms_bcast, 4),
+                               "one_partner_ms": round(ms_fused_one, 4),
+                               "one_partner_gbs": round((Tb.numel() * 4 + Zb.numel() * 4) / (ms_fused_one / 1e3) / 1e9, 1),
                                "bind_direct_ms": round(ms_direct, 4), "bind_direct_tflops": round(direct_tflops, 1),
                                "bind_direct_alu_frac": round(direct_tflops / FP32_PEAK_TFLOPS, 4)}
     del b4, b5, Xb, Yb, Zb

@@ -341,10 +341,18 @@ GS_API gs_status gs_bind(const float* X, long long N, int D, int ldx, const floa
  * Reconstruction followed by binding at the transition into component-wise
  * operators (Sec. 3.3: reconstruction is placed immediately before binding and
  * unbinding): Z = op(T Q, Y) with gs_reconstruct's T (N x r, t_dtype, ldt) and
- * gs_bind's Y, L, op (with its method) and Z.  The rows are processed in chunks
- * whose reconstruction lives in the handle's scratch between the two kernels
- * (the caller needs no N x D buffer for the reconstructed vectors).  flags picks
- * the reconstruction path as in gs_reconstruct.
+ * gs_bind's Y, L, op (with its method) and Z.  With one partner row for more
+ * rows than the basis has (ldy = 0, N > r), binding is applied to the basis
+ * instead of the rows: op(t Q, y) = t op(Q, y) by linearity, so the r basis rows
+ * are bound once and every row is reconstructed straight from them -- the
+ * reconstructed rows are never formed, and the call costs one reconstruction
+ * plus the binding of r rows; its error is then at most (f + eps) ||y_b||
+ * sum_j |t_j| ||q_j,b|| per output of block b, with f the multiplier of
+ * ||x_b|| ||y_b|| in gs_bind's bound for the method, and eps = 2^-10 + r 2^-23 on the tensor-core path (r 2^-23 in fp32).
+ * Otherwise the rows are processed in chunks whose reconstruction lives in the
+ * handle's scratch between the two kernels (the caller needs no N x D buffer
+ * for the reconstructed vectors).  flags picks the reconstruction path as in
+ * gs_reconstruct.
  * Shares the handle's scratch with the other multi-kernel calls: order calls
  * on one handle.
  */

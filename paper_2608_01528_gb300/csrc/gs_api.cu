@@ -560,9 +560,17 @@ gs_status gs_prob_vectorize(const gs_basis* h, const float* P, long long N, int 
     return GS_OK;
 }
 
-// Xhat = T Q with the fp16 copy of T (tensor-core path) in `work` (work_floats floats).
+// Xhat = T B with the fp16 copy of T (tensor-core path) in `work` (work_floats floats).  B is the
+// basis (Qb = h->Q, ldqb = D, Qtb = h->Q16t) or, for the one-partner reconstruct + bind, the basis
+// rows bound with the partner (fp32 r x D rows, ld ldqb, and their transposed fp16 copy).
 static gs_status reconstruct_rows(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt, float* Xhat,
-                                  int ldxh, unsigned flags, cudaStream_t s, float* work, long long work_floats) {
+                                  int ldxh, unsigned flags, cudaStream_t s, float* work, long long work_floats,
+                                  const float* Qb = nullptr, int ldqb = 0, const __half* Qtb = nullptr) {
+    if (!Qb) {
+        Qb = h->Q;
+        ldqb = h->D;
+        Qtb = h->Q16t;
+    }
     const bool tc_ok = h->has_split && h->r >= 1 && t_dtype == GS_F32 && (uintptr_t)T % 16 == 0 && ldt % 4 == 0;
     if (flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && tc_ok && big_gemm(N, h->D, h->r))) {
         if (!tc_ok) return t_dtype != GS_F32 || !h->has_split ? GS_ERR_UNSUPPORTED : GS_ERR_ALIGNMENT;
@@ -582,7 +590,7 @@ static gs_status reconstruct_rows(const gs_basis* h, const void* T, int t_dtype,
             if (st != GS_OK) return st;
             gs::GemmTcArgs a{};
             a.A = work; a.lda = ld16; a.m = nc; a.K = h->r; a.split = false; a.a_half = true;
-            a.B0 = h->Q16t; a.ldb = h->ldr16; a.n = h->D;
+            a.B0 = Qtb; a.ldb = h->ldr16; a.n = h->D;
             a.C = Xhat + (size_t)c0 * ldxh; a.ldc = ldxh; a.c_bf16 = false; a.alpha = 1.f;
             a.rowmul = rowmul;
             st = from_cuda(gs::launch_gemm_tc(a, h->device, s));
@@ -595,7 +603,7 @@ static gs_status reconstruct_rows(const gs_basis* h, const void* T, int t_dtype,
         gs::GemmArgs a{};
         a.A = (const char*)T + (size_t)c0 * ldt * (t_dtype == GS_F32 ? 4 : 2);
         a.a_type = t_dtype == GS_F32 ? gs::MAT_F32 : gs::MAT_BF16; a.lda = ldt;
-        a.B = h->Q; a.b_type = gs::MAT_F32; a.ldb = h->D; a.b_trans = false;
+        a.B = Qb; a.b_type = gs::MAT_F32; a.ldb = ldqb; a.b_trans = false;
         a.C = Xhat + c0 * ldxh; a.c_type = gs::MAT_F32; a.ldc = ldxh;
         a.m = nc; a.n = h->D; a.k = h->r; a.batch = 1; a.alpha = 1.f;
         cudaError_t e = gs::launch_gemm_simt(a, s);
@@ -655,6 +663,32 @@ gs_status gs_bind(const float* X, long long N, int D, int ldx, const float* Y, l
     return bind_rows(X, N, D, ldx, Y, ldy, L, op, Z, ldz, (cudaStream_t)stream);
 }
 
+// Reconstruct + bind with one partner row y for every row: binding is linear in its first
+// operand, so op(t Q, y) = t op(Q, y) -- bind the r basis rows with y once, then reconstruct every
+// row straight from those bound rows.  The reconstructed rows are never formed; the call costs one
+// reconstruction GEMM (on an fp16 copy of op(Q, y), rounded like the basis' own copy) plus the
+// binding of r rows.  Returns GS_ERR_SHAPE, with nothing enqueued, when the scratch cannot hold
+// op(Q, y), its fp16 copy and one 128-row chunk of T.
+static gs_status reconstruct_bind_one_partner(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt,
+                                              const float* Y, int L, int op, float* Z, int ldz, unsigned flags,
+                                              cudaStream_t s) {
+    const int r = h->r, D = h->D, Dp = (D + 3) / 4 * 4, ld16 = (r + 7) / 8 * 8;
+    const long long qy_floats = (long long)r * Dp;
+    const long long qt_floats = ((long long)D * ld16 / 2 + 3) / 4 * 4;  // 16-byte aligned after it
+    const long long work_floats = h->scratch_floats - qy_floats - qt_floats;
+    if (work_floats < 128LL * (ld16 / 2 + 1)) return GS_ERR_SHAPE;
+    float* Qy = h->scratch;
+    __half* Qyt = reinterpret_cast<__half*>(h->scratch + qy_floats);
+    float* work = h->scratch + qy_floats + qt_floats;
+    gs_status st = bind_rows(h->Q, r, D, D, Y, 0, L, op, Qy, Dp, s);
+    if (st != GS_OK) return st;
+    if (h->has_split) {  // the tensor-core reconstruction's operand (the fp32 path reads Qy)
+        st = from_cuda(gs::launch_f16t_dither(Qy, r, D, Dp, Qyt, ld16, s));
+        if (st != GS_OK) return st;
+    }
+    return reconstruct_rows(h, T, t_dtype, N, ldt, Z, ldz, flags, s, work, work_floats, Qy, Dp, Qyt);
+}
+
 gs_status gs_reconstruct_bind(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt, const float* Y,
                               long long ldy, int L, int op, float* Z, int ldz, unsigned flags, void* stream) {
     if (!h || !valid_path(flags)) return GS_ERR_INVALID_ARG;
@@ -673,6 +707,11 @@ gs_status gs_reconstruct_bind(const gs_basis* h, const void* T, int t_dtype, lon
     const int Dp = (h->D + 3) / 4 * 4, ld16 = (h->r + 7) / 8 * 8;
     if ((op & GS_BIND_SPECTRAL) && !gs::bind_spectral_supported(L, h->scratch, Dp, Y, ldy, Z, ldz))
         return spectral_error(L);
+    // one partner for more rows than the basis has: bind the basis instead of the rows
+    if (ldy == 0 && N > h->r && h->r > 0) {
+        st = reconstruct_bind_one_partner(h, T, t_dtype, N, ldt, Y, L, op, Z, ldz, flags, s);
+        if (st != GS_ERR_SHAPE) return st;  // otherwise the scratch is too small: row chunks below
+    }
     long long cr = std::min(h->scratch_floats / (Dp + ld16 / 2 + 1), kMaxGemmRows);
     if (cr >= 128) cr = cr / 128 * 128;
     if (cr < 1) return GS_ERR_SHAPE;

@@ -270,6 +270,26 @@ __global__ void k_q16(const double* __restrict__ Qw, int r, int D, __half* __res
     if (Q16t && d < D) Q16t[(size_t)d * ldt + j] = hv;
 }
 
+// dst[d][j] (cols x ldt fp16) = dithered rounding of src[j][d] (rows x cols fp32, ld lds), through
+// 32 x 32 tiles in shared memory (coalesced reads and writes); the transposed operand of a
+// reconstruction from fp32 rows that are not the basis itself (the basis bound with a partner).
+__global__ void k_f16t_dither(const float* __restrict__ src, int rows, int cols, long long lds,
+                              __half* __restrict__ dst, long long ldt) {
+    __shared__ float tile[32][33];
+    const int j0 = blockIdx.y * 32, d0 = blockIdx.x * 32;
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;  // 256 threads: 8 rows per step
+    for (int k = ty; k < 32; k += 8) {
+        const int j = j0 + k, d = d0 + tx;
+        tile[k][tx] = (j < rows && d < cols) ? src[(size_t)j * lds + d] : 0.f;
+    }
+    __syncthreads();
+    for (int k = ty; k < 32; k += 8) {
+        const int d = d0 + k, j = j0 + tx;
+        if (d < cols && j < rows)
+            dst[(size_t)d * ldt + j] = dither_half((double)tile[tx][k], (unsigned long long)j * cols + d);
+    }
+}
+
 __global__ void k_zero_half(__half* p, long long n) {
     const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (i < n) p[i] = __float2half(0.0f);
@@ -486,6 +506,15 @@ gs_status finalize_basis(const double* Qw, const double* R64, int ldr, const dou
     GS_CK(cudaGetLastError());
     GS_CK(cudaStreamSynchronize(s));
     return GS_OK;
+}
+
+cudaError_t launch_f16t_dither(const float* src, int rows, int cols, long long lds, void* dst, long long ldt,
+                               cudaStream_t s) {
+    if (rows <= 0 || cols <= 0) return cudaSuccess;
+    const dim3 grid((unsigned)((cols + 31) / 32), (unsigned)((rows + 31) / 32));
+    if (grid.y > 65535u) return cudaErrorInvalidConfiguration;
+    k_f16t_dither<<<grid, 256, 0, s>>>(src, rows, cols, lds, static_cast<__half*>(dst), ldt);
+    return cudaGetLastError();
 }
 
 }  // namespace gs

@@ -89,6 +89,10 @@ gs_status build_basis(const float* C, int M, int D, int ldc, double tau, bool no
 // one handle: Q = [Q_0; Q_1; ...], R block diagonal
 gs_status build_basis_grouped(const float* C, int M, int D, int ldc, const int* off, int G, double tau,
                               bool normalize, cudaStream_t s, gs_basis* h);
+// dst[d][j] (cols x ldt fp16) = the basis' unbiased dithered fp16 rounding of src[j][d] (rows x
+// cols fp32, ld lds): the transposed B operand of a reconstruction from other fp32 rows
+cudaError_t launch_f16t_dither(const float* src, int rows, int cols, long long lds, void* dst, long long ldt,
+                               cudaStream_t s);
 // a handle from a saved basis (fp32 Q r x D, R M x r, optional norms), same finalisation as a build
 gs_status import_basis(const float* Q, int ldq, const float* R, int ldr_in, const float* cnorm, int M, int D,
                        int r, cudaStream_t s, gs_basis* h);

@@ -169,6 +169,39 @@ def test_reconstruct_bind_several_chunks(gs, orc):
             check_bind(Z, Zo, Xo, Y, 128, e_rec=1e-4 * np.linalg.norm(Tr, axis=1), method=method)
 
 
+def one_partner_bound(T, Q, Y, L, method, path):
+    """Per output of block b, for op(T Q, y) computed as T op(Q, y) (one partner row): each bound
+    basis row op(q_j, y) carries the binding method's error, f ||q_j,b|| ||y_b||; the
+    reconstruction from those rows adds its own rounding, one fp16 rounding each of T and of
+    op(Q, y) on the tensor core (|op(q_j, y)_k| <= ||q_j,b|| ||y_b||) and the fp32 sum of r
+    products.  Summed with weights |t_j|: (f + eps) ||y_b|| sum_j |t_j| ||q_j,b||."""
+    r = Q.shape[0]
+    eps = r * 2.0 ** -23 + (2.0 ** -10 if path == "tensor" else 0.0)
+    f = bind_error_factor(L, method)
+    return (f + eps) * (np.abs(T.astype(np.float64)) @ block_norms(Q, L)) * block_norms(Y, L)[0][None, :]
+
+
+@pytest.mark.parametrize("path,method", [("simt", "direct"), ("simt", "spectral"), ("tensor", "direct"),
+                                         ("tensor", "auto")])
+def test_reconstruct_bind_one_partner(gs, orc, path, method):
+    """One partner row for 2,000 rows of the attention basis (r = 512 < N): the library binds the
+    basis rows once and reconstructs from them (op(t Q, y) = t op(Q, y)); against the oracle's
+    reconstruction followed by binding, within the bound of that arithmetic."""
+    a = synth.attention(B=1, L=1)
+    b = gs.build_basis(cuda(a["C"]))
+    N, L = 2000, 256
+    T = (synth.attention_probs(13, 1, N, b.M, 1).astype(np.float64) @ host(b.R)).astype(np.float32)
+    Y = np.random.default_rng(12).normal(size=(1, b.D)).astype(np.float32)
+    Qh = host(b.Q)
+    for op in ("bind", "unbind"):
+        Z = gs.reconstruct_bind(b, cuda(T), cuda(Y), L, op, path=path, method=method)
+        gs.stream_status()
+        Zo = orc.reconstruct_bind(T, Qh, Y, L, orc.UNBIND if op == "unbind" else orc.BIND)
+        err = np.abs(host(Z) - Zo).reshape(N, b.D // L, L).max(axis=2)
+        bound = one_partner_bound(T, Qh, Y, L, "direct" if method == "direct" else "spectral", path)
+        assert np.all(err <= bound)
+
+
 def test_bind_argument_errors(gs):
     X = torch.zeros((4, 100), device="cuda:0")
     with pytest.raises(gs.GramSpaceError) as ei:

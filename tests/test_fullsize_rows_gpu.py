@@ -73,6 +73,28 @@ def test_reconstruct_bind_full_size(gs, orc):
     check_bind(Z[idx], Zo, Xo, Yr, L, e_rec=1e-4 * np.linalg.norm(Tr, axis=1), method="spectral")
 
 
+def test_reconstruct_bind_one_partner_full_size(gs, orc):
+    """8,192 rows of the attention basis bound with one partner row in blocks of 256 (the bench's
+    one-partner reconstruct + bind: the basis rows bound once, one reconstruction GEMM), sampled
+    rows against the oracle's reconstruction followed by binding."""
+    from test_bind_gpu import one_partner_bound
+    a = synth.attention(B=1, L=1)
+    b = gs.build_basis(cuda(a["C"]))
+    N, L = 8192, 256
+    P = synth.attention_probs(12, 1, N, b.M, 1)
+    T = (torch.from_numpy(P).to("cuda:0") @ b.R).contiguous()
+    g = torch.Generator().manual_seed(29)
+    Y = torch.randn(1, b.D, generator=g).to("cuda:0")
+    Z = gs.reconstruct_bind(b, T, Y, L)
+    gs.stream_status()
+    rows = sample_rows(N, 64, 6)
+    idx = torch.from_numpy(rows).to(T.device)
+    Tr, Yh, Qh = host(T[idx]), host(Y), host(b.Q)
+    Zo = orc.reconstruct_bind(Tr, Qh, Yh, L)
+    err = np.abs(host(Z[idx]) - Zo).reshape(len(rows), b.D // L, L).max(axis=2)
+    assert np.all(err <= one_partner_bound(Tr, Qh, Yh, L, "spectral", "tensor"))
+
+
 def test_bind_one_partner_full_size(gs, orc):
     """8,192 x 4,096 rows bound with one partner row in blocks of 256 (the bench's one-partner
     binding: the partner's block spectra cached per CTA), sampled rows against the oracle."""

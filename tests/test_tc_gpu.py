@@ -263,3 +263,25 @@ def test_tc_attention(gs, orc, attn_R, B, Lq, Lk, r):
     assert (np.abs(host(A) - ref) / ref).max() <= 2e-2
     assert np.allclose(host(A).sum(axis=2), 1.0, atol=1e-4)
     assert np.abs(host(L) - refl).max() <= 1e-4 * np.abs(refl).max()
+
+
+@pytest.mark.parametrize("M,D", [(256, 1024), (256, 2048), (256, 4096), (100, 1024), (40, 8192), (200, 6000)])
+@pytest.mark.parametrize("outputs", ["lookup", "all"])
+def test_tc_score_paths(gs, orc, M, D, outputs):
+    """The fused kernel across basis sizes (full 256 x 256 TMEM accumulators down to codebooks that
+    are not multiples of 16 or 32) and depths, with argmax / maxval only (the lookup kernel) and
+    with every output, two launches back to back, against the oracle."""
+    rng = np.random.default_rng(M * 7 + D)
+    C = (rng.integers(0, 2, size=(M, D)) * 2 - 1).astype(np.float32)
+    X, labels = synth.noisy_rows(C, 9, 0, 3000, 1.0)
+    b = gs.build_basis(cuda(C))
+    Qo, Ro, cno = orc.build_basis(C)
+    full = outputs == "all"
+    outs = [gs.project_similarity(b, cuda(X), path="tensor", want_S=full, want_Y=full) for _ in range(2)]
+    gs.stream_status()
+    ref = orc.project_similarity(X, Qo, Ro, cno)
+    for out in outs:
+        check_scores(out, ref, X, cno)
+        if full:
+            assert np.all(np.abs(host(out["Y"]) - ref["Y"]) <= TOL_S * ref["xnorm"][:, None])
+    assert torch.equal(outs[0]["argmax"], outs[1]["argmax"])
