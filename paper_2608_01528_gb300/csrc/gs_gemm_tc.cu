@@ -293,15 +293,11 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                     const uint64_t ah = sdesc_sw128(smem_u32(At));
                     if (HALVES == 1) {
                         const int sb0 = rb.idx;
-                        if (!mbar_wait_1t(&c.b_full[sb0], rb.phase, abort_flag, err)) ok = false;
-                        rb.next(p.sb);
-                        int sb1 = sb0;
-                        if (p.nb == 2) {
-                            sb1 = rb.idx;
-                            if (ok && !mbar_wait_1t(&c.b_full[sb1], rb.phase, abort_flag, err)) ok = false;
-                            rb.next(p.sb);
+                        if (!mbar_wait_1t(&c.b_full[sb0], rb.phase, abort_flag, err)) {
+                            ok = false;
+                            break;
                         }
-                        if (!ok) break;
+                        rb.next(p.sb);
                         tc_fence_after();
                         const uint64_t b0 = sdesc_sw128(smem_u32(Bs + (size_t)sb0 * kBStageBytes));
                         if (AMODE != kABF16X2) {
@@ -309,20 +305,34 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                             for (int k = 0; k < kBK / 16; ++k)
                                 mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
                                            (kb != lo || k != 0) ? 1u : 0u);
-                        } else {
-                            const uint64_t al = sdesc_sw128(smem_u32(At + kAPartBytes));
-                            const uint64_t b1 = sdesc_sw128(smem_u32(Bs + (size_t)sb1 * kBStageBytes));
-#pragma unroll
-                            for (int k = 0; k < kBK / 16; ++k) {
-                                mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
-                                           (kb != lo || k != 0) ? 1u : 0u);
-                                mma_f16_ss(d_tmem, al + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc, 1u);
-                                mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b1 + (uint64_t)(2 * k), idesc, 1u);
-                            }
+                            mma_commit(&c.a_empty[sa]);
+                            mma_commit(&c.b_empty[sb0]);
+                            continue;
                         }
-                        mma_commit(&c.a_empty[sa]);
+                        // split operands: the two products with B hi (Ah Bh + Al Bh) go first and
+                        // release B hi's stage, so B lo, one stage behind in the ring, has that long
+                        // to land before Ah Bl needs it
+                        const uint64_t al = sdesc_sw128(smem_u32(At + kAPartBytes));
+#pragma unroll
+                        for (int k = 0; k < kBK / 16; ++k) {
+                            mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc,
+                                       (kb != lo || k != 0) ? 1u : 0u);
+                            mma_f16_ss(d_tmem, al + (uint64_t)(2 * k), b0 + (uint64_t)(2 * k), idesc, 1u);
+                        }
                         mma_commit(&c.b_empty[sb0]);
-                        if (p.nb == 2) mma_commit(&c.b_empty[sb1]);
+                        const int sb1 = rb.idx;
+                        if (!mbar_wait_1t(&c.b_full[sb1], rb.phase, abort_flag, err)) {
+                            ok = false;
+                            break;
+                        }
+                        rb.next(p.sb);
+                        tc_fence_after();
+                        const uint64_t b1 = sdesc_sw128(smem_u32(Bs + (size_t)sb1 * kBStageBytes));
+#pragma unroll
+                        for (int k = 0; k < kBK / 16; ++k)
+                            mma_f16_ss(d_tmem, ah + (uint64_t)(2 * k), b1 + (uint64_t)(2 * k), idesc, 1u);
+                        mma_commit(&c.a_empty[sa]);
+                        mma_commit(&c.b_empty[sb1]);
                         continue;
                     }
                     // 512-column tile (fp16 A, one B per half): the A K-block feeds both halves
