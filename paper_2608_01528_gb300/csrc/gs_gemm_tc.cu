@@ -553,6 +553,219 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
     }
 }
 
+// ----------------------------------------------------------------- CTA-pair GEMM, fp16 A by TMA
+// k_gemm_tc2: C = alpha A B^T (x rowmul[i]) with A already fp16 (reconstruct: the rounded T) on
+// pairs of CTAs (clusters of two): one pair MMA (tcgen05 cta_group::2, M = 256) computes a
+// 256 x nt tile, each CTA staging its own 128 rows of A and half of the tile's nt rows of B, so an
+// SM stages half the B bytes the single-CTA kernel does for the same outputs (B dominated the
+// shared-memory traffic that held reconstruct's MMAs at half rate).  The even CTA's A and B
+// producers expect both CTAs' bytes on its own full barriers, the odd CTA's TMA loads complete on
+// them; the even CTA's MMA thread commits stage releases and accumulator hand-offs to both CTAs;
+// each CTA's epilogue reads its own TMEM rows and releases the accumulator on the even CTA's
+// barrier.  Warp roles (640 threads): 0 A producer, 1 TMEM allocator + MMA issuer (even CTA),
+// 2 B producer, 3 idle, 4-19 epilogue (warp w reads TMEM lanes 32 (w % 4)..+31; the four warps of a
+// lane quadrant take alternate 32-column chunks).  Every wait is bounded.
+constexpr int kP2EpiWarps = 16;
+constexpr int kP2Threads = (4 + kP2EpiWarps) * 32;
+constexpr int kP2StageBytes = 128 * kBK * 2;  // 16 KB: 128 rows of one fp16 K-block (A, or half of B)
+constexpr int kP2MaxS = 6;
+
+struct Gemm2Params {
+    long long m;
+    int n, nkb, nt, tiles_n;
+    long long tiles;  // pair tiles (256 rows x nt columns)
+    int sa, sb, rotate;
+    float* C;
+    long long ldc;
+    float alpha;
+    const float* rowmul;
+};
+
+struct Ctl2 {
+    uint64_t a_full[kP2MaxS], a_empty[kP2MaxS];
+    uint64_t b_full[kP2MaxS], b_empty[kP2MaxS];
+    uint64_t d_full[2], d_empty[2];
+    uint64_t mma_done;
+    uint32_t tmem_base;
+    int abort_flag;
+};
+
+__global__ void __launch_bounds__(kP2Threads, 1)
+    k_gemm_tc2(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
+               const __grid_constant__ Gemm2Params p) {
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+    uint8_t* As = base;
+    uint8_t* Bs = As + (size_t)p.sa * kP2StageBytes;
+    Ctl2& c = *reinterpret_cast<Ctl2*>(Bs + (size_t)p.sb * kP2StageBytes);
+    volatile int* abort_flag = &c.abort_flag;
+    unsigned* err = &g_err_gemm;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    const bool lead = rank == 0;
+    const long long pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+    const int ntiles = p.tiles > pair ? (int)((p.tiles - 1 - pair) / npairs + 1) : 0;
+    auto tile_mn = [&](int lt, long long& tm, int& tn) {
+        const long long tg = pair + (long long)lt * npairs;
+        tm = tg / p.tiles_n;
+        tn = (int)((tg + (p.rotate ? lt : 0)) % p.tiles_n);
+    };
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < p.sa; ++s) {
+            mbar_init(&c.a_full[s], 1);
+            mbar_init(&c.a_empty[s], 1);
+        }
+        for (int s = 0; s < p.sb; ++s) {
+            mbar_init(&c.b_full[s], 1);
+            mbar_init(&c.b_empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&c.d_full[b], 1);
+            mbar_init(&c.d_empty[b], 2 * kP2EpiWarps);  // the epilogue warps of both CTAs
+        }
+        mbar_init(&c.mma_done, 1);
+        c.abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 1) {
+        tmem_alloc2(&c.tmem_base, kTmemCols);
+        tmem_relinquish2();
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync_all();  // the even CTA's barriers exist before the odd CTA signals them
+    tc_fence_after();
+    const uint32_t tmem = c.tmem_base;
+    const uint32_t bbytes = (uint32_t)(p.nt / 2) * kBK * 2;  // one CTA's half of a B K-block
+
+    if (warp == 0 || warp == 2) {
+        // ------------------------------------------------------------- A (warp 0) / B (warp 2) tiles
+        if (lane == 0) {
+            const bool isa = warp == 0;
+            const int depth = isa ? p.sa : p.sb;
+            uint64_t* full = isa ? c.a_full : c.b_full;
+            uint64_t* empty = isa ? c.a_empty : c.b_empty;
+            uint8_t* stages = isa ? As : Bs;
+            const uint32_t bytes = isa ? (uint32_t)kP2StageBytes : bbytes;
+            const CUtensorMap* map = isa ? &tmap_a : &tmap_b;
+            const uint64_t pol = l2_policy_evict_last();
+            int it = 0;
+            RingPos rp;
+            bool ok = true;
+            for (int lt = 0; lt < ntiles && ok; ++lt) {
+                long long tm;
+                int tn;
+                tile_mn(lt, tm, tn);
+                const int y = isa ? (int)(tm * 256 + 128 * rank) : tn * p.nt + (int)rank * (p.nt / 2);
+                for (int kb = 0; kb < p.nkb; ++kb, ++it, rp.next(depth)) {
+                    if (!mbar_wait_1t(&empty[rp.idx], rp.phase ^ 1u, abort_flag, err)) {
+                        ok = false;
+                        break;
+                    }
+                    if (lead) mbar_arrive_expect_tx(&full[rp.idx], 2u * bytes);
+                    tma_load_2d_pair(stages + (size_t)rp.idx * kP2StageBytes, map,
+                                     mapa_shared(smem_u32(&full[rp.idx]), 0), kb * kBK, y, pol);
+                }
+            }
+            // the even CTA waits until every stage it expected (both CTAs' loads) has landed; the
+            // odd CTA's loads land on those barriers, and it leaves only after the closing cluster
+            // barrier, which the even CTA reaches after this drain
+            if (lead)
+                for (int j = std::max(0, it - depth); j < it; ++j)
+                    mbar_drain(&full[j % depth], (uint32_t)(j / depth) & 1u, err);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------- pair MMA issue (even CTA)
+        if (lane == 0 && lead) {
+            const uint32_t idesc = idesc2_f16_f32(p.nt);
+            RingPos ra, rb;
+            bool ok = true;
+            for (int lt = 0; lt < ntiles && ok; ++lt) {
+                const int buf = lt & 1;
+                // both CTAs' epilogues have read this accumulator (arrivals at cluster scope)
+                if (!mbar_wait_cluster(&c.d_empty[buf], ((uint32_t)(lt >> 1) & 1u) ^ 1u, abort_flag, err)) break;
+                tc_fence_after();
+                const uint32_t d_tmem = tmem + (uint32_t)(buf * 256);
+                for (int kb = 0; kb < p.nkb; ++kb, ra.next(p.sa), rb.next(p.sb)) {
+                    if (!mbar_wait_1t(&c.a_full[ra.idx], ra.phase, abort_flag, err) ||
+                        !mbar_wait_1t(&c.b_full[rb.idx], rb.phase, abort_flag, err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint64_t ad = sdesc_sw128(smem_u32(As + (size_t)ra.idx * kP2StageBytes));
+                    const uint64_t bd = sdesc_sw128(smem_u32(Bs + (size_t)rb.idx * kP2StageBytes));
+#pragma unroll
+                    for (int k = 0; k < kBK / 16; ++k)
+                        mma2_f16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc, (kb | k) != 0 ? 1u : 0u);
+                    mma2_commit(&c.a_empty[ra.idx], 3);
+                    mma2_commit(&c.b_empty[rb.idx], 3);
+                }
+                if (ok) mma2_commit(&c.d_full[buf], 3);
+            }
+            mma2_commit(&c.mma_done, 1);
+            mbar_drain(&c.mma_done, 0, err);
+        }
+    } else if (warp >= 4) {
+        // ------------------------------------------------------------- epilogue: this CTA's 128 rows
+        const int quad = warp & 3, chunk = (warp - 4) >> 2;
+        for (int lt = 0; lt < ntiles; ++lt) {
+            const int buf = lt & 1;
+            if (!mbar_wait_warp(&c.d_full[buf], (uint32_t)(lt >> 1) & 1u, abort_flag, err)) break;
+            tc_fence_after();
+            long long tm;
+            int tn;
+            tile_mn(lt, tm, tn);
+            const long long row0 = tm * 256 + 128 * rank;
+            for (int half = 0; half < 2; ++half) {
+                const int lrow = quad * 32 + half * 16;
+                const uint32_t tb = tmem + ((uint32_t)lrow << 16) + (uint32_t)(buf * 256);
+                const long long row[2] = {row0 + lrow + (lane >> 2), row0 + lrow + (lane >> 2) + 8};
+                float rm[2];
+#pragma unroll
+                for (int h = 0; h < 2; ++h) rm[h] = (p.rowmul && row[h] < p.m) ? p.rowmul[row[h]] * p.alpha : p.alpha;
+                for (int jc = 32 * chunk; jc < p.nt; jc += 32 * 4) {
+                    float v[16];
+                    tmem_ld16x256b_x4(tb + (uint32_t)jc, v);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const int col = tn * p.nt + jc + 8 * j + 2 * (lane & 3);
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            if (row[h] >= p.m || col >= p.n) continue;
+                            const float g0 = rm[h] * v[4 * j + 2 * h], g1 = rm[h] * v[4 * j + 2 * h + 1];
+                            float* dst = p.C + (size_t)row[h] * p.ldc + col;
+                            if (col + 1 < p.n && ((uintptr_t)dst & 7u) == 0) {
+                                __stcs(reinterpret_cast<float2*>(dst), make_float2(g0, g1));
+                            } else {
+                                dst[0] = g0;
+                                if (col + 1 < p.n) dst[1] = g1;
+                            }
+                        }
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                if (lead)
+                    mbar_arrive(&c.d_empty[buf]);
+                else
+                    mbar_arrive_cluster(mapa_shared(smem_u32(&c.d_empty[buf]), 0));
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync_all();  // neither CTA leaves while the other may still signal its barriers
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc2(tmem, kTmemCols);
+    }
+}
+
 size_t gemm_smem_bytes(int sx, int sa, int parts, int sb) {
     return 1024 + (size_t)sx * kXStageBytes + (size_t)sa * parts * kAPartBytes + (size_t)sb * kBStageBytes +
            sizeof(Ctl);
@@ -633,8 +846,58 @@ unsigned take_device_error_gemm() {
     return v;
 }
 
+// C = alpha A B^T (x rowmul) with fp16 A on CTA pairs (k_gemm_tc2); fp32 C, no norms, no K trimming.
+static cudaError_t launch_gemm_tc2(const GemmTcArgs& a, int device, cudaStream_t s) {
+    Gemm2Params q;
+    q.m = a.m;
+    q.n = a.n;
+    q.nkb = (a.K + kBK - 1) / kBK;
+    q.nt = a.n >= 256 ? 256 : (a.n + 31) / 32 * 32;  // the pair MMA's N (each CTA stages nt / 2 rows of B)
+    q.tiles_n = (a.n + q.nt - 1) / q.nt;
+    q.tiles = ((a.m + 255) / 256) * (long long)q.tiles_n;
+    q.sa = q.sb = kP2MaxS;
+    q.C = static_cast<float*>(a.C);
+    q.ldc = a.ldc;
+    q.alpha = a.alpha;
+    q.rowmul = a.rowmul;
+    const size_t smem = 1024 + (size_t)(q.sa + q.sb) * kP2StageBytes + sizeof(Ctl2);
+    CUtensorMap ta, tb;
+    if (!make_tmap_2d(&ta, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, a.A, a.m, a.K, a.lda, kBK, 128,
+                      CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_tmap_2d(&tb, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, a.B0, a.n, a.K, a.ldb, kBK, q.nt / 2,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    static bool attr[64];
+    if (device < 0 || device >= 64) return cudaErrorInvalidDevice;
+    if (!attr[device]) {
+        cudaError_t e = cudaFuncSetAttribute(k_gemm_tc2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        attr[device] = true;
+    }
+    int sms = 0;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+    const long long pairs = std::min<long long>(std::max(sms / 2, 1), q.tiles);
+    q.rotate = pairs % q.tiles_n == 0 ? 1 : 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(2 * pairs));
+    cfg.blockDim = dim3(kP2Threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_gemm_tc2, ta, tb, q);
+}
+
 cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     if (a.m <= 0 || a.n <= 0) return cudaSuccess;
+    // fp16 A (T rounded once, the reconstruction): the CTA-pair kernel, whose SMs stage half of B each
+    if (a.a_half && !a.split && !a.c_bf16 && !a.rownorm && !a.colnorm && !a.b_klo && a.m >= 256)
+        return launch_gemm_tc2(a, device, s);
     GemmParams p;
     p.m = a.m;
     p.n = a.n;
