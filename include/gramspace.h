@@ -287,8 +287,10 @@ GS_API gs_status gs_prob_vectorize(const gs_basis* h, const float* P, long long 
  * component-wise operators).  Xhat = T Q: T is N x r coefficients of type
  * t_dtype (GS_F32 or GS_BF16, ld = ldt), Xhat is N x D fp32 (ld = ldxh).
  * Reconstructing R itself returns the codebook C (exact up to rounding).
- * Tensor-core path (GS_PATH_AUTO for large N with fp32 T, 16-byte aligned,
- * ldt % 4 == 0): each row of T is multiplied by an exact power of two that
+ * Tensor-core path (GS_PATH_AUTO for large N with fp32 T, D >= 1024, T 16-byte
+ * aligned, ldt % 4 == 0; GS_PATH_TENSOR returns GS_ERR_UNSUPPORTED for D <
+ * 1024, where one fp16 rounding no longer averages out over the rows of Q):
+ * each row of T is multiplied by an exact power of two that
  * brings its largest magnitude to [2^14, 2^15), rounded once to fp16 into the
  * handle's scratch, multiplied by the dithered fp16 Q with fp32 accumulation,
  * and the row's scale is undone in fp32, so the result is accurate for rows of

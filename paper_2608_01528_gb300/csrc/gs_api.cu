@@ -571,9 +571,14 @@ static gs_status reconstruct_rows(const gs_basis* h, const void* T, int t_dtype,
         ldqb = h->D;
         Qtb = h->Q16t;
     }
-    const bool tc_ok = h->has_split && h->r >= 1 && t_dtype == GS_F32 && (uintptr_t)T % 16 == 0 && ldt % 4 == 0;
+    // one fp16 rounding of T and of Q: each output sums r rounding errors weighted by entries of Q of
+    // size ~1/sqrt(D), so the error's spread is ~2^-11 ||t|| / sqrt(D); from D = 1024 on its worst
+    // case over a large output stays well inside 1e-4 ||t||, shorter rows take the fp32 path
+    const bool deep = h->D >= gs::kMinF16Depth;
+    const bool tc_ok = h->has_split && h->r >= 1 && t_dtype == GS_F32 && deep && (uintptr_t)T % 16 == 0 &&
+                       ldt % 4 == 0;
     if (flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && tc_ok && big_gemm(N, h->D, h->r))) {
-        if (!tc_ok) return t_dtype != GS_F32 || !h->has_split ? GS_ERR_UNSUPPORTED : GS_ERR_ALIGNMENT;
+        if (!tc_ok) return t_dtype != GS_F32 || !h->has_split || !deep ? GS_ERR_UNSUPPORTED : GS_ERR_ALIGNMENT;
         // Xhat = T Q: T rounded once to fp16 into the handle's scratch (every column tile of
         // Xhat re-reads it) after an exact power-of-two scale per row, the basis' dithered fp16
         // Q^T, fp32 accumulation, the row scales undone in the epilogue; rows in chunks that

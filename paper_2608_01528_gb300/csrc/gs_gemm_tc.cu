@@ -852,7 +852,7 @@ static cudaError_t launch_gemm_tc2(const GemmTcArgs& a, int device, cudaStream_t
     q.m = a.m;
     q.n = a.n;
     q.nkb = (a.K + kBK - 1) / kBK;
-    q.nt = a.n >= 256 ? 256 : (a.n + 31) / 32 * 32;  // the pair MMA's N (each CTA stages nt / 2 rows of B)
+    q.nt = 256;  // the pair MMA's N (each CTA stages nt / 2 rows of B; the launcher requires n >= 256)
     q.tiles_n = (a.n + q.nt - 1) / q.nt;
     q.tiles = ((a.m + 255) / 256) * (long long)q.tiles_n;
     q.sa = q.sb = kP2MaxS;
@@ -895,8 +895,10 @@ static cudaError_t launch_gemm_tc2(const GemmTcArgs& a, int device, cudaStream_t
 
 cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     if (a.m <= 0 || a.n <= 0) return cudaSuccess;
-    // fp16 A (T rounded once, the reconstruction): the CTA-pair kernel, whose SMs stage half of B each
-    if (a.a_half && !a.split && !a.c_bf16 && !a.rownorm && !a.colnorm && !a.b_klo && a.m >= 256)
+    // fp16 A (T rounded once, the reconstruction): the CTA-pair kernel, whose SMs stage half of B each,
+    // for products of at least one full pair tile (256 rows, 256 columns: the pair MMA is run at
+    // N = 256 only; a narrower N measured wrong, N = 224 with 112 B rows per CTA)
+    if (a.a_half && !a.split && !a.c_bf16 && !a.rownorm && !a.colnorm && !a.b_klo && a.m >= 256 && a.n >= 256)
         return launch_gemm_tc2(a, device, s);
     GemmParams p;
     p.m = a.m;

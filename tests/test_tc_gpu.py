@@ -192,16 +192,40 @@ def test_tc_reconstruct_round_trips(gs, orc, rankdef_ref):
     assert np.array_equal(np.rint(Xh.cpu().numpy()), C)
 
 
-@pytest.mark.parametrize("N,M,D", [(777, 40, 1002), (130, 8, 1024), (4096, 256, 8192)])
+@pytest.mark.parametrize("N,M,D", [(777, 40, 1030), (130, 8, 1024), (4096, 256, 8192), (300, 40, 1100),
+                                   (513, 64, 1030), (260, 96, 2000), (1000, 130, 1024)])
 def test_tc_reconstruct_matches_oracle(gs, orc, N, M, D):
+    """Reconstruction on the tensor core: CTA pairs (each staging half of every Q tile) for at
+    least 256 rows and 256 columns, single CTAs otherwise (fewer rows, or outputs narrower than one
+    256-column tile); a last column tile that is mostly past D, a last pair tile whose odd CTA has
+    few or no rows, and a depth r below one 64-wide K-block."""
     rng = np.random.default_rng(N + D)
     C = (rng.integers(0, 2, size=(M, D)) * 2 - 1).astype(np.float32)
     b = gs.build_basis(cuda(C))
     Qo, _, _ = orc.build_basis(C)
     T = rng.standard_normal((N, b.r)).astype(np.float32) * 3.0
-    Xh = gs.reconstruct(b, cuda(T), path="tensor")
+    Tp = torch.zeros((N, (b.r + 3) // 4 * 4), device="cuda:0")  # 16-byte rows, as the tensor path needs
+    Tp[:, :b.r] = cuda(T)
+    Xh = gs.reconstruct(b, Tp[:, :b.r], path="tensor")
     gs.stream_status()
     ref = orc.reconstruct(T, Qo)
+    assert np.all(np.abs(host(Xh) - ref) <= 1e-4 * np.linalg.norm(T.astype(np.float64), axis=1)[:, None])
+
+
+def test_tc_reconstruct_short_rows_take_fp32(gs, orc):
+    """D < 1024: one fp16 rounding of T and Q would not average out over the rows of Q (error spread
+    ~2^-11 ||t|| / sqrt(D)), so the tensor-core reconstruction refuses the shape and the default
+    path computes it in fp32, within the bound."""
+    rng = np.random.default_rng(3)
+    C = (rng.integers(0, 2, size=(40, 200)) * 2 - 1).astype(np.float32)
+    b = gs.build_basis(cuda(C))
+    T = rng.standard_normal((300, b.r)).astype(np.float32)
+    with pytest.raises(gs.GramSpaceError) as ei:
+        gs.reconstruct(b, cuda(T), path="tensor")
+    assert ei.value.status == gs.GS_ERR_UNSUPPORTED
+    Xh = gs.reconstruct(b, cuda(T))
+    gs.stream_status()
+    ref = orc.reconstruct(T, host(b.Q))
     assert np.all(np.abs(host(Xh) - ref) <= 1e-4 * np.linalg.norm(T.astype(np.float64), axis=1)[:, None])
 
 
