@@ -309,3 +309,44 @@ def test_tc_score_paths(gs, orc, M, D, outputs):
         if full:
             assert np.all(np.abs(host(out["Y"]) - ref["Y"]) <= TOL_S * ref["xnorm"][:, None])
     assert torch.equal(outs[0]["argmax"], outs[1]["argmax"])
+
+
+@pytest.mark.parametrize("mode", ["raw", "cosine"])
+def test_tc_two_gemm_argmax_without_scores(gs, orc, rankdef_ref, mode):
+    """Argmax / maxval without S on the two-GEMM path (the call the bench times: the scores go to
+    the handle's scratch and a row reduction reads them back).  Identical to the call that writes S
+    (duplicate codewords tie exactly: lowest index; a row of NaN queries: index 0
+    either way, with maxval -FLT_MAX for raw scores, none of which is a number, and 0 for cosine
+    scores, which a norm that is not a number sends to 0), and within the bound of the oracle."""
+    C, (Qo, Ro, cno) = rankdef_ref
+    X, _ = synth.noisy_rows(C, synth.SEEDS["rankdef"], 0, 3000, 1.0)
+    X[5] = np.nan
+    b = gs.build_basis(cuda(C))
+    Xd = cuda(X)
+    only = gs.project_similarity(b, Xd, mode=mode, path="tensor")
+    withS = gs.project_similarity(b, Xd, mode=mode, path="tensor", want_S=True)
+    gs.stream_status()
+    assert torch.equal(only["argmax"], withS["argmax"])
+    assert torch.equal(only["maxval"], withS["maxval"])
+    nan_row_max = -np.finfo(np.float32).max if mode == "raw" else 0.0
+    assert int(only["argmax"][5]) == 0 and float(only["maxval"][5]) == nan_row_max
+    keep = np.arange(3000) != 5
+    ref = orc.project_similarity(X[keep], Qo, Ro, cno, mode=getattr(orc, mode.upper()))
+    idx = torch.from_numpy(np.nonzero(keep)[0]).to(Xd.device)
+    check_scores({k: only[k][idx] for k in ("argmax", "maxval")}, ref, X[keep], cno, mode)
+
+
+def test_tc_two_gemm_argmax_two_codewords(gs, orc):
+    """Two codewords in D = 512 (the split two-GEMM path, D < 1024), argmax / maxval only: the
+    smallest score rows the scratch holds, identical to the call that writes S and within the
+    bound of the oracle."""
+    rng = np.random.default_rng(31)
+    C = (rng.integers(0, 2, size=(2, 512)) * 2 - 1).astype(np.float32)
+    X, _ = synth.noisy_rows(C, 32, 0, 5000, 1.0)
+    b = gs.build_basis(cuda(C))
+    only = gs.project_similarity(b, cuda(X), path="tensor")
+    withS = gs.project_similarity(b, cuda(X), path="tensor", want_S=True)
+    gs.stream_status()
+    assert torch.equal(only["argmax"], withS["argmax"]) and torch.equal(only["maxval"], withS["maxval"])
+    Qo, Ro, cno = orc.build_basis(C)
+    check_scores(only, orc.project_similarity(X, Qo, Ro, cno), X, cno)
