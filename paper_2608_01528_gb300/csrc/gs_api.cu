@@ -694,6 +694,29 @@ static gs_status reconstruct_bind_one_partner(const gs_basis* h, const void* T, 
     return reconstruct_rows(h, T, t_dtype, N, ldt, Z, ldz, flags, s, work, work_floats, Qy, Dp, Qyt);
 }
 
+// Reconstruct + bind with per-row partners in one kernel per chunk of rows (gs_rbind_tc.cu): the
+// chunk's T rows rounded once to fp16 with exact power-of-two row scales (as in gs_reconstruct's
+// tensor path), then each 128 x 256 tile of T Q is bound with its partner columns in tensor memory
+// and only Z is written.  Returns GS_ERR_SHAPE, with nothing enqueued, when the scratch cannot
+// hold one 128-row chunk of the fp16 rows.
+static gs_status reconstruct_bind_fused(const gs_basis* h, const float* T, long long N, int ldt, const float* Y,
+                                        long long ldy, int L, bool unbind, float* Z, int ldz, cudaStream_t s) {
+    const int ld16 = (h->r + 7) / 8 * 8;  // 16-byte rows for TMA
+    const long long chunk = std::min(h->scratch_floats / (ld16 / 2 + 1), kMaxGemmRows) / 128 * 128;
+    if (chunk < 128) return GS_ERR_SHAPE;
+    float* work = h->scratch;
+    float* rowmul = work + (size_t)chunk * ld16 / 2;
+    for (long long c0 = 0; c0 < N; c0 += chunk) {
+        const long long nc = std::min(chunk, N - c0);
+        gs_status st = from_cuda(gs::launch_round_f16(T + (size_t)c0 * ldt, ldt, nc, h->r, work, ld16, rowmul, s));
+        if (st != GS_OK) return st;
+        st = from_cuda(gs::launch_rbind_tc(h, work, ld16, nc, rowmul, Y + (size_t)c0 * ldy, ldy, L, unbind,
+                                           Z + (size_t)c0 * ldz, ldz, h->device, s));
+        if (st != GS_OK) return st;
+    }
+    return GS_OK;
+}
+
 gs_status gs_reconstruct_bind(const gs_basis* h, const void* T, int t_dtype, long long N, int ldt, const float* Y,
                               long long ldy, int L, int op, float* Z, int ldz, unsigned flags, void* stream) {
     if (!h || !valid_path(flags)) return GS_ERR_INVALID_ARG;
@@ -712,6 +735,15 @@ gs_status gs_reconstruct_bind(const gs_basis* h, const void* T, int t_dtype, lon
     const int Dp = (h->D + 3) / 4 * 4, ld16 = (h->r + 7) / 8 * 8;
     if ((op & GS_BIND_SPECTRAL) && !gs::bind_spectral_supported(L, h->scratch, Dp, Y, ldy, Z, ldz))
         return spectral_error(L);
+    // per-row partners on the tensor core: one kernel per chunk, the reconstructed rows kept on chip
+    // (the same rounding of T and Q as gs_reconstruct's tensor path, and the same auto rule)
+    const bool tc_ok = h->has_split && h->r >= 1 && t_dtype == GS_F32 && h->D >= gs::kMinF16Depth &&
+                       (uintptr_t)T % 16 == 0 && ldt % 4 == 0;
+    if (ldy != 0 && !(op & GS_BIND_DIRECT) && tc_ok && gs::rbind_tc_supported(L, h->D, Y, ldy, Z, ldz) &&
+        (flags == GS_PATH_TENSOR || (flags == GS_PATH_AUTO && big_gemm(N, h->D, h->r)))) {
+        st = reconstruct_bind_fused(h, (const float*)T, N, ldt, Y, ldy, L, (op & GS_UNBIND) != 0, Z, ldz, s);
+        if (st != GS_ERR_SHAPE) return st;  // otherwise the scratch is too small: row chunks below
+    }
     // one partner for more rows than the basis has: bind the basis instead of the rows
     if (ldy == 0 && N > h->r && h->r > 0) {
         st = reconstruct_bind_one_partner(h, T, t_dtype, N, ldt, Y, L, op, Z, ldz, flags, s);
@@ -780,7 +812,7 @@ gs_status gs_stream_status(void* stream) {
     cudaError_t e = stream ? cudaStreamSynchronize((cudaStream_t)stream) : cudaDeviceSynchronize();
     if (e != cudaSuccess) return GS_ERR_CUDA;
     const unsigned w = gs::take_device_error_build() | gs::take_device_error_tc() | gs::take_device_error_gemm() |
-                       gs::take_device_error_attn();
+                       gs::take_device_error_attn() | gs::take_device_error_rbind();
     if (w & GS_DEV_ERR_TIMEOUT) return GS_ERR_TIMEOUT;
     if (w & GS_DEV_ERR_RANGE) return GS_ERR_RANGE;
     return GS_OK;

@@ -30,8 +30,7 @@ struct gs_basis {
     __half* Q16t = nullptr;  // D x ldr16 fp16, dithered rounding of Q^T (K-major B of T Q)
     int ldr16 = 0;
     CUtensorMap tmap_q16;    // box {64, 256} over Q16 (valid when r <= 256 and Q16 != null)
-    CUtensorMap tmap_q16t;   // box {64, 256} over Q16t
-    bool has_tmap_q16 = false, has_tmap_q16t = false;
+    bool has_tmap_q16 = false;
     // fused tensor-core similarity: R split into two bf16 matrices (tc_mpad x
     // tc_npad, zero padded), Rh = bf16(R) and Rl = bf16(R - Rh), with tensor maps
     void* tc_Rh = nullptr;
@@ -205,6 +204,15 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s);
 cudaError_t launch_round_f16(const float* X, long long ldx, long long rows, int cols, void* out, long long ldo,
                              float* rowmul, cudaStream_t s);
 
+// ----------------------------------------------------------------- reconstruct + bind on tcgen05 (gs_rbind_tc.cu)
+// Z = op(T Q, Y) with per-row partners in one kernel: T16 (m x r fp16 rows, ld16 halves, each row
+// scaled by an exact power of two whose inverse is rowmul[i]), the basis' Q16t, Y and Z (m rows of
+// D floats, lds ldy / ldz).  L in {64, 128, 256}; Y, Z 16-byte aligned, ldy, ldz multiples of 4.
+bool rbind_tc_supported(int L, int D, const float* Y, long long ldy, const float* Z, int ldz);
+cudaError_t launch_rbind_tc(const gs_basis* h, const void* T16, long long ld16, long long m, const float* rowmul,
+                            const float* Y, long long ldy, int L, bool unbind, float* Z, int ldz, int device,
+                            cudaStream_t s);
+
 // ----------------------------------------------------------------- attention scores on tcgen05 (gs_attn_tc.cu)
 // bf16 Yq (B x Lq x r) and Yk (B x Lk x r), row stride ldy; fp32 A (B x Lq x Lk, dense).
 bool attn_tc_supported(int r, long long ldy, const void* Yq, const void* Yk);
@@ -220,6 +228,7 @@ unsigned take_device_error_tc();
 cudaError_t launch_wait_selftest(cudaStream_t s);
 unsigned take_device_error_gemm();
 unsigned take_device_error_attn();
+unsigned take_device_error_rbind();
 
 }  // namespace gs
 
