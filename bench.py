@@ -514,10 +514,14 @@ def side_rows(gs, dev):
     # the direct sum for comparison: 2 L flops per output on the fp32 lanes
     ms_direct = timeit(lambda: gs.bind(Xb, Yb, Lb, method="direct", out=Zb))
     direct_tflops = 2 * Nb * b5.D * Lb / (ms_direct / 1e3) / 1e12
+    # the fused call (k_rbind_tc: the reconstructed rows stay on chip): T read, Y read, Z written
+    fused_bytes = Tb.numel() * 4 + Yb.numel() * 4 + Zb.numel() * 4
     out["reconstruct_bind"] = {"ms": round(ms_fused, 4), "rows": Nb, "D": b5.D, "r": b5.r, "L": Lb,
+                               "gbs": round(fused_bytes / (ms_fused / 1e3) / 1e9, 1), "bound": "hbm",
+                               "frac": round(fused_bytes / (ms_fused / 1e3) / 1e9 / peaks["hbm_gbs"], 4),
                                "reconstruct_ms": round(ms_rec, 4), "bind_ms": round(ms_bind, 4),
-                               "bind_gbs": round(bind_bytes / (ms_bind / 1e3) / 1e9, 1), "bound": "hbm",
-                               "frac": round(bind_bytes / (ms_bind / 1e3) / 1e9 / peaks["hbm_gbs"], 4),
+                               "bind_gbs": round(bind_bytes / (ms_bind / 1e3) / 1e9, 1),
+                               "bind_frac": round(bind_bytes / (ms_bind / 1e3) / 1e9 / peaks["hbm_gbs"], 4),
                                "bind_one_partner_ms": round(ms_bcast, 4),
                                "one_partner_ms": round(ms_fused_one, 4),
                                "one_partner_gbs": round((Tb.numel() * 4 + Zb.numel() * 4) / (ms_fused_one / 1e3) / 1e9, 1),

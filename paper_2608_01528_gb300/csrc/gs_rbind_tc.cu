@@ -120,22 +120,31 @@ __device__ __forceinline__ bool quad_sync(int quad, bool ok) {
 
 // One strided pass over this warp's groups (b, n2), elements n2 + R2 i (i < R1), in place.
 // Forward (F1): the inputs times `mul` (the row's scale, or none), DFT_R1, then w_H^(n2 k1).
-// Inverse (I2): inverse DFT_R1, then the outputs times `mul`.
+// Inverse (I2): inverse DFT_R1, then the outputs times `mul`.  The next group's loads are in
+// flight while a group is transformed.
 template <int H, bool INV, bool SCALE>
 __device__ __forceinline__ void rb_strided(uint32_t tb, int sub, float mul, const float2* __restrict__ tw) {
     using P = RbPlan<H>;
-    constexpr int R1 = P::R1, R2 = P::R2;
-#pragma unroll 1
-    for (int g = sub; g < P::G; g += kRbSubs) {
-        const int b = g / R2, n2 = g % R2;
-        const uint32_t c0 = tb + (uint32_t)(2 * H * b + 2 * n2);
-        uint32_t r[2 * R1];
+    constexpr int R1 = P::R1, R2 = P::R2, NG = P::G / kRbSubs;
+    uint32_t r[2][2 * R1];
+    auto col = [&](int gi) {
+        const int g = sub + kRbSubs * gi;
+        return tb + (uint32_t)(2 * H * (g / R2) + 2 * (g % R2));
+    };
+    auto issue = [&](int gi, uint32_t (&q)[2 * R1]) {
+        const uint32_t c0 = col(gi);
 #pragma unroll
-        for (int i = 0; i < R1; ++i) tmem_ld2_issue(c0 + (uint32_t)(2 * R2 * i), r[2 * i], r[2 * i + 1]);
-        tmem_wait_ld_regs(r);
+        for (int i = 0; i < R1; ++i) tmem_ld2_issue(c0 + (uint32_t)(2 * R2 * i), q[2 * i], q[2 * i + 1]);
+    };
+    issue(0, r[0]);
+#pragma unroll
+    for (int gi = 0; gi < NG; ++gi) {
+        tmem_wait_ld_regs(r[gi & 1]);
         float2 v[R1];
 #pragma unroll
-        for (int i = 0; i < R1; ++i) v[i] = make_float2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
+        for (int i = 0; i < R1; ++i) v[i] = make_float2(__uint_as_float(r[gi & 1][2 * i]), __uint_as_float(r[gi & 1][2 * i + 1]));
+        if (gi + 1 < NG) issue(gi + 1, r[(gi + 1) & 1]);
+        const int n2 = (sub + kRbSubs * gi) % R2;
         if constexpr (!INV) {
             if constexpr (SCALE) {
 #pragma unroll
@@ -151,6 +160,7 @@ __device__ __forceinline__ void rb_strided(uint32_t tb, int sub, float mul, cons
                 for (int i = 0; i < R1; ++i) v[i] = make_float2(v[i].x * mul, v[i].y * mul);
             }
         }
+        const uint32_t c0 = col(gi);
 #pragma unroll
         for (int i = 0; i < R1; ++i) tmem_st2(c0 + (uint32_t)(2 * R2 * i), v[i].x, v[i].y);
     }
@@ -414,36 +424,51 @@ __global__ void __launch_bounds__(kRbThreads, 1)
         const uint32_t lanes = (uint32_t)(32 * quad) << 16;
         const int rr = 32 * quad + lane;  // this thread's row of the tile
         uint8_t* zst = Zs + (size_t)(warp - kRbEpi0) * kRbZStage;
+        // partner box cc of a tile into TMEM columns `half` + 32 cc of this quadrant's lanes (box cc
+        // sits in stage cc % 4 = sub, in the stage's phase cc / 4: each tile uses a stage twice)
+        auto copy_in = [&](int cc, uint32_t half) -> bool {
+            if (!mbar_wait_warp(&c.y_full[sub], (uint32_t)(cc >> 2), abort_flag, err)) return false;
+            const uint8_t* ys = Ys + (size_t)sub * kRbYStage + (size_t)rr * 128;
+            uint32_t v[32];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const uint4 f = *reinterpret_cast<const uint4*>(ys + ((u ^ (rr & 7)) << 4));
+                v[4 * u] = f.x;
+                v[4 * u + 1] = f.y;
+                v[4 * u + 2] = f.z;
+                v[4 * u + 3] = f.w;
+            }
+            // release the stage only once every lane holds its values (the TMEM store consumes
+            // them) and its reads are ordered before the TMA refill's writes (async proxy)
+            tmem_st32(tmem + lanes + half + (uint32_t)(kRbYCols * cc), v);
+            fence_proxy_async();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&c.y_empty[sub]);
+            return true;
+        };
+        // 16 output columns from registers through this warp's staging to a tensor store
+        auto store_box = [&](const uint32_t* v, int x, long long y) {
+            if (lane == 0) bulk_wait_read_0();  // the previous store has read the staging
+            __syncwarp();
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                *reinterpret_cast<uint4*>(zst + lane * 64 + ((u ^ ((lane >> 1) & 3)) << 4)) =
+                    make_uint4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+            fence_proxy_async();
+            __syncwarp();
+            if (lane == 0) {
+                if (x < p.D && y < p.m) tma_store_2d(&tmap_z, zst, x, (int)y);
+                bulk_commit();
+            }
+        };
+        bool ok = ntiles > 0;
+        if (ok) ok = copy_in(sub, kRbBN) && copy_in(sub + 4, kRbBN);  // tile 0's partner half: 256
         for (int lt = 0; lt < ntiles; ++lt) {
             const uint32_t hx = (uint32_t)((lt & 1) * kRbBN), hy = (uint32_t)kRbBN - hx;
             long long tm;
             int tn;
             tile_mn(lt, tm, tn);
             const long long row0 = tm * kRbBM;
-            bool ok = true;
-            // partner boxes sub and sub + 4 into the partner half (box cc of the tile sits in
-            // stage cc % 4 = sub, in the stage's phase cc / 4)
-            for (int h = 0; h < 2 && ok; ++h) {
-                const int cc = sub + 4 * h;
-                ok = mbar_wait_warp(&c.y_full[sub], (uint32_t)h, abort_flag, err);
-                if (!ok) break;
-                const uint8_t* ys = Ys + (size_t)sub * kRbYStage + (size_t)rr * 128;
-                uint32_t v[32];
-#pragma unroll
-                for (int u = 0; u < 8; ++u) {
-                    const uint4 f = *reinterpret_cast<const uint4*>(ys + ((u ^ (rr & 7)) << 4));
-                    v[4 * u] = f.x;
-                    v[4 * u + 1] = f.y;
-                    v[4 * u + 2] = f.z;
-                    v[4 * u + 3] = f.w;
-                }
-                // release the stage only once every lane holds its values (the TMEM store consumes
-                // them) and its reads are ordered before the TMA refill's writes (async proxy)
-                tmem_st32(tmem + lanes + hy + (uint32_t)(kRbYCols * cc), v);
-                fence_proxy_async();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&c.y_empty[sub]);
-            }
             if (!quad_sync(quad, ok)) break;
             rb_strided<H, false, false>(tmem + lanes + hy, sub, 1.f, tw);
             ok = mbar_wait_warp(&c.d_full, (uint32_t)lt & 1u, abort_flag, err);
@@ -461,30 +486,20 @@ __global__ void __launch_bounds__(kRbThreads, 1)
             if (!quad_sync(quad, true)) break;
             rb_strided<H, true, true>(tmem + lanes + hx, sub, p.zscale, tw);
             if (!quad_sync(quad, true)) break;
-            // output columns 32 cc .. 32 cc + 31 of this quadrant's rows, cc = sub, sub + 4
+            // output columns 32 cc .. 32 cc + 31 of this quadrant's rows (cc = sub, sub + 4); once a
+            // chunk is in registers its TMEM columns take the next tile's partner box cc (this
+            // half is the next tile's partner half), between the chunk's two tensor stores
             const long long y = row0 + 32 * quad;
+            const bool more = lt + 1 < ntiles;
             for (int h = 0; h < 2; ++h) {
                 const int cc = sub + 4 * h;
                 uint32_t v[32];
                 tmem_ld32_issue(tmem + lanes + hx + (uint32_t)(kRbYCols * cc), v);
                 tmem_wait_ld32(v);
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    const int x = tn * kRbBN + cc * kRbYCols + hh * kRbZCols;
-                    if (lane == 0) bulk_wait_read_0();  // the previous store has read the staging
-                    __syncwarp();
-#pragma unroll
-                    for (int u = 0; u < 4; ++u)
-                        *reinterpret_cast<uint4*>(zst + lane * 64 + ((u ^ ((lane >> 1) & 3)) << 4)) =
-                            make_uint4(v[16 * hh + 4 * u], v[16 * hh + 4 * u + 1], v[16 * hh + 4 * u + 2],
-                                       v[16 * hh + 4 * u + 3]);
-                    fence_proxy_async();
-                    __syncwarp();
-                    if (lane == 0) {
-                        if (x < p.D && y < p.m) tma_store_2d(&tmap_z, zst, x, (int)y);
-                        bulk_commit();
-                    }
-                }
+                const int x = tn * kRbBN + cc * kRbYCols;
+                store_box(v, x, y);
+                if (more && ok) ok = copy_in(cc, hx);
+                store_box(v + 16, x + kRbZCols, y);
             }
         }
         if (lane == 0) bulk_wait_all();
