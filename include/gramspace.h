@@ -351,9 +351,15 @@ GS_API gs_status gs_bind(const float* X, long long N, int D, int ldx, const floa
  * plus the binding of r rows; its error is then at most (f + eps) ||y_b||
  * sum_j |t_j| ||q_j,b|| per output of block b, with f the multiplier of
  * ||x_b|| ||y_b|| in gs_bind's bound for the method, and eps = 2^-10 + r 2^-23 on the tensor-core path (r 2^-23 in fp32).
- * Otherwise the rows are processed in chunks whose reconstruction lives in the
- * handle's scratch between the two kernels (the caller needs no N x D buffer
- * for the reconstructed vectors).  flags picks the reconstruction path as in
+ * With per-row partners on the tensor-core path, L in {64, 128, 256}, Y and Z
+ * 16-byte aligned with ldy, ldz multiples of 4, and a spectral (or default)
+ * method, one kernel per chunk of rows reconstructs each 128-row x 256-column
+ * tile on the tensor core and binds it through block spectra held in tensor
+ * memory: only Z is written (the reconstruction's error, 1e-4 ||t||, carried
+ * through the binding, plus the spectral bound).  Otherwise the rows are
+ * processed in chunks whose reconstruction lives in the handle's scratch
+ * between the two kernels (the caller needs no N x D buffer for the
+ * reconstructed vectors).  flags picks the reconstruction path as in
  * gs_reconstruct.
  * Shares the handle's scratch with the other multi-kernel calls: order calls
  * on one handle.
