@@ -564,11 +564,16 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
 // each CTA's epilogue reads its own TMEM rows and releases the accumulator on the even CTA's
 // barrier.  Warp roles (640 threads): 0 A producer, 1 TMEM allocator + MMA issuer (even CTA),
 // 2 B producer, 3 idle, 4-19 epilogue (warp w reads TMEM lanes 32 (w % 4)..+31; the four warps of a
-// lane quadrant take alternate 32-column chunks).  Every wait is bounded.
+// lane quadrant take alternate 32-column chunks, one TMEM row per thread, and write them through
+// two 2 KB staging buffers each (32 rows x 16 floats, 64-byte swizzle) as TMA tensor stores, so the
+// output bytes leave through the TMA unit rather than as per-thread stores through L1).  Every wait
+// is bounded.
 constexpr int kP2EpiWarps = 16;
 constexpr int kP2Threads = (4 + kP2EpiWarps) * 32;
 constexpr int kP2StageBytes = 128 * kBK * 2;  // 16 KB: 128 rows of one fp16 K-block (A, or half of B)
-constexpr int kP2MaxS = 6;
+constexpr int kP2MaxS = 5;
+constexpr int kP2ZCols = 16;                  // an output box: 32 rows x 64 bytes
+constexpr int kP2ZStage = 32 * kP2ZCols * 4;  // 2 KB
 
 struct Gemm2Params {
     long long m;
@@ -592,13 +597,14 @@ struct Ctl2 {
 
 __global__ void __launch_bounds__(kP2Threads, 1)
     k_gemm_tc2(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
-               const __grid_constant__ Gemm2Params p) {
+               const __grid_constant__ CUtensorMap tmap_c, const __grid_constant__ Gemm2Params p) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
     uint8_t* As = base;
     uint8_t* Bs = As + (size_t)p.sa * kP2StageBytes;
-    Ctl2& c = *reinterpret_cast<Ctl2*>(Bs + (size_t)p.sb * kP2StageBytes);
+    uint8_t* Cs = Bs + (size_t)p.sb * kP2StageBytes;
+    Ctl2& c = *reinterpret_cast<Ctl2*>(Cs + (size_t)kP2EpiWarps * 2 * kP2ZStage);
     volatile int* abort_flag = &c.abort_flag;
     unsigned* err = &g_err_gemm;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -710,6 +716,9 @@ __global__ void __launch_bounds__(kP2Threads, 1)
     } else if (warp >= 4) {
         // ------------------------------------------------------------- epilogue: this CTA's 128 rows
         const int quad = warp & 3, chunk = (warp - 4) >> 2;
+        const uint32_t lanes = (uint32_t)(32 * quad) << 16;
+        uint8_t* zst = Cs + (size_t)(warp - 4) * 2 * kP2ZStage;
+        int zb = 0;
         for (int lt = 0; lt < ntiles; ++lt) {
             const int buf = lt & 1;
             if (!mbar_wait_warp(&c.d_full[buf], (uint32_t)(lt >> 1) & 1u, abort_flag, err)) break;
@@ -718,43 +727,46 @@ __global__ void __launch_bounds__(kP2Threads, 1)
             int tn;
             tile_mn(lt, tm, tn);
             const long long row0 = tm * 256 + 128 * rank;
-            for (int half = 0; half < 2; ++half) {
-                const int lrow = quad * 32 + half * 16;
-                const uint32_t tb = tmem + ((uint32_t)lrow << 16) + (uint32_t)(buf * 256);
-                const long long row[2] = {row0 + lrow + (lane >> 2), row0 + lrow + (lane >> 2) + 8};
-                float rm[2];
+            const long long row = row0 + 32 * quad + lane, y = row0 + 32 * quad;
+            const float rm = (p.rowmul && row < p.m) ? p.rowmul[row] * p.alpha : p.alpha;
+            for (int jc = 32 * chunk; jc < p.nt; jc += 32 * 4) {
+                uint32_t v[32];
+                tmem_ld32_issue(tmem + lanes + (uint32_t)(buf * 256 + jc), v);
+                tmem_wait_ld32(v);
+                if (jc + 32 * 4 >= p.nt) {  // this warp's last read of the accumulator: back to the MMA
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) {
+                        if (lead)
+                            mbar_arrive(&c.d_empty[buf]);
+                        else
+                            mbar_arrive_cluster(mapa_shared(smem_u32(&c.d_empty[buf]), 0));
+                    }
+                }
 #pragma unroll
-                for (int h = 0; h < 2; ++h) rm[h] = (p.rowmul && row[h] < p.m) ? p.rowmul[row[h]] * p.alpha : p.alpha;
-                for (int jc = 32 * chunk; jc < p.nt; jc += 32 * 4) {
-                    float v[16];
-                    tmem_ld16x256b_x4(tb + (uint32_t)jc, v);
+                for (int hh = 0; hh < 2; ++hh) {
+                    const int x = tn * p.nt + jc + kP2ZCols * hh;
+                    if (lane == 0) bulk_wait_read_1();  // the store two boxes back has read this buffer
+                    __syncwarp();
+                    uint8_t* sb = zst + (size_t)zb * kP2ZStage;
+                    zb ^= 1;
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const int col = tn * p.nt + jc + 8 * j + 2 * (lane & 3);
-#pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-                            if (row[h] >= p.m || col >= p.n) continue;
-                            const float g0 = rm[h] * v[4 * j + 2 * h], g1 = rm[h] * v[4 * j + 2 * h + 1];
-                            float* dst = p.C + (size_t)row[h] * p.ldc + col;
-                            if (col + 1 < p.n && ((uintptr_t)dst & 7u) == 0) {
-                                __stcs(reinterpret_cast<float2*>(dst), make_float2(g0, g1));
-                            } else {
-                                dst[0] = g0;
-                                if (col + 1 < p.n) dst[1] = g1;
-                            }
-                        }
+                    for (int u = 0; u < 4; ++u) {
+                        const uint32_t* w = v + 16 * hh + 4 * u;
+                        *reinterpret_cast<float4*>(sb + lane * 64 + ((u ^ ((lane >> 1) & 3)) << 4)) =
+                            make_float4(rm * __uint_as_float(w[0]), rm * __uint_as_float(w[1]),
+                                        rm * __uint_as_float(w[2]), rm * __uint_as_float(w[3]));
+                    }
+                    fence_proxy_async();
+                    __syncwarp();
+                    if (lane == 0) {
+                        if (x < p.n && y < p.m) tma_store_2d(&tmap_c, sb, x, (int)y);
+                        bulk_commit();
                     }
                 }
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) {
-                if (lead)
-                    mbar_arrive(&c.d_empty[buf]);
-                else
-                    mbar_arrive_cluster(mapa_shared(smem_u32(&c.d_empty[buf]), 0));
-            }
         }
+        if (lane == 0) bulk_wait_all();
     }
 
     tc_fence_before();
@@ -860,12 +872,15 @@ static cudaError_t launch_gemm_tc2(const GemmTcArgs& a, int device, cudaStream_t
     q.ldc = a.ldc;
     q.alpha = a.alpha;
     q.rowmul = a.rowmul;
-    const size_t smem = 1024 + (size_t)(q.sa + q.sb) * kP2StageBytes + sizeof(Ctl2);
-    CUtensorMap ta, tb;
+    const size_t smem = 1024 + (size_t)(q.sa + q.sb) * kP2StageBytes + (size_t)kP2EpiWarps * 2 * kP2ZStage +
+                        sizeof(Ctl2);
+    CUtensorMap ta, tb, tc;
     if (!make_tmap_2d(&ta, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, a.A, a.m, a.K, a.lda, kBK, 128,
                       CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_tmap_2d(&tb, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, a.B0, a.n, a.K, a.ldb, kBK, q.nt / 2,
-                      CU_TENSOR_MAP_SWIZZLE_128B))
+                      CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_tmap_2d(&tc, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, a.C, a.m, a.n, a.ldc, kP2ZCols, 32,
+                      CU_TENSOR_MAP_SWIZZLE_64B))
         return cudaErrorInvalidValue;
     static bool attr[64];
     if (device < 0 || device >= 64) return cudaErrorInvalidDevice;
@@ -890,7 +905,7 @@ static cudaError_t launch_gemm_tc2(const GemmTcArgs& a, int device, cudaStream_t
     at[0].val.clusterDim.z = 1;
     cfg.attrs = at;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, k_gemm_tc2, ta, tb, q);
+    return cudaLaunchKernelEx(&cfg, k_gemm_tc2, ta, tb, tc, q);
 }
 
 cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
@@ -898,7 +913,8 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     // fp16 A (T rounded once, the reconstruction): the CTA-pair kernel, whose SMs stage half of B each,
     // for products of at least one full pair tile (256 rows, 256 columns: the pair MMA is run at
     // N = 256 only, the only width its tests cover; the reconstruction needs D >= 1024 anyway)
-    if (a.a_half && !a.split && !a.c_bf16 && !a.rownorm && !a.colnorm && !a.b_klo && a.m >= 256 && a.n >= 256)
+    if (a.a_half && !a.split && !a.c_bf16 && !a.rownorm && !a.colnorm && !a.b_klo && a.m >= 256 && a.n >= 256 &&
+        (uintptr_t)a.C % 16 == 0 && a.ldc % 4 == 0)  // the output's tensor map: 16-byte rows
         return launch_gemm_tc2(a, device, s);
     GemmParams p;
     p.m = a.m;

@@ -215,6 +215,10 @@ static __device__ __forceinline__ void bulk_commit() {
 static __device__ __forceinline__ void bulk_wait_read_0() {
     asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
+// Until at most the most recent one of this thread's bulk groups is still reading shared memory.
+static __device__ __forceinline__ void bulk_wait_read_1() {
+    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
 // Until all of this thread's bulk groups have completed.
 static __device__ __forceinline__ void bulk_wait_all() {
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
