@@ -693,6 +693,15 @@ __global__ void __launch_bounds__(kP2Threads, 1)
                 if (!mbar_wait_cluster(&c.d_empty[buf], ((uint32_t)(lt >> 1) & 1u) ^ 1u, abort_flag, err)) break;
                 tc_fence_after();
                 const uint32_t d_tmem = tmem + (uint32_t)(buf * 256);
+                // a narrow last column tile (w <= nt / 2 valid columns) takes all of them from the even
+                // CTA's half of B, so an MMA of N = 2 ceil(w / 8) 8 covers them; the odd CTA's half
+                // (rows beyond n, zero) and the accumulator columns it leaves stale map to output
+                // columns at or beyond n, which the tensor stores clip
+                long long tm;
+                int tn;
+                tile_mn(lt, tm, tn);
+                const int w = p.n - tn * p.nt;
+                const uint32_t idesc_t = w <= p.nt / 2 ? idesc2_f16_f32(std::max(32, 2 * ((w + 7) / 8 * 8))) : idesc;
                 for (int kb = 0; kb < p.nkb; ++kb, ra.next(p.sa), rb.next(p.sb)) {
                     if (!mbar_wait_1t(&c.a_full[ra.idx], ra.phase, abort_flag, err) ||
                         !mbar_wait_1t(&c.b_full[rb.idx], rb.phase, abort_flag, err)) {
@@ -704,7 +713,7 @@ __global__ void __launch_bounds__(kP2Threads, 1)
                     const uint64_t bd = sdesc_sw128(smem_u32(Bs + (size_t)rb.idx * kP2StageBytes));
 #pragma unroll
                     for (int k = 0; k < kBK / 16; ++k)
-                        mma2_f16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc, (kb | k) != 0 ? 1u : 0u);
+                        mma2_f16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc_t, (kb | k) != 0 ? 1u : 0u);
                     mma2_commit(&c.a_empty[ra.idx], 3);
                     mma2_commit(&c.b_empty[rb.idx], 3);
                 }

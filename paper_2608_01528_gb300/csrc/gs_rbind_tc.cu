@@ -167,28 +167,33 @@ __device__ __forceinline__ void rb_strided(uint32_t tb, int sub, float mul, cons
 }
 
 // One pair (k, k' = H - k) of the middle step.  From W (the packed transforms of x and of y) at k
-// and k', the doubled real spectra
-//   E = W_k + conj(W_k'),  O = -i (W_k - conj(W_k')),  X_k = E + t O,  X_k' = conj(E - t O)
-// (t = w_L^k), the product Z = X Y (unbind: X conj(Y)) at both, and the doubled packed spectrum
-// of the product's real inverse transform
+// and k', the doubled real spectra at k and the conjugates of those at k':
+//   E = W_k + conj(W_k'),  O = -i (W_k - conj(W_k')),  P = X_k = E + t O,  Q = conj(X_k') = E - t O
+// (t = w_L^k; R = Y_k and S = conj(Y_k') the same way), the product Z = X Y (unbind: X conj(Y)) as
+// Z_k = P R and conj(Z_k') = Q S (unbind: P conj(R), Q conj(S)), and the doubled packed spectrum of
+// the product's real inverse transform
 //   V_k = A + C,  V_k' = conj(A - C),  A = Z_k + conj(Z_k'),  C = i conj(t) (Z_k - conj(Z_k')).
 // For k = 0 (k' = 0 mod H, the second spectrum being X_H) and k = H / 2 (k' = k) both outputs are
 // the same value.
 template <bool UNB>
 __device__ __forceinline__ void rb_pair(float2 wxk, float2 wxc, float2 wyk, float2 wyc, float2 t, float2& vk,
                                         float2& vc) {
-    const float2 ex = c_add(wxk, c_conj(wxc)), ox = c_mul_negi(c_sub(wxk, c_conj(wxc)));
-    const float2 ey = c_add(wyk, c_conj(wyc)), oy = c_mul_negi(c_sub(wyk, c_conj(wyc)));
-    const float2 tox = c_mul(t, ox), toy = c_mul(t, oy);
-    const float2 xk = c_add(ex, tox), xc = c_conj(c_sub(ex, tox));
-    const float2 yk = c_add(ey, toy), yc = c_conj(c_sub(ey, toy));
-    const float2 zk = UNB ? c_mulconj(xk, yk) : c_mul(xk, yk);
-    const float2 zc = UNB ? c_mulconj(xc, yc) : c_mul(xc, yc);
-    const float2 a = c_add(zk, c_conj(zc));
-    const float2 bm = c_mulconj(c_sub(zk, c_conj(zc)), t);  // (Z_k - conj(Z_k')) conj(t)
-    const float2 cc = make_float2(-bm.y, bm.x);              // times i
+    auto spectra = [&](float2 wk, float2 wc, float2& pk, float2& qc) {
+        const float2 e = make_float2(wk.x + wc.x, wk.y - wc.y);
+        const float2 o = make_float2(wk.y + wc.y, wc.x - wk.x);
+        const float2 to = c_mul(t, o);
+        pk = c_add(e, to);
+        qc = c_sub(e, to);
+    };
+    float2 P, Q, R, S;
+    spectra(wxk, wxc, P, Q);
+    spectra(wyk, wyc, R, S);
+    const float2 zk = UNB ? c_mulconj(P, R) : c_mul(P, R);
+    const float2 zc = UNB ? c_mulconj(Q, S) : c_mul(Q, S);  // conj(Z_k')
+    const float2 a = c_add(zk, zc), b = c_sub(zk, zc);
+    const float2 cc = make_float2(fmaf(t.y, b.x, -t.x * b.y), fmaf(t.x, b.x, t.y * b.y));  // i conj(t) b
     vk = c_add(a, cc);
-    vc = c_conj(c_sub(a, cc));
+    vc = make_float2(a.x - cc.x, cc.y - a.y);
 }
 
 template <int N>
