@@ -64,7 +64,10 @@ typedef enum gs_status {
                                 entry near 2^64 or beyond, or an infinity); results of
                                 that call are invalid, rerun it with GS_PATH_SIMT
                                 (device word)                                        */
-    GS_ERR_UNSUPPORTED = 8   /* no sm_103 device, or a forced path cannot run      */
+    GS_ERR_UNSUPPORTED = 8   /* no sm_103 device, or a forced path cannot run (or,
+                                as a device word, a kernel found its shared-memory
+                                window placed so that its buffers do not fit; it
+                                returned without writing)                          */
 } gs_status;
 
 typedef enum gs_dtype { GS_F32 = 0, GS_BF16 = 1 } gs_dtype;

@@ -815,6 +815,7 @@ gs_status gs_stream_status(void* stream) {
                        gs::take_device_error_attn() | gs::take_device_error_rbind();
     if (w & GS_DEV_ERR_TIMEOUT) return GS_ERR_TIMEOUT;
     if (w & GS_DEV_ERR_RANGE) return GS_ERR_RANGE;
+    if (w & GS_DEV_ERR_LAYOUT) return GS_ERR_UNSUPPORTED;
     return GS_OK;
 }
 

@@ -234,3 +234,4 @@ unsigned take_device_error_rbind();
 
 #define GS_DEV_ERR_TIMEOUT 0x1u
 #define GS_DEV_ERR_RANGE 0x2u
+#define GS_DEV_ERR_LAYOUT 0x4u  // a kernel's shared-memory buffers did not fit where they landed

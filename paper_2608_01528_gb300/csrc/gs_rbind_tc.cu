@@ -3,11 +3,13 @@
 //
 // Sec. 3.3 reconstructs x_hat = t Q from Gram-loc coefficients and binds it with a partner row y
 // block by block (Sec. 2.2: circular convolution of blocks of L; unbinding: circular
-// correlation).  Here each persistent CTA computes a 128-row x 256-column tile of X_hat = T Q on
-// the tensor core (fp16 T rows scaled by exact powers of two, the basis' fp16 Q^T, fp32
-// accumulation in TMEM) and binds it where it lies: the tile holds 256 / L whole blocks of each
-// of its 128 rows, and the binding runs through block spectra (convolution theorem, real blocks
-// packed as H = L / 2 complex points) with TMEM as the transforms' working storage:
+// correlation).  Here persistent pairs of CTAs (clusters of two) compute 256-row x 256-column
+// tiles of X_hat = T Q on the tensor core (one tcgen05 cta_group::2 MMA: fp16 T rows scaled by
+// exact powers of two, the basis' fp16 Q^T, fp32 accumulation in TMEM; each CTA stages its own 128
+// rows of T and half of the tile's rows of Q^T), and each CTA binds its 128 x 256 part where it
+// lies: it holds 256 / L whole blocks of each of the CTA's rows, and the binding runs through block
+// spectra (convolution theorem, real blocks packed as H = L / 2 complex points) with TMEM as the
+// transforms' working storage:
 //
 //   z = IDFT_L(DFT_L(x) . DFT_L(y))          bind
 //   z = IDFT_L(DFT_L(x) . conj(DFT_L(y)))    unbind
@@ -36,9 +38,11 @@
 // The spectra carry a factor 2 each (real split without halves), the product 4, its packing 2,
 // the unnormalised inverse H: z = v / (8 H) = v / (4 L), an exact power of two.
 //
-// Warp roles (608 threads): 0 TMA producer of T and Q K-blocks, 1 TMEM allocator + MMA issuer,
-// 2 TMA producer of the partner rows (and an L2 prefetch of the next tile's), 3-18 transforms
-// (warp w reads TMEM lanes 32 (w % 4)..+31).  Every mbarrier wait is bounded (gs_tc_ptx.cuh); a
+// Warp roles (608 threads): 0 TMA producer of T and Q K-blocks (both CTAs' loads complete on the even
+// CTA's barriers), 1 TMEM allocator + pair MMA issuer (even CTA; its commits release both CTAs'
+// stages and hand both accumulators over), 2 TMA producer of the partner rows (and an L2 prefetch of
+// the next tile's), 3-18 transforms (warp w reads TMEM lanes 32 (w % 4)..+31; the next MMA waits for
+// the transform warps of both CTAs).  Every mbarrier wait is bounded (gs_tc_ptx.cuh); a
 // quadrant's four warps decide together, at the named barrier between passes, whether to go on,
 // so a timeout unwinds them without leaving one behind.
 
@@ -64,15 +68,13 @@ constexpr int kRbBK = 64;                                // K-block of the MMA o
 constexpr int kRbSubs = 4;                               // transform warps per lane quadrant
 constexpr int kRbEpi0 = 3;                               // first transform warp
 constexpr int kRbThreads = (kRbEpi0 + 4 * kRbSubs) * 32;  // 608
-constexpr int kRbStages = 2;                             // T / Q K-block stages
-constexpr int kRbAStage = kRbBM * kRbBK * 2;             // 16 KB of fp16 T
-constexpr int kRbBStage = kRbBN * kRbBK * 2;             // 32 KB of fp16 Q^T
-constexpr int kRbYStages = 4;
+constexpr int kRbStages = 3;                             // T / Q K-block stages
+constexpr int kRbAStage = kRbBM * kRbBK * 2;             // 16 KB of fp16 T (this CTA's 128 rows)
+constexpr int kRbBStage = kRbBN / 2 * kRbBK * 2;         // 16 KB of fp16 Q^T (this CTA's half of the tile)
+constexpr int kRbYStages = 8;                            // a whole tile of partner boxes (box cc in stage cc)
 constexpr int kRbYCols = 32;                             // a partner box: 128 rows x 128 bytes
 constexpr int kRbYStage = kRbBM * kRbYCols * 4;          // 16 KB
 constexpr int kRbChunks = kRbBN / kRbYCols;              // 8 partner boxes per tile
-constexpr int kRbZCols = 16;                             // an output box: 32 rows x 64 bytes
-constexpr int kRbZStage = 32 * kRbZCols * 4;             // 2 KB per transform warp
 constexpr int kRbMaxL = 256;
 
 struct RbParams {
@@ -86,17 +88,21 @@ struct RbParams {
 struct RbCtl {
     uint64_t full[kRbStages], empty[kRbStages];
     uint64_t y_full[kRbYStages], y_empty[kRbYStages];
-    uint64_t d_full;    // the tile's accumulator is complete (MMA commit)
-    uint64_t y_free;    // the partner half has been read: the next tile's MMA may write it
+    uint64_t d_full;    // the tile's accumulator is complete (MMA commit, to both CTAs)
+    uint64_t y_free;    // both CTAs' partner halves have been read: the next tile's MMA may write them
     uint64_t mma_done;
     uint32_t tmem_base;
     int abort_flag;
 };
 
-constexpr size_t rb_smem_bytes() {
-    return 1024 + (size_t)kRbStages * (kRbAStage + kRbBStage) + (size_t)kRbYStages * kRbYStage +
-           (size_t)4 * kRbSubs * kRbZStage + kRbMaxL * sizeof(float2) + sizeof(RbCtl);
-}
+// shared memory: the control block and the twiddle table, then (from the next 1024-byte boundary)
+// the T / Q stages and the partner stages.  Dynamic shared memory starts 1024-aligned in practice,
+// so the request is the whole per-block limit and the kernel checks that its layout fits (else it
+// records GS_DEV_ERR_LAYOUT and returns before touching anything).
+constexpr size_t kRbHead = (sizeof(RbCtl) + 15) / 16 * 16 + kRbMaxL * sizeof(float2);
+constexpr size_t kRbData = (size_t)kRbStages * (kRbAStage + kRbBStage) + (size_t)kRbYStages * kRbYStage;
+constexpr size_t kRbSmemBytes = 227 * 1024;
+static_assert(kRbHead + kRbData <= kRbSmemBytes, "layout");
 
 // the transform plan of a block of L = 2 H reals
 template <int H>
@@ -290,19 +296,26 @@ __global__ void __launch_bounds__(kRbThreads, 1)
                const __grid_constant__ RbParams p) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
-    uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
-    uint8_t* As = base;
+    RbCtl& c = *reinterpret_cast<RbCtl*>(smem_raw);
+    float2* tw = reinterpret_cast<float2*>(smem_raw + (sizeof(RbCtl) + 15) / 16 * 16);
+    const uint32_t off = ((raw + (uint32_t)kRbHead + 1023u) & ~1023u) - raw;
+    unsigned* err = &g_err_rbind;
+    if (off + kRbData > kRbSmemBytes) {  // uniform over the grid: every thread leaves here
+        if (threadIdx.x == 0 && blockIdx.x == 0) atomicOr(err, GS_DEV_ERR_LAYOUT);
+        return;
+    }
+    uint8_t* As = smem_raw + off;
     uint8_t* Bs = As + (size_t)kRbStages * kRbAStage;
     uint8_t* Ys = Bs + (size_t)kRbStages * kRbBStage;
-    uint8_t* Zs = Ys + (size_t)kRbYStages * kRbYStage;
-    float2* tw = reinterpret_cast<float2*>(Zs + (size_t)4 * kRbSubs * kRbZStage);
-    RbCtl& c = *reinterpret_cast<RbCtl*>(tw + kRbMaxL);
     volatile int* abort_flag = &c.abort_flag;
-    unsigned* err = &g_err_rbind;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int ntiles = p.tiles > blockIdx.x ? (int)((p.tiles - 1 - blockIdx.x) / gridDim.x + 1) : 0;
+    const uint32_t rank = cluster_ctarank();
+    const bool lead = rank == 0;
+    const long long pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+    const int ntiles = p.tiles > pair ? (int)((p.tiles - 1 - pair) / npairs + 1) : 0;
+    // pair tile lt: rows tm 256 + [0, 256) (this CTA's: + 128 rank), columns tn 256 + [0, 256)
     auto tile_mn = [&](int lt, long long& tm, int& tn) {
-        const long long tg = blockIdx.x + (long long)lt * gridDim.x;
+        const long long tg = pair + (long long)lt * npairs;
         tm = tg / p.tiles_n;
         tn = (int)(tg % p.tiles_n);
     };
@@ -316,7 +329,7 @@ __global__ void __launch_bounds__(kRbThreads, 1)
             mbar_init(&c.y_empty[s], 4);  // one transform warp of each lane quadrant reads a box
         }
         mbar_init(&c.d_full, 1);
-        mbar_init(&c.y_free, 4 * kRbSubs);
+        mbar_init(&c.y_free, 2 * 4 * kRbSubs);  // the transform warps of both CTAs (the even CTA's is used)
         mbar_init(&c.mma_done, 1);
         c.abort_flag = 0;
         fence_barrier_init();
@@ -328,11 +341,12 @@ __global__ void __launch_bounds__(kRbThreads, 1)
         tw[j] = make_float2(co, -s);
     }
     if (warp == 1) {
-        tmem_alloc(&c.tmem_base, 512);
-        tmem_relinquish();
+        tmem_alloc2(&c.tmem_base, 512);
+        tmem_relinquish2();
     }
     tc_fence_before();
     __syncthreads();
+    cluster_sync_all();  // the even CTA's barriers exist before the odd CTA signals them
     tc_fence_after();
     const uint32_t tmem = c.tmem_base;
 
@@ -352,25 +366,32 @@ __global__ void __launch_bounds__(kRbThreads, 1)
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(&c.full[rp.idx], (uint32_t)(kRbAStage + kRbBStage));
-                    tma_load_2d(As + (size_t)rp.idx * kRbAStage, &tmap_a, &c.full[rp.idx], kb * kRbBK,
-                                (int)(tm * kRbBM), pol);
-                    tma_load_2d(Bs + (size_t)rp.idx * kRbBStage, &tmap_b, &c.full[rp.idx], kb * kRbBK, tn * kRbBN,
-                                pol);
+                    // both CTAs' halves complete on the even CTA's full barrier
+                    if (lead) mbar_arrive_expect_tx(&c.full[rp.idx], 2u * (kRbAStage + kRbBStage));
+                    const uint32_t fb = mapa_shared(smem_u32(&c.full[rp.idx]), 0);
+                    tma_load_2d_pair(As + (size_t)rp.idx * kRbAStage, &tmap_a, fb, kb * kRbBK,
+                                     (int)(tm * 2 * kRbBM + kRbBM * rank), pol);
+                    tma_load_2d_pair(Bs + (size_t)rp.idx * kRbBStage, &tmap_b, fb, kb * kRbBK,
+                                     tn * kRbBN + (kRbBN / 2) * (int)rank, pol);
                 }
             }
-            for (int j = std::max(0, it - kRbStages); j < it; ++j)
-                mbar_drain(&c.full[j % kRbStages], (uint32_t)(j / kRbStages) & 1u, err);
+            // the even CTA waits until every stage it expected (both CTAs' loads) has landed; the
+            // odd CTA leaves only after the closing cluster barrier, which the even CTA reaches
+            // after this drain
+            if (lead)
+                for (int j = std::max(0, it - kRbStages); j < it; ++j)
+                    mbar_drain(&c.full[j % kRbStages], (uint32_t)(j / kRbStages) & 1u, err);
         }
     } else if (warp == 1) {
-        // ------------------------------------------------------------- MMA issue
-        if (lane == 0) {
-            const uint32_t idesc = idesc_f16_f32(kRbBN);
+        // ------------------------------------------------------------- pair MMA issue (even CTA)
+        if (lane == 0 && lead) {
+            const uint32_t idesc = idesc2_f16_f32(kRbBN);
             RingPos rp;
             bool ok = true;
             for (int lt = 0; lt < ntiles && ok; ++lt) {
-                // the half this tile accumulates into held the previous tile's partner spectra
-                if (lt > 0 && !mbar_wait_1t(&c.y_free, (uint32_t)(lt - 1) & 1u, abort_flag, err)) break;
+                // the half this tile accumulates into held the previous tile's partner spectra, in both
+                // CTAs (arrivals at cluster scope)
+                if (lt > 0 && !mbar_wait_cluster(&c.y_free, (uint32_t)(lt - 1) & 1u, abort_flag, err)) break;
                 tc_fence_after();
                 const uint32_t d_tmem = tmem + (uint32_t)((lt & 1) * kRbBN);
                 for (int kb = 0; kb < p.nkb; ++kb, rp.next(kRbStages)) {
@@ -383,12 +404,12 @@ __global__ void __launch_bounds__(kRbThreads, 1)
                     const uint64_t bd = sdesc_sw128(smem_u32(Bs + (size_t)rp.idx * kRbBStage));
 #pragma unroll
                     for (int k = 0; k < kRbBK / 16; ++k)
-                        mma_f16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc, (kb | k) != 0 ? 1u : 0u);
-                    mma_commit(&c.empty[rp.idx]);
+                        mma2_f16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc, (kb | k) != 0 ? 1u : 0u);
+                    mma2_commit(&c.empty[rp.idx], 3);
                 }
-                if (ok) mma_commit(&c.d_full);
+                if (ok) mma2_commit(&c.d_full, 3);
             }
-            mma_commit(&c.mma_done);
+            mma2_commit(&c.mma_done, 1);
             mbar_drain(&c.mma_done, 0, err);
         }
     } else if (warp == 2) {
@@ -408,7 +429,7 @@ __global__ void __launch_bounds__(kRbThreads, 1)
                     tile_mn(lt + 1, tm2, tn2);
                     for (int cc = 0; cc < kRbChunks; ++cc)
                         if (tn2 * kRbBN + cc * kRbYCols < p.D)
-                            tma_prefetch_2d(&tmap_y, tn2 * kRbBN + cc * kRbYCols, (int)(tm2 * kRbBM));
+                            tma_prefetch_2d(&tmap_y, tn2 * kRbBN + cc * kRbYCols, (int)(tm2 * 2 * kRbBM + kRbBM * rank));
                 }
                 for (int cc = 0; cc < kRbChunks; ++cc, ++it, rp.next(kRbYStages)) {
                     if (!mbar_wait_1t(&c.y_empty[rp.idx], rp.phase ^ 1u, abort_flag, err)) {
@@ -417,7 +438,7 @@ __global__ void __launch_bounds__(kRbThreads, 1)
                     }
                     mbar_arrive_expect_tx(&c.y_full[rp.idx], (uint32_t)kRbYStage);
                     tma_load_2d(Ys + (size_t)rp.idx * kRbYStage, &tmap_y, &c.y_full[rp.idx],
-                                tn * kRbBN + cc * kRbYCols, (int)(tm * kRbBM), pol);
+                                tn * kRbBN + cc * kRbYCols, (int)(tm * 2 * kRbBM + kRbBM * rank), pol);
                 }
             }
             for (int j = std::max(0, it - kRbYStages); j < it; ++j)
@@ -428,12 +449,11 @@ __global__ void __launch_bounds__(kRbThreads, 1)
         const int quad = warp & 3, sub = (warp - kRbEpi0) >> 2;
         const uint32_t lanes = (uint32_t)(32 * quad) << 16;
         const int rr = 32 * quad + lane;  // this thread's row of the tile
-        uint8_t* zst = Zs + (size_t)(warp - kRbEpi0) * kRbZStage;
-        // partner box cc of a tile into TMEM columns `half` + 32 cc of this quadrant's lanes (box cc
-        // sits in stage cc % 4 = sub, in the stage's phase cc / 4: each tile uses a stage twice)
-        auto copy_in = [&](int cc, uint32_t half) -> bool {
-            if (!mbar_wait_warp(&c.y_full[sub], (uint32_t)(cc >> 2), abort_flag, err)) return false;
-            const uint8_t* ys = Ys + (size_t)sub * kRbYStage + (size_t)rr * 128;
+        // partner box cc of tile 0 into TMEM columns 256 + 32 cc of this quadrant's lanes; the stage
+        // goes back to the producer at once (box cc of every tile sits in stage cc, phase lt & 1)
+        auto copy_in0 = [&](int cc) -> bool {
+            if (!mbar_wait_warp(&c.y_full[cc], 0u, abort_flag, err)) return false;
+            const uint8_t* ys = Ys + (size_t)cc * kRbYStage + (size_t)rr * 128;
             uint32_t v[32];
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
@@ -445,35 +465,20 @@ __global__ void __launch_bounds__(kRbThreads, 1)
             }
             // release the stage only once every lane holds its values (the TMEM store consumes
             // them) and its reads are ordered before the TMA refill's writes (async proxy)
-            tmem_st32(tmem + lanes + half + (uint32_t)(kRbYCols * cc), v);
+            tmem_st32(tmem + lanes + (uint32_t)(kRbBN + kRbYCols * cc), v);
             fence_proxy_async();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&c.y_empty[sub]);
+            if (lane == 0) mbar_arrive(&c.y_empty[cc]);
             return true;
         };
-        // 16 output columns from registers through this warp's staging to a tensor store
-        auto store_box = [&](const uint32_t* v, int x, long long y) {
-            if (lane == 0) bulk_wait_read_0();  // the previous store has read the staging
-            __syncwarp();
-#pragma unroll
-            for (int u = 0; u < 4; ++u)
-                *reinterpret_cast<uint4*>(zst + lane * 64 + ((u ^ ((lane >> 1) & 3)) << 4)) =
-                    make_uint4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
-            fence_proxy_async();
-            __syncwarp();
-            if (lane == 0) {
-                if (x < p.D && y < p.m) tma_store_2d(&tmap_z, zst, x, (int)y);
-                bulk_commit();
-            }
-        };
         bool ok = ntiles > 0;
-        if (ok) ok = copy_in(sub, kRbBN) && copy_in(sub + 4, kRbBN);  // tile 0's partner half: 256
+        if (ok) ok = copy_in0(sub) && copy_in0(sub + 4);
         for (int lt = 0; lt < ntiles; ++lt) {
             const uint32_t hx = (uint32_t)((lt & 1) * kRbBN), hy = (uint32_t)kRbBN - hx;
             long long tm;
             int tn;
             tile_mn(lt, tm, tn);
-            const long long row0 = tm * kRbBM;
+            const long long row0 = tm * 2 * kRbBM + kRbBM * rank;
             if (!quad_sync(quad, ok)) break;
             rb_strided<H, false, false>(tmem + lanes + hy, sub, 1.f, tw);
             ok = mbar_wait_warp(&c.d_full, (uint32_t)lt & 1u, abort_flag, err);
@@ -487,24 +492,64 @@ __global__ void __launch_bounds__(kRbThreads, 1)
             rb_middle<H, UNB>(tmem + lanes + hx, tmem + lanes + hy, sub, tw);
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&c.y_free);  // this warp is done with the partner half
+            if (lane == 0) {  // this warp is done with the partner half
+                if (lead)
+                    mbar_arrive(&c.y_free);
+                else
+                    mbar_arrive_cluster(mapa_shared(smem_u32(&c.y_free), 0));
+            }
             if (!quad_sync(quad, true)) break;
             rb_strided<H, true, true>(tmem + lanes + hx, sub, p.zscale, tw);
             if (!quad_sync(quad, true)) break;
-            // output columns 32 cc .. 32 cc + 31 of this quadrant's rows (cc = sub, sub + 4); once a
-            // chunk is in registers its TMEM columns take the next tile's partner box cc (this
-            // half is the next tile's partner half), between the chunk's two tensor stores
+            // output columns 32 cc .. 32 cc + 31 of this quadrant's rows (cc = sub, sub + 4).  Sixteen
+            // columns at a time: the outputs come out of TMEM, the next tile's partner values for the
+            // same columns come out of this warp's 32 rows of stage cc and go into TMEM in their place
+            // (this half is the next tile's partner half), and the outputs take their place in the
+            // stage; the 32 x 32 box then leaves by one tensor store (128-byte swizzle, as loaded).
+            // After the last tile the stage has no refill pending, so its rows are free.
             const long long y = row0 + 32 * quad;
             const bool more = lt + 1 < ntiles;
             for (int h = 0; h < 2; ++h) {
                 const int cc = sub + 4 * h;
-                uint32_t v[32];
-                tmem_ld32_issue(tmem + lanes + hx + (uint32_t)(kRbYCols * cc), v);
-                tmem_wait_ld32(v);
+                uint8_t* slice = Ys + (size_t)cc * kRbYStage + (size_t)(32 * quad) * 128;
+                if (more && ok) ok = mbar_wait_warp(&c.y_full[cc], (uint32_t)(lt + 1) & 1u, abort_flag, err);
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh) {
+                    const uint32_t col = tmem + lanes + hx + (uint32_t)(kRbYCols * cc + 16 * hh);
+                    float z[16];
+                    tmem_ld16(col, z);
+                    uint8_t* rowp = slice + lane * 128;
+                    if (more && ok) {
+                        uint32_t v[16];
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) {
+                            const uint4 f = *reinterpret_cast<const uint4*>(rowp + (((4 * hh + u) ^ (lane & 7)) << 4));
+                            v[4 * u] = f.x;
+                            v[4 * u + 1] = f.y;
+                            v[4 * u + 2] = f.z;
+                            v[4 * u + 3] = f.w;
+                        }
+                        tmem_st16(col, v);
+                    }
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+                        *reinterpret_cast<float4*>(rowp + (((4 * hh + u) ^ (lane & 7)) << 4)) =
+                            make_float4(z[4 * u], z[4 * u + 1], z[4 * u + 2], z[4 * u + 3]);
+                }
+                fence_proxy_async();
+                __syncwarp();
                 const int x = tn * kRbBN + cc * kRbYCols;
-                store_box(v, x, y);
-                if (more && ok) ok = copy_in(cc, hx);
-                store_box(v + 16, x + kRbZCols, y);
+                if (lane == 0) {
+                    if (x < p.D && y < p.m) tma_store_2d(&tmap_z, slice, x, (int)y);
+                    bulk_commit();
+                }
+            }
+            // both boxes read: the stages go back to the producer for the tile after next
+            if (lane == 0) bulk_wait_read_0();
+            __syncwarp();
+            if (more && lane == 0) {
+                mbar_arrive(&c.y_empty[sub]);
+                mbar_arrive(&c.y_empty[sub + 4]);
             }
         }
         if (lane == 0) bulk_wait_all();
@@ -512,9 +557,10 @@ __global__ void __launch_bounds__(kRbThreads, 1)
 
     tc_fence_before();
     __syncthreads();
+    cluster_sync_all();  // neither CTA leaves while the other may still signal its barriers
     if (warp == 1) {
         tc_fence_after();
-        tmem_dealloc(tmem, 512);
+        tmem_dealloc2(tmem, 512);
     }
 }
 
@@ -536,8 +582,19 @@ static cudaError_t rb_launch(int grid, size_t smem, cudaStream_t s, const CUtens
         if (e != cudaSuccess) return e;
         attr[device] = true;
     }
-    k_rbind_tc<H, UNB><<<grid, kRbThreads, smem, s>>>(ta, tb, ty, tz, p);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kRbThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_rbind_tc<H, UNB>, ta, tb, ty, tz, p);
 }
 
 cudaError_t launch_rbind_tc(const gs_basis* h, const void* T16, long long ld16, long long m, const float* rowmul,
@@ -551,22 +608,22 @@ cudaError_t launch_rbind_tc(const gs_basis* h, const void* T16, long long ld16, 
     p.D = h->D;
     p.nkb = (h->r + kRbBK - 1) / kRbBK;
     p.tiles_n = (h->D + kRbBN - 1) / kRbBN;
-    p.tiles = ((m + kRbBM - 1) / kRbBM) * (long long)p.tiles_n;
+    p.tiles = ((m + 2 * kRbBM - 1) / (2 * kRbBM)) * (long long)p.tiles_n;  // pair tiles of 256 rows
     p.zscale = 1.0f / (4.0f * (float)L);
     p.rowmul = rowmul;
     CUtensorMap ta, tb, ty, tz;
     if (!make_tmap_2d(&ta, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, T16, m, h->r, ld16, kRbBK, kRbBM,
                       CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_tmap_2d(&tb, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, h->Q16t, h->D, h->r, h->ldr16, kRbBK, kRbBN,
+        !make_tmap_2d(&tb, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, h->Q16t, h->D, h->r, h->ldr16, kRbBK, kRbBN / 2,
                       CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_tmap_2d(&ty, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, Y, m, h->D, ldy, kRbYCols, kRbBM,
                       CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_tmap_2d(&tz, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, Z, m, h->D, ldz, kRbZCols, 32, CU_TENSOR_MAP_SWIZZLE_64B))
+        !make_tmap_2d(&tz, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, Z, m, h->D, ldz, kRbYCols, 32, CU_TENSOR_MAP_SWIZZLE_128B))
         return cudaErrorInvalidValue;
     int sms = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
-    const int grid = (int)std::min<long long>(sms > 0 ? sms : 1, p.tiles);
-    const size_t smem = rb_smem_bytes();
+    const int grid = 2 * (int)std::min<long long>(std::max(sms / 2, 1), p.tiles);  // CTA pairs
+    const size_t smem = kRbSmemBytes;
     switch (L) {
         case 64:
             return unbind ? rb_launch<32, true>(grid, smem, s, ta, tb, ty, tz, p, device)
