@@ -164,6 +164,26 @@ def test_tc_two_gemm_rank_deficient(gs, orc, rankdef_ref, mode):
     assert np.all(np.abs(host(out["Y"]) - ref["Y"]) <= TOL_S * ref["xnorm"][:, None])
 
 
+@pytest.mark.parametrize("M,D,N", [(600, 2048, 700), (1024, 2048, 1100), (300, 2304, 257)])
+def test_tc_two_gemm_widths(gs, orc, M, D, N):
+    """The projection of the two-GEMM path for r > 256 (128 x 512 tiles, two 256-column
+    accumulators fed by each converted K-block): r = 600 (a second tile 88 columns wide), 1,024 (two
+    full tiles) and 300 (one tile, the second accumulator 44 columns wide); N = 700, 1,100 and 257
+    end in a partial row tile."""
+    rng = np.random.default_rng(M + D)
+    C = np.where(rng.random((M, D)) < 0.5, -1.0, 1.0).astype(np.float32)
+    X, _ = synth.noisy_rows(C, 23, 0, N, 1.0)
+    b = gs.build_basis(cuda(C))
+    Qo, Ro, cno = orc.build_basis(C)
+    assert b.r == M
+    for mode in ("raw", "cosine"):
+        out = gs.project_similarity(b, cuda(X), mode=mode, path="tensor", want_S=True, want_Y=True)
+        gs.stream_status()
+        ref = orc.project_similarity(X, Qo, Ro, cno, mode=getattr(orc, mode.upper()))
+        check_scores(out, ref, X, cno, mode)
+        assert np.all(np.abs(host(out["Y"]) - ref["Y"]) <= TOL_S * ref["xnorm"][:, None])
+
+
 def test_tc_two_gemm_wide_codebook(gs, orc):
     """M = 300 > 256 codewords in D = 200 (rank 200 < M, Sec. 3.1's D < M case)."""
     rng = np.random.default_rng(21)
