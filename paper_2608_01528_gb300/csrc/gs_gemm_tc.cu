@@ -422,11 +422,24 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
             }
             const uint8_t* Xt = Xs + (size_t)sx * kXStageBytes;
             uint8_t* At = As + (size_t)sa * p.parts * kAPartBytes;
+            // fp16 A: the whole K-block into registers first, so the staging stage goes back to
+            // the A producer before the conversion rather than after it (the split mode, with
+            // twice the stores per element, keeps the loads inside the loop: its registers are
+            // spoken for)
+            constexpr bool kEarlyX = AMODE == kAF16;
+            float4 xv[kCvtRows];
+            if (kEarlyX) {
+#pragma unroll
+                for (int u = 0; u < kCvtRows; ++u)
+                    xv[u] = *reinterpret_cast<const float4*>(Xt + (rbase + kCvtRowStep * u) * (kBK * 4) + c4 * 16);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&c.x_empty[sx]);
+            }
             float nrm[kCvtRows];  // this K-block's part of ||a||^2 of each of the thread's rows
 #pragma unroll
             for (int u = 0; u < kCvtRows; ++u) {
                 const int row = rbase + kCvtRowStep * u;
-                const float4 x = *reinterpret_cast<const float4*>(Xt + row * (kBK * 4) + c4 * 16);
+                const float4 x = kEarlyX ? xv[u] : *reinterpret_cast<const float4*>(Xt + row * (kBK * 4) + c4 * 16);
                 const int off = row * 128 + (((c4 >> 1) ^ (row & 7)) * 16) + (c4 & 1) * 8;
                 uint2 hi;
                 if (AMODE == kAF16) {
@@ -451,7 +464,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
             __syncwarp();
             if (lane == 0) {
                 mbar_arrive(&c.a_full[sa]);
-                mbar_arrive(&c.x_empty[sx]);
+                if (!kEarlyX) mbar_arrive(&c.x_empty[sx]);
             }
             if (want_xn2) {
                 // butterfly over the 16 lanes of a row phase: after the step with lane bit b, a
