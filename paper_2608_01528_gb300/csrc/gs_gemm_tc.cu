@@ -425,17 +425,25 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
             // fp16 A: the whole K-block into registers first, so the staging stage goes back to
             // the A producer before the conversion rather than after it (the split mode, with
             // twice the stores per element, keeps the loads inside the loop: its registers are
-            // spoken for)
+            // spoken for).  Every loaded value is used (range, norm) before the stage is released:
+            // an arrive issued while loads were still outstanding let the TMA refill overwrite
+            // the stage under them
             constexpr bool kEarlyX = AMODE == kAF16;
             float4 xv[kCvtRows];
+            float nrm[kCvtRows];  // this K-block's part of ||a||^2 of each of the thread's rows
             if (kEarlyX) {
 #pragma unroll
                 for (int u = 0; u < kCvtRows; ++u)
                     xv[u] = *reinterpret_cast<const float4*>(Xt + (rbase + kCvtRowStep * u) * (kBK * 4) + c4 * 16);
+#pragma unroll
+                for (int u = 0; u < kCvtRows; ++u) {
+                    const float4 x = xv[u];
+                    amax = fmaxf(amax, fmaxf(fmaxf(fabsf(x.x), fabsf(x.y)), fmaxf(fabsf(x.z), fabsf(x.w))));
+                    nrm[u] = fmaf(x.x, x.x, fmaf(x.y, x.y, fmaf(x.z, x.z, x.w * x.w)));
+                }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&c.x_empty[sx]);
             }
-            float nrm[kCvtRows];  // this K-block's part of ||a||^2 of each of the thread's rows
 #pragma unroll
             for (int u = 0; u < kCvtRows; ++u) {
                 const int row = rbase + kCvtRowStep * u;
@@ -443,8 +451,6 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                 const int off = row * 128 + (((c4 >> 1) ^ (row & 7)) * 16) + (c4 & 1) * 8;
                 uint2 hi;
                 if (AMODE == kAF16) {
-                    amax = fmaxf(amax, fmaxf(fmaxf(fabsf(x.x), fabsf(x.y)), fmaxf(fabsf(x.z), fabsf(x.w))));
-                    nrm[u] = fmaf(x.x, x.x, fmaf(x.y, x.y, fmaf(x.z, x.z, x.w * x.w)));
                     const __half2 h0 = __floats2half2_rn(x.x, x.y), h1 = __floats2half2_rn(x.z, x.w);
                     hi.x = *reinterpret_cast<const uint32_t*>(&h0);
                     hi.y = *reinterpret_cast<const uint32_t*>(&h1);

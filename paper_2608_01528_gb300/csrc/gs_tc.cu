@@ -384,21 +384,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!wait_warp(&c.x_full[sx], rx.phase) || !wait_warp(&c.a_empty[sa], ra.phase ^ 1u)) return false;
                 const uint8_t* Xt = Xs + (size_t)sx * p.xstage;
                 uint8_t* At = As + (size_t)sa * kAStageBytes;
-                // the whole K-block into registers first, so the staging stage goes back to the X
-                // producer before the conversion rather than after it
-                float4 xv[kCvtRows];
 #pragma unroll
                 for (int u = 0; u < kCvtRows; ++u) {
                     const int row = rbase + kCvtRowStep * u;
-                    xv[u] = row < tr.nrows ? *reinterpret_cast<const float4*>(Xt + row * (kBK * 4) + c4 * 16)
-                                           : make_float4(0.f, 0.f, 0.f, 0.f);
-                }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&c.x_empty[sx]);
-#pragma unroll
-                for (int u = 0; u < kCvtRows; ++u) {
-                    const int row = rbase + kCvtRowStep * u;
-                    float4 x = xv[u];
+                    float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (row < tr.nrows) x = *reinterpret_cast<const float4*>(Xt + row * (kBK * 4) + c4 * 16);
                     if (redo) {  // exact power-of-two scale: the fp16 rounding below loses nothing to range
                         const float sc = pow2f(rs[row]);
                         x.x *= sc;
@@ -418,7 +408,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 fence_proxy_async();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&c.a_full[sa]);
+                if (lane == 0) {
+                    mbar_arrive(&c.a_full[sa]);
+                    mbar_arrive(&c.x_empty[sx]);
+                }
             }
             // tile finished: this group's part of ||x||^2 of each row is added into shared memory
 #pragma unroll
