@@ -8,12 +8,13 @@
 //   2. twice (reorthogonalisation): H = V Q_old^T (tiled fp64 dot products
 //      over D-slices, then a slice reduction that also accumulates R), and
 //      V -= H Q_old -- a block projection against the basis built so far;
-//   3. one CTA runs modified Gram-Schmidt with two passes over the panel's own
-//      new directions, row by row, decides rank (||v|| > tol * ||c_i||),
-//      normalises and appends accepted rows to Q.
+//   3. a cluster of CTAs (each owning a slice of the columns) runs Gram-Schmidt
+//      with two passes over the panel's own new directions, row by row, decides
+//      rank (||v|| > tol * ||c_i||), normalises and appends accepted rows to Q.
 // In exact arithmetic this is the row-wise two-pass Gram-Schmidt of the
 // paper's construction (projections onto orthonormal directions commute);
-// the block passes against the old basis are what make it data-parallel.
+// the block passes against the old basis and the column slices within the
+// panel are what make it data-parallel.
 // The only host synchronisation is the read of the final rank r.
 //
 // Afterwards fp32 copies of Q and R are made for the caller, plus the
@@ -164,41 +165,139 @@ __global__ void __launch_bounds__(256) k_panel_update(double* __restrict__ V,
     }
 }
 
-// 3. modified Gram-Schmidt (two passes) inside the panel, rank decision,
-//    normalisation and append.  One CTA of 1024 threads; thread t owns the
-//    columns d = t, t + 1024, ... of every vector it touches.
-__global__ void __launch_bounds__(1024) k_panel_mgs(double* __restrict__ V, double* __restrict__ Qw,
-                                                     int D, int bp, int p0, double tau,
-                                                     const double* __restrict__ cn,
-                                                     double* __restrict__ R64, int ldr,
-                                                     int* __restrict__ r_dev, int rmax) {
-    __shared__ double sh[33];
+// 3. Gram-Schmidt with two passes inside the panel, rank decision, normalisation and append, on a
+//    cluster of kMgsCtas CTAs: CTA c owns columns [c S, (c + 1) S) of every vector (S = ceil(D /
+//    kMgsCtas)), so the fp64 arithmetic of a row is spread over kMgsCtas SMs (GB300's fp64 rate
+//    per SM is low: one CTA doing this took 1.5 ms per 16-row panel of 10,000-wide rows).  Each
+//    pass takes the projections of v on all of the panel's new directions at once (classical
+//    Gram-Schmidt, twice: the same factorisation as the row-by-row passes in exact arithmetic, and
+//    as stable with the second pass), so a row needs three sums over the whole row: the two passes'
+//    projections and the norm.  A sum is reduced in each CTA, posted into every CTA's shared memory
+//    and added there in CTA order after a cluster barrier, so every CTA holds the same values, takes
+//    the same rank decisions and runs the same number of barriers (3 per row): no wait can be left
+//    without its partners.  Partial sums alternate between two buffers, so one barrier per sum
+//    suffices (a buffer is written again only after the next sum's barrier, which every CTA reaches
+//    once it has read the buffer).
+constexpr int kMgsCtas = 8;
+constexpr int kMgsThreads = 256;
+static_assert(kPanel == 16, "the sums' butterfly gives lane l entry l & 15");
+
+__device__ __forceinline__ void st_cluster_f64(uint32_t caddr, double v) {
+    asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(caddr), "d"(v) : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ uint32_t map_to_rank(const void* p, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
+                 : "=r"(r)
+                 : "r"((uint32_t)__cvta_generic_to_shared(p)), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ void cluster_barrier() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__global__ void __launch_bounds__(kMgsThreads) k_panel_gs2(double* __restrict__ V, double* __restrict__ Qw, int D,
+                                                          int bp, int p0, double tau, const double* __restrict__ cn,
+                                                          double* __restrict__ R64, int ldr, int* __restrict__ r_dev,
+                                                          int rmax) {
+    __shared__ double part[2][kMgsCtas][kPanel];  // per sum: every CTA's partials (posted by that CTA)
+    __shared__ double red[kMgsThreads / 32][kPanel];
+    const uint32_t rank = cluster_rank();
+    const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+    const int S = (D + kMgsCtas - 1) / kMgsCtas;
+    const int c0 = (int)rank * S, c1 = min(D, c0 + S);
     const int r0 = *r_dev;
-    int r = r0;
+    int r = r0, nsum = 0;
+    cluster_barrier();  // every CTA of the cluster is running before anyone posts into its memory
+
+    // the sum over the cluster of acc[0..kPanel) (this thread's part): reduced in the CTA, posted to
+    // every CTA, added in CTA order; the result is identical in every thread of every CTA
+    auto cluster_sum = [&](double (&acc)[kPanel], double (&out)[kPanel]) {
+        // warp: a butterfly over the lane bits 3..0 leaves lane l with the sum of entry l & 15 over
+        // its half-warp (after the step with lane bit b a lane keeps the entries whose index has bit
+        // b equal to its own), then the two half-warps are added: 16 shuffles instead of 80
+#pragma unroll
+        for (int wb = kPanel / 2; wb >= 1; wb >>= 1) {
+            const bool up = (lane & wb) != 0;
+#pragma unroll
+            for (int j = 0; j < wb; ++j) {
+                const double send = up ? acc[j] : acc[j + wb];
+                const double keep = up ? acc[j + wb] : acc[j];
+                acc[j] = keep + __shfl_xor_sync(0xffffffffu, send, wb);
+            }
+        }
+        acc[0] += __shfl_xor_sync(0xffffffffu, acc[0], 16);
+        __syncthreads();  // red is free (its previous readers are past this point)
+        if (lane < kPanel) red[w][lane] = acc[0];
+        __syncthreads();
+        const int slot = nsum & 1;
+        if (tid < kPanel * kMgsCtas) {
+            const int j = tid % kPanel, dest = tid / kPanel;
+            double v = 0.0;
+            for (int ww = 0; ww < kMgsThreads / 32; ++ww) v += red[ww][j];
+            st_cluster_f64(map_to_rank(&part[slot][rank][j], (uint32_t)dest), v);
+        }
+        cluster_barrier();
+#pragma unroll
+        for (int j = 0; j < kPanel; ++j) {
+            double v = 0.0;
+            for (int c = 0; c < kMgsCtas; ++c) v += part[slot][c][j];
+            out[j] = v;
+        }
+        ++nsum;
+    };
+
     for (int k = 0; k < bp; ++k) {
         double* v = V + (size_t)k * D;
         double* Rrow = R64 + (size_t)(p0 + k) * ldr;
+        const int nj = r - r0;  // the panel's new directions so far
         for (int pass = 0; pass < 2; ++pass) {
-            for (int j = r0; j < r; ++j) {
-                const double* q = Qw + (size_t)j * D;
-                double part = 0.0;
-                for (int d = threadIdx.x; d < D; d += 1024) part += q[d] * v[d];
-                const double h = block_sum<1024>(part, sh);
-                for (int d = threadIdx.x; d < D; d += 1024) v[d] -= h * q[d];
-                if (threadIdx.x == 0) Rrow[j] += h;
+            double acc[kPanel], h[kPanel];
+#pragma unroll
+            for (int j = 0; j < kPanel; ++j) acc[j] = 0.0;
+            for (int d = c0 + tid; d < c1; d += kMgsThreads) {
+                const double x = v[d];
+#pragma unroll
+                for (int j = 0; j < kPanel; ++j)
+                    if (j < nj) acc[j] += Qw[(size_t)(r0 + j) * D + d] * x;
+            }
+            cluster_sum(acc, h);
+            for (int d = c0 + tid; d < c1; d += kMgsThreads) {
+                double x = v[d];
+#pragma unroll
+                for (int j = 0; j < kPanel; ++j)
+                    if (j < nj) x -= h[j] * Qw[(size_t)(r0 + j) * D + d];
+                v[d] = x;
+            }
+            if (rank == 0 && tid < nj) {
+                double hv = 0.0;  // h[tid] without a dynamic index (which would move h to local memory)
+#pragma unroll
+                for (int j = 0; j < kPanel; ++j)
+                    if (j == tid) hv = h[j];
+                Rrow[r0 + tid] += hv;
             }
         }
-        double part = 0.0;
-        for (int d = threadIdx.x; d < D; d += 1024) part += v[d] * v[d];
-        const double nu = sqrt(block_sum<1024>(part, sh));
+        double acc[kPanel], nn[kPanel];
+#pragma unroll
+        for (int j = 0; j < kPanel; ++j) acc[j] = 0.0;
+        for (int d = c0 + tid; d < c1; d += kMgsThreads) acc[0] += v[d] * v[d];
+        cluster_sum(acc, nn);
+        const double nu = sqrt(nn[0]);
         if (nu > tau * cn[p0 + k] && r < rmax) {
             double* q = Qw + (size_t)r * D;
-            for (int d = threadIdx.x; d < D; d += 1024) q[d] = v[d] / nu;
-            if (threadIdx.x == 0) Rrow[r] = nu;
+            for (int d = c0 + tid; d < c1; d += kMgsThreads) q[d] = v[d] / nu;
+            if (rank == 0 && tid == 0) Rrow[r] = nu;
             ++r;
         }
+        __syncthreads();  // this CTA's columns of the new direction are written before they are read
     }
-    if (threadIdx.x == 0) *r_dev = r;
+    if (rank == 0 && tid == 0) *r_dev = r;
+    cluster_barrier();  // no CTA leaves while a peer may still post into its memory
 }
 
 // ----------------------------------------------------------------- finalisation
@@ -395,7 +494,23 @@ gs_status factor_rows(const float* C, int M, int D, int ldc, double tau, bool no
                 k_panel_update<<<grid1(D, kUpdCols), 256, 0, s>>>(V, Qw, D, bp, r_dev, H, ldh);
             }
         }
-        k_panel_mgs<<<1, 1024, 0, s>>>(V, Qw, D, bp, p0, tau, cn, R64, ldr, r_dev, rmax);
+        {
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3(kMgsCtas);
+            cfg.blockDim = dim3(kMgsThreads);
+            cfg.stream = s;
+            cudaLaunchAttribute at[1];
+            at[0].id = cudaLaunchAttributeClusterDimension;
+            at[0].val.clusterDim.x = kMgsCtas;
+            at[0].val.clusterDim.y = 1;
+            at[0].val.clusterDim.z = 1;
+            cfg.attrs = at;
+            cfg.numAttrs = 1;
+            if (kMgsCtas > 8)
+                GS_CK(cudaFuncSetAttribute(k_panel_gs2, cudaFuncAttributeNonPortableClusterSizeAllowed, 1));
+            GS_CK(cudaLaunchKernelEx(&cfg, k_panel_gs2, V, Qw, D, bp, p0, tau, (const double*)cn, R64, ldr, r_dev,
+                                     rmax));
+        }
     }
     GS_CK(cudaGetLastError());
     int r = 0;
