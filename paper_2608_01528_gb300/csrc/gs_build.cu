@@ -27,6 +27,7 @@
 #include <vector>
 
 #include "gs_internal.h"
+#include "gs_tc_ptx.cuh"
 
 namespace gs {
 namespace {
@@ -172,50 +173,42 @@ __global__ void __launch_bounds__(256) k_panel_update(double* __restrict__ V,
 //    pass takes the projections of v on all of the panel's new directions at once (classical
 //    Gram-Schmidt, twice: the same factorisation as the row-by-row passes in exact arithmetic, and
 //    as stable with the second pass), so a row needs three sums over the whole row: the two passes'
-//    projections and the norm.  A sum is reduced in each CTA, posted into every CTA's shared memory
-//    and added there in CTA order after a cluster barrier, so every CTA holds the same values, takes
-//    the same rank decisions and runs the same number of barriers (3 per row): no wait can be left
-//    without its partners.  Partial sums alternate between two buffers, so one barrier per sum
-//    suffices (a buffer is written again only after the next sum's barrier, which every CTA reaches
-//    once it has read the buffer).
+//    projections and the norm.  A sum is reduced in each CTA (a 16-lane butterfly, then across the
+//    warps), and each CTA's partials are stored into every CTA's shared memory with st.async, whose
+//    bytes complete on the receiver's mbarrier for that buffer (no release fence on the sending
+//    side; a cluster barrier per sum cost ~11 us); every CTA adds the partials in CTA order, so all
+//    hold the same values, take the same rank decisions and run the same sums.  Partial sums
+//    alternate between two buffers: a CTA posts sum n + 2 only after it has every partial of sum
+//    n + 1, which each CTA posts after reading sum n, so a buffer is never overwritten while read.
+//    Every wait is bounded (on expiry: GS_DEV_ERR_TIMEOUT, and the kernel runs on to its end).
 constexpr int kMgsCtas = 8;
 constexpr int kMgsThreads = 256;
 static_assert(kPanel == 16, "the sums' butterfly gives lane l entry l & 15");
-
-__device__ __forceinline__ void st_cluster_f64(uint32_t caddr, double v) {
-    asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(caddr), "d"(v) : "memory");
-}
-__device__ __forceinline__ uint32_t cluster_rank() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
-}
-__device__ __forceinline__ uint32_t map_to_rank(const void* p, uint32_t rank) {
-    uint32_t r;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
-                 : "=r"(r)
-                 : "r"((uint32_t)__cvta_generic_to_shared(p)), "r"(rank));
-    return r;
-}
-__device__ __forceinline__ void cluster_barrier() {
-    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
 
 __global__ void __launch_bounds__(kMgsThreads) k_panel_gs2(double* __restrict__ V, double* __restrict__ Qw, int D,
                                                           int bp, int p0, double tau, const double* __restrict__ cn,
                                                           double* __restrict__ R64, int ldr, int* __restrict__ r_dev,
                                                           int rmax) {
-    __shared__ double part[2][kMgsCtas][kPanel];  // per sum: every CTA's partials (posted by that CTA)
+    using namespace ptx;
+    __shared__ double part[2][kMgsCtas][kPanel];  // per sum: every CTA's partials (stored by that CTA)
     __shared__ double red[kMgsThreads / 32][kPanel];
-    const uint32_t rank = cluster_rank();
+    __shared__ uint64_t pbar[2];                  // one barrier per partial buffer: 1 arrival + the bytes
+    __shared__ double total[kPanel];              // the last sum, added once for the whole CTA
+    const uint32_t rank = cluster_ctarank();
     const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
     const int S = (D + kMgsCtas - 1) / kMgsCtas;
     const int c0 = (int)rank * S, c1 = min(D, c0 + S);
     const int r0 = *r_dev;
     int r = r0, nsum = 0;
-    cluster_barrier();  // every CTA of the cluster is running before anyone posts into its memory
+    bool ok = true;  // false once a wait has run out (the results are then flagged as an error)
+    if (tid == 0) {
+        mbar_init(&pbar[0], 1);
+        mbar_init(&pbar[1], 1);
+        fence_barrier_init();
+    }
+    cluster_sync_all();  // every CTA's barriers exist before anyone stores into its memory
 
-    // the sum over the cluster of acc[0..kPanel) (this thread's part): reduced in the CTA, posted to
+    // the sum over the cluster of acc[0..kPanel) (this thread's part): reduced in the CTA, stored into
     // every CTA, added in CTA order; the result is identical in every thread of every CTA
     auto cluster_sum = [&](double (&acc)[kPanel], double (&out)[kPanel]) {
         // warp: a butterfly over the lane bits 3..0 leaves lane l with the sum of entry l & 15 over
@@ -232,23 +225,38 @@ __global__ void __launch_bounds__(kMgsThreads) k_panel_gs2(double* __restrict__ 
             }
         }
         acc[0] += __shfl_xor_sync(0xffffffffu, acc[0], 16);
-        __syncthreads();  // red is free (its previous readers are past this point)
+        __syncthreads();  // red and the last sum's buffer have been read by every thread of this CTA
         if (lane < kPanel) red[w][lane] = acc[0];
         __syncthreads();
         const int slot = nsum & 1;
+        const uint32_t parity = (uint32_t)(nsum >> 1) & 1u;
+        if (tid == 0) mbar_arrive_expect_tx(&pbar[slot], (uint32_t)(kMgsCtas * kPanel * sizeof(double)));
         if (tid < kPanel * kMgsCtas) {
             const int j = tid % kPanel, dest = tid / kPanel;
             double v = 0.0;
             for (int ww = 0; ww < kMgsThreads / 32; ++ww) v += red[ww][j];
-            st_cluster_f64(map_to_rank(&part[slot][rank][j], (uint32_t)dest), v);
+            st_async_f64(mapa_shared(smem_u32(&part[slot][rank][j]), (uint32_t)dest), v,
+                         mapa_shared(smem_u32(&pbar[slot]), (uint32_t)dest));
         }
-        cluster_barrier();
-#pragma unroll
-        for (int j = 0; j < kPanel; ++j) {
+        // sixteen threads wait for every CTA's partials and add them (fp64 adds run at a low rate
+        // on GB300: every thread adding all 128 had cost ~9 us a sum)
+        if (tid < kPanel) {
+            if (ok) {
+                const unsigned long long t0 = globaltimer();
+                for (uint32_t it = 0; !mbar_try_wait_cluster(&pbar[slot], parity); ++it)
+                    if ((it & 255u) == 255u && globaltimer() - t0 > kWaitLimitNs) {
+                        atomicOr(&g_err_build, GS_DEV_ERR_TIMEOUT);
+                        ok = false;
+                        break;
+                    }
+            }
             double v = 0.0;
-            for (int c = 0; c < kMgsCtas; ++c) v += part[slot][c][j];
-            out[j] = v;
+            for (int c = 0; c < kMgsCtas; ++c) v += part[slot][c][tid];
+            total[tid] = v;
         }
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < kPanel; ++j) out[j] = total[j];
         ++nsum;
     };
 
@@ -294,10 +302,9 @@ __global__ void __launch_bounds__(kMgsThreads) k_panel_gs2(double* __restrict__ 
             if (rank == 0 && tid == 0) Rrow[r] = nu;
             ++r;
         }
-        __syncthreads();  // this CTA's columns of the new direction are written before they are read
     }
     if (rank == 0 && tid == 0) *r_dev = r;
-    cluster_barrier();  // no CTA leaves while a peer may still post into its memory
+    cluster_sync_all();  // no CTA leaves while a peer may still store into its memory
 }
 
 // ----------------------------------------------------------------- finalisation

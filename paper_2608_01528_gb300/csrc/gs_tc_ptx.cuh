@@ -134,6 +134,12 @@ static __device__ __forceinline__ void st_async_f32x2(uint32_t caddr, float a, f
                  "f"(a), "f"(b), "r"(cbar)
                  : "memory");
 }
+// The same for one double.
+static __device__ __forceinline__ void st_async_f64(uint32_t caddr, double a, uint32_t cbar) {
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b64 [%0], %1, [%2];" ::"r"(caddr),
+                 "l"(__double_as_longlong(a)), "r"(cbar)
+                 : "memory");
+}
 // Non-blocking test (test_wait, not try_wait): a thread suspended in try_wait on a
 // barrier that only other SMs arrive on was observed to wake late, by microseconds.
 static __device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
