@@ -24,7 +24,7 @@
 // vectorization V = P R (split, B0 / B1 = bf16 hi / lo of R^T).
 //
 // Tiles are 128 x nt (nt <= 256) with the fp32 accumulator double-buffered in
-// TMEM (2 x 256 columns), or, for a long K with A rounded to fp16 and n > 256, 128 x 512
+// TMEM (2 x 256 columns), or, for a long K with A rounded to fp16 and n > 256, 128 x 2 nt (nt <= 256)
 // (two 256-column accumulators filling TMEM, single-buffered: each converted A K-block
 // feeds both); one persistent CTA per SM walks the tiles with the n index fastest (rotated
 // each wave so that no CTA keeps one column tile), so
@@ -112,7 +112,7 @@ struct Ctl {
     int abort_flag;
 };
 
-// AMODE: kAF16, kABF16X2 or kAF16T; HALVES = 2: 128 x 512 tiles (two accumulators, fp16 A, one
+// AMODE: kAF16, kABF16X2 or kAF16T; HALVES = 2: 128 x 2 nt tiles (two accumulators, fp16 A, one
 // B).  Template parameters, so that each kernel carries only its own mode's control flow.
 template <int AMODE, int HALVES>
 __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see kThreads)
@@ -278,7 +278,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
             const uint32_t idesc = AMODE == kABF16X2 ? idesc_bf16_f32(p.nt) : idesc_f16_f32(p.nt);
             RingPos ra, rb;
             bool ok = true;
-            const int nbuf = HALVES == 2 ? 1 : 2;  // a 512-column tile fills TMEM
+            const int nbuf = HALVES == 2 ? 1 : 2;  // a tile of two halves fills TMEM
             for (int lt = 0; lt < ntiles && ok; ++lt) {
                 const int buf = lt % nbuf;
                 if (!mbar_wait_1t(&c.d_empty[buf], ((uint32_t)(lt / nbuf) & 1u) ^ 1u, abort_flag, err)) break;
@@ -340,7 +340,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                         mma_commit(&c.b_empty[sb1]);
                         continue;
                     }
-                    // 512-column tile (fp16 A, one B per half): the A K-block feeds both halves
+                    // wide tile (fp16 A, one B per half): the A K-block feeds both halves
                     for (int hf = 0; hf < 2 && ok; ++hf) {
                         const int sb0 = rb.idx;
                         if (!mbar_wait_1t(&c.b_full[sb0], rb.phase, abort_flag, err)) {
@@ -349,7 +349,7 @@ __global__ void __maxnreg__(96)  // 608 threads: at most 96 registers each (see 
                         }
                         rb.next(p.sb);
                         tc_fence_after();
-                        const uint32_t dh = d_tmem + (uint32_t)(hf * 256);
+                        const uint32_t dh = d_tmem + (uint32_t)(hf * p.nt);  // the halves side by side
                         const uint64_t b0 = sdesc_sw128(smem_u32(Bs + (size_t)sb0 * kBStageBytes));
 #pragma unroll
                         for (int k = 0; k < kBK / 16; ++k)
@@ -955,10 +955,17 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& a, int device, cudaStream_t s) {
     p.K = a.K;
     p.nkb = (a.K + kBK - 1) / kBK;
     p.nt = a.n >= 256 ? 256 : (a.n + 31) / 32 * 32;
-    // a long K with fp32 A rounded to fp16 and more than 256 columns: 512-column tiles, so each
-    // converted A K-block feeds two 256-column MMAs (half the A loads and conversions per
-    // output; the single TMEM accumulator costs one epilogue per tile, small against the K loop)
+    // a long K with fp32 A rounded to fp16 and more than 256 columns: tiles of two column halves
+    // (up to 512 columns), so each converted A K-block feeds two MMAs (half the A loads and
+    // conversions per output; the single TMEM accumulator costs one epilogue per tile, small
+    // against the K loop)
     const int halves = (!a.a_half && !a.split && a.n > 256 && p.nkb >= 32) ? 2 : 1;
+    if (halves == 2) {
+        // the columns split evenly over the wide tiles, each half rounded up to 16 (r = 922: two
+        // tiles of 2 x 240 columns rather than of 2 x 256, whose last 102 columns would be padding)
+        const int nw = (a.n + 511) / 512;
+        p.nt = std::min(256, ((a.n + nw - 1) / nw + 31) / 32 * 16);
+    }
     p.tiles_n = (a.n + p.nt * halves - 1) / (p.nt * halves);
     p.tiles = ((a.m + kBM - 1) / kBM) * (long long)p.tiles_n;
     p.amode = a.a_half ? kAF16T : a.split ? kABF16X2 : kAF16;
