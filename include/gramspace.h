@@ -108,7 +108,8 @@ typedef struct gs_basis gs_basis;
  *      copies of the tensor-core kernels.  Destroy with gs_basis_destroy.
  * Synchronises `stream` once (to learn r).  Requires 1 <= M, 1 <= D, ldc >= D.
  * Errors: GS_ERR_INVALID_ARG, GS_ERR_SHAPE, GS_ERR_NOMEM, GS_ERR_CUDA,
- *         GS_ERR_UNSUPPORTED (no sm_103 device).
+ *         GS_ERR_UNSUPPORTED (no sm_103 device), GS_ERR_TIMEOUT (a bounded wait
+ *         between the cooperating blocks of the build ran out; no handle).
  */
 GS_API gs_status gs_build_basis(const float* C, int M, int D, int ldc, float rank_tol,
                          unsigned flags, void* stream, gs_basis** out);

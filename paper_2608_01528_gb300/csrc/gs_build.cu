@@ -523,6 +523,8 @@ gs_status factor_rows(const float* C, int M, int D, int ldc, double tau, bool no
     int r = 0;
     GS_CK(cudaMemcpyAsync(&r, r_dev, sizeof(int), cudaMemcpyDeviceToHost, s));
     GS_CK(cudaStreamSynchronize(s));
+    // a bounded wait of the panel kernel that ran out leaves the factorisation unusable
+    if (take_device_error_build() & GS_DEV_ERR_TIMEOUT) return GS_ERR_TIMEOUT;
     f.r = r;
     f.ldr = ldr;
     return GS_OK;
